@@ -1,0 +1,377 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle through a route that is independent of the
+oracle's own formula: a different equation of the paper for the same
+quantity, a closed form, a brute-force bit-plane evaluation (the paper's
+bit-serial engine, Algorithm "Bit-plane schedules"), or a library routine in
+a special case.  A plausible mistake in the oracle (a dropped term, a wrong
+sign, a transposed operand, a wrong rounding) fails at least one of them.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+
+from paper_2608_03057_gb300 import schedule, workloads
+
+ALL_CODES = np.arange(-128, 128, dtype=np.int64).astype(np.int8)
+
+
+# ---------------------------------------------------------------- LSB mask --
+
+def test_mask_b8_is_identity(oracle):
+    # b = b_max keeps every plane: the operating weight is the stored weight.
+    assert np.array_equal(oracle.mask(ALL_CODES, 8), ALL_CODES)
+
+
+@pytest.mark.parametrize("b", range(2, 9))
+def test_mask_grid_and_idempotent(oracle, b):
+    m = oracle.mask(ALL_CODES, b).astype(np.int64)
+    k = 8 - b
+    # the value stays on the stored 8-bit grid and is a multiple of 2^k there
+    assert np.all((m + 128) % (1 << k) == 0)
+    # truncation only removes magnitude from the unsigned code
+    assert np.all(m <= ALL_CODES.astype(np.int64)) and np.all(ALL_CODES - m < (1 << k))
+    # idempotent, and chains of truncation compose to the smaller precision
+    assert np.array_equal(oracle.mask(m.astype(np.int8), b), m.astype(np.int8))
+    for b2 in range(2, 9):
+        assert np.array_equal(oracle.mask(oracle.mask(ALL_CODES, b), b2), oracle.mask(ALL_CODES, min(b, b2)))
+    # exactly 2^b distinct operating values
+    assert len(np.unique(m)) == 1 << b
+
+
+def _recursive_lsb_removal(Q, k, n=8):
+    """Eq. lsb_extraction + Eq. lsb_masking with M = 0 applied to the k least
+    significant planes one after another: at level j the (n-j)-bit code is
+    Q_{n-j} = floor(Q / 2^j), its LSB is Q_{n-j} - 2 Q_{n-j-1}, and removing it
+    subtracts 2^j * LSB on the stored grid."""
+    out = Q
+    for j in range(k):
+        q_hi = Q // (1 << j)
+        q_lo = Q // (1 << (j + 1))
+        lsb = q_hi - 2 * q_lo
+        assert lsb in (0, 1)
+        out = out - (1 << j) * lsb
+    return out
+
+
+@pytest.mark.parametrize("b", range(2, 9))
+def test_mask_equals_recursive_lsb_masking(oracle, b):
+    for s in range(-128, 128):
+        Q = s + 128
+        want = _recursive_lsb_removal(Q, 8 - b) - 128
+        assert oracle.mask_scalar(s, b) == want
+        # Eq. hw_multi_lsb: the dropped block is the sum of the low bit-planes
+        lsb_k = sum((1 << p) * ((Q >> p) & 1) for p in range(8 - b))
+        assert Q - lsb_k - 128 == want
+
+
+# ------------------------------------------------------------ quantizers --
+
+def test_truncquant_lsb_is_a_bit():
+    # Eq. truncquant on a normalized weight W in [0,1): Q_{n-1} = floor(Q_n / 2)
+    # is the direct (n-1)-bit quantization, and Eq. lsb_extraction is 0 or 1.
+    W = np.arange(0, 4096) / 4096.0
+    for n in range(2, 9):
+        Qn = np.floor(W * 2 ** n)
+        Qn1 = np.floor(Qn / 2)
+        assert np.array_equal(Qn1, np.floor(W * 2 ** (n - 1)))
+        lsb = Qn - 2 * Qn1
+        assert set(np.unique(lsb)) <= {0.0, 1.0}
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_weight_quant_nests_under_truncation(oracle, mode):
+    # The 2^n (not 2^n - 1) denominator of Eq. weight_scale makes the b-bit
+    # code equal the truncated 8-bit code (Eq. hw_rightshift), in fp32 too.
+    w = workloads.normal((64, 257), seed=11, std=0.02)
+    w[3] += 0.05  # an all-positive row for the asymmetric mode
+    q8 = oracle.quant_weight(w, 8, mode)["q"]
+    for k in range(1, 7):
+        qb = oracle.quant_weight(w, 8 - k, mode)["q"]
+        assert np.array_equal(q8 >> k, qb), k
+
+
+def test_weight_quant_matches_truncquant_on_a_dyadic_grid(oracle):
+    # With max|w| = 1 every step below is exact, so the symmetric-range
+    # quantizer must equal Eq. truncquant on W = (w - min) / (max - min).
+    j = np.arange(-1024, 1025)
+    w = (j / 1024.0).astype(np.float32)[None, :]
+    d = oracle.quant_weight(w, 8, 0)
+    W = (j + 1024) / 2048.0
+    want = np.minimum(np.floor(W * 256), 255)
+    assert np.array_equal(d["q"][0], want)
+    assert d["alpha"][0] == np.float32(1 / 128) and d["z"][0] == 128.0
+
+
+def test_weight_quant_closed_form(oracle):
+    w = workloads.normal((32, 1152), seed=1, std=0.02)
+    d = oracle.quant_weight(w, 8, 0)
+    amax = np.abs(w).max(1)
+    assert np.array_equal(d["alpha"], (amax / 128).astype(np.float32))
+    assert np.all(d["z"] == 128.0)
+    assert np.array_equal(d["s"].astype(np.int32), d["q"] - 128)
+    # floor: alpha (Q - z) lies in (w - alpha, w], except the clamped top code
+    rec = d["alpha"][:, None].astype(np.float64) * (d["q"] - 128)
+    err = w.astype(np.float64) - rec
+    top = d["q"] == 255
+    a = np.broadcast_to(d["alpha"][:, None].astype(np.float64), w.shape)
+    # slack: w/alpha + z is rounded to fp32 (ulp <= 2^-15 below 256) before the floor
+    slack = 2.0 ** -14 * a
+    assert np.all((err[~top] > -slack[~top]) & (err[~top] < a[~top] + slack[~top]))
+    assert np.all(np.abs(err[top]) <= a[top] + slack[top])
+    # the channel minimum maps to code 0, the maximum to 2^n - 1 (Eq. weight_quant clamp)
+    for n in range(32):
+        assert d["q"][n, np.argmax(np.abs(w[n]))] in (0, 255)
+    # Eq. weight_dequant scale: 2^n / (2^n - 1) * alpha
+    np.testing.assert_allclose(d["c"], d["alpha"].astype(np.float64) * 256 / 255, rtol=2e-7)
+
+
+def test_weight_quant_degenerate_row(oracle):
+    w = np.zeros((2, 16), np.float32)
+    w[1] = 0.5
+    d = oracle.quant_weight(w, 8, 0)
+    assert np.all(d["s"][0] == 0) and d["alpha"][0] == 1.0
+    da = oracle.quant_weight(w, 8, 1)
+    # asymmetric degenerate row dequantizes back to its constant value
+    assert np.allclose(da["alpha"][1] * (da["q"][1] - da["z"][1]), 0.5)
+
+
+def test_act_quant_round_half_even(oracle):
+    # min = 0, max = 255 gives alpha = 1, z = 0: codes are rint(x) with ties to even.
+    x = np.array([[0.0, 255.0, 2.5, 3.5, 0.5, 1.5, 254.5, 100.49999]], np.float32)
+    s, alpha, zc = oracle.quant_act(x, 8, 1, 0)
+    assert alpha[0] == 1.0 and zc[0] == 128.0
+    assert list(s[0].astype(int) + 128) == [0, 255, 2, 4, 0, 2, 254, 100]
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("n_bits", [8, 4])
+def test_act_quant_closed_form(oracle, mode, n_bits):
+    x = workloads.normal((64, 1152), seed=0)
+    x[5] = np.abs(x[5]) + 0.1  # a row that does not straddle zero
+    s, alpha, zc = oracle.quant_act(x, n_bits, mode, 0)
+    half = 1 << (n_bits - 1)
+    Q = s.astype(np.int64) + half
+    assert Q.min() >= 0 and Q.max() <= 2 ** n_bits - 1
+    lo = x.min(1) if mode else -np.abs(x).max(1)
+    hi = x.max(1) if mode else np.abs(x).max(1)
+    np.testing.assert_allclose(alpha, (hi.astype(np.float64) - lo) / (2 ** n_bits - 1), rtol=1e-6)
+    z = half - zc.astype(np.float64)
+    np.testing.assert_allclose(z, -lo / alpha.astype(np.float64), rtol=1e-6, atol=1e-5)
+    # round to nearest: |x - alpha (Q - z)| <= alpha / 2 (plus fp32 slack)
+    rec = alpha[:, None].astype(np.float64) * (Q - z[:, None])
+    assert np.all(np.abs(x - rec) <= alpha[:, None] * (0.5 + 1e-4))
+    # the range ends land on the extreme codes
+    if mode:
+        assert np.all(Q[np.arange(64), x.argmin(1)] == 0)
+        assert np.all(Q[np.arange(64), x.argmax(1)] == 2 ** n_bits - 1)
+
+
+def test_act_quant_per_tensor_equals_single_row(oracle):
+    x = workloads.normal((7, 33), seed=3)
+    s_t, a_t, z_t = oracle.quant_act(x, 8, 0, 1)
+    s_r, a_r, z_r = oracle.quant_act(x.reshape(1, -1), 8, 0, 0)
+    assert np.array_equal(s_t.reshape(-1), s_r.reshape(-1)) and a_t[0] == a_r[0] and z_t[0] == z_r[0]
+
+
+# ------------------------------------------------------------ contraction --
+
+def _engine_bitserial(Qx, Qw, a_bits=8, w_planes=range(8)):
+    """The bit-serial schedule of the paper's engine on unsigned codes:
+    sum over weight planes i and activation planes j of
+    2^(i+j) * popcount(W_i AND A_j)."""
+    total = 0
+    for i in w_planes:
+        Wi = [(q >> i) & 1 for q in Qw]
+        for j in range(a_bits):
+            Aj = [(q >> j) & 1 for q in Qx]
+            total += (1 << (i + j)) * sum(wi & aj for wi, aj in zip(Wi, Aj))
+    return total
+
+
+@pytest.mark.parametrize("b", [8, 6, 5, 3, 2])
+def test_gemm_equals_bitserial_engine(oracle, b):
+    M, N, K = 3, 4, 37
+    s_x = workloads.uniform_codes((M, K), seed=5, lo=-128, hi=127)
+    s_w = workloads.uniform_codes((N, K), seed=6, lo=-128, hi=127)
+    acc = oracle.gemm(s_x, s_w, b)
+    k = 8 - b
+    for m in range(M):
+        for n in range(N):
+            Qx = [int(v) + 128 for v in s_x[m]]
+            Qw8 = [int(v) + 128 for v in s_w[n]]
+            # the engine streams only the top b stored planes (App. F.2)
+            E = _engine_bitserial(Qx, Qw8, 8, range(k, 8))
+            wm = [((q >> k) << k) for q in Qw8]  # operating code on the stored grid
+            # E = sum (s_x + 128)(w' + 128) with w' the signed operating weight
+            want = E - 128 * sum(int(v) for v in s_x[m]) - 128 * sum(q - 128 for q in wm) - 128 * 128 * K
+            assert acc[m, n] == want
+
+
+def test_gemm_signed_planes_brute_force(oracle):
+    # Two's-complement plane decomposition of the masked weight (plane 7 weighs -128).
+    M, N, K = 4, 5, 50
+    s_x = workloads.uniform_codes((M, K), seed=8, lo=-128, hi=127).astype(np.int64)
+    s_w = workloads.uniform_codes((N, K), seed=9, lo=-128, hi=127)
+    for b in (8, 4):
+        wm = oracle.mask(s_w, b).astype(np.int64) & 0xFF
+        acc = oracle.gemm(s_x.astype(np.int8), s_w, b)
+        for m in range(M):
+            for n in range(N):
+                tot = 0
+                for p in range(8):
+                    plane = (wm[n] >> p) & 1
+                    weight = -(1 << p) if p == 7 else (1 << p)
+                    tot += weight * int(np.dot(plane, s_x[m]))
+                assert acc[m, n] == tot
+
+
+def test_gemm_closed_forms(oracle):
+    K = 1024
+    a = np.full((2, K), -128, np.int8)
+    w = np.full((3, K), -128, np.int8)
+    assert np.all(oracle.gemm(a, w, 8) == 16384 * K)
+    assert np.all(oracle.gemm(a, w, 2) == 16384 * K)  # -128 survives every mask
+    one = np.ones((2, K), np.int8)
+    w7 = np.full((3, K), 127, np.int8)
+    for b in range(2, 9):
+        assert np.all(oracle.gemm(one, w7, b) == K * (127 & ~((1 << (8 - b)) - 1)))
+    # operand order: acc[m][n] pairs row m of s_x with row n of s_w
+    x = np.zeros((2, 4), np.int8)
+    x[1, 2] = 1
+    ww = np.zeros((3, 4), np.int8)
+    ww[2, 2] = 64
+    acc = oracle.gemm(x, ww, 8)
+    assert acc[1, 2] == 64 and acc.sum() == 64
+
+
+def test_gemm_int32_overflow_is_reported(oracle):
+    K = 131073  # 16384 * K > 2^31 - 1
+    a = np.full((1, K), -128, np.int8)
+    with pytest.raises(OverflowError):
+        oracle.gemm(a, a, 8)
+
+
+# --------------------------------------------------------------- epilogue --
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("b", [8, 5, 3])
+def test_epilogue_f32_matches_definition(oracle, mode, b):
+    M, N, K = 48, 40, 1152
+    x = workloads.normal((M, K), seed=21)
+    w = workloads.normal((N, K), seed=22, std=0.02)
+    bias = workloads.normal((N,), seed=23, std=0.02)
+    wq = oracle.quant_weight(w, 8, 0)
+    s_x, alpha, zc = oracle.quant_act(x, 8, mode, 0)
+    acc = oracle.gemm(s_x, wq["s"], b)
+    rs = oracle.row_sums(wq["s"], b)
+    y32, ybf = oracle.epilogue_f32(acc, alpha, zc, rs, wq["c"], bias)
+    y64 = oracle.linear_def_f64(s_x, alpha, zc, wq["s"], wq["c"], bias, b)
+    # the factored fp32 sequence is the definition up to a few fp32 roundings
+    scale = np.abs(alpha)[:, None] * np.abs(wq["c"])[None, :] * (np.abs(acc) + np.abs(zc)[:, None] * np.abs(rs)[None, :])
+    assert np.all(np.abs(y32 - y64) <= 8 * 2.0 ** -24 * (scale + np.abs(y64)) + 1e-9)
+    # bf16 output is within half a bf16 ulp of the definition, plus that slack
+    yb = oracle.bf16_bits_to_f32(ybf).astype(np.float64)
+    ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(y64), 1e-30))) - 7)
+    assert np.all(np.abs(yb - y64) <= 0.5 * ulp + 8 * 2.0 ** -24 * (scale + np.abs(y64)) + 1e-9)
+
+
+def test_epilogue_real_domain_error_is_quantization_sized(oracle):
+    # End to end at b = 8 the dequantized layer approximates x @ w^T + bias.
+    M, N, K = 16, 24, 512
+    x = workloads.normal((M, K), seed=31)
+    w = workloads.normal((N, K), seed=32, std=0.02)
+    out = oracle.linear_layer(x, oracle.quant_weight(w)["s"], oracle.quant_weight(w)["c"], None, 8)
+    ref = x.astype(np.float64) @ w.astype(np.float64).T
+    rel = np.linalg.norm(out["y"] - ref) / np.linalg.norm(ref)
+    assert rel < 0.02
+
+
+def test_bf16_rounding_ties_to_even(oracle):
+    # 1 + 2^-8 is halfway between bf16 neighbours 1 and 1 + 2^-7: ties go to even (1.0)
+    v = np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -(1.0 + 2 ** -8), 1.0 + 2 ** -8 + 2 ** -20], np.float32)
+    got = oracle.bf16_bits_to_f32(oracle.f32_to_bf16_bits(v))
+    assert list(got) == [1.0, 1.0 + 2 ** -6, -1.0, 1.0 + 2 ** -7]
+
+
+# ------------------------------------------------------------------- conv --
+
+def test_conv_definition_matches_torch_conv2d(oracle):
+    torch = pytest.importorskip("torch")
+    B, H, W, Cin, Cout = 2, 5, 6, 8, 7
+    x = workloads.normal((B, H, W, Cin), seed=41)
+    w = workloads.normal((Cout, 9 * Cin), seed=42, std=0.05)
+    bias = workloads.normal((Cout,), seed=43, std=0.02)
+    wq = oracle.quant_weight(w)
+    s_x, alpha, zc = oracle.quant_act(x.reshape(1, -1), 8, 1, 0)
+    s_x = s_x.reshape(B, H, W, Cin)
+    for b in (8, 4):
+        y64 = oracle.conv3x3_def_f64(s_x, alpha[0], zc[0], wq["s"], wq["c"], bias, b)
+        xh = torch.tensor(alpha[0], dtype=torch.float64) * (torch.tensor(s_x, dtype=torch.float64) + float(zc[0]))
+        wh = torch.tensor(wq["c"], dtype=torch.float64)[:, None] * torch.tensor(oracle.mask(wq["s"], b), dtype=torch.float64)
+        wh = wh.reshape(Cout, 3, 3, Cin).permute(0, 3, 1, 2)
+        ref = torch.nn.functional.conv2d(xh.permute(0, 3, 1, 2), wh, torch.tensor(bias, dtype=torch.float64), padding=1)
+        ref = ref.permute(0, 2, 3, 1).reshape(-1, Cout).numpy()
+        np.testing.assert_allclose(y64, ref, rtol=1e-12, atol=1e-12)
+        # codes + border-aware row sums + fp32 epilogue reproduce the definition
+        acc, rs = oracle.conv3x3(s_x, wq["s"], b)
+        y32, _ = oracle.epilogue_f32(acc, alpha, zc, rs, wq["c"], bias, per_tensor=True, rs_per_row=True)
+        np.testing.assert_allclose(y32, y64, rtol=1e-5, atol=1e-6)
+
+
+def test_conv_1x1_image_is_center_tap_linear(oracle):
+    Cin, Cout = 16, 5
+    s_x = workloads.uniform_codes((3, 1, 1, Cin), seed=51, lo=-128, hi=127)
+    s_w = workloads.uniform_codes((Cout, 9 * Cin), seed=52, lo=-128, hi=127)
+    acc, rs = oracle.conv3x3(s_x, s_w, 6)
+    center = s_w.reshape(Cout, 9, Cin)[:, 4, :]
+    assert np.array_equal(acc, oracle.gemm(s_x.reshape(3, Cin), center, 6))
+    assert np.array_equal(rs, np.broadcast_to(oracle.row_sums(center, 6), (3, Cout)))
+
+
+def test_conv_interior_pixel_is_full_im2col_row(oracle):
+    B, H, W, Cin, Cout = 1, 4, 4, 8, 3
+    s_x = workloads.uniform_codes((B, H, W, Cin), seed=53, lo=-128, hi=127)
+    s_w = workloads.uniform_codes((Cout, 9 * Cin), seed=54, lo=-128, hi=127)
+    acc, rs = oracle.conv3x3(s_x, s_w, 5)
+    h, w = 2, 1
+    patch = np.concatenate([s_x[0, h + dh, w + dw] for dh in (-1, 0, 1) for dw in (-1, 0, 1)])[None]
+    assert np.array_equal(acc[h * W + w], oracle.gemm(patch, s_w, 5)[0])
+    assert np.array_equal(rs[h * W + w], oracle.row_sums(s_w, 5))
+
+
+# --------------------------------------------------------------- schedule --
+
+def _golden_rows(name):
+    here = os.path.join(os.path.dirname(__file__), "golden", name)
+    for line in open(here):
+        line = line.split("#")[0].strip()
+        if line:
+            parts = line.split()
+            yield int(parts[0]), float(parts[1]), float(parts[2])
+
+
+def test_rel_bitops_reproduces_paper_table():
+    rows = list(_golden_rows("rel_bitops_table.txt"))
+    assert len(rows) >= 6
+    for a_bits, eff_w, rel in rows:
+        assert round(schedule.rel_bitops(eff_w, a_bits) + 1e-9, 2) == rel
+
+
+def test_stage_partition_is_contiguous():
+    # 20 steps in 4 stages: 5 consecutive steps each, stage 0 first (noisiest)
+    st = [schedule.stage_of_step(t, 20, 4) for t in range(20)]
+    assert st == sorted(st) and [st.count(s) for s in range(4)] == [5, 5, 5, 5] and st[0] == 0
+    # SDXL-Turbo: four steps, each its own stage
+    assert [schedule.stage_of_step(t, 4, 4) for t in range(4)] == [0, 1, 2, 3]
+    # uneven split still covers every stage in order
+    st = [schedule.stage_of_step(t, 7, 3) for t in range(7)]
+    assert st == sorted(st) and set(st) == {0, 1, 2}
+
+
+def test_effective_bits_weights_by_ops():
+    tab = np.array([[8, 4], [2, 4]], np.uint8)
+    eb = schedule.effective_bits(tab, [3, 1])
+    assert eb[0] == pytest.approx((8 * 3 + 2) / 4) and eb[1] == 4.0
