@@ -1,0 +1,239 @@
+/*
+ * tasq.h -- C ABI of the GB300 (sm_103a) masked-W8A8 library for TASQ
+ * (Temporal-Adaptive Bit Sparsification Quantization, arXiv 2608.03057).
+ *
+ * What the library computes.  Each quantized layer keeps ONE shared 8-bit
+ * weight buffer (Sec. 3.1, Eq. truncquant; App. F.1).  At denoising stage s
+ * the layer runs at an operating precision b = table[layer][s] in 2..8 (the
+ * bit-allocation map of App. F.1): the 8 - b least-significant planes of the
+ * stored code are dropped (Eqs. lsb_extraction, lsb_masking, hw_rightshift,
+ * hw_multi_lsb) and the truncated weight multiplies the quantized activations
+ * (Eq. qalora, Y = Q(X) Q(W)), with the dequantization of App. A.1 folded
+ * into an epilogue that writes bf16.
+ *
+ * Conventions shared by every call:
+ *  - Pointers named d_* are DEVICE pointers on the context's device; h_* are
+ *    host pointers.  The caller owns every buffer it passes; the library never
+ *    keeps a caller pointer beyond the call, except d_stage of
+ *    tasq_set_stage_device (documented there).
+ *  - Calls that take a `stream` only enqueue work on that stream (a
+ *    cudaStream_t; NULL is the legacy default stream).  They do not allocate,
+ *    do not synchronize, and return as soon as the work is queued.  Calls
+ *    without a stream are set-up calls and may allocate or synchronize, as
+ *    documented on each.
+ *  - The context's device must be the current CUDA device of the calling
+ *    thread; a mismatch returns TASQ_ERR_INVALID_ARG.
+ *  - Every call returns TASQ_OK (0) or an error code; tasq_last_error() then
+ *    describes the failure.  Arguments are validated on the host before
+ *    anything is launched: an invalid call launches nothing.
+ *  - Errors that only the device can see (an out-of-range stage read from
+ *    device memory, a packed buffer that does not match N/K, a pipeline wait
+ *    that ran past its time limit) are recorded in a device status word that
+ *    tasq_device_status() reads; the kernel then returns early without
+ *    trapping, and the CUDA context stays usable.
+ *  - A context may be used from one host thread at a time.  Per-tensor
+ *    activation quantization uses a small per-context reduction scratch, so
+ *    two such calls on different streams of one context must not overlap.
+ *
+ * Data layouts: row-major, innermost index last.  Activations of a linear
+ * layer are [M][K] (M tokens); of a conv, NHWC [B][H][W][Cin].  Weights are
+ * [N][K] (linear) or [Cout][3][3][Cin] = [N][9*Cin] (conv).  Outputs are bf16
+ * [M][N] (linear) or NHWC [B][H][W][Cout] (conv), as uint16_t bit patterns.
+ * Shape rules: K % 16 == 0 and N % 8 == 0 (conv: Cin % 16 == 0); M >= 0 may
+ * be anything (M == 0 is a no-op).  Every device pointer must be 16-byte
+ * aligned.
+ */
+#ifndef TASQ_H
+#define TASQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TASQ_ABI_VERSION 1
+
+/* Return codes. */
+enum {
+    TASQ_OK = 0,
+    TASQ_ERR_INVALID_ARG = 1,    /* bad pointer, range, enum or device */
+    TASQ_ERR_UNSUPPORTED = 2,    /* legal but unsupported shape, alignment or mode */
+    TASQ_ERR_CUDA = 3,           /* a CUDA runtime call or launch failed */
+    TASQ_ERR_DEVICE_TIMEOUT = 4, /* (device status) a pipeline wait ran past its limit */
+    TASQ_ERR_DEVICE = 5          /* (device status) a check inside a kernel failed */
+};
+
+enum { TASQ_LINEAR = 0, TASQ_CONV3X3 = 1 };               /* layer kinds */
+enum { TASQ_F32 = 0, TASQ_BF16 = 1 };                     /* float tensor dtypes */
+enum { TASQ_SYMRANGE = 0, TASQ_ASYM = 1 };                /* quantization range */
+enum { TASQ_PER_TOKEN = 0, TASQ_PER_TENSOR = 1 };         /* activation granularity */
+/* Storage of activation codes s = Q - 2^(n-1): one signed byte, or the same
+ * integer held exactly in an IEEE fp16 (the operand type of the tensor-core
+ * route; every integer in [-128, 127] is exact in fp16). */
+enum { TASQ_CODES_S8 = 0, TASQ_CODES_F16 = 1 };
+/* Contraction routes.  TC: tcgen05 MMA on fp16-held integer codes with fp32
+ * accumulation in tensor memory, drained to int32 in chunks whose exactness
+ * is certified at pack time (needs TASQ_CODES_F16).  MMA_S8: warp-level
+ * mma.sync with int8 operands and int32 accumulators (needs TASQ_CODES_S8).
+ * AUTO picks the route that matches the code storage. */
+enum { TASQ_ROUTE_AUTO = 0, TASQ_ROUTE_TC = 1, TASQ_ROUTE_MMA_S8 = 2 };
+
+typedef struct tasq_ctx_s* tasq_ctx;
+typedef void* tasq_stream; /* cudaStream_t */
+
+/* ABI version of the loaded library (TASQ_ABI_VERSION). */
+int tasq_version(void);
+
+/* Create a context on CUDA device `device`.  Set-up call: allocates the
+ * context's device status word and reduction scratch (a few bytes) and
+ * leaves the calling thread's current device unchanged.  *out is NULL on
+ * failure. */
+int tasq_create(tasq_ctx* out, int device);
+
+/* Destroy a context and free what it allocated.  Synchronizes the device.
+ * NULL is ignored. */
+void tasq_destroy(tasq_ctx ctx);
+
+/* Text of the last error on this context (valid until the next call on it);
+ * with ctx == NULL, the last tasq_create failure of this thread. */
+const char* tasq_last_error(tasq_ctx ctx);
+
+/* Device status: synchronizes the device, returns TASQ_OK or the first
+ * device-side error code recorded since the last read (TASQ_ERR_DEVICE_TIMEOUT,
+ * TASQ_ERR_DEVICE) in *out, then clears it.  Set-up call. */
+int tasq_device_status(tasq_ctx ctx, int* out);
+
+/* Route used by tasq_masked_gemm / tasq_masked_conv3x3 (TASQ_ROUTE_*). */
+int tasq_set_route(tasq_ctx ctx, int route);
+
+/* Time limit of every pipeline wait inside the kernels, in nanoseconds
+ * (default 2e9; 0 restores the default).  A wait that runs past it records
+ * TASQ_ERR_DEVICE_TIMEOUT in the device status and its kernel returns. */
+int tasq_set_timeout_ns(tasq_ctx ctx, uint64_t ns);
+
+/* Failure-detection self test: launches one block that waits on a barrier
+ * nothing ever arrives at, bounded by `timeout_ns`.  The wait gives up,
+ * records TASQ_ERR_DEVICE_TIMEOUT in the device status and the kernel
+ * returns, leaving the context usable.  Enqueue call. */
+int tasq_selftest_timeout(tasq_ctx ctx, uint64_t timeout_ns, tasq_stream stream);
+
+/*
+ * Weight quantization, App. A.1.1 (Eqs. weight_quant, weight_scale,
+ * weight_dequant), per output channel, with the range taken symmetric,
+ * [-max|w|, +max|w|] (so alpha = max|w| / 128 and z = 128):
+ *   Q = clamp(floor(w / alpha + z), 0, 255),  stored s_w = Q - 128 (int8),
+ *   c_w = (256/255) * alpha   so that   w_hat = c_w * s_w.
+ * fp32 operation order (each step rounds to nearest even): alpha =
+ * (hi - lo) / 256, z = -lo / alpha, Q = floor((w / alpha) + z),
+ * c_w = alpha * (256/255).  An all-zero channel gets alpha = 1, z = 128.
+ * d_w: [N][K] of `dtype` (TASQ_F32 or TASQ_BF16).  Outputs d_sw [N][K] int8,
+ * d_cw [N] fp32, d_alpha [N] fp32 (may be NULL).  Enqueue call.
+ */
+int tasq_quant_weights(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, int8_t* d_sw, float* d_cw,
+                       float* d_alpha, tasq_stream stream);
+
+/*
+ * Bytes of the packed form of one layer (see tasq_pack_weights), for
+ * kind TASQ_LINEAR (K = in features) or TASQ_CONV3X3 (K = 9*Cin).
+ * Returns 0 for invalid shapes.
+ */
+size_t tasq_packed_bytes(int kind, int N, int K);
+
+/*
+ * Pack one layer's stored 8-bit weights once (App. F.1: the stored buffer is
+ * not copied per stage).  d_packed (caller-allocated, tasq_packed_bytes
+ * bytes, 256-byte aligned) receives:
+ *   - a copy of d_sw [N][K] (the shared buffer every stage reads),
+ *   - c_w [N] and bias [N] (zeros when d_bias is NULL),
+ *   - for each b in 2..8 the row sums rs_b[n] = sum_k mask_b(s_w[n][k])
+ *     (they carry the activation zero point through the integer sum), and
+ *     for a conv the per-tap sums of the same,
+ *   - for each b the exactness certificate of the TC route: the longest run
+ *     of 64-wide K blocks over which 128 * sum |mask_b(s_w[n][k])| <= 2^24
+ *     for every channel n, so that fp32 partial sums of int8 x int8 products
+ *     stay exact integers (|s_x| <= 128).
+ * mask_b(v) drops the 8-b low planes of the unsigned code v + 128
+ * (Eq. hw_rightshift); on the signed byte this is v & (0xFF << (8-b)).
+ * kind: TASQ_LINEAR (K = in features, Cin ignored) or TASQ_CONV3X3
+ * (K = 9*Cin, weights ordered (kh, kw, cin)).  Enqueue call.
+ */
+int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_bias, int N,
+                      int K, int Cin, void* d_packed, tasq_stream stream);
+
+/*
+ * Bit-allocation map (App. F.1): h_bits [L][S] uint8, each value in 2..8,
+ * copied into device memory owned by the context.  Set-up call: allocates
+ * (only when L*S grows), copies synchronously, validates every entry first.
+ * Changing stage afterwards needs no host work: it is an argument of the
+ * next call, or a device int (tasq_set_stage_device).
+ */
+int tasq_set_schedule(tasq_ctx ctx, const uint8_t* h_bits, int L, int S);
+
+/*
+ * Optional device-resident stage: with d_stage set, a call whose `stage`
+ * argument is -1 reads the stage from *d_stage when its kernel runs, so one
+ * captured CUDA graph serves every stage.  The context keeps the pointer
+ * until it is replaced or cleared (NULL); the caller keeps it alive.
+ */
+int tasq_set_stage_device(tasq_ctx ctx, const int32_t* d_stage);
+
+/*
+ * Activation quantization, App. A.1.2 (Eqs. act_quant, act_scale):
+ *   alpha = (max - min) / (2^n - 1),  z = -min / alpha,
+ *   Q = clamp(round_half_even(x / alpha + z), 0, 2^n - 1),
+ * stored as the signed code s = Q - 2^(n-1), with zc = 2^(n-1) - z so that
+ * x_hat = alpha * (Q - z) = alpha * (s + zc).
+ * fp32 order (each step rounds to nearest even): alpha = (hi - lo) / (2^n-1),
+ * z = -lo / alpha, u = (x / alpha) + z, Q = rint(u), zc = 2^(n-1) - z.
+ * A constant group gets alpha = 1 and z = 2^(n-1) (SYMRANGE) or -min (ASYM).
+ * mode: TASQ_SYMRANGE ([lo, hi] = [-max|x|, max|x|]) or TASQ_ASYM (min, max).
+ * gran: TASQ_PER_TOKEN (one alpha/zc per row of d_x [M][K]) or
+ * TASQ_PER_TENSOR (one for the whole tensor; d_x may then be any [M][K] view
+ * of a contiguous tensor, e.g. NHWC with M = B*H*W, K = Cin).
+ * n_bits in 2..8.  d_x: [M][K] of `dtype`; d_codes: [M][K] int8 or fp16 per
+ * code_fmt; d_alpha, d_zc: [M] (per token) or [1] (per tensor) fp32.
+ * Enqueue call (per tensor: two kernels and a 16-byte memset).
+ */
+int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode, int gran,
+                   void* d_codes, int code_fmt, float* d_alpha, float* d_zc, tasq_stream stream);
+
+/*
+ * Masked linear layer (Eq. qalora with the Temporal-Spatial LSB mask of
+ * Eq. lsb_masking at operating precision b = table[layer][stage]):
+ *   acc[m][n] = sum_k s_x[m][k] * mask_b(s_w[n][k])            (exact int32)
+ *   y[m][n]   = bf16( ((float(acc) + zc[m]*float(rs_b[n])) * (alpha[m]*c_w[n])) + bias[n] )
+ * with every fp32 operation rounded to nearest even in that order.
+ * stage: 0..S-1, or -1 to read it from the device int of
+ * tasq_set_stage_device.  d_codes: [M][K] activation codes (code_fmt);
+ * d_alpha/d_zc: [M] per-token scales from tasq_quant_act.  d_packed: from
+ * tasq_pack_weights with kind TASQ_LINEAR and the same N, K.  d_y: [M][N]
+ * bf16 bits.  d_acc: [M][N] int32, or NULL (then acc is not written).
+ * The mask is applied inside the kernel as each weight tile is loaded; the
+ * stored buffer is never modified.  Enqueue call.
+ */
+int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt, const float* d_alpha,
+                     const float* d_zc, int M, const void* d_packed, int N, int K, uint16_t* d_y, int32_t* d_acc,
+                     tasq_stream stream);
+
+/*
+ * Masked 3x3 convolution, stride 1, padding 1, as an implicit GEMM over
+ * K = 9*Cin (kh, kw, cin): same contraction and epilogue as
+ * tasq_masked_gemm with one activation scale for the tensor (d_alpha[0],
+ * d_zc[0], from a TASQ_PER_TENSOR quantization).  Padding is zero in the real
+ * domain: a tap outside the image contributes nothing, so its weights are
+ * left out of the row sum of that output pixel.
+ * d_codes: NHWC [B][H][W][Cin]; d_y: NHWC [B][H][W][Cout] bf16 bits;
+ * d_acc: [B*H*W][Cout] int32 or NULL.  d_packed: kind TASQ_CONV3X3 with
+ * N = Cout, K = 9*Cin.  Enqueue call.
+ */
+int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt, const float* d_alpha,
+                        const float* d_zc, int B, int H, int W, int Cin, const void* d_packed, int Cout, uint16_t* d_y,
+                        int32_t* d_acc, tasq_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TASQ_H */

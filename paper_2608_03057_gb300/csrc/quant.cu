@@ -1,0 +1,416 @@
+// Quantizers (App. A.1), weight packing (App. F.1) and the failure-detection
+// self test.  All kernels here are bandwidth-bound: 16-byte vector loads and
+// stores, warp-shuffle reductions, one warp per row.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "tasq_internal.cuh"
+
+namespace tasq {
+namespace {
+
+constexpr int kRowWarps = 8;  // rows per 256-thread block
+
+// Eight consecutive input floats (as fp32) from a 16-byte (bf16) or two
+// 16-byte (fp32) chunks.  `i` counts 8-element groups along the row.
+__device__ inline void load8(const void* row, int dtype, int64_t i, float v[8]) {
+    if (dtype == TASQ_F32) {
+        const float4* p = reinterpret_cast<const float4*>(row) + 2 * i;
+        float4 a = __ldg(p), b = __ldg(p + 1);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    } else {
+        uint4 r = __ldg(reinterpret_cast<const uint4*>(row) + i);
+        uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            v[2 * j] = __uint_as_float(w[j] << 16);
+            v[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+        }
+    }
+}
+
+__device__ inline float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ inline float warp_min(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+// Quantization range of a group: [lo, hi] -> (alpha, z) in the fp32 order
+// alpha = (hi - lo) / denom, z = -lo / alpha; a constant group gets alpha = 1
+// and z = half (symmetric range) or -lo.
+__device__ inline void scale_of_range(float lo, float hi, float denom, float half, int mode, float* alpha,
+                                      float* z) {
+    float range = __fsub_rn(hi, lo);
+    if (range == 0.0f) {
+        *alpha = 1.0f;
+        *z = (mode == TASQ_SYMRANGE) ? half : -lo;
+    } else {
+        *alpha = __fdiv_rn(range, denom);
+        *z = __fdiv_rn(-lo, *alpha);
+    }
+}
+
+// Activation code: Q = clamp(rint(x / alpha + z), 0, qmax), s = Q - half.
+__device__ inline int act_code(float x, float alpha, float z, int qmax, int half) {
+    float u = __fadd_rn(__fdiv_rn(x, alpha), z);
+    int q = __float2int_rn(u);  // round half to even
+    q = min(max(q, 0), qmax);
+    return q - half;
+}
+
+__device__ inline void store8_codes(void* out, int code_fmt, int64_t i, const int s[8]) {
+    if (code_fmt == TASQ_CODES_S8) {
+        uint2 pk;
+        pk.x = (s[0] & 0xFF) | ((s[1] & 0xFF) << 8) | ((s[2] & 0xFF) << 16) | ((uint32_t)(s[3] & 0xFF) << 24);
+        pk.y = (s[4] & 0xFF) | ((s[5] & 0xFF) << 8) | ((s[6] & 0xFF) << 16) | ((uint32_t)(s[7] & 0xFF) << 24);
+        reinterpret_cast<uint2*>(out)[i] = pk;
+    } else {
+        uint4 pk;
+        uint32_t h[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) h[j] = __half_as_ushort(__int2half_rn(s[j]));
+        pk.x = h[0] | (h[1] << 16);
+        pk.y = h[2] | (h[3] << 16);
+        pk.z = h[4] | (h[5] << 16);
+        pk.w = h[6] | (h[7] << 16);
+        reinterpret_cast<uint4*>(out)[i] = pk;
+    }
+}
+
+// ---------------------------------------------------------------- weights --
+__global__ void __launch_bounds__(256) quant_weights_kernel(const void* __restrict__ w, int dtype, int N, int K,
+                                                            int8_t* __restrict__ sw, float* __restrict__ cw,
+                                                            float* __restrict__ alpha_out) {
+    int lane = threadIdx.x & 31;
+    int n = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (n >= N) return;
+    const char* row = reinterpret_cast<const char*>(w) + int64_t(n) * K * (dtype == TASQ_F32 ? 4 : 2);
+    int groups = K / 8;
+    float amax = 0.0f;
+    for (int i = lane; i < groups; i += 32) {
+        float v[8];
+        load8(row, dtype, i, v);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) amax = fmaxf(amax, fabsf(v[j]));
+    }
+    amax = warp_max(amax);
+    float alpha, z;
+    scale_of_range(-amax, amax, 256.0f, 128.0f, TASQ_SYMRANGE, &alpha, &z);
+    int8_t* srow = sw + int64_t(n) * K;
+    for (int i = lane; i < groups; i += 32) {
+        float v[8];
+        load8(row, dtype, i, v);
+        uint32_t pk[2] = {0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            float u = __fadd_rn(__fdiv_rn(v[j], alpha), z);
+            int q = __float2int_rd(u);  // floor
+            q = min(max(q, 0), 255) - 128;
+            pk[j >> 2] |= uint32_t(q & 0xFF) << (8 * (j & 3));
+        }
+        reinterpret_cast<uint2*>(srow)[i] = make_uint2(pk[0], pk[1]);
+    }
+    if (lane == 0) {
+        cw[n] = __fmul_rn(alpha, __fdiv_rn(256.0f, 255.0f));
+        if (alpha_out) alpha_out[n] = alpha;
+    }
+}
+
+// ------------------------------------------------------ activations, token --
+__global__ void __launch_bounds__(256) quant_act_token_kernel(const void* __restrict__ x, int dtype, int M, int K,
+                                                              int n_bits, int mode, void* __restrict__ codes,
+                                                              int code_fmt, float* __restrict__ alpha_out,
+                                                              float* __restrict__ zc_out) {
+    int lane = threadIdx.x & 31;
+    int m = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (m >= M) return;
+    const char* row = reinterpret_cast<const char*>(x) + int64_t(m) * K * (dtype == TASQ_F32 ? 4 : 2);
+    int groups = K / 8;
+    float lo = INFINITY, hi = -INFINITY;
+    for (int i = lane; i < groups; i += 32) {
+        float v[8];
+        load8(row, dtype, i, v);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            lo = fminf(lo, v[j]);
+            hi = fmaxf(hi, v[j]);
+        }
+    }
+    lo = warp_min(lo);
+    hi = warp_max(hi);
+    if (mode == TASQ_SYMRANGE) {
+        hi = fmaxf(fabsf(lo), fabsf(hi));
+        lo = -hi;
+    }
+    const int half = 1 << (n_bits - 1), qmax = (1 << n_bits) - 1;
+    float alpha, z;
+    scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
+    char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (code_fmt == TASQ_CODES_S8 ? 1 : 2);
+    for (int i = lane; i < groups; i += 32) {
+        float v[8];
+        load8(row, dtype, i, v);
+        int s[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, z, qmax, half);
+        store8_codes(out, code_fmt, i, s);
+    }
+    if (lane == 0) {
+        alpha_out[m] = alpha;
+        zc_out[m] = __fsub_rn(float(half), z);
+    }
+}
+
+// ----------------------------------------------------- activations, tensor --
+// Order-preserving map of a float onto an unsigned key.
+__device__ inline uint32_t order_key(float f) {
+    uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ inline float key_value(uint32_t k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+// scratch[0] = ~key(min), scratch[1] = key(max); both start at 0.
+__global__ void __launch_bounds__(256) tensor_range_kernel(const void* __restrict__ x, int dtype, int64_t groups,
+                                                           unsigned int* scratch) {
+    float lo = INFINITY, hi = -INFINITY;
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < groups; i += int64_t(gridDim.x) * blockDim.x) {
+        float v[8];
+        load8(x, dtype, i, v);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            lo = fminf(lo, v[j]);
+            hi = fmaxf(hi, v[j]);
+        }
+    }
+    lo = warp_min(lo);
+    hi = warp_max(hi);
+    __shared__ float slo[8], shi[8];
+    int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        slo[warp] = lo;
+        shi[warp] = hi;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int i = 1; i < int(blockDim.x >> 5); ++i) {
+            lo = fminf(lo, slo[i]);
+            hi = fmaxf(hi, shi[i]);
+        }
+        if (lo <= hi) {
+            atomicMax(&scratch[0], ~order_key(lo));
+            atomicMax(&scratch[1], order_key(hi));
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) quant_act_tensor_kernel(const void* __restrict__ x, int dtype, int64_t groups,
+                                                               int n_bits, int mode, void* __restrict__ codes,
+                                                               int code_fmt, float* __restrict__ alpha_out,
+                                                               float* __restrict__ zc_out,
+                                                               const unsigned int* __restrict__ scratch) {
+    float lo = key_value(~scratch[0]);
+    float hi = key_value(scratch[1]);
+    if (mode == TASQ_SYMRANGE) {
+        hi = fmaxf(fabsf(lo), fabsf(hi));
+        lo = -hi;
+    }
+    const int half = 1 << (n_bits - 1), qmax = (1 << n_bits) - 1;
+    float alpha, z;
+    scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < groups; i += int64_t(gridDim.x) * blockDim.x) {
+        float v[8];
+        load8(x, dtype, i, v);
+        int s[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, z, qmax, half);
+        store8_codes(codes, code_fmt, i, s);
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        alpha_out[0] = alpha;
+        zc_out[0] = __fsub_rn(float(half), z);
+    }
+}
+
+// -------------------------------------------------------------------- pack --
+__global__ void pack_header_kernel(int kind, int N, int K, PackedHeader* hdr) {
+    PackedHeader h = packed_layout(kind, N, K);
+    for (int b = 0; b <= kBMax; ++b) h.chunk_kb[b] = (b >= kBMin) ? 0x7FFFFFFF : 0;
+    *hdr = h;
+}
+
+// One block per output channel: row sums and per-tap sums for every b, and
+// the channel's longest certified chunk (in 64-wide K blocks) for every b.
+__global__ void __launch_bounds__(256) pack_sums_kernel(const int8_t* __restrict__ sw, int kind, int N, int K, int Cin,
+                                                        char* packed) {
+    extern __shared__ int smem_sums[];  // [kNumB][KB] block abs sums
+    const PackedHeader lay = packed_layout(kind, N, K);
+    PackedHeader* hdr = reinterpret_cast<PackedHeader*>(packed);
+    int32_t* rs = reinterpret_cast<int32_t*>(packed + lay.off_rs);
+    int32_t* ts = reinterpret_cast<int32_t*>(packed + lay.off_ts);
+    const int n = blockIdx.x;
+    const int KB = (K + kCertKBlock - 1) / kCertKBlock;
+    const int8_t* row = sw + int64_t(n) * K;
+    __shared__ int red[kNumB][9];
+    if (threadIdx.x < kNumB * 9) red[threadIdx.x / 9][threadIdx.x % 9] = 0;
+    for (int i = threadIdx.x; i < kNumB * KB; i += blockDim.x) smem_sums[i] = 0;
+    __syncthreads();
+    // per-thread partials: [b][tap] signed sums; block abs sums via shared atomics
+    int part[kNumB][9];
+#pragma unroll
+    for (int bi = 0; bi < kNumB; ++bi)
+#pragma unroll
+        for (int t = 0; t < 9; ++t) part[bi][t] = 0;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) {
+        int v = row[k];
+        int tap = (kind == TASQ_CONV3X3) ? k / Cin : 0;
+        int kb = k / kCertKBlock;
+#pragma unroll
+        for (int bi = 0; bi < kNumB; ++bi) {
+            int m = mask_code(v, bi + kBMin);
+#pragma unroll
+            for (int t = 0; t < 9; ++t)
+                if (t == tap) part[bi][t] += m;
+            atomicAdd(&smem_sums[bi * KB + kb], abs(m));
+        }
+    }
+#pragma unroll
+    for (int bi = 0; bi < kNumB; ++bi)
+#pragma unroll
+        for (int t = 0; t < 9; ++t) {
+            int s = part[bi][t];
+#pragma unroll
+            for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+            if ((threadIdx.x & 31) == 0 && s) atomicAdd(&red[bi][t], s);
+        }
+    __syncthreads();
+    if (threadIdx.x < kNumB) {
+        int bi = threadIdx.x;
+        int tot = 0;
+        for (int t = 0; t < 9; ++t) tot += red[bi][t];
+        rs[bi * N + n] = tot;
+        if (kind == TASQ_CONV3X3)
+            for (int t = 0; t < 9; ++t) ts[(int64_t(bi) * N + n) * 9 + t] = red[bi][t];
+    }
+    // Longest chunk length C (in K blocks) such that EVERY window of C
+    // consecutive blocks stays within the bound.  Windows (not only aligned
+    // chunks) make the property monotone in C, so the minimum over channels is
+    // valid for every channel.  C = (shortest window whose sum exceeds the
+    // bound) - 1, found by two pointers over the non-negative block sums.
+    __syncthreads();
+    if (threadIdx.x < kNumB) {
+        const int bi = threadIdx.x;
+        const int* S = smem_sums + bi * KB;
+        int shortest = KB + 1;
+        int64_t sum = 0;
+        int l = 0;
+        for (int r = 0; r < KB; ++r) {
+            sum += S[r];
+            while (sum > kCertLimit) {
+                shortest = min(shortest, r - l + 1);
+                sum -= S[l++];
+            }
+        }
+        atomicMin(&hdr->chunk_kb[bi + kBMin], max(1, shortest - 1));
+    }
+}
+
+// ------------------------------------------------------------- self test --
+__global__ void selftest_timeout_kernel(int* status, unsigned long long timeout_ns) {
+    __shared__ __align__(8) unsigned long long bar;
+    if (threadIdx.x == 0) {
+        uint32_t a = (uint32_t)__cvta_generic_to_shared(&bar);
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(1));
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        unsigned long long t0;
+        asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+        uint32_t done = 0;
+        while (!done) {
+            asm volatile(
+                "{\n.reg .pred p;\n"
+                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+                "selp.u32 %0, 1, 0, p;\n}\n"
+                : "=r"(done)
+                : "r"(a), "r"(0u)
+                : "memory");
+            if (done) break;
+            unsigned long long t;
+            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+            if (t - t0 > timeout_ns) {
+                set_status(status, TASQ_ERR_DEVICE_TIMEOUT);
+                break;
+            }
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int8_t* sw, float* cw, float* alpha,
+                                 cudaStream_t st) {
+    if (N == 0) return cudaSuccess;
+    quant_weights_kernel<<<(N + kRowWarps - 1) / kRowWarps, 256, 0, st>>>(w, dtype, N, K, sw, cw, alpha);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_quant_act_token(const void* x, int dtype, int M, int K, int n_bits, int mode, void* codes,
+                                   int code_fmt, float* alpha, float* zc, cudaStream_t st) {
+    if (M == 0) return cudaSuccess;
+    quant_act_token_kernel<<<(M + kRowWarps - 1) / kRowWarps, 256, 0, st>>>(x, dtype, M, K, n_bits, mode, codes,
+                                                                            code_fmt, alpha, zc);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_quant_act_tensor(const void* x, int dtype, int64_t count, int n_bits, int mode, void* codes,
+                                    int code_fmt, float* alpha, float* zc, unsigned int* scratch, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(scratch, 0, 16, st);
+    if (e != cudaSuccess) return e;
+    int64_t groups = count / 8;
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    int64_t want = (groups + 255) / 256;
+    int grid = int(want < 4 * sms ? (want > 0 ? want : 1) : 4 * sms);
+    tensor_range_kernel<<<grid, 256, 0, st>>>(x, dtype, groups, scratch);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    quant_act_tensor_kernel<<<grid, 256, 0, st>>>(x, dtype, groups, n_bits, mode, codes, code_fmt, alpha, zc,
+                                                  scratch);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* bias, int N, int K, int Cin,
+                        void* packed, cudaStream_t st) {
+    const PackedHeader lay = packed_layout(kind, N, K);
+    char* p = reinterpret_cast<char*>(packed);
+    cudaError_t e = cudaMemsetAsync(p, 0, lay.total, st);
+    if (e != cudaSuccess) return e;
+    pack_header_kernel<<<1, 1, 0, st>>>(kind, N, K, reinterpret_cast<PackedHeader*>(p));
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (N == 0) return cudaSuccess;
+    if ((e = cudaMemcpyAsync(p + lay.off_w, sw, size_t(N) * K, cudaMemcpyDeviceToDevice, st)) != cudaSuccess) return e;
+    if ((e = cudaMemcpyAsync(p + lay.off_cw, cw, size_t(N) * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess) return e;
+    if (bias && (e = cudaMemcpyAsync(p + lay.off_bias, bias, size_t(N) * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+        return e;
+    int KB = (K + kCertKBlock - 1) / kCertKBlock;
+    size_t smem = size_t(kNumB) * KB * sizeof(int);
+    if (smem > 48 * 1024) {
+        e = cudaFuncSetAttribute(pack_sums_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+        if (e != cudaSuccess) return e;
+    }
+    pack_sums_kernel<<<N, 256, smem, st>>>(sw, kind, N, K, Cin, p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, cudaStream_t st) {
+    selftest_timeout_kernel<<<1, 32, 0, st>>>(status, timeout_ns);
+    return cudaGetLastError();
+}
+
+}  // namespace tasq

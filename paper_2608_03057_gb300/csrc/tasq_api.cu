@@ -1,0 +1,323 @@
+// Host side of the C ABI declared in include/tasq.h: the context, argument
+// validation (nothing is launched for an invalid call) and kernel launches.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+
+#include "tasq_internal.cuh"
+
+#define TASQ_API extern "C" __attribute__((visibility("default")))
+
+struct tasq_ctx_s {
+    int device = 0;
+    int num_sms = 0;
+    int* d_words = nullptr;  // [0] status, [16..19] reduction scratch
+    uint8_t* d_table = nullptr;
+    size_t table_cap = 0;
+    int L = 0, S = 0;
+    const int32_t* d_stage = nullptr;
+    int route = TASQ_ROUTE_AUTO;
+    unsigned long long timeout_ns = 2000000000ull;
+    std::string err;
+};
+
+namespace {
+
+thread_local std::string g_create_err;
+
+int fail(tasq_ctx ctx, int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (ctx) ctx->err = buf;
+    else g_create_err = buf;
+    return code;
+}
+
+int cuda_fail(tasq_ctx ctx, cudaError_t e, const char* what) {
+    return fail(ctx, TASQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_ctx(tasq_ctx ctx) {
+    if (!ctx) return TASQ_ERR_INVALID_ARG;
+    int cur = -1;
+    cudaError_t e = cudaGetDevice(&cur);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaGetDevice");
+    if (cur != ctx->device)
+        return fail(ctx, TASQ_ERR_INVALID_ARG, "current device %d is not the context's device %d", cur, ctx->device);
+    ctx->err.clear();
+    return TASQ_OK;
+}
+
+#define CHECK_CTX(ctx)                      \
+    do {                                    \
+        int rc_ = check_ctx(ctx);           \
+        if (rc_ != TASQ_OK) return rc_;     \
+    } while (0)
+
+#define REQUIRE(cond, code, ...)                          \
+    do {                                                  \
+        if (!(cond)) return fail(ctx, code, __VA_ARGS__); \
+    } while (0)
+
+}  // namespace
+
+TASQ_API int tasq_version(void) { return TASQ_ABI_VERSION; }
+
+TASQ_API int tasq_create(tasq_ctx* out, int device) {
+    if (!out) return fail(nullptr, TASQ_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    int count = 0;
+    cudaError_t e = cudaGetDeviceCount(&count);
+    if (e != cudaSuccess) return fail(nullptr, TASQ_ERR_CUDA, "cudaGetDeviceCount: %s", cudaGetErrorString(e));
+    if (device < 0 || device >= count) return fail(nullptr, TASQ_ERR_INVALID_ARG, "device %d out of range", device);
+    cudaDeviceProp prop;
+    if ((e = cudaGetDeviceProperties(&prop, device)) != cudaSuccess)
+        return fail(nullptr, TASQ_ERR_CUDA, "cudaGetDeviceProperties: %s", cudaGetErrorString(e));
+    if (prop.major != 10 || prop.minor != 3)
+        return fail(nullptr, TASQ_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a", device,
+                    prop.major, prop.minor);
+    int prev = 0;
+    cudaGetDevice(&prev);
+    if ((e = cudaSetDevice(device)) != cudaSuccess)
+        return fail(nullptr, TASQ_ERR_CUDA, "cudaSetDevice: %s", cudaGetErrorString(e));
+    tasq_ctx ctx = new tasq_ctx_s();
+    ctx->device = device;
+    ctx->num_sms = prop.multiProcessorCount;
+    e = cudaMalloc(&ctx->d_words, 256);
+    if (e == cudaSuccess) e = cudaMemset(ctx->d_words, 0, 256);
+    cudaSetDevice(prev);
+    if (e != cudaSuccess) {
+        delete ctx;
+        return fail(nullptr, TASQ_ERR_CUDA, "allocating the status word: %s", cudaGetErrorString(e));
+    }
+    *out = ctx;
+    return TASQ_OK;
+}
+
+TASQ_API void tasq_destroy(tasq_ctx ctx) {
+    if (!ctx) return;
+    int prev = 0;
+    cudaGetDevice(&prev);
+    cudaSetDevice(ctx->device);
+    cudaDeviceSynchronize();
+    cudaFree(ctx->d_words);
+    cudaFree(ctx->d_table);
+    cudaSetDevice(prev);
+    delete ctx;
+}
+
+TASQ_API const char* tasq_last_error(tasq_ctx ctx) { return ctx ? ctx->err.c_str() : g_create_err.c_str(); }
+
+TASQ_API int tasq_device_status(tasq_ctx ctx, int* out) {
+    CHECK_CTX(ctx);
+    REQUIRE(out, TASQ_ERR_INVALID_ARG, "out is NULL");
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaDeviceSynchronize");
+    int v = 0;
+    if ((e = cudaMemcpy(&v, ctx->d_words, sizeof v, cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_fail(ctx, e, "reading the status word");
+    if ((e = cudaMemset(ctx->d_words, 0, sizeof v)) != cudaSuccess) return cuda_fail(ctx, e, "clearing the status word");
+    *out = v;
+    return TASQ_OK;
+}
+
+TASQ_API int tasq_set_route(tasq_ctx ctx, int route) {
+    CHECK_CTX(ctx);
+    REQUIRE(route >= TASQ_ROUTE_AUTO && route <= TASQ_ROUTE_MMA_S8, TASQ_ERR_INVALID_ARG, "route %d", route);
+    ctx->route = route;
+    return TASQ_OK;
+}
+
+TASQ_API int tasq_set_timeout_ns(tasq_ctx ctx, uint64_t ns) {
+    CHECK_CTX(ctx);
+    ctx->timeout_ns = ns ? ns : 2000000000ull;
+    return TASQ_OK;
+}
+
+TASQ_API int tasq_selftest_timeout(tasq_ctx ctx, uint64_t timeout_ns, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(timeout_ns > 0 && timeout_ns <= 10000000000ull, TASQ_ERR_INVALID_ARG, "timeout_ns must be in (0, 1e10]");
+    cudaError_t e = tasq::launch_selftest_timeout(ctx->d_words, timeout_ns, (cudaStream_t)stream);
+    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "selftest launch");
+}
+
+TASQ_API int tasq_quant_weights(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, int8_t* d_sw, float* d_cw,
+                                float* d_alpha, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(dtype == TASQ_F32 || dtype == TASQ_BF16, TASQ_ERR_INVALID_ARG, "dtype %d", dtype);
+    REQUIRE(N >= 0 && K > 0, TASQ_ERR_INVALID_ARG, "N=%d K=%d", N, K);
+    REQUIRE(K % 16 == 0, TASQ_ERR_UNSUPPORTED, "K=%d must be a multiple of 16", K);
+    REQUIRE(N == 0 || (d_w && d_sw && d_cw), TASQ_ERR_INVALID_ARG, "NULL pointer");
+    REQUIRE(aligned16(d_w) && aligned16(d_sw) && aligned16(d_cw) && aligned16(d_alpha), TASQ_ERR_UNSUPPORTED,
+            "pointers must be 16-byte aligned");
+    cudaError_t e = tasq::launch_quant_weights(d_w, dtype, N, K, d_sw, d_cw, d_alpha, (cudaStream_t)stream);
+    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "quant_weights launch");
+}
+
+TASQ_API size_t tasq_packed_bytes(int kind, int N, int K) {
+    if ((kind != TASQ_LINEAR && kind != TASQ_CONV3X3) || N < 0 || K <= 0) return 0;
+    if (kind == TASQ_CONV3X3 && K % 9) return 0;
+    return (size_t)tasq::packed_layout(kind, N, K).total;
+}
+
+TASQ_API int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_bias,
+                               int N, int K, int Cin, void* d_packed, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(kind == TASQ_LINEAR || kind == TASQ_CONV3X3, TASQ_ERR_INVALID_ARG, "kind %d", kind);
+    REQUIRE(N > 0 && K > 0, TASQ_ERR_INVALID_ARG, "N=%d K=%d", N, K);
+    REQUIRE(K % 16 == 0 && N % 8 == 0, TASQ_ERR_UNSUPPORTED, "need K %% 16 == 0 and N %% 8 == 0 (N=%d K=%d)", N, K);
+    if (kind == TASQ_CONV3X3) {
+        REQUIRE(Cin > 0 && K == 9 * Cin, TASQ_ERR_INVALID_ARG, "conv: K=%d must be 9*Cin (Cin=%d)", K, Cin);
+        REQUIRE(Cin % 16 == 0, TASQ_ERR_UNSUPPORTED, "conv: Cin=%d must be a multiple of 16", Cin);
+    }
+    REQUIRE(d_sw && d_cw && d_packed, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    REQUIRE((reinterpret_cast<uintptr_t>(d_packed) & 255u) == 0, TASQ_ERR_UNSUPPORTED, "d_packed must be 256-byte aligned");
+    REQUIRE(aligned16(d_sw) && aligned16(d_cw) && aligned16(d_bias), TASQ_ERR_UNSUPPORTED,
+            "pointers must be 16-byte aligned");
+    cudaError_t e = tasq::launch_pack(kind, d_sw, d_cw, d_bias, N, K, kind == TASQ_CONV3X3 ? Cin : 0, d_packed,
+                                      (cudaStream_t)stream);
+    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "pack launch");
+}
+
+TASQ_API int tasq_set_schedule(tasq_ctx ctx, const uint8_t* h_bits, int L, int S) {
+    CHECK_CTX(ctx);
+    REQUIRE(h_bits && L > 0 && S > 0, TASQ_ERR_INVALID_ARG, "need h_bits, L > 0, S > 0");
+    REQUIRE((int64_t)L * S <= (int64_t(1) << 30), TASQ_ERR_INVALID_ARG, "table too large");
+    for (int64_t i = 0; i < (int64_t)L * S; ++i)
+        REQUIRE(h_bits[i] >= tasq::kBMin && h_bits[i] <= tasq::kBMax, TASQ_ERR_INVALID_ARG,
+                "bits[%lld] = %d is outside 2..8", (long long)i, (int)h_bits[i]);
+    cudaError_t e = cudaDeviceSynchronize();  // no kernel may be reading the old table
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaDeviceSynchronize");
+    size_t bytes = (size_t)L * S;
+    if (bytes > ctx->table_cap) {
+        cudaFree(ctx->d_table);
+        ctx->d_table = nullptr;
+        ctx->table_cap = 0;
+        if ((e = cudaMalloc(&ctx->d_table, bytes)) != cudaSuccess) return cuda_fail(ctx, e, "allocating the table");
+        ctx->table_cap = bytes;
+    }
+    if ((e = cudaMemcpy(ctx->d_table, h_bits, bytes, cudaMemcpyHostToDevice)) != cudaSuccess)
+        return cuda_fail(ctx, e, "copying the table");
+    ctx->L = L;
+    ctx->S = S;
+    return TASQ_OK;
+}
+
+TASQ_API int tasq_set_stage_device(tasq_ctx ctx, const int32_t* d_stage) {
+    CHECK_CTX(ctx);
+    REQUIRE((reinterpret_cast<uintptr_t>(d_stage) & 3u) == 0, TASQ_ERR_INVALID_ARG, "d_stage must be 4-byte aligned");
+    ctx->d_stage = d_stage;
+    return TASQ_OK;
+}
+
+TASQ_API int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode, int gran,
+                            void* d_codes, int code_fmt, float* d_alpha, float* d_zc, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(dtype == TASQ_F32 || dtype == TASQ_BF16, TASQ_ERR_INVALID_ARG, "dtype %d", dtype);
+    REQUIRE(mode == TASQ_SYMRANGE || mode == TASQ_ASYM, TASQ_ERR_INVALID_ARG, "mode %d", mode);
+    REQUIRE(gran == TASQ_PER_TOKEN || gran == TASQ_PER_TENSOR, TASQ_ERR_INVALID_ARG, "gran %d", gran);
+    REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16, TASQ_ERR_INVALID_ARG, "code_fmt %d", code_fmt);
+    REQUIRE(n_bits >= 2 && n_bits <= 8, TASQ_ERR_INVALID_ARG, "n_bits %d outside 2..8", n_bits);
+    REQUIRE(M >= 0 && K > 0, TASQ_ERR_INVALID_ARG, "M=%d K=%d", M, K);
+    REQUIRE(K % 16 == 0, TASQ_ERR_UNSUPPORTED, "K=%d must be a multiple of 16", K);
+    if (M == 0) return TASQ_OK;
+    REQUIRE(d_x && d_codes && d_alpha && d_zc, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    REQUIRE(aligned16(d_x) && aligned16(d_codes), TASQ_ERR_UNSUPPORTED, "pointers must be 16-byte aligned");
+    cudaError_t e;
+    if (gran == TASQ_PER_TOKEN)
+        e = tasq::launch_quant_act_token(d_x, dtype, M, K, n_bits, mode, d_codes, code_fmt, d_alpha, d_zc,
+                                         (cudaStream_t)stream);
+    else
+        e = tasq::launch_quant_act_tensor(d_x, dtype, (int64_t)M * K, n_bits, mode, d_codes, code_fmt, d_alpha, d_zc,
+                                          reinterpret_cast<unsigned int*>(ctx->d_words + 16), (cudaStream_t)stream);
+    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "quant_act launch");
+}
+
+namespace {
+
+int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void* d_codes, int code_fmt,
+                       const float* d_alpha, const float* d_zc, int M, const void* d_packed, int N, int K, int B,
+                       int H, int W, int Cin, uint16_t* d_y, int32_t* d_acc, tasq_stream stream) {
+    REQUIRE(ctx->d_table, TASQ_ERR_INVALID_ARG, "no schedule: call tasq_set_schedule first");
+    REQUIRE(layer >= 0 && layer < ctx->L, TASQ_ERR_INVALID_ARG, "layer %d outside 0..%d", layer, ctx->L - 1);
+    REQUIRE(stage >= -1 && stage < ctx->S, TASQ_ERR_INVALID_ARG, "stage %d outside -1..%d", stage, ctx->S - 1);
+    REQUIRE(stage >= 0 || ctx->d_stage, TASQ_ERR_INVALID_ARG, "stage -1 needs tasq_set_stage_device");
+    REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16, TASQ_ERR_INVALID_ARG, "code_fmt %d", code_fmt);
+    REQUIRE(M >= 0 && N > 0 && K > 0, TASQ_ERR_INVALID_ARG, "M=%d N=%d K=%d", M, N, K);
+    REQUIRE(K % 16 == 0 && N % 8 == 0, TASQ_ERR_UNSUPPORTED, "need K %% 16 == 0 and N %% 8 == 0 (N=%d K=%d)", N, K);
+    int route = ctx->route;
+    if (route == TASQ_ROUTE_AUTO) route = code_fmt == TASQ_CODES_F16 ? TASQ_ROUTE_TC : TASQ_ROUTE_MMA_S8;
+    REQUIRE((route == TASQ_ROUTE_TC) == (code_fmt == TASQ_CODES_F16), TASQ_ERR_UNSUPPORTED,
+            "route %d cannot read code format %d", route, code_fmt);
+    if (M == 0) return TASQ_OK;
+    REQUIRE(d_codes && d_alpha && d_zc && d_packed && d_y, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    REQUIRE(aligned16(d_codes) && aligned16(d_y) && aligned16(d_acc), TASQ_ERR_UNSUPPORTED,
+            "pointers must be 16-byte aligned");
+    REQUIRE((reinterpret_cast<uintptr_t>(d_packed) & 255u) == 0, TASQ_ERR_UNSUPPORTED, "d_packed must be 256-byte aligned");
+
+    const tasq::PackedHeader lay = tasq::packed_layout(kind, N, K);
+    const char* p = reinterpret_cast<const char*>(d_packed);
+    tasq::GemmArgs a{};
+    a.x = d_codes;
+    a.alpha = d_alpha;
+    a.zc = d_zc;
+    a.w = reinterpret_cast<const int8_t*>(p + lay.off_w);
+    a.cw = reinterpret_cast<const float*>(p + lay.off_cw);
+    a.bias = reinterpret_cast<const float*>(p + lay.off_bias);
+    a.rs = reinterpret_cast<const int32_t*>(p + lay.off_rs);
+    a.ts = kind == TASQ_CONV3X3 ? reinterpret_cast<const int32_t*>(p + lay.off_ts) : nullptr;
+    a.hdr = reinterpret_cast<const tasq::PackedHeader*>(p);
+    a.table = ctx->d_table;
+    a.d_stage = ctx->d_stage;
+    a.layer = layer;
+    a.stage = stage;
+    a.S = ctx->S;
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.B = B;
+    a.H = H;
+    a.W = W;
+    a.Cin = Cin;
+    a.per_tensor = kind == TASQ_CONV3X3;
+    a.y = d_y;
+    a.acc = d_acc;
+    a.status = ctx->d_words;
+    a.timeout_ns = ctx->timeout_ns;
+    cudaError_t e;
+    if (route == TASQ_ROUTE_TC) {
+        const char* why = nullptr;
+        e = tasq::launch_gemm_tc(a, ctx->num_sms, (cudaStream_t)stream, &why);
+        if (why) return fail(ctx, TASQ_ERR_UNSUPPORTED, "tensor-core route: %s", why);
+    } else {
+        e = tasq::launch_gemm_s8(a, ctx->num_sms, (cudaStream_t)stream);
+    }
+    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "masked contraction launch");
+}
+
+}  // namespace
+
+TASQ_API int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
+                              const float* d_alpha, const float* d_zc, int M, const void* d_packed, int N, int K,
+                              uint16_t* d_y, int32_t* d_acc, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    return masked_contraction(ctx, TASQ_LINEAR, layer, stage, d_codes, code_fmt, d_alpha, d_zc, M, d_packed, N, K, 1,
+                              0, 0, 0, d_y, d_acc, stream);
+}
+
+TASQ_API int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
+                                 const float* d_alpha, const float* d_zc, int B, int H, int W, int Cin,
+                                 const void* d_packed, int Cout, uint16_t* d_y, int32_t* d_acc, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(B >= 0 && H > 0 && W > 0 && Cin > 0, TASQ_ERR_INVALID_ARG, "B=%d H=%d W=%d Cin=%d", B, H, W, Cin);
+    REQUIRE(Cin % 16 == 0, TASQ_ERR_UNSUPPORTED, "conv: Cin=%d must be a multiple of 16", Cin);
+    REQUIRE((int64_t)B * H * W <= 0x7FFFFFFF && (int64_t)9 * Cin <= 0x7FFFFFFF, TASQ_ERR_UNSUPPORTED, "too large");
+    return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, B * H * W, d_packed,
+                              Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
+}

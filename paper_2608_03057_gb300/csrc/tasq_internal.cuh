@@ -1,0 +1,150 @@
+// Internal declarations shared by the translation units of libtasq.
+// Nothing here is part of the C ABI (include/tasq.h is).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/tasq.h"
+
+namespace tasq {
+
+// ---------------------------------------------------------------------------
+// Packed layer layout (one contiguous, caller-allocated buffer per layer).
+// ---------------------------------------------------------------------------
+constexpr uint32_t kPackedMagic = 0x51534154u;  // "TASQ"
+constexpr int kBMin = 2, kBMax = 8, kNumB = kBMax - kBMin + 1;
+constexpr int kCertKBlock = 64;   // K block of the exactness certificate (TC route BK)
+constexpr int64_t kCertLimit = int64_t(1) << 17;  // 2^24 / 128: sum |w| bound per chunk
+
+struct PackedHeader {
+    uint32_t magic;
+    int32_t kind, N, K, Cin;
+    int32_t chunk_kb[kBMax + 1];  // TC route: K blocks per exact fp32 chunk, indexed by b
+    int64_t off_w, off_cw, off_bias, off_rs, off_ts, total;
+};
+static_assert(sizeof(PackedHeader) <= 256, "header must fit in 256 bytes");
+
+__host__ __device__ inline int64_t align_up(int64_t v, int64_t a) { return (v + a - 1) / a * a; }
+
+__host__ __device__ inline PackedHeader packed_layout(int kind, int N, int K) {
+    PackedHeader h{};
+    h.magic = kPackedMagic;
+    h.kind = kind;
+    h.N = N;
+    h.K = K;
+    h.Cin = kind == TASQ_CONV3X3 ? K / 9 : 0;
+    h.off_w = 1024;
+    h.off_cw = align_up(h.off_w + int64_t(N) * K, 256);
+    h.off_bias = align_up(h.off_cw + 4 * int64_t(N), 256);
+    h.off_rs = align_up(h.off_bias + 4 * int64_t(N), 256);          // int32 [kNumB][N]
+    h.off_ts = align_up(h.off_rs + 4 * int64_t(kNumB) * N, 256);     // int32 [kNumB][N][9] (conv)
+    h.total = align_up(h.off_ts + (kind == TASQ_CONV3X3 ? 4 * int64_t(kNumB) * N * 9 : 0), 256);
+    return h;
+}
+
+// Signed stored code with the low 8-b planes of the unsigned code cleared.
+// (v + 128) has the same low planes as v, and 128 is a multiple of 2^(8-b).
+__host__ __device__ inline int mask_code(int v, int b) { return v & ~((1 << (8 - b)) - 1); }
+// Byte mask replicated over a 32-bit word of four codes.
+__host__ __device__ inline uint32_t mask_word(int b) { return 0x01010101u * (0xFFu & (0xFFu << (8 - b))); }
+
+// ---------------------------------------------------------------------------
+// Device status word: first error wins.
+// ---------------------------------------------------------------------------
+__device__ inline void set_status(int* status, int code) {
+    if (status) atomicCAS(status, 0, code);
+}
+
+// ---------------------------------------------------------------------------
+// Arguments of the masked contraction kernels (both routes, linear and conv).
+// ---------------------------------------------------------------------------
+struct GemmArgs {
+    const void* x;            // codes: [M][K] (linear) or NHWC (conv)
+    const float* alpha;       // [M] or [1]
+    const float* zc;
+    const int8_t* w;          // stored codes [N][K]
+    const float* cw;          // [N]
+    const float* bias;        // [N]
+    const int32_t* rs;        // [kNumB][N]
+    const int32_t* ts;        // conv: [kNumB][N][9]
+    const PackedHeader* hdr;  // device copy of the header
+    const uint8_t* table;     // [L][S]
+    const int32_t* d_stage;   // used when stage < 0
+    int layer, stage, S;
+    int M, N, K;
+    int B, H, W, Cin;         // conv geometry (Cin == 0 for a linear layer)
+    int per_tensor;
+    uint16_t* y;              // bf16 bits
+    int32_t* acc;             // optional int32 accumulators
+    int* status;
+    unsigned long long timeout_ns;
+};
+
+// Resolves b for this launch on the device; returns 0 (and records an error)
+// when the stage or the table entry is out of range or the header mismatches.
+__device__ inline int resolve_bits(const GemmArgs& a) {
+    int stage = a.stage >= 0 ? a.stage : (a.d_stage ? *a.d_stage : -1);
+    if (stage < 0 || stage >= a.S) {
+        set_status(a.status, TASQ_ERR_DEVICE);
+        return 0;
+    }
+    int b = a.table[a.layer * a.S + stage];
+    if (b < kBMin || b > kBMax || a.hdr->magic != kPackedMagic || a.hdr->N != a.N || a.hdr->K != a.K) {
+        set_status(a.status, TASQ_ERR_DEVICE);
+        return 0;
+    }
+    return b;
+}
+
+// Fused dequantization epilogue, fp32 with one rounding per operation:
+// y = ((float(acc) + zc * float(rs)) * (alpha * cw)) + bias.
+__device__ inline float epilogue_value(int acc, float alpha, float zc, int rs, float cw, float bias) {
+    float a = __int2float_rn(acc);
+    float t = __fmul_rn(zc, __int2float_rn(rs));
+    float u = __fadd_rn(a, t);
+    float s = __fmul_rn(alpha, cw);
+    float v = __fmul_rn(u, s);
+    return __fadd_rn(v, bias);
+}
+
+// fp32 -> bf16 bits, round to nearest even (finite inputs).
+__device__ inline uint16_t bf16_bits(float f) {
+    uint32_t u = __float_as_uint(f);
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+// Sum of the in-bounds taps' per-tap weight sums for output pixel (h, w).
+__device__ inline int conv_row_sum(const int32_t* ts_n, int h, int w, int H, int W) {
+    int s = 0;
+#pragma unroll
+    for (int dh = 0; dh < 3; ++dh) {
+        int ih = h + dh - 1;
+        if (ih < 0 || ih >= H) continue;
+#pragma unroll
+        for (int dw = 0; dw < 3; ++dw) {
+            int iw = w + dw - 1;
+            if (iw < 0 || iw >= W) continue;
+            s += ts_n[dh * 3 + dw];
+        }
+    }
+    return s;
+}
+
+// ---------------------------------------------------------------------------
+// Host-side launchers implemented in the kernel translation units.
+// ---------------------------------------------------------------------------
+cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int8_t* sw, float* cw, float* alpha,
+                                 cudaStream_t st);
+cudaError_t launch_quant_act_token(const void* x, int dtype, int M, int K, int n_bits, int mode, void* codes,
+                                   int code_fmt, float* alpha, float* zc, cudaStream_t st);
+cudaError_t launch_quant_act_tensor(const void* x, int dtype, int64_t count, int n_bits, int mode, void* codes,
+                                    int code_fmt, float* alpha, float* zc, unsigned int* scratch, cudaStream_t st);
+cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* bias, int N, int K, int Cin,
+                        void* packed, cudaStream_t st);
+cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why);
+cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, cudaStream_t st);
+
+}  // namespace tasq

@@ -1,0 +1,400 @@
+"""GPU parity: every step of the path, called through the C ABI, against the
+CPU oracle on the same seeded inputs.
+
+Bar: int8 codes, int32 accumulators, row sums and the packed certificate are
+bit-exact; bf16 outputs are within |d| <= 1e-2 + 1e-3 |ref| of the oracle's
+fp32-order epilogue (and are expected to be bit-identical, since both sides
+round every fp32 operation to nearest even in the same order).
+"""
+import numpy as np
+import pytest
+
+from paper_2608_03057_gb300 import tasq, workloads
+from tests import gpu_layer as G
+
+pytestmark = pytest.mark.gpu
+
+ROUTES = [pytest.param(tasq.TASQ_CODES_S8, id="mma_s8"), pytest.param(tasq.TASQ_CODES_F16, id="tc")]
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    c = G.Ctx()
+    yield c
+    assert tasq.tasq_device_status(c.h) == tasq.TASQ_OK
+    c.close()
+
+
+# ------------------------------------------------------------ quantizers --
+
+@pytest.mark.parametrize("dtype", [tasq.TASQ_F32, tasq.TASQ_BF16])
+def test_quant_weights_bitexact(ctx, oracle, dtype):
+    torch = G.torch()
+    N, K = 136, 1168
+    w = workloads.normal((N, K), seed=1, std=0.02)
+    w[5] = 0.0  # degenerate channel
+    if dtype == tasq.TASQ_BF16:
+        wd, w = G.to_bf16(w)
+    else:
+        wd = G.dev(w)
+    sw, cw, al = G.quant_weights(ctx, wd, dtype, N, K)
+    ref = oracle.quant_weight(w, 8, oracle.SYMRANGE)
+    assert np.array_equal(sw.cpu().numpy(), ref["s"])
+    assert np.array_equal(cw.cpu().numpy(), ref["c"])
+    assert np.array_equal(al.cpu().numpy(), ref["alpha"])
+
+
+@pytest.mark.parametrize("code_fmt", [tasq.TASQ_CODES_S8, tasq.TASQ_CODES_F16])
+@pytest.mark.parametrize("mode", [tasq.TASQ_SYMRANGE, tasq.TASQ_ASYM])
+@pytest.mark.parametrize("n_bits", [8, 4])
+@pytest.mark.parametrize("dtype", [tasq.TASQ_F32, tasq.TASQ_BF16])
+def test_quant_act_per_token_bitexact(ctx, oracle, code_fmt, mode, n_bits, dtype):
+    M, K = 203, 1152
+    x = workloads.normal((M, K), seed=0)
+    x[7] = 0.0          # constant row
+    x[9] = np.abs(x[9]) + 0.5  # one-signed row
+    x[11, :] = 3.0
+    x[11, 5] = 2.5      # exact ties of the rounding
+    if dtype == tasq.TASQ_BF16:
+        xd, x = G.to_bf16(x)
+    else:
+        xd = G.dev(x)
+    codes, alpha, zc = G.quant_act(ctx, xd, dtype, M, K, n_bits, mode, tasq.TASQ_PER_TOKEN, code_fmt)
+    s, a, z = oracle.quant_act(x, n_bits, mode, oracle.PER_TOKEN)
+    assert np.array_equal(G.codes_to_int8(codes), s)
+    assert np.array_equal(alpha.cpu().numpy(), a)
+    assert np.array_equal(zc.cpu().numpy(), z)
+
+
+@pytest.mark.parametrize("mode", [tasq.TASQ_SYMRANGE, tasq.TASQ_ASYM])
+@pytest.mark.parametrize("code_fmt", [tasq.TASQ_CODES_S8, tasq.TASQ_CODES_F16])
+def test_quant_act_per_tensor_bitexact(ctx, oracle, mode, code_fmt):
+    B, H, W, C = 1, 64, 64, 320
+    x = workloads.normal((B, H, W, C), seed=2)
+    codes, alpha, zc = G.quant_act(ctx, G.dev(x), tasq.TASQ_F32, B * H * W, C, 8, mode, tasq.TASQ_PER_TENSOR, code_fmt)
+    s, a, z = oracle.quant_act(x.reshape(1, -1), 8, mode, oracle.PER_TOKEN)
+    assert np.array_equal(G.codes_to_int8(codes).reshape(-1), s.reshape(-1))
+    assert alpha.cpu().numpy()[0] == a[0] and zc.cpu().numpy()[0] == z[0]
+
+
+# ------------------------------------------------------------------ pack --
+
+def _expected_chunk(masked_abs_blocks, limit=1 << 17):
+    """Longest window length (in 64-wide K blocks) all of whose windows stay
+    within the limit, minimized over channels."""
+    best = None
+    for row in masked_abs_blocks:
+        KB = len(row)
+        c = KB
+        for L in range(1, KB + 1):
+            if max(row[i:i + L].sum() for i in range(KB - L + 1)) > limit:
+                c = L - 1
+                break
+        best = c if best is None else min(best, c)
+    return max(best, 1)
+
+
+@pytest.mark.parametrize("kind", [tasq.TASQ_LINEAR, tasq.TASQ_CONV3X3])
+def test_pack_row_sums_and_certificate(ctx, oracle, kind):
+    torch = G.torch()
+    if kind == tasq.TASQ_LINEAR:
+        N, K, Cin = 72, 4096, 0
+    else:
+        N, Cin = 48, 320
+        K = 9 * Cin
+    s_w = workloads.uniform_codes((N, K), seed=3, lo=-128, hi=127)
+    cw = workloads.uniform((N,), 4, 1e-4, 1e-3)
+    packed = G.pack(ctx, kind, G.dev(s_w), G.dev(cw), None, N, K, Cin)
+    torch.cuda.synchronize()
+    chunk, off = G.packed_header(packed)
+    raw = packed.cpu().numpy()
+    assert np.array_equal(raw[off["off_w"]:off["off_w"] + N * K].view(np.int8).reshape(N, K), s_w)
+    rs = raw[off["off_rs"]:off["off_rs"] + 4 * 7 * N].view(np.int32).reshape(7, N)
+    for b in range(2, 9):
+        masked = oracle.mask(s_w, b).astype(np.int64)
+        assert np.array_equal(rs[b - 2], oracle.row_sums(s_w, b)), b
+        KB = (K + 63) // 64
+        blocks = np.abs(np.pad(masked, ((0, 0), (0, KB * 64 - K)))).reshape(N, KB, 64).sum(2)
+        assert chunk[b] == _expected_chunk(blocks), b
+        if kind == tasq.TASQ_CONV3X3:
+            ts = raw[off["off_ts"]:off["off_ts"] + 4 * 7 * N * 9].view(np.int32).reshape(7, N, 9)
+            assert np.array_equal(ts[b - 2], masked.reshape(N, 9, Cin).sum(2)), b
+
+
+# ---------------------------------------------------------- linear layer --
+
+def _setup_linear(ctx, oracle, M, N, K, bits, seed=0, x_std=1.0, w_std=0.02, dtype=tasq.TASQ_F32, code_fmt=None,
+                  mode=tasq.TASQ_SYMRANGE):
+    w = workloads.normal((N, K), seed + 1, w_std)
+    bias = workloads.normal((N,), seed + 2, 0.02)
+    x = workloads.normal((M, K), seed, x_std)
+    if dtype == tasq.TASQ_BF16:
+        xd, x = G.to_bf16(x)
+    else:
+        xd = G.dev(x)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, G.dev(bias), N, K)
+    tasq.tasq_set_schedule(ctx.h, np.asarray([bits], np.uint8), 1, len(bits))
+    codes, alpha, zc = G.quant_act(ctx, xd, dtype, M, K, 8, mode, tasq.TASQ_PER_TOKEN, code_fmt)
+    wq = oracle.quant_weight(w)
+    s_x, a_ref, z_ref = oracle.quant_act(x, 8, mode, oracle.PER_TOKEN)
+    return dict(packed=packed, codes=codes, alpha=alpha, zc=zc, wq=wq, s_x=s_x, a=a_ref, z=z_ref, bias=bias)
+
+
+def _check_layer(oracle, st, b, y, acc, rows=None):
+    s_x, a, z = st["s_x"], st["a"], st["z"]
+    if rows is not None:
+        s_x, a, z = s_x[rows], a[rows], z[rows]
+    ref_acc = oracle.gemm(s_x, st["wq"]["s"], b)
+    got_acc = acc.cpu().numpy() if rows is None else acc.cpu().numpy()[rows]
+    assert np.array_equal(got_acc, ref_acc), f"b={b}: {(got_acc != ref_acc).sum()} int32 mismatches"
+    rs = oracle.row_sums(st["wq"]["s"], b)
+    _, yb = oracle.epilogue_f32(ref_acc, a, z, rs, st["wq"]["c"], st["bias"])
+    got_y = G.bf16_bits_host(y) if rows is None else G.bf16_bits_host(y)[rows]
+    same = G.assert_bf16_close(got_y, yb)
+    assert same == yb.size, f"b={b}: {yb.size - same} bf16 outputs differ in the last bit"
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_single_linear_all_stages(ctx, oracle, code_fmt):
+    """256 tokens x 1152 -> 1152, stages at b = 8, 6, 4, 3 on one shared buffer."""
+    M, N, K = 256, 1152, 1152
+    st = _setup_linear(ctx, oracle, M, N, K, [8, 6, 4, 3], code_fmt=code_fmt)
+    for stage, b in enumerate([8, 6, 4, 3]):
+        y, acc = G.gemm(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+        _check_layer(oracle, st, b, y, acc)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("M,N,K", [(1, 8, 16), (77, 24, 48), (300, 136, 1168), (129, 264, 2240), (513, 72, 64)])
+def test_ragged_shapes(ctx, oracle, code_fmt, M, N, K):
+    bits = [2, 5, 7, 8]
+    st = _setup_linear(ctx, oracle, M, N, K, bits, seed=M + N, code_fmt=code_fmt, mode=tasq.TASQ_ASYM)
+    for stage, b in enumerate(bits):
+        y, acc = G.gemm(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+        _check_layer(oracle, st, b, y, acc)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_output_without_acc(ctx, oracle, code_fmt):
+    M, N, K = 200, 128, 256
+    st = _setup_linear(ctx, oracle, M, N, K, [6], code_fmt=code_fmt)
+    y0, acc = G.gemm(ctx, 0, 0, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+    y1, _ = G.gemm(ctx, 0, 0, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K, want_acc=False)
+    assert np.array_equal(G.bf16_bits_host(y0), G.bf16_bits_host(y1))
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_empty_batch_is_a_noop(ctx, code_fmt):
+    torch = G.torch()
+    N, K = 64, 64
+    sw = torch.zeros((N, K), dtype=torch.int8, device="cuda")
+    cw = torch.ones((N,), dtype=torch.float32, device="cuda")
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K)
+    tasq.tasq_set_schedule(ctx.h, np.array([[8]], np.uint8), 1, 1)
+    one = torch.zeros((16,), dtype=torch.float32, device="cuda")
+    tasq.tasq_masked_gemm(ctx.h, 0, 0, one, code_fmt, one, one, 0, packed, N, K, one, None)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_extreme_codes_exact(ctx, oracle, code_fmt):
+    """All activation and weight codes at -128 (|acc| = 16384 K) and
+    alternating-sign rows: the accumulators must stay exact."""
+    torch = G.torch()
+    M, N, K = 130, 136, 1024
+    s_w = np.full((N, K), -128, np.int8)
+    s_w[1::2, 1::2] = 127
+    s_x = np.full((M, K), -128, np.int8)
+    s_x[1::3, ::2] = 127
+    cw = np.full((N,), 1e-6, np.float32)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, G.dev(s_w), G.dev(cw), None, N, K)
+    tasq.tasq_set_schedule(ctx.h, np.array([[8, 2, 5]], np.uint8), 1, 3)
+    codes = G.dev(s_x) if code_fmt == tasq.TASQ_CODES_S8 else G.dev(s_x.astype(np.float16))
+    alpha = G.dev(np.full((M,), 1e-3, np.float32))
+    zc = G.dev(np.full((M,), 0.5, np.float32))
+    for stage, b in enumerate([8, 2, 5]):
+        y, acc = G.gemm(ctx, 0, stage, codes, code_fmt, alpha, zc, M, packed, N, K)
+        assert np.array_equal(acc.cpu().numpy(), oracle.gemm(s_x, s_w, b)), b
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_uniform_codes_long_k_exact(ctx, oracle, code_fmt):
+    """Uniform [-127, 127] codes with K = 4096: sums of |w| exceed the fp32
+    exact range, so the tensor-core route must drain in certified chunks."""
+    M, N, K = 256, 256, 4096
+    s_x = workloads.uniform_codes((M, K), seed=61)
+    s_w = workloads.uniform_codes((N, K), seed=62)
+    cw = workloads.uniform((N,), 63, 1e-4, 2e-4)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, G.dev(s_w), G.dev(cw), None, N, K)
+    tasq.tasq_set_schedule(ctx.h, np.array([[8, 7, 4, 2]], np.uint8), 1, 4)
+    codes = G.dev(s_x) if code_fmt == tasq.TASQ_CODES_S8 else G.dev(s_x.astype(np.float16))
+    alpha = G.dev(workloads.uniform((M,), 64, 1e-3, 2e-3))
+    zc = G.dev(np.full((M,), 0.5, np.float32))
+    for stage, b in enumerate([8, 7, 4, 2]):
+        y, acc = G.gemm(ctx, 0, stage, codes, code_fmt, alpha, zc, M, packed, N, K)
+        assert np.array_equal(acc.cpu().numpy(), oracle.gemm(s_x, s_w, b)), b
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_stage_from_device_int(ctx, oracle, code_fmt):
+    torch = G.torch()
+    M, N, K = 128, 256, 512
+    bits = [3, 8, 5]
+    st = _setup_linear(ctx, oracle, M, N, K, bits, code_fmt=code_fmt)
+    d_stage = torch.zeros((4,), dtype=torch.int32, device="cuda")
+    tasq.tasq_set_stage_device(ctx.h, d_stage)
+    try:
+        for stage, b in enumerate(bits):
+            d_stage.fill_(stage)
+            y, acc = G.gemm(ctx, 0, -1, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+            _check_layer(oracle, st, b, y, acc)
+        d_stage.fill_(7)  # out of range: recorded on the device, nothing written
+        G.gemm(ctx, 0, -1, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+        assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_ERR_DEVICE
+        assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+    finally:
+        tasq.tasq_set_stage_device(ctx.h, None)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("M,N,K", [(4096, 3456, 1152), (4096, 1152, 4608), (1200, 2240, 2240), (77, 1280, 2048)])
+def test_full_size_sampled_rows(ctx, oracle, code_fmt, M, N, K):
+    """Full-size layer shapes of the backbones, checked on sampled token rows
+    (the oracle computes those rows one by one)."""
+    bits = [3, 8]
+    st = _setup_linear(ctx, oracle, M, N, K, bits, seed=K, dtype=tasq.TASQ_BF16, code_fmt=code_fmt)
+    rows = np.unique(np.concatenate([np.arange(0, M, max(1, M // 40)), [M - 1]]))
+    for stage, b in enumerate(bits):
+        y, acc = G.gemm(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+        _check_layer(oracle, st, b, y, acc, rows=rows)
+
+
+# ------------------------------------------------------------------ conv --
+
+def _run_conv(ctx, oracle, B, H, W, Cin, Cout, bits, code_fmt, seed=0, rows=None):
+    torch = G.torch()
+    K = 9 * Cin
+    x = workloads.normal((B, H, W, Cin), seed)
+    w = workloads.normal((Cout, K), seed + 1, 0.02)
+    bias = workloads.normal((Cout,), seed + 2, 0.02)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, Cout, K)
+    packed = G.pack(ctx, tasq.TASQ_CONV3X3, sw, cw, G.dev(bias), Cout, K, Cin)
+    tasq.tasq_set_schedule(ctx.h, np.asarray([bits], np.uint8), 1, len(bits))
+    codes, alpha, zc = G.quant_act(ctx, G.dev(x), tasq.TASQ_F32, B * H * W, Cin, 8, tasq.TASQ_SYMRANGE,
+                                   tasq.TASQ_PER_TENSOR, code_fmt)
+    wq = oracle.quant_weight(w)
+    s_x, a, z = oracle.quant_act(x.reshape(1, -1), 8, 0, 0)
+    s_x = s_x.reshape(B, H, W, Cin)
+    assert np.array_equal(G.codes_to_int8(codes).reshape(B, H, W, Cin), s_x)
+    for stage, b in enumerate(bits):
+        y, acc = G.conv(ctx, 0, stage, codes, code_fmt, alpha, zc, B, H, W, Cin, packed, Cout)
+        if rows is None:
+            ref_acc, rs = oracle.conv3x3(s_x, wq["s"], b)
+            got_acc, got_y = acc.cpu().numpy(), G.bf16_bits_host(y)
+        else:
+            ref_acc, rs = _conv_rows(oracle, s_x, wq["s"], b, rows)
+            got_acc, got_y = acc.cpu().numpy()[rows], G.bf16_bits_host(y)[rows]
+        assert np.array_equal(got_acc, ref_acc), f"b={b}: {(got_acc != ref_acc).sum()} int32 mismatches"
+        _, yb = oracle.epilogue_f32(ref_acc, a, z, rs, wq["c"], bias, per_tensor=True, rs_per_row=True)
+        same = G.assert_bf16_close(got_y, yb)
+        assert same == yb.size
+
+
+def _conv_rows(oracle, s_x, s_w, b, rows):
+    """Oracle conv restricted to output pixels `rows`: each pixel's 3x3
+    neighbourhood is cut out (zero code padding outside the image) and run
+    through the oracle conv on a 3x3 image, whose centre pixel is the wanted one."""
+    B, H, W, Cin = s_x.shape
+    acc_out, rs_out = [], []
+    for p in rows:
+        bb, h, w = p // (H * W), (p // W) % H, p % W
+        patch = np.zeros((1, 3, 3, Cin), np.int8)
+        valid = np.zeros((3, 3), bool)
+        for dh in range(3):
+            for dw in range(3):
+                ih, iw = h + dh - 1, w + dw - 1
+                if 0 <= ih < H and 0 <= iw < W:
+                    patch[0, dh, dw] = s_x[bb, ih, iw]
+                    valid[dh, dw] = True
+        acc, _ = oracle.conv3x3(patch, s_w, b)
+        acc_out.append(acc[4])
+        m = oracle.mask(s_w, b).astype(np.int64).reshape(s_w.shape[0], 3, 3, Cin).sum(3)
+        rs_out.append((m * valid[None]).sum((1, 2)).astype(np.int32))
+    return np.stack(acc_out), np.stack(rs_out)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("B,H,W,Cin,Cout", [(1, 8, 8, 32, 16), (2, 5, 7, 16, 24), (1, 1, 1, 48, 8), (1, 3, 1, 64, 136)])
+def test_conv_small_full(ctx, oracle, code_fmt, B, H, W, Cin, Cout):
+    _run_conv(ctx, oracle, B, H, W, Cin, Cout, [8, 4, 6], code_fmt)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("C,HW", [(320, 64), (640, 32), (1280, 16)])
+def test_conv_full_size_sampled(ctx, oracle, code_fmt, C, HW):
+    rng = workloads.rng(C)
+    P = HW * HW
+    border = [0, HW - 1, HW * (HW - 1), P - 1, HW // 2, HW * (HW // 2)]
+    rows = np.unique(np.concatenate([border, rng.integers(0, P, 24)]))
+    _run_conv(ctx, oracle, 1, HW, HW, C, C, [5, 8], code_fmt, seed=C, rows=rows)
+
+
+# ------------------------------------------------------ failure handling --
+
+def test_invalid_arguments_launch_nothing(ctx):
+    torch = G.torch()
+    buf = torch.zeros((1 << 16,), dtype=torch.uint8, device="cuda")
+    with pytest.raises(tasq.TasqError) as e:
+        tasq.tasq_set_schedule(ctx.h, np.array([[9]], np.uint8), 1, 1)
+    assert e.value.code == tasq.TASQ_ERR_INVALID_ARG
+    tasq.tasq_set_schedule(ctx.h, np.array([[8, 4]], np.uint8), 1, 2)
+    cases = [
+        dict(layer=1, stage=0, K=64, N=64, code=tasq.TASQ_ERR_INVALID_ARG),
+        dict(layer=0, stage=2, K=64, N=64, code=tasq.TASQ_ERR_INVALID_ARG),
+        dict(layer=0, stage=-1, K=64, N=64, code=tasq.TASQ_ERR_INVALID_ARG),
+        dict(layer=0, stage=0, K=40, N=64, code=tasq.TASQ_ERR_UNSUPPORTED),
+        dict(layer=0, stage=0, K=64, N=60, code=tasq.TASQ_ERR_UNSUPPORTED),
+    ]
+    for c in cases:
+        with pytest.raises(tasq.TasqError) as e:
+            tasq.tasq_masked_gemm(ctx.h, c["layer"], c["stage"], buf, tasq.TASQ_CODES_S8, buf, buf, 16, buf, c["N"],
+                                  c["K"], buf, None)
+        assert e.value.code == c["code"], c
+    with pytest.raises(tasq.TasqError) as e:  # misaligned output pointer
+        tasq.tasq_masked_gemm(ctx.h, 0, 0, buf, tasq.TASQ_CODES_S8, buf, buf, 16, buf, 64, 64, buf.data_ptr() + 2, None)
+    assert e.value.code == tasq.TASQ_ERR_UNSUPPORTED
+    with pytest.raises(tasq.TasqError) as e:  # route and code storage disagree
+        tasq.tasq_set_route(ctx.h, tasq.TASQ_ROUTE_TC)
+        tasq.tasq_masked_gemm(ctx.h, 0, 0, buf, tasq.TASQ_CODES_S8, buf, buf, 16, buf, 64, 64, buf, None)
+    tasq.tasq_set_route(ctx.h, tasq.TASQ_ROUTE_AUTO)
+    assert e.value.code == tasq.TASQ_ERR_UNSUPPORTED
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+def test_packed_buffer_mismatch_is_caught_on_device(ctx, oracle):
+    torch = G.torch()
+    N, K = 64, 128
+    sw = torch.zeros((N, K), dtype=torch.int8, device="cuda")
+    cw = torch.ones((N,), dtype=torch.float32, device="cuda")
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K)
+    tasq.tasq_set_schedule(ctx.h, np.array([[8]], np.uint8), 1, 1)
+    codes = torch.zeros((16, 64), dtype=torch.int8, device="cuda")
+    al = torch.ones((16,), dtype=torch.float32, device="cuda")
+    y = torch.zeros((16, 64), dtype=torch.int16, device="cuda")
+    tasq.tasq_masked_gemm(ctx.h, 0, 0, codes, tasq.TASQ_CODES_S8, al, al, 16, packed, 64, 64, y, None)  # K mismatch
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_ERR_DEVICE
+
+
+def test_device_wait_timeout_is_reported_and_context_survives(ctx, oracle):
+    tasq.tasq_selftest_timeout(ctx.h, 50_000_000)  # 50 ms wait on a barrier nothing arrives at
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_ERR_DEVICE_TIMEOUT
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+    # the context still computes correctly afterwards
+    M, N, K = 64, 64, 128
+    st = _setup_linear(ctx, oracle, M, N, K, [7], code_fmt=tasq.TASQ_CODES_S8)
+    y, acc = G.gemm(ctx, 0, 0, st["codes"], tasq.TASQ_CODES_S8, st["alpha"], st["zc"], M, st["packed"], N, K)
+    _check_layer(oracle, st, 7, y, acc)
