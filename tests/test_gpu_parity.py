@@ -328,9 +328,20 @@ def _conv_rows(oracle, s_x, s_w, b, rows):
 
 
 @pytest.mark.parametrize("code_fmt", ROUTES)
-@pytest.mark.parametrize("B,H,W,Cin,Cout", [(1, 8, 8, 32, 16), (2, 5, 7, 16, 24), (1, 1, 1, 48, 8), (1, 3, 1, 64, 136)])
+@pytest.mark.parametrize("B,H,W,Cin,Cout", [(1, 8, 8, 64, 16), (2, 5, 7, 64, 24), (1, 1, 1, 128, 8), (1, 3, 1, 64, 136),
+                                            (1, 9, 13, 192, 40), (2, 16, 16, 64, 256)])
 def test_conv_small_full(ctx, oracle, code_fmt, B, H, W, Cin, Cout):
     _run_conv(ctx, oracle, B, H, W, Cin, Cout, [8, 4, 6], code_fmt)
+
+
+@pytest.mark.parametrize("B,H,W,Cin,Cout", [(1, 8, 8, 32, 16), (2, 5, 7, 16, 24), (1, 1, 1, 48, 8)])
+def test_conv_narrow_channels(ctx, oracle, B, H, W, Cin, Cout):
+    """Cin % 16 == 0 but not % 64: the int8 route runs it; the tensor-core
+    route (whose 64-wide K blocks must not straddle a tap) refuses it."""
+    _run_conv(ctx, oracle, B, H, W, Cin, Cout, [8, 4, 6], tasq.TASQ_CODES_S8)
+    with pytest.raises(tasq.TasqError) as e:
+        _run_conv(ctx, oracle, B, H, W, Cin, Cout, [8], tasq.TASQ_CODES_F16)
+    assert e.value.code == tasq.TASQ_ERR_UNSUPPORTED
 
 
 @pytest.mark.parametrize("code_fmt", ROUTES)
