@@ -1,0 +1,465 @@
+#!/usr/bin/env python3
+"""Benchmark of the TASQ masked-W8A8 path on GB300.
+
+One step = one denoising step of a synthetic backbone: for every quantized
+layer, activation quantization (per token; per tensor for a 3x3 conv) and the
+masked contraction at that layer's operating precision for the step's stage,
+read from the device-resident bit table.  The whole step is captured once as
+a CUDA graph; the stage comes from a device int written before each replay,
+so a stage switch is a 4-byte write and never a weight copy.
+
+Default workload: the PixArt-Sigma-shaped DiT at 1024 px (224 layers, 4096
+image tokens, 300 text tokens, 20 stages, learned-style schedule).  The JSON
+line reports throughput in int8-equivalent TOPS (2*M*N*K per layer call,
+independent of b), ms per step, the same step under the all-8-bit schedule,
+the roofline of the dominant kernel, an end-to-end figure through the C ABI
+with host buffers, and the CPU oracle's throughput on a bounded sample.
+
+--impl reference times the CPU oracle (the reference arm of this repository)
+on a bounded sample of the same workload, on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np
+
+METRIC = "masked W8A8 GEMM TOPS and % int8 tensor peak vs effective bits b; ms/denoise step"
+UNIT = "TOPS"
+WORKLOAD_NAMES = {
+    "pixart": "pixart_sigma_1024px_denoise_step",
+    "sana": "sana_1600m_1024px_denoise_step",
+    "sdxl": "sdxl_turbo_512px_denoise_step",
+    "single": "single_linear_256x1152x1152",
+}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=list(WORKLOAD_NAMES), default="pixart")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU oracle sample budget")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--blocks", type=int, default=0, help="keep only the first N transformer blocks (small cases)")
+    ap.add_argument("--no-all8", action="store_true", help="skip the all-8-bit schedule comparison")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d.get("hbm_gbs", 6800.0), bf16=d.get("bf16_tflops", 1900.0),
+                    bf16_sus=d.get("bf16_tflops_sustained", 1700.0), src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+# ------------------------------------------------------------------ clocks --
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons during a region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.out = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if not self.proc:
+            return None
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                rows.append(dict(sm=float(f[1]), smax=float(f[2]), util=float(f[4]), hw=f[6], hwt=f[7], swt=f[8],
+                                 swp=f[9]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        load = [r for r in rows if r["util"] >= 50] or rows
+        reasons = set()
+        for r in load:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"), ("swt", "sw_thermal_slowdown"),
+                              ("swp", "sw_power_cap")):
+                if r[key].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in load), "sm_max_mhz": max(r["smax"] for r in load),
+                "reasons": sorted(reasons), "samples": len(load)}
+
+
+# --------------------------------------------------------------- workload --
+class Step:
+    """Device-resident workload of one denoising step and its launch sequence."""
+
+    def __init__(self, torch, tasq, workloads, name: str, seed: int, blocks: int = 0):
+        self.torch, self.tasq = torch, tasq
+        self.layers = workloads.inventory(name)
+        self.table = workloads.schedule_for(name, len(self.layers))
+        if blocks:
+            keep = len(workloads.inventory_blocks(name, blocks))
+            self.layers, self.table = self.layers[:keep], np.ascontiguousarray(self.table[:keep])
+        self.S = self.table.shape[1]
+        self.ctx = tasq.tasq_create(torch.cuda.current_device())
+        tasq.tasq_set_schedule(self.ctx, self.table, len(self.layers), self.S)
+        dev = "cuda"
+        self.packed, self.x, self.y = [], [], []
+        max_mk = max(l.M * (l.Cin if l.Cin else l.K) for l in self.layers)
+        max_m = max(l.M for l in self.layers)
+        self.codes = torch.empty((max_mk,), dtype=torch.float16, device=dev)
+        self.alpha = torch.empty((max_m,), dtype=torch.float32, device=dev)
+        self.zc = torch.empty((max_m,), dtype=torch.float32, device=dev)
+        for i, l in enumerate(self.layers):
+            w = workloads.device_normal((l.N, l.K), seed * 100003 + 2 * i + 1, 0.02)
+            sw = torch.empty((l.N, l.K), dtype=torch.int8, device=dev)
+            cw = torch.empty((l.N,), dtype=torch.float32, device=dev)
+            tasq.tasq_quant_weights(self.ctx, w, tasq.TASQ_F32, l.N, l.K, sw, cw)
+            bias = workloads.device_normal((l.N,), seed * 100003 + 2 * i + 2, 0.02)
+            kind = tasq.TASQ_CONV3X3 if l.kind == workloads.CONV3X3 else tasq.TASQ_LINEAR
+            pk = torch.empty((tasq.tasq_packed_bytes(kind, l.N, l.K),), dtype=torch.uint8, device=dev)
+            tasq.tasq_pack_weights(self.ctx, kind, sw, cw, bias, l.N, l.K, l.Cin, pk)
+            self.packed.append(pk)
+            xs = (l.B, l.H, l.W, l.Cin) if l.kind == workloads.CONV3X3 else (l.M, l.K)
+            self.x.append(workloads.device_normal(xs, seed * 100003 + 1000003 + i, 1.0, torch.bfloat16))
+            self.y.append(torch.empty((l.M, l.N), dtype=torch.int16, device=dev))
+            del w, sw, cw, bias
+        self.d_stage = torch.zeros((4,), dtype=torch.int32, device=dev)
+        tasq.tasq_set_stage_device(self.ctx, self.d_stage)
+        torch.cuda.synchronize()
+        self.ops = sum(l.ops for l in self.layers)
+        self.gemm_ops = [l.ops for l in self.layers]
+        self.conv = workloads.CONV3X3
+
+    def launch(self, events=None):
+        """Enqueue one step on the current stream (stage read from d_stage)."""
+        t = self.tasq
+        for i, l in enumerate(self.layers):
+            if l.kind == self.conv:
+                t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.Cin, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TENSOR,
+                                 self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
+                if events:
+                    events[i][0].record()
+                t.tasq_masked_conv3x3(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B, l.H,
+                                      l.W, l.Cin, self.packed[i], l.N, self.y[i], None)
+            else:
+                t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.K, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TOKEN,
+                                 self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
+                if events:
+                    events[i][0].record()
+                t.tasq_masked_gemm(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
+                                   self.packed[i], l.N, l.K, self.y[i], None)
+            if events:
+                events[i][1].record()
+
+    def launches_per_step(self):
+        # per-token quant: 1 kernel; per-tensor quant: 2 kernels (+ a memset); contraction: 1 kernel
+        return sum(3 if l.kind == self.conv else 2 for l in self.layers)
+
+    def act_bytes(self):
+        """HBM bytes of activation quantization per step (bf16 in, fp16 codes out, scales)."""
+        return sum(l.M * (l.Cin if l.Cin else l.K) * 4 + 8 * l.M for l in self.layers)
+
+    def gemm_bytes(self):
+        """Algorithmic HBM bytes of the contractions per step: fp16 codes in, int8 weights,
+        bf16 out, per-channel and per-token scalars."""
+        tot = 0
+        for l in self.layers:
+            k_in = l.Cin if l.Cin else l.K
+            tot += l.M * k_in * 2 + l.N * l.K + 2 * l.M * l.N + 12 * l.N + 8 * l.M
+        return tot
+
+    def close(self):
+        self.tasq.tasq_destroy(self.ctx)
+
+
+def make_events(torch, n, external):
+    kw = dict(enable_timing=True)
+    if external:
+        kw["external"] = True
+    return [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(n)]
+
+
+def capture(torch, step, events=None):
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+        step.launch(events)
+    return g
+
+
+def timed_replays(torch, g, step, steps, stage_of):
+    s = torch.cuda.current_stream()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0.record(s)
+    for k in range(steps):
+        step.d_stage.fill_(stage_of(k))
+        g.replay()
+    t1.record(s)
+    torch.cuda.synchronize()
+    return t0.elapsed_time(t1) / steps
+
+
+# ------------------------------------------------------------ CPU oracle --
+def oracle_sample(workload: str, budget_s: float, rows: int = 32, seed: int = 0, max_layers=None):
+    """Time the CPU oracle (act quant, int32 contraction, row sums, fp32
+    epilogue) on `rows` token rows of successive layers of the workload until
+    the budget is spent.  Returns (ops, seconds, layers_done, rows, threads)."""
+    from oracle import oracle
+    from paper_2608_03057_gb300 import workloads
+
+    layers = workloads.inventory(workload)
+    table = workloads.schedule_for(workload, len(layers))
+    oracle.build()
+    ops = 0
+    spent = 0.0
+    done = 0
+    for i, l in enumerate(layers):
+        if (max_layers is not None and done >= max_layers) or spent >= budget_s:
+            break
+        w = workloads.normal((l.N, l.K), seed + 2 * i + 1, 0.02)
+        wq = oracle.quant_weight(w)
+        b = int(table[i, 0])
+        if l.kind == workloads.CONV3X3:
+            # `rows` 3x3 images: 9 output pixels each with 4 (corner), 6 (edge) or 9 valid taps
+            x = workloads.normal((rows, 3, 3, l.Cin), seed + 7 * i + 3)
+            t0 = time.perf_counter()
+            s_x, a, z = oracle.quant_act(x.reshape(1, -1), 8, oracle.SYMRANGE, oracle.PER_TOKEN)
+            acc, rs = oracle.conv3x3(s_x.reshape(rows, 3, 3, l.Cin), wq["s"], b)
+            oracle.epilogue_f32(acc, a, z, rs, wq["c"], None, per_tensor=True, rs_per_row=True)
+            spent += time.perf_counter() - t0
+            ops += 2 * rows * (4 * 4 + 4 * 6 + 9) * l.Cin * l.N
+        else:
+            x = workloads.normal((rows, l.K), seed + 7 * i + 3)
+            t0 = time.perf_counter()
+            oracle.linear_layer(x, wq["s"], wq["c"], None, b)
+            spent += time.perf_counter() - t0
+            ops += 2 * rows * l.N * l.K
+        done += 1
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return ops, spent, done, rows, threads
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    # warm-up samples, then K timed samples of one layer-row block each
+    per_step = max(0.5, min(5.0, 60.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        oracle_sample(args.workload, per_step / 4, seed=args.seed)
+    ops = secs = 0.0
+    layers_done = 0
+    threads = 1
+    rows = 32
+    for k in range(args.steps):
+        o, s, d, rows, threads = oracle_sample(args.workload, per_step, seed=args.seed + k)
+        ops += o
+        secs += s
+        layers_done += d
+    value = ops / secs / 1e12
+    sample = (f"{rows} token rows x the first layers of the {WORKLOAD_NAMES[args.workload]} inventory per step "
+              f"({layers_done} layer calls in {args.steps} steps, ~{per_step:.1f} s each); act quant + int32 "
+              f"contraction + fp32 epilogue")
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": secs * 1e3 / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+            "config": {"workload": WORKLOAD_NAMES[args.workload], "sample": "bounded CPU sample"},
+            "impl": "reference",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------- main --
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+
+    from paper_2608_03057_gb300 import tasq, workloads
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    peaks = load_peaks()
+
+    step = Step(torch, tasq, workloads, args.workload, args.seed, args.blocks)
+    S = step.S
+    stage_of = lambda k: k % S
+
+    # eager warm-up (first launches set kernel attributes), then capture
+    for k in range(2):
+        step.d_stage.fill_(stage_of(k))
+        step.launch()
+    torch.cuda.synchronize()
+    assert tasq.tasq_device_status(step.ctx) == tasq.TASQ_OK
+    external = True
+    try:
+        events = make_events(torch, len(step.layers), True)
+        g = capture(torch, step, events)
+    except (TypeError, RuntimeError):
+        external = False
+        events = None
+        g = capture(torch, step, None)
+    for k in range(args.warmup):
+        step.d_stage.fill_(stage_of(k))
+        g.replay()
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    if rank == 0:
+        clocks.start()
+    if dist:
+        dist.barrier()
+    ms = timed_replays(torch, g, step, args.steps, stage_of)
+    clk = clocks.stop() if rank == 0 else None
+    status = tasq.tasq_device_status(step.ctx)
+    if status != tasq.TASQ_OK:
+        raise SystemExit(f"device status {status} after the timed region")
+
+    # per-kernel durations of the last timed replay
+    if external:
+        gemm_ms = [events[i][0].elapsed_time(events[i][1]) for i in range(len(step.layers))]
+    else:  # eager pass with events around each contraction
+        events = make_events(torch, len(step.layers), False)
+        step.d_stage.fill_(stage_of(args.steps - 1))
+        step.launch(events)
+        torch.cuda.synchronize()
+        gemm_ms = [events[i][0].elapsed_time(events[i][1]) for i in range(len(step.layers))]
+
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * step.ops / (ms * 1e-3) / 1e12
+
+    # the all-8-bit schedule on the same captured graph (same table buffer)
+    L = len(step.layers)
+    ms8 = None
+    if not args.no_all8:
+        tasq.tasq_set_schedule(step.ctx, workloads.schedule_constant(L, S, 8), L, S)
+        ms8 = timed_replays(torch, g, step, max(10, args.steps // 2), stage_of)
+        tasq.tasq_set_schedule(step.ctx, step.table, L, S)
+
+    # end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e:
+        xh = [x.cpu().pin_memory() for x in step.x]
+        yh = [torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for y in step.y]
+        s = torch.cuda.current_stream()
+        def e2e_step():
+            for i in range(L):
+                step.x[i].copy_(xh[i], non_blocking=True)
+            step.launch()
+            for i in range(L):
+                yh[i].copy_(step.y[i], non_blocking=True)
+        e2e_step()
+        torch.cuda.synchronize()
+        ge = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(ge, capture_error_mode="thread_local"):
+            e2e_step()
+        n_e2e = max(5, args.steps // 10)
+        ms_e2e = timed_replays(torch, ge, step, n_e2e, stage_of)
+        if dist:
+            t = torch.tensor([ms_e2e], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms_e2e = float(t.item())
+        e2e = {"value": world * step.ops / (ms_e2e * 1e-3) / 1e12, "unit": UNIT,
+               "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in xh)),
+               "d2h_bytes_per_step": int(sum(y.numel() * y.element_size() for y in yh)),
+               "ms_per_step": ms_e2e}
+        del xh, yh, ge
+
+    gemm_total_ms = sum(gemm_ms)
+    achieved = step.ops / (gemm_total_ms * 1e-3) / 1e12
+    peak = peaks["bf16_sus"]
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": None, "kernel": "gemm_tc_kernel",
+                "peak_source": f"{peaks['src']} bf16 sustained (fp16 MMA runs at the bf16 rate)",
+                "timing": "CUDA events around each contraction in the last timed replay" if external
+                else "CUDA events around each contraction in an eager pass after the timed region"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        o, s, d, rows, threads = oracle_sample(args.workload, args.cpu_seconds, seed=args.seed)
+        cpu = {"value": o / s / 1e12, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"{rows} token rows of each of the first {d} layers of the step ({s:.1f} s)"}
+
+    if rank == 0:
+        bits = step.table.astype(np.float64)
+        ops_w = np.array(step.gemm_ops, np.float64)
+        eff_w = float((bits * ops_w[:, None]).sum() / (ops_w.sum() * S))
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f16-exact-int8", "data": "synthetic",
+            "config": {"workload": WORKLOAD_NAMES[args.workload], "layers": L, "stages": S,
+                       "schedule": "seeded learned-style per-(layer, stage) bits", "effective_w_bits": eff_w,
+                       "rel_bitops": eff_w * 8 / 64, "route": "tcgen05 fp16 MMA, exact int32",
+                       "activations": "bf16 in HBM, per-token int8 codes held as fp16",
+                       "l2": "inputs larger than L2 (per-step activations and weights exceed 129 MB)",
+                       "graph": "whole step captured once; stage from a device int",
+                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+            "ms_per_step_all8": ms8,
+            "roofline": roofline,
+            "roofline_quant_act": {"bound": "hbm", "bytes_per_step": step.act_bytes(),
+                                   "note": "quantization kernels share the step with the contractions"},
+            "e2e": e2e,
+            "gpu_launches": step.launches_per_step() * args.steps,
+            "cpu_baseline": cpu,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    step.close()
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

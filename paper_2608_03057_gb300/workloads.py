@@ -61,6 +61,18 @@ def uniform(shape, seed: int, lo: float, hi: float) -> np.ndarray:
     return rng(seed).uniform(lo, hi, size=shape).astype(np.float32)
 
 
+def device_normal(shape, seed: int, std: float = 1.0, dtype=None, device="cuda"):
+    """N(0, std^2) drawn on the GPU with torch's seeded Philox generator (for
+    benchmark-sized tensors that would take too long to draw on the host)."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    t = torch.randn(shape, generator=g, device=device, dtype=torch.float32)
+    if std != 1.0:
+        t.mul_(std)
+    return t if dtype is None else t.to(dtype)
+
+
 # ----------------------------------------------------------------------------
 # Layer inventories
 # ----------------------------------------------------------------------------
@@ -127,7 +139,7 @@ def sdxl_turbo() -> List[Layer]:
     out: List[Layer] = []
     # down 320 @ 64x64: conv_in + 2 resnets (2 convs each) + downsample
     out += [_conv(f"down0.conv{i}", 320, 64, 64) for i in range(5)]
-    # down 640 @ 32x32: 2 resnets with 1 transformer block each... 2 blocks/resnet
+    # down 640 @ 32x32: 2 resnets with 2 transformer blocks each
     out += [_conv(f"down1.conv{i}", 640, 32, 32) for i in range(5)]
     for r in range(2):
         for t in range(2):
@@ -196,6 +208,15 @@ def schedule_for(config: str, L: int, seed: int = 7) -> np.ndarray:
     if config == "sweep":
         return np.array([[2, 3, 4, 5, 6, 7, 8, 8]], np.uint8)
     raise KeyError(config)
+
+
+def inventory_blocks(config: str, blocks: int) -> List[Layer]:
+    """The first `blocks` transformer blocks of a DiT inventory (small cases)."""
+    if config == "pixart":
+        return pixart_sigma(blocks=blocks)
+    if config == "sana":
+        return sana_1600m(blocks=blocks)
+    return inventory(config)
 
 
 def inventory(config: str) -> List[Layer]:
