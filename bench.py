@@ -170,6 +170,8 @@ class Step:
         t = self.tasq
         for i, l in enumerate(self.layers):
             if l.kind == self.conv:
+                if events:
+                    events[i][2].record()
                 t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.Cin, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TENSOR,
                                  self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
                 if events:
@@ -177,6 +179,8 @@ class Step:
                 t.tasq_masked_conv3x3(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B, l.H,
                                       l.W, l.Cin, self.packed[i], l.N, self.y[i], None)
             else:
+                if events:
+                    events[i][2].record()
                 t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.K, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TOKEN,
                                  self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
                 if events:
@@ -211,7 +215,7 @@ def make_events(torch, n, external):
     kw = dict(enable_timing=True)
     if external:
         kw["external"] = True
-    return [(torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(n)]
+    return [(torch.cuda.Event(**kw), torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(n)]
 
 
 def capture(torch, step, events=None):
@@ -337,14 +341,17 @@ def main():
         step.launch()
     torch.cuda.synchronize()
     assert tasq.tasq_device_status(step.ctx) == tasq.TASQ_OK
+    # the timed graph holds only the kernels (event nodes between kernels would
+    # block programmatic dependent launch); a second capture of the same launch
+    # sequence with an event around every kernel gives per-kernel durations
+    g = capture(torch, step, None)
     external = True
     try:
         events = make_events(torch, len(step.layers), True)
-        g = capture(torch, step, events)
+        g_ev = capture(torch, step, events)
     except (TypeError, RuntimeError):
         external = False
         events = None
-        g = capture(torch, step, None)
     for k in range(args.warmup):
         step.d_stage.fill_(stage_of(k))
         g.replay()
@@ -362,14 +369,18 @@ def main():
         raise SystemExit(f"device status {status} after the timed region")
 
     # per-kernel durations of the last timed replay
-    if external:
-        gemm_ms = [events[i][0].elapsed_time(events[i][1]) for i in range(len(step.layers))]
-    else:  # eager pass with events around each contraction
+    if external:  # instrumented replays right after the timed region
+        for k in range(3):
+            step.d_stage.fill_(stage_of(args.steps + k))
+            g_ev.replay()
+        torch.cuda.synchronize()
+    else:  # eager pass with events around each kernel
         events = make_events(torch, len(step.layers), False)
         step.d_stage.fill_(stage_of(args.steps - 1))
         step.launch(events)
         torch.cuda.synchronize()
-        gemm_ms = [events[i][0].elapsed_time(events[i][1]) for i in range(len(step.layers))]
+    gemm_ms = [events[i][0].elapsed_time(events[i][1]) for i in range(len(step.layers))]
+    quant_ms = [events[i][2].elapsed_time(events[i][0]) for i in range(len(step.layers))]
 
     if dist:
         t = torch.tensor([ms], device="cuda")
@@ -420,7 +431,8 @@ def main():
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "traffic": None, "kernel": "gemm_tc_kernel",
                 "peak_source": f"{peaks['src']} bf16 sustained (fp16 MMA runs at the bf16 rate)",
-                "timing": "CUDA events around each contraction in the last timed replay" if external
+                "timing": "CUDA events around each contraction in a replay of the step with event nodes "
+                          "between kernels, right after the timed region" if external
                 else "CUDA events around each contraction in an eager pass after the timed region"}
 
     cpu = None
@@ -447,7 +459,15 @@ def main():
             "ms_per_step_all8": ms8,
             "roofline": roofline,
             "roofline_quant_act": {"bound": "hbm", "bytes_per_step": step.act_bytes(),
-                                   "note": "quantization kernels share the step with the contractions"},
+                                   "achieved": step.act_bytes() / (sum(quant_ms) * 1e-3) / 1e9,
+                                   "peak": peaks["hbm"], "unit": "GB/s",
+                                   "frac": step.act_bytes() / (sum(quant_ms) * 1e-3) / 1e9 / peaks["hbm"],
+                                   "ms_per_step": sum(quant_ms)},
+            "step_breakdown_ms": {"contractions": sum(gemm_ms), "act_quant": sum(quant_ms),
+                                  "timed_step": ms,
+                                  "note": "per-kernel sums come from the instrumented replay, where kernels "
+                                          "cannot overlap; the timed step lets each launch overlap the "
+                                          "previous kernel's tail"},
             "e2e": e2e,
             "gpu_launches": step.launches_per_step() * args.steps,
             "cpu_baseline": cpu,

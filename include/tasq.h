@@ -31,9 +31,12 @@
  *    that ran past its time limit) are recorded in a device status word that
  *    tasq_device_status() reads; the kernel then returns early without
  *    trapping, and the CUDA context stays usable.
- *  - A context may be used from one host thread at a time.  Per-tensor
- *    activation quantization uses a small per-context reduction scratch, so
- *    two such calls on different streams of one context must not overlap.
+ *  - A context may be used from one host thread at a time.  Two kinds of
+ *    call use per-context device scratch: per-tensor activation quantization
+ *    (a 16-byte reduction) and tensor-core contractions whose certificate
+ *    splits K into several chunks (int32 running sums, 96 KB per SM).  Calls
+ *    of either kind on different streams of one context must not overlap;
+ *    use one context per concurrent stream.
  *
  * Data layouts: row-major, innermost index last.  Activations of a linear
  * layer are [M][K] (M tokens); of a conv, NHWC [B][H][W][Cin].  Weights are
@@ -87,7 +90,8 @@ typedef void* tasq_stream; /* cudaStream_t */
 int tasq_version(void);
 
 /* Create a context on CUDA device `device`.  Set-up call: allocates the
- * context's device status word and reduction scratch (a few bytes) and
+ * context's device status word, its reduction scratch and the tensor-core
+ * route's accumulator scratch (96 KB per SM: about 14.6 MB on a GB300), and
  * leaves the calling thread's current device unchanged.  *out is NULL on
  * failure. */
 int tasq_create(tasq_ctx* out, int device);
@@ -118,6 +122,15 @@ int tasq_set_timeout_ns(tasq_ctx ctx, uint64_t ns);
  * records TASQ_ERR_DEVICE_TIMEOUT in the device status and the kernel
  * returns, leaving the context usable.  Enqueue call. */
 int tasq_selftest_timeout(tasq_ctx ctx, uint64_t timeout_ns, tasq_stream stream);
+
+/* Arithmetic self test of the activation quantizer: the quantizer divides
+ * x / alpha with a reciprocal computed once per group followed by two exact
+ * remainder corrections (Markstein's method) instead of a hardware division
+ * per element.  For every pair (d_x[i], d_a[j]), i < nx, j < na, this adds 1
+ * to *d_mismatches (caller-zeroed uint64 on the device) when that quotient's
+ * bit pattern differs from IEEE round-to-nearest division.  Enqueue call. */
+int tasq_selftest_quotients(tasq_ctx ctx, const float* d_x, int nx, const float* d_a, int na,
+                            unsigned long long* d_mismatches, tasq_stream stream);
 
 /*
  * Weight quantization, App. A.1.1 (Eqs. weight_quant, weight_scale,

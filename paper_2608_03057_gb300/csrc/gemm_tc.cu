@@ -30,34 +30,57 @@
 // bounded by the context's time limit; a wait that gives up records
 // TASQ_ERR_DEVICE_TIMEOUT, the CTA drains its copies in flight, frees its
 // tensor memory and returns.
+#include <cstdio>
+
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cudaTypedefs.h>
 
 #include "tasq_internal.cuh"
 #include "tc_ptx.cuh"
 
+// Optional per-role timestamps of CTA 0 (build with -DTASQ_TRACE; compiled
+// out otherwise): role 0 producer, 1 MMA, 2 converter warp, 3 epilogue warp.
+#ifdef TASQ_TRACE
+__device__ unsigned long long g_tasq_trace[4][256][8];
+#define TQ(role, it, k)                                                          \
+    do {                                                                         \
+        if (blockIdx.x == 0 && (it) < 256) g_tasq_trace[role][it][k] = clock64(); \
+    } while (0)
+#else
+#define TQ(role, it, k) \
+    do {                \
+    } while (0)
+#endif
+
 namespace tasq {
 namespace {
 
-constexpr int BCH = 128;         // output channels per tile (MMA M)
-constexpr int BTOK = 128;        // tokens / output pixels per tile (MMA N)
-constexpr int BK = 64;           // K per pipeline stage
-constexpr int STAGES = 6;        // shared-memory stages
-constexpr int ASLOTS = 4;        // tensor-memory slots of converted weights
-constexpr int THREADS = 320;
-constexpr int X_STAGE = BTOK * BK * 2;  // 16 KB fp16 codes
-constexpr int W_STAGE = BCH * BK;       // 8 KB int8 codes
+constexpr int BCH = 128;          // output channels per tile (MMA M)
+constexpr int BTOK = 192;         // tokens / output pixels per tile (MMA N)
+constexpr int BK = 128;           // K per pipeline stage (two 64-wide swizzle atoms)
+constexpr int STAGES = 3;         // shared-memory stages
+constexpr int ASLOTS = 2;         // tensor-memory slots of converted weights
+constexpr int EPI_WARPS = 12;     // three per tensor-memory lane quadrant
+constexpr int THREADS = (6 + EPI_WARPS) * 32;
+constexpr int X_HALF = BTOK * 64 * 2;   // 24 KB: one 64-wide K atom of fp16 codes
+constexpr int X_STAGE = 2 * X_HALF;     // 48 KB
+constexpr int W_STAGE = BCH * BK;       // 16 KB int8 codes, 128-byte rows
+constexpr int GROUPS = BTOK / 32;       // 32-token column groups of the accumulator
+static_assert(GROUPS == 2 * EPI_WARPS / 4, "each epilogue warp drains two groups");
 // tensor memory columns
-constexpr uint32_t ACC_COL = 0;                         // 2 x BTOK fp32 accumulators
-constexpr uint32_t A_COL = 2 * BTOK;                    // ASLOTS x 32 (64 fp16 per row)
-constexpr uint32_t SUM_COL = A_COL + ASLOTS * (BK / 2);  // BTOK int32 running sums
+constexpr uint32_t ACC_COL = 0;           // 2 x BTOK fp32 accumulators
+constexpr uint32_t A_COL = 2 * BTOK;      // ASLOTS x 64 columns (128 fp16 per row)
+constexpr uint32_t A_SLOT_COLS = BK / 2;
 constexpr uint32_t TMEM_COLS = 512;
-static_assert(SUM_COL + BTOK <= TMEM_COLS, "tensor memory budget");
+static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
 constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BTOK);
 
 struct Smem {
     uint8_t x[STAGES][X_STAGE];  // 1024-aligned (128B swizzle atoms)
     uint8_t w[STAGES][W_STAGE];
+    float ep_al[EPI_WARPS][32], ep_zc[EPI_WARPS][32];
+    int ep_tok[EPI_WARPS][32], ep_tap[EPI_WARPS][32];
     uint64_t full[STAGES], empty[STAGES];
     uint64_t afull[ASLOTS], aempty[ASLOTS];
     uint64_t accfull[2], accempty[2];
@@ -71,7 +94,7 @@ struct TcParams {
     GemmArgs a;
     int conv;
     int tiles_ch, tiles_tok;
-    int bw, bh, tiles_w, tiles_h;  // conv: token tile = bh x bw pixel rectangle
+    int bw_log2, bh, tiles_w, tiles_h;  // conv: token tile = bh x 2^bw_log2 pixel rectangle
 };
 
 struct Waiter {
@@ -97,6 +120,19 @@ struct Waiter {
     }
 };
 
+// Ring position: slot index and phase parity, advanced without divisions.
+template <int N>
+struct Ring {
+    int slot = 0;
+    uint32_t phase = 0;
+    __device__ __forceinline__ void next() {
+        if (++slot == N) {
+            slot = 0;
+            phase ^= 1u;
+        }
+    }
+};
+
 // fp16 bit patterns of four masked codes: (w & m) ^ 0x80 per byte gives the
 // unsigned code u = v + 128; 0x64uu is the fp16 value 1024 + u; subtracting
 // 1152 leaves v exactly.
@@ -111,7 +147,27 @@ __device__ __forceinline__ void widen4(uint32_t w, uint32_t m, uint32_t& lo, uin
     hi = *reinterpret_cast<uint32_t*>(&h);
 }
 
-__global__ void __launch_bounds__(THREADS, 1)
+struct TileCoord {
+    int ch0, tok0, img, h0, w0;
+};
+
+__device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
+    TileCoord c;
+    c.ch0 = (t % p.tiles_ch) * BCH;
+    const int tt = t / p.tiles_ch;
+    c.tok0 = c.img = c.h0 = c.w0 = 0;
+    if (p.conv) {
+        const int per_img = p.tiles_h * p.tiles_w;
+        c.img = tt / per_img;
+        c.h0 = ((tt % per_img) / p.tiles_w) * p.bh;
+        c.w0 = (tt % p.tiles_w) << p.bw_log2;
+    } else {
+        c.tok0 = tt * BTOK;
+    }
+    return c;
+}
+
+__global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w) {
     extern __shared__ uint8_t smem_raw[];
@@ -123,7 +179,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int b = resolve_bits(a);
     if (b == 0) return;  // uniform across the CTA: nothing allocated yet
     const int KT = (a.K + BK - 1) / BK;
-    int chunk = a.hdr->chunk_kb[b];
+    // certificate is in 64-wide K blocks; a run of c64 of them covers c64/2 of ours
+    int chunk = a.hdr->chunk_kb[b] / (BK / kCertKBlock);
     chunk = chunk < 1 ? 1 : (chunk > KT ? KT : chunk);
     const int nchunks = (KT + chunk - 1) / chunk;
     const int tiles = p.tiles_ch * p.tiles_tok;
@@ -139,7 +196,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(ptx::smem_u32(&s->accfull[i]), 1);
-            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), 4);
+            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS);
         }
         ptx::mbar_init(ptx::smem_u32(&s->drain), 1);
         s->abort = 0;
@@ -155,50 +212,56 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem_base;
+    // the prologue above overlaps the previous kernel; inputs are read only after it
+    ptx::grid_dependency_wait();
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
         if (lane == 0) {
+            Ring<STAGES> rs;
             int it = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-                const int ch0 = (t % p.tiles_ch) * BCH;
-                const int tt = t / p.tiles_ch;
-                int tok0 = 0, img = 0, h0 = 0, w0 = 0;
-                if (p.conv) {
-                    const int per_img = p.tiles_h * p.tiles_w;
-                    img = tt / per_img;
-                    h0 = ((tt % per_img) / p.tiles_w) * p.bh;
-                    w0 = (tt % p.tiles_w) * p.bw;
-                } else {
-                    tok0 = tt * BTOK;
-                }
-                for (int kb = 0; kb < KT; ++kb, ++it) {
-                    const int st = it % STAGES;
-                    if (!wt.wait(&s->empty[st], ((it / STAGES) & 1) ^ 1)) {
+                const TileCoord tc = tile_coord(p, t);
+                for (int kb = 0; kb < KT; ++kb, ++it, rs.next()) {
+                    TQ(0, it, 0);
+                    if (!wt.wait(&s->empty[rs.slot], rs.phase ^ 1)) {
                         ok = false;
                         break;
                     }
-                    const uint32_t fb = ptx::smem_u32(&s->full[st]);
+                    TQ(0, it, 1);
+                    const uint32_t fb = ptx::smem_u32(&s->full[rs.slot]);
                     ptx::mbar_arrive_expect_tx(fb, X_STAGE + W_STAGE);
+                    const uint32_t xdst = ptx::smem_u32(s->x[rs.slot]);
                     const int k0 = kb * BK;
-                    if (p.conv) {
-                        const int tap = k0 / a.Cin, c0 = k0 - tap * a.Cin;
-                        ptx::tma_load_4d(ptx::smem_u32(s->x[st]), &tm_x, fb, c0, w0 + tap % 3 - 1, h0 + tap / 3 - 1,
-                                         img);
-                    } else {
-                        ptx::tma_load_2d(ptx::smem_u32(s->x[st]), &tm_x, fb, k0, tok0);
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh) {
+                        const int kh = k0 + 64 * hh;
+                        if (p.conv) {
+                            // a 128-wide K block may straddle two taps when Cin % 128 == 64
+                            const int tap = kh / a.Cin, c0 = kh - tap * a.Cin;
+                            ptx::tma_load_4d(xdst + hh * X_HALF, &tm_x, fb, c0, tc.w0 + tap % 3 - 1,
+                                             tc.h0 + tap / 3 - 1, tc.img);
+                        } else {
+                            ptx::tma_load_2d(xdst + hh * X_HALF, &tm_x, fb, kh, tc.tok0);
+                        }
                     }
-                    ptx::tma_load_2d(ptx::smem_u32(s->w[st]), &tm_w, fb, k0, ch0);
+                    ptx::tma_load_2d(ptx::smem_u32(s->w[rs.slot]), &tm_w, fb, k0, tc.ch0);
                 }
             }
             // copies still in flight must land before the CTA may exit
-            const int first = it > STAGES ? it - STAGES : 0;
-            for (int j = first; j < it; ++j) wt.wait(&s->full[j % STAGES], (j / STAGES) & 1, true);
+            for (int j = 0; j < STAGES && j < it; ++j) {
+                // the last STAGES stages issued, oldest first
+                const int jj = it - STAGES + j;
+                if (jj < 0) continue;
+                wt.wait(&s->full[jj % STAGES], (jj / STAGES) & 1, true);
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
         if (lane == 0) {
+            Ring<STAGES> rs;
+            Ring<ASLOTS> ra;
             int it = 0, cc = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
@@ -210,26 +273,36 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
                     ptx::tc_fence_after();
                     const uint32_t d = tmem + ACC_COL + buf * BTOK;
-                    const int kb_end = min(KT, (c + 1) * chunk);
-                    for (int kb = c * chunk; kb < kb_end; ++kb, ++it) {
-                        const int st = it % STAGES, sl = it % ASLOTS;
-                        if (!wt.wait(&s->full[st], (it / STAGES) & 1) ||
-                            !wt.wait(&s->afull[sl], (it / ASLOTS) & 1)) {
+                    const int kb0 = c * chunk, kb_end = min(KT, kb0 + chunk);
+                    for (int kb = kb0; kb < kb_end; ++kb, ++it, rs.next(), ra.next()) {
+                        TQ(1, it, 0);
+                        if (!wt.wait(&s->full[rs.slot], rs.phase)) {
                             ok = false;
                             break;
                         }
+                        TQ(1, it, 1);
+                        if (!wt.wait(&s->afull[ra.slot], ra.phase)) {
+                            ok = false;
+                            break;
+                        }
+                        TQ(1, it, 2);
                         ptx::tc_fence_after();
-                        const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[st]));
+                        const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[rs.slot]));
+                        const uint32_t acol = tmem + A_COL + ra.slot * A_SLOT_COLS;
 #pragma unroll
                         for (int k = 0; k < BK / 16; ++k)
-                            ptx::mma_f16_ts(d, tmem + A_COL + sl * (BK / 2) + k * 8, bdesc + uint64_t((k * 32) >> 4),
-                                            IDESC, (kb > c * chunk || k > 0) ? 1u : 0u);
-                        ptx::mma_commit(ptx::smem_u32(&s->empty[st]));
-                        ptx::mma_commit(ptx::smem_u32(&s->aempty[sl]));
+                            ptx::mma_f16_ts(d, acol + k * 8,
+                                            bdesc + uint64_t(((k >> 2) * X_HALF + (k & 3) * 32) >> 4), IDESC,
+                                            (kb > kb0 || k > 0) ? 1u : 0u);
+                        ptx::mma_commit(ptx::smem_u32(&s->empty[rs.slot]));
+                        ptx::mma_commit(ptx::smem_u32(&s->aempty[ra.slot]));
+                        TQ(1, it, 3);
                     }
                     if (ok) ptx::mma_commit(ptx::smem_u32(&s->accfull[buf]));
                 }
             }
+            // the next kernel may be launched while the last epilogue runs
+            ptx::grid_launch_dependents();
             // every MMA issued must finish before tensor memory is released
             ptx::mma_commit(ptx::smem_u32(&s->drain));
             wt.wait(&s->drain, 0, true);
@@ -240,54 +313,71 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int r = q * 32 + lane;        // channel row within the tile
         const uint32_t m = mask_word(b);
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
+        Ring<STAGES> rs;
+        Ring<ASLOTS> ra;
         int it = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-            for (int kb = 0; kb < KT; ++kb, ++it) {
-                const int st = it % STAGES, sl = it % ASLOTS;
-                if (!wt.wait(&s->full[st], (it / STAGES) & 1)) {
+            for (int kb = 0; kb < KT; ++kb, ++it, rs.next(), ra.next()) {
+                if (warp == 2 && lane == 0) TQ(2, it, 0);
+                if (!wt.wait(&s->full[rs.slot], rs.phase)) {
                     ok = false;
                     break;
                 }
-                // 64 codes of row r; 16-byte chunk c sits at c ^ ((r >> 1) & 3) (64-byte swizzle)
-                uint4 v[4];
-                const uint8_t* row = s->w[st] + r * BK;
+                if (warp == 2 && lane == 0) TQ(2, it, 1);
+                // 128 codes of row r; 16-byte chunk c sits at c ^ (r & 7) (128-byte swizzle)
+                uint4 v[8];
+                const uint8_t* row = s->w[rs.slot] + r * BK;
 #pragma unroll
-                for (int c = 0; c < 4; ++c) v[c] = *reinterpret_cast<const uint4*>(row + ((c ^ ((r >> 1) & 3)) << 4));
+                for (int c = 0; c < 8; ++c) v[c] = *reinterpret_cast<const uint4*>(row + ((c ^ (r & 7)) << 4));
                 __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->empty[st]));
-                if (!wt.wait(&s->aempty[sl], ((it / ASLOTS) & 1) ^ 1)) {
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->empty[rs.slot]));
+                if (warp == 2 && lane == 0) TQ(2, it, 2);
+                if (!wt.wait(&s->aempty[ra.slot], ra.phase ^ 1)) {
                     ok = false;
                     break;
                 }
-                uint32_t f[32];
+                if (warp == 2 && lane == 0) TQ(2, it, 3);
+                const uint32_t dst = lane_base + A_COL + ra.slot * A_SLOT_COLS;
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    widen4(v[c].x, m, f[8 * c + 0], f[8 * c + 1]);
-                    widen4(v[c].y, m, f[8 * c + 2], f[8 * c + 3]);
-                    widen4(v[c].z, m, f[8 * c + 4], f[8 * c + 5]);
-                    widen4(v[c].w, m, f[8 * c + 6], f[8 * c + 7]);
+                for (int hh = 0; hh < 2; ++hh) {
+                    uint32_t f[32];
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        const uint4 u = v[4 * hh + c];
+                        widen4(u.x, m, f[8 * c + 0], f[8 * c + 1]);
+                        widen4(u.y, m, f[8 * c + 2], f[8 * c + 3]);
+                        widen4(u.z, m, f[8 * c + 4], f[8 * c + 5]);
+                        widen4(u.w, m, f[8 * c + 6], f[8 * c + 7]);
+                    }
+                    ptx::tmem_st32(dst + hh * 32, f);
                 }
-                ptx::tmem_st32(lane_base + A_COL + sl * (BK / 2), f);
+                if (warp == 2 && lane == 0) TQ(2, it, 4);
                 ptx::tmem_wait_st();
+                if (warp == 2 && lane == 0) TQ(2, it, 5);
                 ptx::tc_fence_before();
                 __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->afull[sl]));
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->afull[ra.slot]));
             }
         }
     } else {
         // ------------------------------------- accumulator drain + epilogue
-        const int q = warp & 3;
+        const int e = warp - 6;              // 0..EPI_WARPS-1
+        const int q = warp & 3;              // lane quadrant: channels q*32 .. q*32+31
+        const int part = e >> 2;             // which pair of 32-token groups
         const int r = q * 32 + lane;
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
         const int32_t* ts_b = p.conv ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
+        float* my_al = s->ep_al[e];
+        float* my_zc = s->ep_zc[e];
+        int* my_tok = s->ep_tok[e];
+        int* my_tap = s->ep_tap[e];
         int cc = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-            const int ch0 = (t % p.tiles_ch) * BCH;
-            const int tt = t / p.tiles_ch;
-            const int n = ch0 + r;
+            const TileCoord tc = tile_coord(p, t);
+            const int n = tc.ch0 + r;
             const bool n_ok = n < a.N;
             float cw = 0.f, bias = 0.f;
             int rs = 0;
@@ -304,80 +394,147 @@ __global__ void __launch_bounds__(THREADS, 1)
                     rs = rs_b[n];
                 }
             }
-            int img = 0, h0 = 0, w0 = 0, tok0 = 0;
-            if (p.conv) {
-                const int per_img = p.tiles_h * p.tiles_w;
-                img = tt / per_img;
-                h0 = ((tt % per_img) / p.tiles_w) * p.bh;
-                w0 = (tt % p.tiles_w) * p.bw;
-            } else {
-                tok0 = tt * BTOK;
+
+            // Token index, (conv) in-bounds taps and per-token scales of column j = lane of
+            // each of this warp's two groups, fetched before the accumulator is ready so
+            // the loads' latency hides under the MMAs.
+            int tok_r[2], tap_r[2];
+            float al_r[2], zc_r[2];
+#pragma unroll
+            for (int gi = 0; gi < 2; ++gi) {
+                const int jt = (2 * part + gi) * 32 + lane;
+                int tok = -1, tap = 0;
+                if (p.conv) {
+                    const int hh = tc.h0 + (jt >> p.bw_log2), ww = tc.w0 + (jt & ((1 << p.bw_log2) - 1));
+                    if (hh < a.H && ww < a.W) {
+                        tok = (tc.img * a.H + hh) * a.W + ww;
+#pragma unroll
+                        for (int dh = 0; dh < 3; ++dh)
+#pragma unroll
+                            for (int dw = 0; dw < 3; ++dw) {
+                                const int ih = hh + dh - 1, iw = ww + dw - 1;
+                                if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W) tap |= 1 << (dh * 3 + dw);
+                            }
+                    }
+                } else {
+                    tok = tc.tok0 + jt < a.M ? tc.tok0 + jt : -1;
+                }
+                tok_r[gi] = tok;
+                tap_r[gi] = tap;
+                al_r[gi] = tok >= 0 ? (a.per_tensor ? a.alpha[0] : a.alpha[tok]) : 0.f;
+                zc_r[gi] = tok >= 0 ? (a.per_tensor ? a.zc[0] : a.zc[tok]) : 0.f;
             }
+            // stage group gi's per-token values in this warp's scratch for broadcast reads
+            auto stage_tokens = [&](int gi) -> bool {
+                __syncwarp();
+                my_tok[lane] = tok_r[gi];
+                my_tap[lane] = tap_r[gi];
+                my_al[lane] = al_r[gi];
+                my_zc[lane] = zc_r[gi];
+                __syncwarp();
+                return __all_sync(0xffffffffu, tok_r[gi] >= 0);
+            };
+            // Epilogue of 16 consecutive columns j0..j0+15 of group g from exact
+            // accumulator values (float-held integers when `fl`, else int32).
+            auto finish16 = [&](int g, int j0, const uint32_t (&v)[16], bool fl, bool all_tok) {
+                uint32_t yb2[8];
+#pragma unroll
+                for (int j4 = 0; j4 < 4; ++j4) {
+                    const float4 al4 = *reinterpret_cast<const float4*>(my_al + j0 + 4 * j4);
+                    const float4 zc4 = *reinterpret_cast<const float4*>(my_zc + j0 + 4 * j4);
+                    const float al[4] = {al4.x, al4.y, al4.z, al4.w};
+                    const float zc[4] = {zc4.x, zc4.y, zc4.z, zc4.w};
+                    int4 tp4 = make_int4(0, 0, 0, 0);
+                    if (p.conv) tp4 = *reinterpret_cast<const int4*>(my_tap + j0 + 4 * j4);
+                    const int tp[4] = {tp4.x, tp4.y, tp4.z, tp4.w};
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        int rsum = rs;
+                        if (p.conv) {
+                            rsum = 0;
+#pragma unroll
+                            for (int k9 = 0; k9 < 9; ++k9) rsum += (tp[u] >> k9) & 1 ? ts[k9] : 0;
+                        }
+                        const uint32_t raw = v[4 * j4 + u];
+                        const float acc_f = fl ? __uint_as_float(raw) : __int2float_rn(int(raw));
+                        const float tz = __fmul_rn(zc[u], __int2float_rn(rsum));
+                        const float y = __fadd_rn(__fmul_rn(__fadd_rn(acc_f, tz), __fmul_rn(al[u], cw)), bias);
+                        const uint32_t h = __bfloat16_as_ushort(__float2bfloat16_rn(y));
+                        const int jj = 4 * j4 + u;
+                        yb2[jj >> 1] = (jj & 1) ? (yb2[jj >> 1] | (h << 16)) : h;
+                    }
+                }
+                if (!n_ok) return;
+                if (!p.conv && all_tok) {
+                    const int64_t row0 = int64_t(tc.tok0 + g * 32 + j0);
+                    uint16_t* yp = a.y + row0 * a.N + n;
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) yp[int64_t(j) * a.N] = uint16_t(yb2[j >> 1] >> (16 * (j & 1)));
+                    if (a.acc) {
+                        int32_t* ap = a.acc + row0 * a.N + n;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            ap[int64_t(j) * a.N] = fl ? __float2int_rn(__uint_as_float(v[j])) : int(v[j]);
+                    }
+                } else {
+#pragma unroll
+                    for (int j4 = 0; j4 < 4; ++j4) {
+                        const int4 tk = *reinterpret_cast<const int4*>(my_tok + j0 + 4 * j4);
+                        const int tks[4] = {tk.x, tk.y, tk.z, tk.w};
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            if (tks[u] < 0) continue;
+                            const int jj = 4 * j4 + u;
+                            a.y[int64_t(tks[u]) * a.N + n] = uint16_t(yb2[jj >> 1] >> (16 * (jj & 1)));
+                            if (a.acc)
+                                a.acc[int64_t(tks[u]) * a.N + n] =
+                                    fl ? __float2int_rn(__uint_as_float(v[jj])) : int(v[jj]);
+                        }
+                    }
+                }
+            };
+
+            // Multi-chunk tiles keep their int32 running sums in this warp's slice of the
+            // per-CTA scratch (32 channels x 64 tokens); each value is only re-read by
+            // the thread that wrote it.
+            int32_t* my_part = a.part + (int64_t(blockIdx.x) * EPI_WARPS + e) * (64 * 32) + lane;
             for (int c = 0; c < nchunks; ++c, ++cc) {
                 const int buf = cc & 1;
+                if (warp == 6 && lane == 0) TQ(3, cc, 0);
                 if (!wt.wait(&s->accfull[buf], (cc >> 1) & 1)) {
                     ok = false;
                     break;
                 }
+                if (warp == 6 && lane == 0) TQ(3, cc, 1);
                 ptx::tc_fence_after();
+                const uint32_t acc_base = lane_base + ACC_COL + buf * BTOK;
                 const bool last = c == nchunks - 1;
 #pragma unroll 1
-                for (int g = 0; g < BTOK / 32; ++g) {
-                    uint32_t v[32];
-                    ptx::tmem_ld32(lane_base + ACC_COL + buf * BTOK + g * 32, v);
-                    ptx::tmem_wait_ld();
-                    int iv[32];
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) iv[j] = __float2int_rn(__uint_as_float(v[j]));
-                    if (c > 0) {
-                        uint32_t sv[32];
-                        ptx::tmem_ld32(lane_base + SUM_COL + g * 32, sv);
+                for (int gi = 0; gi < 2; ++gi) {
+                    const int g = 2 * part + gi;
+                    const bool all_tok = last ? stage_tokens(gi) : false;
+#pragma unroll 1
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t v[16];
+                        ptx::tmem_ld16(acc_base + g * 32 + h * 16, v);
                         ptx::tmem_wait_ld();
+                        if (nchunks > 1) {
+                            int32_t* pp = my_part + (gi * 32 + h * 16) * 32;
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) iv[j] += int(sv[j]);
-                    }
-                    if (!last) {
-                        uint32_t sv[32];
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) sv[j] = uint32_t(iv[j]);
-                        ptx::tmem_st32(lane_base + SUM_COL + g * 32, sv);
-                        ptx::tmem_wait_st();
-                        continue;
-                    }
-                    // final: fused dequantization epilogue for 32 tokens of channel n
-                    int tok_lane;  // token (or output pixel) index held by this lane, -1 if none
-                    if (p.conv) {
-                        const int j = g * 32 + lane;
-                        const int h = h0 + j / p.bw, w = w0 + j % p.bw;
-                        tok_lane = (h < a.H && w < a.W) ? (img * a.H + h) * a.W + w : -1;
-                    } else {
-                        const int m = tok0 + g * 32 + lane;
-                        tok_lane = m < a.M ? m : -1;
-                    }
-                    float al_lane = 0.f, zc_lane = 0.f;
-                    if (tok_lane >= 0) {
-                        al_lane = a.per_tensor ? a.alpha[0] : a.alpha[tok_lane];
-                        zc_lane = a.per_tensor ? a.zc[0] : a.zc[tok_lane];
-                    }
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int m = __shfl_sync(0xffffffffu, tok_lane, j);
-                        const float al = __shfl_sync(0xffffffffu, al_lane, j);
-                        const float zc = __shfl_sync(0xffffffffu, zc_lane, j);
-                        if (m < 0 || !n_ok) continue;
-                        int rsum = rs;
-                        if (p.conv) {
-                            const int jj = g * 32 + j;
-                            rsum = conv_row_sum(ts, h0 + jj / p.bw, w0 + jj % p.bw, a.H, a.W);
+                            for (int j = 0; j < 16; ++j) {
+                                int x = __float2int_rn(__uint_as_float(v[j]));
+                                if (c > 0) x += pp[j * 32];
+                                if (last) v[j] = uint32_t(x);
+                                else pp[j * 32] = x;
+                            }
                         }
-                        const float y = epilogue_value(iv[j], al, zc, rsum, cw, bias);
-                        a.y[int64_t(m) * a.N + n] = bf16_bits(y);
-                        if (a.acc) a.acc[int64_t(m) * a.N + n] = iv[j];
+                        if (last) finish16(g, h * 16, v, nchunks == 1, all_tok);
                     }
                 }
                 ptx::tc_fence_before();
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->accempty[buf]));
+                if (warp == 6 && lane == 0) TQ(3, cc, 2);
             }
         }
     }
@@ -404,8 +561,14 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 
 }  // namespace
 
+size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * EPI_WARPS * 64 * 32 * sizeof(int32_t); }
+
 cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
     *why = nullptr;
+    if (!a.part) {
+        *why = "no accumulator scratch";
+        return cudaSuccess;
+    }
     if (a.M == 0 || a.N == 0) return cudaSuccess;
     auto encode = get_encode();
     if (!encode) {
@@ -419,15 +582,16 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     CUtensorMap tm_x, tm_w;
     CUresult r;
     if (p.conv) {
-        if (a.Cin % BK) {
+        if (a.Cin % 64) {
             *why = "convolution needs Cin % 64 == 0";
             return cudaSuccess;
         }
-        int bw = 1;
-        while (bw < a.W && bw < BTOK) bw <<= 1;
-        p.bw = bw;
-        p.bh = BTOK / bw;
-        p.tiles_w = (a.W + p.bw - 1) / p.bw;
+        int bwl = 0;
+        while ((1 << bwl) < a.W && (1 << bwl) < 64) ++bwl;  // 2^bwl divides BTOK = 192
+        p.bw_log2 = bwl;
+        p.bh = BTOK >> bwl;
+        const int bw = 1 << bwl;
+        p.tiles_w = (a.W + bw - 1) / bw;
         p.tiles_h = (a.H + p.bh - 1) / p.bh;
         const int64_t tok_tiles = int64_t(a.B) * p.tiles_h * p.tiles_w;
         if (tok_tiles * p.tiles_ch > 0x7FFFFFFF) {
@@ -437,7 +601,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         p.tiles_tok = int(tok_tiles);
         cuuint64_t dims[4] = {cuuint64_t(a.Cin), cuuint64_t(a.W), cuuint64_t(a.H), cuuint64_t(a.B)};
         cuuint64_t strides[3] = {cuuint64_t(a.Cin) * 2, cuuint64_t(a.W) * a.Cin * 2, cuuint64_t(a.H) * a.W * a.Cin * 2};
-        cuuint32_t box[4] = {BK, cuuint32_t(p.bw), cuuint32_t(p.bh), 1};
+        cuuint32_t box[4] = {64, cuuint32_t(bw), cuuint32_t(p.bh), 1};
         cuuint32_t es[4] = {1, 1, 1, 1};
         r = encode(&tm_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void*>(a.x), dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -446,7 +610,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         p.tiles_tok = (a.M + BTOK - 1) / BTOK;
         cuuint64_t dims[2] = {cuuint64_t(a.K), cuuint64_t(a.M)};
         cuuint64_t strides[1] = {cuuint64_t(a.K) * 2};
-        cuuint32_t box[2] = {BK, BTOK};
+        cuuint32_t box[2] = {64, BTOK};
         cuuint32_t es[2] = {1, 1};
         r = encode(&tm_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(a.x), dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -462,7 +626,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         cuuint32_t box[2] = {BK, BCH};
         cuuint32_t es[2] = {1, 1};
         r = encode(&tm_w, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t*>(a.w), dims, strides, box, es,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) {
             *why = "weight tensor map rejected";
@@ -473,8 +637,39 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     const int grid = int(tiles < num_sms ? tiles : num_sms);
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    gemm_tc_kernel<<<grid, THREADS, SMEM_BYTES, st>>>(p, tm_x, tm_w);
-    return cudaGetLastError();
+    // programmatic dependent launch: the grid may start while the previous
+    // kernel drains; it waits (griddepcontrol.wait) before reading inputs
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel, p, tm_x, tm_w);
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e == cudaErrorLaunchOutOfResources) {
+        // report what the kernel asked for, to make the failure actionable
+        static char msg[256];
+        cudaFuncAttributes fa{};
+        cudaFuncGetAttributes(&fa, gemm_tc_kernel);
+        snprintf(msg, sizeof msg,
+                 "launch out of resources: %d threads x %d registers, %d B dynamic smem (kernel max %d threads, "
+                 "%zu B static smem)",
+                 THREADS, fa.numRegs, SMEM_BYTES, fa.maxThreadsPerBlock, fa.sharedSizeBytes);
+        *why = msg;
+        return cudaSuccess;
+    }
+    return e;
 }
+
+#ifdef TASQ_TRACE
+extern "C" __attribute__((visibility("default"))) int tasq_debug_trace(void* host, size_t bytes) {
+    return (int)cudaMemcpyFromSymbol(host, g_tasq_trace, bytes < sizeof(g_tasq_trace) ? bytes : sizeof(g_tasq_trace));
+}
+#endif
 
 }  // namespace tasq

@@ -5,6 +5,7 @@
 #include <cuda_fp16.h>
 
 #include "tasq_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace tasq {
 namespace {
@@ -57,11 +58,13 @@ __device__ inline void scale_of_range(float lo, float hi, float denom, float hal
 }
 
 // Activation code: Q = clamp(rint(x / alpha + z), 0, qmax), s = Q - half.
-__device__ inline int act_code(float x, float alpha, float z, int qmax, int half) {
-    float u = __fadd_rn(__fdiv_rn(x, alpha), z);
-    int q = __float2int_rn(u);  // round half to even
-    q = min(max(q, 0), qmax);
-    return q - half;
+// ralpha = RN(1 / alpha); x / alpha is still rounded exactly as IEEE division.
+__device__ inline int act_code(float x, float alpha, float ralpha, float z, int qmax, int half) {
+    const float u = __fadd_rn(div_rn_by(x, alpha, ralpha), z);
+    // u lies in [-1, qmax + 1] up to rounding for x inside the quantization range;
+    // clamp first so the bit trick's |u| <= 2^22 precondition always holds
+    const int q = rint_small(fminf(fmaxf(u, -2.0f), float(qmax) + 2.0f));
+    return min(max(q, 0), qmax) - half;
 }
 
 __device__ inline void store8_codes(void* out, int code_fmt, int64_t i, const int s[8]) {
@@ -151,19 +154,153 @@ __global__ void __launch_bounds__(256) quant_act_token_kernel(const void* __rest
     const int half = 1 << (n_bits - 1), qmax = (1 << n_bits) - 1;
     float alpha, z;
     scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
+    const float ralpha = __frcp_rn(alpha);
     char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (code_fmt == TASQ_CODES_S8 ? 1 : 2);
     for (int i = lane; i < groups; i += 32) {
         float v[8];
         load8(row, dtype, i, v);
         int s[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, z, qmax, half);
+        for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, ralpha, z, qmax, half);
         store8_codes(out, code_fmt, i, s);
     }
     if (lane == 0) {
         alpha_out[m] = alpha;
         zc_out[m] = __fsub_rn(float(half), z);
     }
+}
+
+// Single-pass per-token quantization: one warp per row, the whole row held in
+// registers as NPL 16-byte chunks per lane (chunk c of the row is lane c % 32,
+// slot c / 32), so every load is issued before the min/max reduction.
+template <int NPL, int DTYPE, int CODES>
+__global__ void __launch_bounds__(256) quant_act_rowreg_kernel(const void* __restrict__ x, int M, int K, int n_bits,
+                                                               int mode, void* __restrict__ codes,
+                                                               float* __restrict__ alpha_out,
+                                                               float* __restrict__ zc_out) {
+    constexpr int EPC = DTYPE == TASQ_F32 ? 4 : 8;  // elements per 16-byte chunk
+    const int lane = threadIdx.x & 31;
+    const int m = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    // launched with programmatic dependent launch: wait for the previous kernel
+    // (which may still read the code buffer) before touching memory
+    ptx::grid_dependency_wait();
+    if (m >= M) return;
+    const int chunks = K / EPC;
+    const uint4* row = reinterpret_cast<const uint4*>(x) + int64_t(m) * chunks;
+    uint4 d[NPL];
+#pragma unroll
+    for (int k = 0; k < NPL; ++k) {
+        const int c = lane + 32 * k;
+        d[k] = c < chunks ? __ldg(row + c) : make_uint4(0, 0, 0, 0);
+    }
+    auto elem = [&](const uint4& v, int j) -> float {
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+        if (DTYPE == TASQ_F32) return __uint_as_float(w[j]);
+        return __uint_as_float((j & 1) ? (w[j >> 1] & 0xFFFF0000u) : (w[j >> 1] << 16));
+    };
+    float lo = INFINITY, hi = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < NPL; ++k) {
+        if (lane + 32 * k < chunks) {
+#pragma unroll
+            for (int j = 0; j < EPC; ++j) {
+                const float f = elem(d[k], j);
+                lo = fminf(lo, f);
+                hi = fmaxf(hi, f);
+            }
+        }
+    }
+    lo = warp_min(lo);
+    hi = warp_max(hi);
+    if (mode == TASQ_SYMRANGE) {
+        hi = fmaxf(fabsf(lo), fabsf(hi));
+        lo = -hi;
+    }
+    const int half = 1 << (n_bits - 1), qmax = (1 << n_bits) - 1;
+    float alpha, z;
+    scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
+    const float ralpha = __frcp_rn(alpha);
+    char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (CODES == TASQ_CODES_S8 ? 1 : 2);
+#pragma unroll
+    for (int k = 0; k < NPL; ++k) {
+        const int c = lane + 32 * k;
+        if (c >= chunks) continue;
+        int q[EPC];
+#pragma unroll
+        for (int j = 0; j < EPC; ++j) q[j] = act_code(elem(d[k], j), alpha, ralpha, z, qmax, half);
+        if (CODES == TASQ_CODES_S8) {
+            if (EPC == 8) {
+                uint2 pk;
+                pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((uint32_t)(q[3] & 0xFF) << 24);
+                pk.y = (q[4 % EPC] & 0xFF) | ((q[5 % EPC] & 0xFF) << 8) | ((q[6 % EPC] & 0xFF) << 16) |
+                       ((uint32_t)(q[7 % EPC] & 0xFF) << 24);
+                reinterpret_cast<uint2*>(out)[c] = pk;
+            } else {
+                reinterpret_cast<uint32_t*>(out)[c] =
+                    (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2 % EPC] & 0xFF) << 16) | ((uint32_t)(q[3 % EPC] & 0xFF) << 24);
+            }
+        } else {
+            // fp16 of a small integer s: the bits 0x6400 + (s + half) hold 1024 + s + half
+            // exactly; one packed subtraction of 1024 + half leaves s
+            uint32_t h[EPC];
+#pragma unroll
+            for (int j = 0; j < EPC; ++j) h[j] = 0x6400u + uint32_t(q[j] + half);
+            const uint32_t off = 0x6400u + uint32_t(half);
+            const __half2 bias2 = __halves2half2(__ushort_as_half(uint16_t(off)), __ushort_as_half(uint16_t(off)));
+            auto sub2 = [&](uint32_t lo16, uint32_t hi16) -> uint32_t {
+                uint32_t w = lo16 | (hi16 << 16);
+                __half2 r = __hsub2(*reinterpret_cast<__half2*>(&w), bias2);
+                return *reinterpret_cast<uint32_t*>(&r);
+            };
+            if (EPC == 8) {
+                uint4 pk;
+                pk.x = sub2(h[0], h[1]);
+                pk.y = sub2(h[2], h[3]);
+                pk.z = sub2(h[4 % EPC], h[5 % EPC]);
+                pk.w = sub2(h[6 % EPC], h[7 % EPC]);
+                reinterpret_cast<uint4*>(out)[c] = pk;
+            } else {
+                reinterpret_cast<uint2*>(out)[c] = make_uint2(sub2(h[0], h[1]), sub2(h[2 % EPC], h[3 % EPC]));
+            }
+        }
+    }
+    if (lane == 0) {
+        alpha_out[m] = alpha;
+        zc_out[m] = __fsub_rn(float(half), z);
+    }
+    ptx::grid_launch_dependents();
+}
+
+template <int NPL, int DTYPE>
+cudaError_t launch_rowreg(const void* x, int M, int K, int n_bits, int mode, void* codes, int code_fmt, float* alpha,
+                          float* zc, cudaStream_t st) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((M + kRowWarps - 1) / kRowWarps);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = code_fmt == TASQ_CODES_S8
+                        ? cudaLaunchKernelEx(&cfg, quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_S8>, x, M, K, n_bits,
+                                             mode, codes, alpha, zc)
+                        : cudaLaunchKernelEx(&cfg, quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16>, x, M, K, n_bits,
+                                             mode, codes, alpha, zc);
+    return e == cudaSuccess ? cudaGetLastError() : e;
+}
+
+template <int DTYPE>
+bool dispatch_rowreg(int chunks_per_lane, const void* x, int M, int K, int n_bits, int mode, void* codes, int code_fmt,
+                     float* alpha, float* zc, cudaStream_t st, cudaError_t* e) {
+    if (chunks_per_lane <= 2) *e = launch_rowreg<2, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
+    else if (chunks_per_lane <= 5) *e = launch_rowreg<5, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
+    else if (chunks_per_lane <= 9) *e = launch_rowreg<9, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
+    else if (chunks_per_lane <= 18) *e = launch_rowreg<18, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
+    else if (chunks_per_lane <= 24) *e = launch_rowreg<24, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
+    else return false;
+    return true;
 }
 
 // ----------------------------------------------------- activations, tensor --
@@ -224,12 +361,13 @@ __global__ void __launch_bounds__(256) quant_act_tensor_kernel(const void* __res
     const int half = 1 << (n_bits - 1), qmax = (1 << n_bits) - 1;
     float alpha, z;
     scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
+    const float ralpha = __frcp_rn(alpha);
     for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < groups; i += int64_t(gridDim.x) * blockDim.x) {
         float v[8];
         load8(x, dtype, i, v);
         int s[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, z, qmax, half);
+        for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, ralpha, z, qmax, half);
         store8_codes(codes, code_fmt, i, s);
     }
     if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -350,7 +488,28 @@ __global__ void selftest_timeout_kernel(int* status, unsigned long long timeout_
     }
 }
 
+// Counts x / a pairs where the activation quantizer's quotient differs from
+// IEEE division (bit patterns compared).
+__global__ void selftest_quotients_kernel(const float* __restrict__ x, int nx, const float* __restrict__ a, int na,
+                                          unsigned long long* mismatches) {
+    unsigned long long bad = 0;
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < int64_t(nx) * na;
+         i += int64_t(gridDim.x) * blockDim.x) {
+        const float xv = x[i % nx], av = a[i / nx];
+        const float ra = __frcp_rn(av);
+        bad += __float_as_uint(div_rn_by(xv, av, ra)) != __float_as_uint(__fdiv_rn(xv, av));
+    }
+    for (int o = 16; o; o >>= 1) bad += __shfl_xor_sync(0xffffffffu, bad, o);
+    if ((threadIdx.x & 31) == 0 && bad) atomicAdd(mismatches, bad);
+}
+
 }  // namespace
+
+cudaError_t launch_selftest_quotients(const float* x, int nx, const float* a, int na, unsigned long long* mismatches,
+                                      cudaStream_t st) {
+    selftest_quotients_kernel<<<1024, 256, 0, st>>>(x, nx, a, na, mismatches);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int8_t* sw, float* cw, float* alpha,
                                  cudaStream_t st) {
@@ -362,6 +521,14 @@ cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int8_t*
 cudaError_t launch_quant_act_token(const void* x, int dtype, int M, int K, int n_bits, int mode, void* codes,
                                    int code_fmt, float* alpha, float* zc, cudaStream_t st) {
     if (M == 0) return cudaSuccess;
+    // rows that fit in registers: one pass over HBM
+    const int chunks = K * (dtype == TASQ_F32 ? 4 : 2) / 16;
+    const int per_lane = (chunks + 31) / 32;
+    cudaError_t e = cudaSuccess;
+    if (dtype == TASQ_F32 ? dispatch_rowreg<TASQ_F32>(per_lane, x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st, &e)
+                          : dispatch_rowreg<TASQ_BF16>(per_lane, x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st, &e))
+        return e;
+    // longer rows: two passes (the second mostly from L2)
     quant_act_token_kernel<<<(M + kRowWarps - 1) / kRowWarps, 256, 0, st>>>(x, dtype, M, K, n_bits, mode, codes,
                                                                             code_fmt, alpha, zc);
     return cudaGetLastError();

@@ -13,6 +13,7 @@ struct tasq_ctx_s {
     int device = 0;
     int num_sms = 0;
     int* d_words = nullptr;  // [0] status, [16..19] reduction scratch
+    int32_t* d_part = nullptr;  // tensor-core route: int32 running sums of multi-chunk tiles
     uint8_t* d_table = nullptr;
     size_t table_cap = 0;
     int L = 0, S = 0;
@@ -91,10 +92,13 @@ TASQ_API int tasq_create(tasq_ctx* out, int device) {
     ctx->num_sms = prop.multiProcessorCount;
     e = cudaMalloc(&ctx->d_words, 256);
     if (e == cudaSuccess) e = cudaMemset(ctx->d_words, 0, 256);
+    if (e == cudaSuccess) e = cudaMalloc(&ctx->d_part, tasq::gemm_tc_part_bytes(ctx->num_sms));
     cudaSetDevice(prev);
     if (e != cudaSuccess) {
+        cudaFree(ctx->d_words);
+        cudaFree(ctx->d_part);
         delete ctx;
-        return fail(nullptr, TASQ_ERR_CUDA, "allocating the status word: %s", cudaGetErrorString(e));
+        return fail(nullptr, TASQ_ERR_CUDA, "allocating context buffers: %s", cudaGetErrorString(e));
     }
     *out = ctx;
     return TASQ_OK;
@@ -107,6 +111,7 @@ TASQ_API void tasq_destroy(tasq_ctx ctx) {
     cudaSetDevice(ctx->device);
     cudaDeviceSynchronize();
     cudaFree(ctx->d_words);
+    cudaFree(ctx->d_part);
     cudaFree(ctx->d_table);
     cudaSetDevice(prev);
     delete ctx;
@@ -144,6 +149,14 @@ TASQ_API int tasq_selftest_timeout(tasq_ctx ctx, uint64_t timeout_ns, tasq_strea
     CHECK_CTX(ctx);
     REQUIRE(timeout_ns > 0 && timeout_ns <= 10000000000ull, TASQ_ERR_INVALID_ARG, "timeout_ns must be in (0, 1e10]");
     cudaError_t e = tasq::launch_selftest_timeout(ctx->d_words, timeout_ns, (cudaStream_t)stream);
+    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "selftest launch");
+}
+
+TASQ_API int tasq_selftest_quotients(tasq_ctx ctx, const float* d_x, int nx, const float* d_a, int na,
+                                    unsigned long long* d_mismatches, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(nx > 0 && na > 0 && d_x && d_a && d_mismatches, TASQ_ERR_INVALID_ARG, "need nx, na > 0 and pointers");
+    cudaError_t e = tasq::launch_selftest_quotients(d_x, nx, d_a, na, d_mismatches, (cudaStream_t)stream);
     return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "selftest launch");
 }
 
@@ -288,6 +301,7 @@ int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void*
     a.per_tensor = kind == TASQ_CONV3X3;
     a.y = d_y;
     a.acc = d_acc;
+    a.part = ctx->d_part;
     a.status = ctx->d_words;
     a.timeout_ns = ctx->timeout_ns;
     cudaError_t e;

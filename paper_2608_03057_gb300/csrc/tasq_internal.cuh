@@ -77,6 +77,7 @@ struct GemmArgs {
     int per_tensor;
     uint16_t* y;              // bf16 bits
     int32_t* acc;             // optional int32 accumulators
+    int32_t* part;            // TC route: per-CTA int32 running sums of multi-chunk tiles
     int* status;
     unsigned long long timeout_ns;
 };
@@ -95,6 +96,25 @@ __device__ inline int resolve_bits(const GemmArgs& a) {
         return 0;
     }
     return b;
+}
+
+// x / a rounded to nearest even, from ra = RN(1/a): the quotient estimate
+// q = RN(x * ra) is refined twice by the exact FMA remainder r = x - q * a
+// (Markstein's correction, q <- RN(q + r * ra)), which reaches the correctly
+// rounded quotient for normal operands.  Checked against IEEE division by
+// tasq_selftest_quotients over every finite bf16 input.
+__device__ __forceinline__ float div_rn_by(float x, float a, float ra) {
+    float q = __fmul_rn(x, ra);
+    float r = __fmaf_rn(-q, a, x);
+    q = __fmaf_rn(r, ra, q);
+    r = __fmaf_rn(-q, a, x);
+    return __fmaf_rn(r, ra, q);
+}
+
+// Round half to even of |u| <= 2^22, returned as an int: adding 1.5 * 2^23
+// leaves the rounded integer in the low mantissa bits.
+__device__ __forceinline__ int rint_small(float u) {
+    return int(__float_as_uint(__fadd_rn(u, 12582912.0f)) - 0x4B400000u);
 }
 
 // Fused dequantization epilogue, fp32 with one rounding per operation:
@@ -145,6 +165,9 @@ cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float
                         void* packed, cudaStream_t st);
 cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why);
+size_t gemm_tc_part_bytes(int num_sms);  // scratch the TC route needs for `num_sms` persistent CTAs
 cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, cudaStream_t st);
+cudaError_t launch_selftest_quotients(const float* x, int nx, const float* a, int na, unsigned long long* mismatches,
+                                      cudaStream_t st);
 
 }  // namespace tasq

@@ -57,6 +57,7 @@ def lib():
                 "tasq_set_route": ([P, I], I),
                 "tasq_set_timeout_ns": ([P, U64], I),
                 "tasq_selftest_timeout": ([P, U64, P], I),
+                "tasq_selftest_quotients": ([P, P, I, P, I, P, P], I),
                 "tasq_quant_weights": ([P, P, I, I, I, P, P, P, P], I),
                 "tasq_packed_bytes": ([I, I, I], SZ),
                 "tasq_pack_weights": ([P, I, P, P, P, I, I, I, P, P], I),
@@ -137,6 +138,11 @@ def tasq_set_timeout_ns(ctx, ns: int) -> None:
 
 def tasq_selftest_timeout(ctx, timeout_ns: int, stream=None) -> None:
     _check(ctx, lib().tasq_selftest_timeout(ctx, int(timeout_ns), _stream(stream)))
+
+
+def tasq_selftest_quotients(ctx, x, nx, a, na, mismatches, stream=None) -> None:
+    _check(ctx, lib().tasq_selftest_quotients(ctx, _ptr(x), int(nx), _ptr(a), int(na), _ptr(mismatches),
+                                              _stream(stream)))
 
 
 def tasq_quant_weights(ctx, w, dtype, N, K, sw, cw, alpha=None, stream=None) -> None:

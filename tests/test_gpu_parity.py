@@ -409,3 +409,21 @@ def test_device_wait_timeout_is_reported_and_context_survives(ctx, oracle):
     st = _setup_linear(ctx, oracle, M, N, K, [7], code_fmt=tasq.TASQ_CODES_S8)
     y, acc = G.gemm(ctx, 0, 0, st["codes"], tasq.TASQ_CODES_S8, st["alpha"], st["zc"], M, st["packed"], N, K)
     _check_layer(oracle, st, 7, y, acc)
+
+
+def test_quotient_routine_matches_ieee_division(ctx):
+    """The activation quantizer's x / alpha (reciprocal once per group, two
+    exact remainder corrections) equals IEEE round-to-nearest division for
+    every finite bf16 dividend against divisors spanning the normal range."""
+    torch = G.torch()
+    bits = np.arange(1 << 16, dtype=np.uint32)
+    xs = (bits << 16).view(np.float32)
+    e = (bits >> 7) & 0xFF
+    xs = xs[(e > 30) & (e < 225)]  # normal dividends, quotients stay normal
+    rng = workloads.rng(5)
+    a = np.concatenate([np.exp2(rng.uniform(-30, 30, 2000)), 2.0 ** np.arange(-30, 31),
+                        rng.uniform(1e-3, 5e-2, 1000)]).astype(np.float32)
+    mism = torch.zeros((1,), dtype=torch.int64, device="cuda")
+    tasq.tasq_selftest_quotients(ctx.h, G.dev(xs), xs.size, G.dev(a), a.size, mism)
+    torch.cuda.synchronize()
+    assert int(mism.item()) == 0
