@@ -245,6 +245,33 @@ int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void* d_codes,
                         const float* d_zc, int B, int H, int W, int Cin, const void* d_packed, int Cout, uint16_t* d_y,
                         int32_t* d_acc, tasq_stream stream);
 
+/*
+ * Per-tensor activation quantization without any allocation (no context).
+ * The paper has no counterpart to this call: it exists for callers that
+ * cannot allocate device memory at run time -- for example an inference
+ * plugin whose host framework forbids allocation while it enqueues work, or
+ * a deployment whose device memory is planned once before serving -- and so
+ * cannot create a context (tasq_create allocates).
+ * It computes exactly what tasq_quant_act computes with gran =
+ * TASQ_PER_TENSOR (same arguments and layouts; d_alpha and d_zc hold one
+ * value each), but its reduction scratch is a 16 KB array compiled into the
+ * library, which every GPU that loads the library keeps until the process
+ * exits.  The call itself allocates nothing: it enqueues two kernels on
+ * `stream` and returns.
+ *  - Limit: M * K <= 67,108,864 elements (2048 slices of 32,768); larger
+ *    tensors return TASQ_ERR_UNSUPPORTED without launching anything.
+ *  - The first call on a device looks up the array's device address once
+ *    (cudaGetSymbolAddress, with that device current); make that first call
+ *    before capturing a stream into a CUDA graph.
+ *  - Every call uses the same array, and each call rewrites the slots it
+ *    reads, so nothing carries over between calls; but calls whose kernels
+ *    overlap on the GPU (different streams, or one device used from several
+ *    threads without ordering) race on the array and must be serialized.
+ *  - Errors are described by tasq_last_error(NULL) on the calling thread.
+ */
+int tasq_quant_act_tensor_noalloc(const void* d_x, int dtype, int M, int K, int n_bits, int mode, void* d_codes,
+                                  int code_fmt, float* d_alpha, float* d_zc, tasq_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -4,6 +4,9 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include <cstdio>
+#include <mutex>
+
 #include "tasq_internal.cuh"
 #include "tc_ptx.cuh"
 
@@ -580,4 +583,165 @@ cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, 
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Per-tensor activation quantization that allocates nothing.
+//
+// For callers that cannot allocate device memory at run time (an inference
+// plugin whose host framework forbids allocation inside enqueue, a process
+// whose memory is planned once up front, code that must not create a
+// context-owned buffer), the reduction scratch of per-tensor quantization
+// lives in a file-scope device array instead of context memory.  Each block
+// of the first kernel writes the (min, max) of its own slice into its slot;
+// the second kernel folds the slots in a fixed order, so the result does not
+// depend on timing and no slot needs clearing between calls.  The array is
+// 16 KB and stays resident on every GPU that loads the library, until exit.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr int kNoAllocMaxBlocks = 2048;
+constexpr int64_t kNoAllocSlice = 32768;  // elements reduced per block
+static __device__ __align__(256) float2 g_noalloc_ranges[kNoAllocMaxBlocks];
+
+__global__ void __launch_bounds__(256) noalloc_range_kernel(const void* __restrict__ x, int dtype, int64_t count,
+                                                            float2* ranges) {
+    const int64_t g0 = blockIdx.x * (kNoAllocSlice / 8);
+    const int64_t g1 = min(count / 8, g0 + kNoAllocSlice / 8);
+    float lo = INFINITY, hi = -INFINITY;
+    for (int64_t i = g0 + threadIdx.x; i < g1; i += blockDim.x) {
+        float v[8];
+        load8(x, dtype, i, v);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            lo = fminf(lo, v[j]);
+            hi = fmaxf(hi, v[j]);
+        }
+    }
+    lo = warp_min(lo);
+    hi = warp_max(hi);
+    __shared__ float slo[8], shi[8];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        slo[warp] = lo;
+        shi[warp] = hi;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int i = 1; i < int(blockDim.x >> 5); ++i) {
+            lo = fminf(lo, slo[i]);
+            hi = fmaxf(hi, shi[i]);
+        }
+        ranges[blockIdx.x] = make_float2(lo, hi);
+    }
+}
+
+__global__ void __launch_bounds__(256) noalloc_quant_kernel(const void* __restrict__ x, int dtype, int64_t count,
+                                                            int nranges, int n_bits, int mode, void* __restrict__ codes,
+                                                            int code_fmt, float* __restrict__ alpha_out,
+                                                            float* __restrict__ zc_out,
+                                                            const float2* __restrict__ ranges) {
+    __shared__ float s_lo, s_hi;
+    if (threadIdx.x < 32) {
+        float lo = INFINITY, hi = -INFINITY;
+        for (int i = threadIdx.x; i < nranges; i += 32) {
+            const float2 r = ranges[i];
+            lo = fminf(lo, r.x);
+            hi = fmaxf(hi, r.y);
+        }
+        lo = warp_min(lo);
+        hi = warp_max(hi);
+        if (threadIdx.x == 0) {
+            s_lo = lo;
+            s_hi = hi;
+        }
+    }
+    __syncthreads();
+    float lo = s_lo, hi = s_hi;
+    if (mode == TASQ_SYMRANGE) {
+        hi = fmaxf(fabsf(lo), fabsf(hi));
+        lo = -hi;
+    }
+    const int half = 1 << (n_bits - 1), qmax = (1 << n_bits) - 1;
+    float alpha, z;
+    scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
+    const float ralpha = __frcp_rn(alpha);
+    const int64_t groups = count / 8;
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < groups; i += int64_t(gridDim.x) * blockDim.x) {
+        float v[8];
+        load8(x, dtype, i, v);
+        int sv[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) sv[j] = act_code(v[j], alpha, ralpha, z, qmax, half);
+        store8_codes(codes, code_fmt, i, sv);
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        alpha_out[0] = alpha;
+        zc_out[0] = __fsub_rn(float(half), z);
+    }
+}
+
+// Device address of g_noalloc_ranges, looked up once per device (the host-side
+// name is only a stand-in for the device array).
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[64] = {};
+
+int noalloc_fail(int code, const char* msg) {
+    set_noctx_error(msg);
+    return code;
+}
+
+}  // namespace
+
 }  // namespace tasq
+
+extern "C" __attribute__((visibility("default"))) int tasq_quant_act_tensor_noalloc(
+    const void* d_x, int dtype, int M, int K, int n_bits, int mode, void* d_codes, int code_fmt, float* d_alpha,
+    float* d_zc, tasq_stream stream) {
+    using namespace tasq;
+    if (dtype != TASQ_F32 && dtype != TASQ_BF16) return noalloc_fail(TASQ_ERR_INVALID_ARG, "dtype must be F32 or BF16");
+    if (mode != TASQ_SYMRANGE && mode != TASQ_ASYM) return noalloc_fail(TASQ_ERR_INVALID_ARG, "mode must be SYMRANGE or ASYM");
+    if (code_fmt != TASQ_CODES_S8 && code_fmt != TASQ_CODES_F16)
+        return noalloc_fail(TASQ_ERR_INVALID_ARG, "code_fmt must be CODES_S8 or CODES_F16");
+    if (n_bits < 2 || n_bits > 8) return noalloc_fail(TASQ_ERR_INVALID_ARG, "n_bits must be in 2..8");
+    if (M < 0 || K <= 0) return noalloc_fail(TASQ_ERR_INVALID_ARG, "need M >= 0 and K > 0");
+    if (K % 16) return noalloc_fail(TASQ_ERR_UNSUPPORTED, "K must be a multiple of 16");
+    const int64_t count = int64_t(M) * K;
+    if (count > int64_t(kNoAllocMaxBlocks) * kNoAllocSlice) {
+        char msg[160];
+        snprintf(msg, sizeof msg, "tensor of %lld elements exceeds the %lld-element limit of quantization without allocation",
+                 (long long)count, (long long)(int64_t(kNoAllocMaxBlocks) * kNoAllocSlice));
+        return noalloc_fail(TASQ_ERR_UNSUPPORTED, msg);
+    }
+    if (M == 0) return TASQ_OK;
+    if (!d_x || !d_codes || !d_alpha || !d_zc) return noalloc_fail(TASQ_ERR_INVALID_ARG, "NULL pointer");
+    if ((reinterpret_cast<uintptr_t>(d_x) | reinterpret_cast<uintptr_t>(d_codes)) & 15u)
+        return noalloc_fail(TASQ_ERR_UNSUPPORTED, "d_x and d_codes must be 16-byte aligned");
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return noalloc_fail(TASQ_ERR_CUDA, cudaGetErrorString(e));
+    if (dev < 0 || dev >= 64) return noalloc_fail(TASQ_ERR_UNSUPPORTED, "device index above 63");
+    void* ranges = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_noalloc_mu);
+        if (!g_noalloc_addr[dev]) {
+            e = cudaGetSymbolAddress(&g_noalloc_addr[dev], g_noalloc_ranges);
+            if (e != cudaSuccess) {
+                g_noalloc_addr[dev] = nullptr;
+                return noalloc_fail(TASQ_ERR_CUDA, cudaGetErrorString(e));
+            }
+        }
+        ranges = g_noalloc_addr[dev];
+    }
+    const int nranges = int((count + kNoAllocSlice - 1) / kNoAllocSlice);
+    cudaStream_t st = (cudaStream_t)stream;
+    noalloc_range_kernel<<<nranges, 256, 0, st>>>(d_x, dtype, count, reinterpret_cast<float2*>(ranges));
+    if ((e = cudaGetLastError()) != cudaSuccess) return noalloc_fail(TASQ_ERR_CUDA, cudaGetErrorString(e));
+    int sms = 148;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t want = (count / 8 + 255) / 256;
+    const int grid = int(want < 4 * sms ? want : 4 * sms);
+    noalloc_quant_kernel<<<grid, 256, 0, st>>>(d_x, dtype, count, nranges, n_bits, mode, d_codes, code_fmt, d_alpha,
+                                               d_zc, reinterpret_cast<const float2*>(ranges));
+    if ((e = cudaGetLastError()) != cudaSuccess) return noalloc_fail(TASQ_ERR_CUDA, cudaGetErrorString(e));
+    return TASQ_OK;
+}
+

@@ -119,6 +119,11 @@ TASQ_API void tasq_destroy(tasq_ctx ctx) {
 
 TASQ_API const char* tasq_last_error(tasq_ctx ctx) { return ctx ? ctx->err.c_str() : g_create_err.c_str(); }
 
+namespace tasq {
+// Error text of calls made without a context (read by tasq_last_error(NULL)).
+void set_noctx_error(const char* msg) { g_create_err = msg; }
+}  // namespace tasq
+
 TASQ_API int tasq_device_status(tasq_ctx ctx, int* out) {
     CHECK_CTX(ctx);
     REQUIRE(out, TASQ_ERR_INVALID_ARG, "out is NULL");

@@ -167,6 +167,7 @@ cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why);
 size_t gemm_tc_part_bytes(int num_sms);  // scratch the TC route needs for `num_sms` persistent CTAs
 cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, cudaStream_t st);
+void set_noctx_error(const char* msg);
 cudaError_t launch_selftest_quotients(const float* x, int nx, const float* a, int na, unsigned long long* mismatches,
                                       cudaStream_t st);
 

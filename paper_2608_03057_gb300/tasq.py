@@ -66,6 +66,7 @@ def lib():
                 "tasq_quant_act": ([P, P, I, I, I, I, I, I, P, I, P, P, P], I),
                 "tasq_masked_gemm": ([P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_conv3x3": ([P, I, I, P, I, P, P, I, I, I, I, P, I, P, P, P], I),
+                "tasq_quant_act_tensor_noalloc": ([P, I, I, I, I, I, P, I, P, P, P], I),
             }
             for name, (args, res) in sigs.items():
                 f = getattr(L, name)
@@ -183,3 +184,10 @@ def tasq_masked_conv3x3(ctx, layer, stage, codes, code_fmt, alpha, zc, B, H, W, 
     _check(ctx, lib().tasq_masked_conv3x3(ctx, int(layer), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
                                           _ptr(zc), int(B), int(H), int(W), int(Cin), _ptr(packed), int(Cout), _ptr(y),
                                           _ptr(acc), _stream(stream)))
+
+
+def tasq_quant_act_tensor_noalloc(x, dtype, M, K, n_bits, mode, codes, code_fmt, alpha, zc, stream=None) -> None:
+    """Per-tensor activation quantization that allocates nothing (no context)."""
+    _check(None, lib().tasq_quant_act_tensor_noalloc(_ptr(x), int(dtype), int(M), int(K), int(n_bits), int(mode),
+                                                     _ptr(codes), int(code_fmt), _ptr(alpha), _ptr(zc),
+                                                     _stream(stream)))
