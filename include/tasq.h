@@ -216,8 +216,10 @@ int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n
  * Masked linear layer (Eq. qalora with the Temporal-Spatial LSB mask of
  * Eq. lsb_masking at operating precision b = table[layer][stage]):
  *   acc[m][n] = sum_k s_x[m][k] * mask_b(s_w[n][k])            (exact int32)
- *   y[m][n]   = bf16( ((float(acc) + zc[m]*float(rs_b[n])) * (alpha[m]*c_w[n])) + bias[n] )
- * with every fp32 operation rounded to nearest even in that order.
+ *   u = fma(zc[m], float(rs_b[n]), float(acc)),  s = alpha[m] * c_w[n],
+ *   y[m][n] = bf16(fma(u, s, bias[n]))
+ * with every fp32 operation (and each fused multiply-add) rounded once to
+ * nearest even, in that order; y = alpha*c_w*(acc + zc*rs_b) + bias.
  * stage: 0..S-1, or -1 to read it from the device int of
  * tasq_set_stage_device.  d_codes: [M][K] activation codes (code_fmt);
  * d_alpha/d_zc: [M] per-token scales from tasq_quant_act.  d_packed: from

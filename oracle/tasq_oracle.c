@@ -13,7 +13,8 @@
  * precision; the dequantized result is given twice: in the kernel's fp32
  * rounding order (oq_epilogue_f32) and by the definition in fp64
  * (oq_linear_def_f64 / oq_conv3x3_def_f64).  Compile with -ffp-contract=off so
- * that no multiply-add is fused: every operation rounds once to nearest-even.
+ * that the compiler fuses nothing: every operation rounds once to nearest-even,
+ * and the only fused multiply-adds are the explicit fmaf calls of the epilogue.
  *
  * Readings of the paper taken here (the paper is silent on them):
  *  - Weights are quantized per output channel, activations per token (linear)
@@ -215,8 +216,10 @@ void oq_row_sums(const int8_t* s_w, int N, int K, int b, int32_t* rs) {
 
 /*
  * Dequantization (Eqs. act_dequant and weight_dequant) folded around the
- * integer contraction, in the kernel's fp32 rounding order:
- *   y = bf16_rne( RN( RN( RN(float(acc) + RN(zc * float(rs))) * RN(alpha * c) ) + bias ) )
+ * integer contraction, in the kernel's fp32 rounding order (two fused
+ * multiply-adds, each rounded once):
+ *   u = RN(zc * float(rs) + float(acc)),  s = RN(alpha * c),  y = RN(u * s + bias),
+ *   output bf16_rne(y),
  * because sum_k alpha(s_x + zc) * c * mask(s_w) = alpha * c * (acc + zc * rs).
  * alpha/zc are indexed by row_of(m) = m (per token) or 0 (per tensor);
  * rs[m*rs_stride_m + n] lets a conv pass one row sum per output pixel.
@@ -228,11 +231,9 @@ void oq_epilogue_f32(const int32_t* acc, int M, int N, const float* alpha, const
         int r = per_tensor ? 0 : m;
         for (int n = 0; n < N; ++n) {
             float a = (float)acc[(int64_t)m * N + n];
-            float t = zc[r] * (float)rs[(int64_t)m * rs_stride_m + n];
-            float u = a + t;
+            float u = fmaf(zc[r], (float)rs[(int64_t)m * rs_stride_m + n], a);
             float s = alpha[r] * c_w[n];
-            float v = u * s;
-            float y = v + (bias ? bias[n] : 0.0f);
+            float y = fmaf(u, s, bias ? bias[n] : 0.0f);
             if (y_f32) y_f32[(int64_t)m * N + n] = y;
             if (y_bf16) y_bf16[(int64_t)m * N + n] = oq_bf16_rne(y);
         }

@@ -31,6 +31,7 @@
 // TASQ_ERR_DEVICE_TIMEOUT, the CTA drains its copies in flight, frees its
 // tensor memory and returns.
 #include <cstdio>
+#include <cstdlib>
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -56,31 +57,48 @@ __device__ unsigned long long g_tasq_trace[4][256][8];
 namespace tasq {
 namespace {
 
-constexpr int BCH = 128;          // output channels per tile (MMA M)
+constexpr int BCH = 128;          // output channels per CTA (MMA M per CTA)
 constexpr int BTOK = 192;         // tokens / output pixels per tile (MMA N)
 constexpr int BK = 128;           // K per pipeline stage (two 64-wide swizzle atoms)
-constexpr int STAGES = 3;         // shared-memory stages
-constexpr int ASLOTS = 2;         // tensor-memory slots of converted weights
+constexpr int SLOT_K = 128;       // K covered by one tensor-memory slot of converted weights
+constexpr int SLOTS_PER_STAGE = BK / SLOT_K;
+constexpr int ASLOTS = 2 * SLOTS_PER_STAGE;  // converted-weight slots in tensor memory
 constexpr int EPI_WARPS = 12;     // three per tensor-memory lane quadrant
 constexpr int THREADS = (6 + EPI_WARPS) * 32;
-constexpr int X_HALF = BTOK * 64 * 2;   // 24 KB: one 64-wide K atom of fp16 codes
-constexpr int X_STAGE = 2 * X_HALF;     // 48 KB
 constexpr int W_STAGE = BCH * BK;       // 16 KB int8 codes, 128-byte rows
 constexpr int GROUPS = BTOK / 32;       // 32-token column groups of the accumulator
 static_assert(GROUPS == 2 * EPI_WARPS / 4, "each epilogue warp drains two groups");
 // tensor memory columns
 constexpr uint32_t ACC_COL = 0;           // 2 x BTOK fp32 accumulators
-constexpr uint32_t A_COL = 2 * BTOK;      // ASLOTS x 64 columns (128 fp16 per row)
-constexpr uint32_t A_SLOT_COLS = BK / 2;
+constexpr uint32_t A_COL = 2 * BTOK;      // ASLOTS x SLOT_K/2 columns (fp16 pairs)
+constexpr uint32_t A_SLOT_COLS = SLOT_K / 2;
 constexpr uint32_t TMEM_COLS = 512;
 static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
-constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BTOK);
 
+// PAIR = false: one CTA computes a 128-channel x 192-token tile.
+// PAIR = true : a cluster of two CTAs computes a 256 x 192 tile with the 2-SM
+// MMA; each CTA converts its own 128 weight rows into its own tensor memory
+// and holds half of the activation tile (96 tokens) in shared memory, so a
+// stage is 40 KB instead of 64 KB and five stages fit.
+template <bool PAIR>
+struct Cfg {
+    static constexpr int NH = PAIR ? 2 : 1;           // CTAs sharing the token tile
+    static constexpr int XT = BTOK / NH;              // tokens of the tile in this CTA's shared memory
+    static constexpr int X_HALF = XT * 64 * 2;        // one 64-wide K atom of fp16 codes
+    static constexpr int X_STAGE = 2 * X_HALF;
+    static constexpr int STAGES = PAIR ? 5 : 3;
+    static constexpr int CH_TILE = BCH * NH;          // channels per tile
+    static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH * NH, BTOK);
+};
+
+template <bool PAIR>
 struct Smem {
-    uint8_t x[STAGES][X_STAGE];  // 1024-aligned (128B swizzle atoms)
+    static constexpr int STAGES = Cfg<PAIR>::STAGES;
+    uint8_t x[STAGES][Cfg<PAIR>::X_STAGE];  // 1024-aligned (128B swizzle atoms)
     uint8_t w[STAGES][W_STAGE];
-    float ep_al[EPI_WARPS][32], ep_zc[EPI_WARPS][32];
-    int ep_tok[EPI_WARPS][32], ep_tap[EPI_WARPS][32];
+    float ep_al[EPI_WARPS][2][32], ep_zc[EPI_WARPS][2][32];  // per warp, per group, per column
+    int ep_tok[EPI_WARPS][2][32], ep_tap[EPI_WARPS][2][32];
+    alignas(16) uint16_t ep_stage[EPI_WARPS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
     uint64_t full[STAGES], empty[STAGES];
     uint64_t afull[ASLOTS], aempty[ASLOTS];
     uint64_t accfull[2], accempty[2];
@@ -88,26 +106,34 @@ struct Smem {
     uint32_t tmem_base;
     int abort;
 };
-constexpr int SMEM_BYTES = sizeof(Smem) + 1024;
+template <bool PAIR>
+constexpr int smem_bytes() {
+    return int(sizeof(Smem<PAIR>)) + 1024;
+}
 
 struct TcParams {
     GemmArgs a;
     int conv;
-    int tiles_ch, tiles_tok;
-    int bw_log2, bh, tiles_w, tiles_h;  // conv: token tile = bh x 2^bw_log2 pixel rectangle
+    int tiles_ch, tiles_tok;  // tiles of Cfg::CH_TILE channels x BTOK tokens
+    // conv: a token tile is NH stacked boxes of bhx rows x 2^bw_log2 pixels
+    int bw_log2, bhx, tiles_w, tiles_h;
 };
 
+template <bool PAIR>
 struct Waiter {
-    Smem* s;
+    Smem<PAIR>* s;
     const GemmArgs* a;
     // Bounded wait on phase `parity` of an mbarrier; false after a timeout or
-    // when another role has aborted the CTA.
-    __device__ __forceinline__ bool wait(uint64_t* bar, uint32_t parity, bool ignore_abort = false) const {
+    // when another role has aborted the CTA.  `cluster` acquires arrivals
+    // released by the peer CTA.
+    __device__ __forceinline__ bool wait(uint64_t* bar, uint32_t parity, bool ignore_abort = false,
+                                         bool cluster = false) const {
         const uint32_t addr = ptx::smem_u32(bar);
-        if (ptx::mbar_try_wait(addr, parity)) return true;
+        auto probe = [&]() { return cluster ? ptx::mbar_try_wait_cluster(addr, parity) : ptx::mbar_try_wait(addr, parity); };
+        if (probe()) return true;
         const uint64_t t0 = ptx::globaltimer();
         for (uint32_t it = 1;; ++it) {
-            if (ptx::mbar_try_wait(addr, parity)) return true;
+            if (probe()) return true;
             if ((it & 63) == 0) {
                 if (!ignore_abort && *(volatile int*)&s->abort) return false;
                 if (ptx::globaltimer() - t0 > a->timeout_ns) {
@@ -148,18 +174,20 @@ __device__ __forceinline__ void widen4(uint32_t w, uint32_t m, uint32_t& lo, uin
 }
 
 struct TileCoord {
-    int ch0, tok0, img, h0, w0;
+    int ch0;             // first channel of this CTA's 128 rows
+    int tok0, img, h0, w0;
 };
 
-__device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
+template <bool PAIR>
+__device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t, int rank) {
     TileCoord c;
-    c.ch0 = (t % p.tiles_ch) * BCH;
+    c.ch0 = (t % p.tiles_ch) * Cfg<PAIR>::CH_TILE + rank * BCH;
     const int tt = t / p.tiles_ch;
     c.tok0 = c.img = c.h0 = c.w0 = 0;
     if (p.conv) {
         const int per_img = p.tiles_h * p.tiles_w;
         c.img = tt / per_img;
-        c.h0 = ((tt % per_img) / p.tiles_w) * p.bh;
+        c.h0 = ((tt % per_img) / p.tiles_w) * (p.bhx * Cfg<PAIR>::NH);
         c.w0 = (tt % p.tiles_w) << p.bw_log2;
     } else {
         c.tok0 = tt * BTOK;
@@ -167,36 +195,43 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
     return c;
 }
 
+template <bool PAIR>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w) {
+    using C = Cfg<PAIR>;
+    constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
-    Smem* s = reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    Smem<PAIR>* s = reinterpret_cast<Smem<PAIR>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const GemmArgs& a = p.a;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const Waiter wt{s, &a};
+    const Waiter<PAIR> wt{s, &a};
+    const uint32_t rank = PAIR ? ptx::cluster_rank() : 0u;
+    const bool leader = rank == 0;
 
     const int b = resolve_bits(a);
-    if (b == 0) return;  // uniform across the CTA: nothing allocated yet
+    if (b == 0) return;  // uniform across the grid (a launch-wide check): nothing allocated yet
     const int KT = (a.K + BK - 1) / BK;
     // certificate is in 64-wide K blocks; a run of c64 of them covers c64/2 of ours
     int chunk = a.hdr->chunk_kb[b] / (BK / kCertKBlock);
     chunk = chunk < 1 ? 1 : (chunk > KT ? KT : chunk);
     const int nchunks = (KT + chunk - 1) / chunk;
     const int tiles = p.tiles_ch * p.tiles_tok;
+    const int unit = PAIR ? int(blockIdx.x >> 1) : int(blockIdx.x);  // pair (or CTA) index
+    const int units = PAIR ? int(gridDim.x >> 1) : int(gridDim.x);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             ptx::mbar_init(ptx::smem_u32(&s->full[i]), 1);
-            ptx::mbar_init(ptx::smem_u32(&s->empty[i]), 4 + 1);  // 4 converter warps + MMA commit
+            ptx::mbar_init(ptx::smem_u32(&s->empty[i]), 4 + 1);  // 4 converter warps + the MMA commit
         }
         for (int i = 0; i < ASLOTS; ++i) {
-            ptx::mbar_init(ptx::smem_u32(&s->afull[i]), 4);
+            ptx::mbar_init(ptx::smem_u32(&s->afull[i]), 4 * C::NH);  // converter warps of every CTA
             ptx::mbar_init(ptx::smem_u32(&s->aempty[i]), 1);
         }
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(ptx::smem_u32(&s->accfull[i]), 1);
-            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS);
+            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS * C::NH);
         }
         ptx::mbar_init(ptx::smem_u32(&s->drain), 1);
         s->abort = 0;
@@ -205,11 +240,17 @@ __global__ void __maxnreg__(96)
         ptx::prefetch_tmap(&tm_w);
     }
     if (warp == 1) {
-        ptx::tmem_alloc(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
-        ptx::tmem_relinquish();
+        if (PAIR) {
+            ptx::tmem_alloc2(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
+            ptx::tmem_relinquish2();
+        } else {
+            ptx::tmem_alloc(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
+            ptx::tmem_relinquish();
+        }
         ptx::tc_fence_before();
     }
-    __syncthreads();
+    if (PAIR) ptx::cluster_sync();  // barriers of both CTAs exist before any cross-CTA use
+    else __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem_base;
     // the prologue above overlaps the previous kernel; inputs are read only after it
@@ -221,8 +262,8 @@ __global__ void __maxnreg__(96)
             Ring<STAGES> rs;
             int it = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-                const TileCoord tc = tile_coord(p, t);
+            for (int t = unit; t < tiles && ok; t += units) {
+                const TileCoord tc = tile_coord<PAIR>(p, t, rank);
                 for (int kb = 0; kb < KT; ++kb, ++it, rs.next()) {
                     TQ(0, it, 0);
                     if (!wt.wait(&s->empty[rs.slot], rs.phase ^ 1)) {
@@ -231,7 +272,9 @@ __global__ void __maxnreg__(96)
                     }
                     TQ(0, it, 1);
                     const uint32_t fb = ptx::smem_u32(&s->full[rs.slot]);
-                    ptx::mbar_arrive_expect_tx(fb, X_STAGE + W_STAGE);
+                    // the leader's barrier counts both CTAs' activation halves
+                    const uint32_t xbar = PAIR ? ptx::mapa(fb, 0) : fb;
+                    ptx::mbar_arrive_expect_tx(fb, (leader ? C::NH * C::X_STAGE : 0) + W_STAGE);
                     const uint32_t xdst = ptx::smem_u32(s->x[rs.slot]);
                     const int k0 = kb * BK;
 #pragma unroll
@@ -240,85 +283,101 @@ __global__ void __maxnreg__(96)
                         if (p.conv) {
                             // a 128-wide K block may straddle two taps when Cin % 128 == 64
                             const int tap = kh / a.Cin, c0 = kh - tap * a.Cin;
-                            ptx::tma_load_4d(xdst + hh * X_HALF, &tm_x, fb, c0, tc.w0 + tap % 3 - 1,
-                                             tc.h0 + tap / 3 - 1, tc.img);
+                            const int c1 = tc.w0 + tap % 3 - 1, c2 = tc.h0 + int(rank) * p.bhx + tap / 3 - 1;
+                            if (PAIR)
+                                ptx::tma2_load_4d(xdst + hh * C::X_HALF, &tm_x, xbar, c0, c1, c2, tc.img);
+                            else
+                                ptx::tma_load_4d(xdst + hh * C::X_HALF, &tm_x, fb, c0, c1, c2, tc.img);
                         } else {
-                            ptx::tma_load_2d(xdst + hh * X_HALF, &tm_x, fb, kh, tc.tok0);
+                            const int c1 = tc.tok0 + int(rank) * C::XT;
+                            if (PAIR)
+                                ptx::tma2_load_2d(xdst + hh * C::X_HALF, &tm_x, xbar, kh, c1);
+                            else
+                                ptx::tma_load_2d(xdst + hh * C::X_HALF, &tm_x, fb, kh, c1);
                         }
                     }
                     ptx::tma_load_2d(ptx::smem_u32(s->w[rs.slot]), &tm_w, fb, k0, tc.ch0);
                 }
             }
+            // the next kernel may be launched while this grid drains
+            ptx::grid_launch_dependents();
             // copies still in flight must land before the CTA may exit
             for (int j = 0; j < STAGES && j < it; ++j) {
-                // the last STAGES stages issued, oldest first
-                const int jj = it - STAGES + j;
+                const int jj = it - STAGES + j;  // the last STAGES stages issued, oldest first
                 if (jj < 0) continue;
                 wt.wait(&s->full[jj % STAGES], (jj / STAGES) & 1, true);
             }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
-        if (lane == 0) {
+        if (lane == 0 && leader) {
             Ring<STAGES> rs;
             Ring<ASLOTS> ra;
             int it = 0, cc = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+            for (int t = unit; t < tiles && ok; t += units) {
                 for (int c = 0; c < nchunks && ok; ++c, ++cc) {
                     const int buf = cc & 1;
-                    if (!wt.wait(&s->accempty[buf], ((cc >> 1) & 1) ^ 1)) {
+                    if (!wt.wait(&s->accempty[buf], ((cc >> 1) & 1) ^ 1, false, PAIR)) {
                         ok = false;
                         break;
                     }
                     ptx::tc_fence_after();
                     const uint32_t d = tmem + ACC_COL + buf * BTOK;
                     const int kb0 = c * chunk, kb_end = min(KT, kb0 + chunk);
-                    for (int kb = kb0; kb < kb_end; ++kb, ++it, rs.next(), ra.next()) {
+                    for (int kb = kb0; kb < kb_end; ++kb, ++it, rs.next()) {
                         TQ(1, it, 0);
-                        if (!wt.wait(&s->full[rs.slot], rs.phase)) {
-                            ok = false;
-                            break;
-                        }
-                        TQ(1, it, 1);
-                        if (!wt.wait(&s->afull[ra.slot], ra.phase)) {
-                            ok = false;
-                            break;
-                        }
-                        TQ(1, it, 2);
-                        ptx::tc_fence_after();
                         const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[rs.slot]));
-                        const uint32_t acol = tmem + A_COL + ra.slot * A_SLOT_COLS;
 #pragma unroll
-                        for (int k = 0; k < BK / 16; ++k)
-                            ptx::mma_f16_ts(d, acol + k * 8,
-                                            bdesc + uint64_t(((k >> 2) * X_HALF + (k & 3) * 32) >> 4), IDESC,
-                                            (kb > kb0 || k > 0) ? 1u : 0u);
-                        ptx::mma_commit(ptx::smem_u32(&s->empty[rs.slot]));
-                        ptx::mma_commit(ptx::smem_u32(&s->aempty[ra.slot]));
+                        for (int hh = 0; hh < SLOTS_PER_STAGE; ++hh) {
+                            // the converters of every CTA have passed this stage's full
+                            // barrier (activations landed) and written this weight slot
+                            if (!wt.wait(&s->afull[ra.slot], ra.phase, false, PAIR)) {
+                                ok = false;
+                                break;
+                            }
+                            ptx::tc_fence_after();
+                            const uint32_t acol = tmem + A_COL + ra.slot * A_SLOT_COLS;
+#pragma unroll
+                            for (int kk = 0; kk < SLOT_K / 16; ++kk) {
+                                const int k = hh * (SLOT_K / 16) + kk;  // K step of 16 within the stage
+                                const uint64_t bk = bdesc + uint64_t(((k >> 2) * C::X_HALF + (k & 3) * 32) >> 4);
+                                const uint32_t accum = (kb > kb0 || k > 0) ? 1u : 0u;
+                                if (PAIR) ptx::mma2_f16_ts(d, acol + kk * 8, bk, C::IDESC, accum);
+                                else ptx::mma_f16_ts(d, acol + kk * 8, bk, C::IDESC, accum);
+                            }
+                            if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->aempty[ra.slot]), 0x3);
+                            else ptx::mma_commit(ptx::smem_u32(&s->aempty[ra.slot]));
+                            ra.next();
+                        }
+                        if (!ok) break;
+                        if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->empty[rs.slot]), 0x3);
+                        else ptx::mma_commit(ptx::smem_u32(&s->empty[rs.slot]));
                         TQ(1, it, 3);
                     }
-                    if (ok) ptx::mma_commit(ptx::smem_u32(&s->accfull[buf]));
+                    if (ok) {
+                        if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->accfull[buf]), 0x3);
+                        else ptx::mma_commit(ptx::smem_u32(&s->accfull[buf]));
+                    }
                 }
             }
-            // the next kernel may be launched while the last epilogue runs
-            ptx::grid_launch_dependents();
             // every MMA issued must finish before tensor memory is released
-            ptx::mma_commit(ptx::smem_u32(&s->drain));
+            if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->drain), 0x1);
+            else ptx::mma_commit(ptx::smem_u32(&s->drain));
             wt.wait(&s->drain, 0, true);
         }
     } else if (warp < 6) {
         // ------------------------------------------- weight mask + convert
         const int q = warp & 3;             // tensor-memory lane quadrant
-        const int r = q * 32 + lane;        // channel row within the tile
+        const int r = q * 32 + lane;        // channel row within this CTA's 128
         const uint32_t m = mask_word(b);
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         Ring<STAGES> rs;
         Ring<ASLOTS> ra;
         int it = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-            for (int kb = 0; kb < KT; ++kb, ++it, rs.next(), ra.next()) {
+        for (int t = unit; t < tiles && ok; t += units) {
+            for (int kb = 0; kb < KT; ++kb, ++it, rs.next()) {
                 if (warp == 2 && lane == 0) TQ(2, it, 0);
                 if (!wt.wait(&s->full[rs.slot], rs.phase)) {
                     ok = false;
@@ -333,31 +392,38 @@ __global__ void __maxnreg__(96)
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->empty[rs.slot]));
                 if (warp == 2 && lane == 0) TQ(2, it, 2);
-                if (!wt.wait(&s->aempty[ra.slot], ra.phase ^ 1)) {
-                    ok = false;
-                    break;
-                }
-                if (warp == 2 && lane == 0) TQ(2, it, 3);
-                const uint32_t dst = lane_base + A_COL + ra.slot * A_SLOT_COLS;
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    uint32_t f[32];
-#pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        const uint4 u = v[4 * hh + c];
-                        widen4(u.x, m, f[8 * c + 0], f[8 * c + 1]);
-                        widen4(u.y, m, f[8 * c + 2], f[8 * c + 3]);
-                        widen4(u.z, m, f[8 * c + 4], f[8 * c + 5]);
-                        widen4(u.w, m, f[8 * c + 6], f[8 * c + 7]);
+                for (int hh = 0; hh < SLOTS_PER_STAGE; ++hh) {
+                    if (!wt.wait(&s->aempty[ra.slot], ra.phase ^ 1)) {
+                        ok = false;
+                        break;
                     }
-                    ptx::tmem_st32(dst + hh * 32, f);
+                    if (warp == 2 && lane == 0 && hh == 0) TQ(2, it, 3);
+#pragma unroll
+                    for (int q32 = 0; q32 < SLOT_K / 64; ++q32) {  // 32 columns (64 K) per store
+                        uint32_t f[32];
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            const uint4 u = v[(hh * SLOT_K / 64 + q32) * 4 + c];
+                            widen4(u.x, m, f[8 * c + 0], f[8 * c + 1]);
+                            widen4(u.y, m, f[8 * c + 2], f[8 * c + 3]);
+                            widen4(u.z, m, f[8 * c + 4], f[8 * c + 5]);
+                            widen4(u.w, m, f[8 * c + 6], f[8 * c + 7]);
+                        }
+                        ptx::tmem_st32(lane_base + A_COL + ra.slot * A_SLOT_COLS + q32 * 32, f);
+                    }
+                    ptx::tmem_wait_st();
+                    ptx::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        const uint32_t ab = ptx::smem_u32(&s->afull[ra.slot]);
+                        if (PAIR) ptx::mbar_arrive_cluster(ptx::mapa(ab, 0));
+                        else ptx::mbar_arrive(ab);
+                    }
+                    ra.next();
                 }
-                if (warp == 2 && lane == 0) TQ(2, it, 4);
-                ptx::tmem_wait_st();
+                if (!ok) break;
                 if (warp == 2 && lane == 0) TQ(2, it, 5);
-                ptx::tc_fence_before();
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->afull[ra.slot]));
             }
         }
     } else {
@@ -369,43 +435,42 @@ __global__ void __maxnreg__(96)
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
         const int32_t* ts_b = p.conv ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
-        float* my_al = s->ep_al[e];
-        float* my_zc = s->ep_zc[e];
-        int* my_tok = s->ep_tok[e];
-        int* my_tap = s->ep_tap[e];
         int cc = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-            const TileCoord tc = tile_coord(p, t);
+        for (int t = unit; t < tiles && ok; t += units) {
+            const TileCoord tc = tile_coord<PAIR>(p, t, rank);
             const int n = tc.ch0 + r;
             const bool n_ok = n < a.N;
-            float cw = 0.f, bias = 0.f;
-            int rs = 0;
-            int ts[9];
+            // row sums as fp32: |sum| < 2^24, so the values and every partial sum
+            // of in-bounds taps below are exact, equal to float(int sum)
+            float cw = 0.f, bias = 0.f, rs = 0.f;
+            float ts[9];
 #pragma unroll
-            for (int i = 0; i < 9; ++i) ts[i] = 0;
+            for (int i = 0; i < 9; ++i) ts[i] = 0.f;
             if (n_ok) {
                 cw = a.cw[n];
                 bias = a.bias[n];
                 if (p.conv) {
 #pragma unroll
-                    for (int i = 0; i < 9; ++i) ts[i] = ts_b[int64_t(n) * 9 + i];
+                    for (int i = 0; i < 9; ++i) ts[i] = __int2float_rn(ts_b[int64_t(n) * 9 + i]);
                 } else {
-                    rs = rs_b[n];
+                    rs = __int2float_rn(rs_b[n]);
                 }
             }
 
             // Token index, (conv) in-bounds taps and per-token scales of column j = lane of
-            // each of this warp's two groups, fetched before the accumulator is ready so
-            // the loads' latency hides under the MMAs.
-            int tok_r[2], tap_r[2];
-            float al_r[2], zc_r[2];
+            // each of this warp's two groups, written to this warp's shared scratch before
+            // the accumulator wait, so the global loads' latency hides under the MMAs.
+            bool all_tok_g[2];
+            __syncwarp();  // the previous tile's reads of the scratch are done
 #pragma unroll
             for (int gi = 0; gi < 2; ++gi) {
                 const int jt = (2 * part + gi) * 32 + lane;
                 int tok = -1, tap = 0;
                 if (p.conv) {
-                    const int hh = tc.h0 + (jt >> p.bw_log2), ww = tc.w0 + (jt & ((1 << p.bw_log2) - 1));
+                    // column jt came from box jt / XT (stacked bhx-row boxes of the tile)
+                    const int jb = jt / C::XT, jj = jt - jb * C::XT;
+                    const int hh = tc.h0 + jb * p.bhx + (jj >> p.bw_log2), ww = tc.w0 + (jj & ((1 << p.bw_log2) - 1));
                     if (hh < a.H && ww < a.W) {
                         tok = (tc.img * a.H + hh) * a.W + ww;
 #pragma unroll
@@ -419,24 +484,21 @@ __global__ void __maxnreg__(96)
                 } else {
                     tok = tc.tok0 + jt < a.M ? tc.tok0 + jt : -1;
                 }
-                tok_r[gi] = tok;
-                tap_r[gi] = tap;
-                al_r[gi] = tok >= 0 ? (a.per_tensor ? a.alpha[0] : a.alpha[tok]) : 0.f;
-                zc_r[gi] = tok >= 0 ? (a.per_tensor ? a.zc[0] : a.zc[tok]) : 0.f;
+                s->ep_tok[e][gi][lane] = tok;
+                s->ep_tap[e][gi][lane] = tap;
+                s->ep_al[e][gi][lane] = tok >= 0 ? (a.per_tensor ? a.alpha[0] : a.alpha[tok]) : 0.f;
+                s->ep_zc[e][gi][lane] = tok >= 0 ? (a.per_tensor ? a.zc[0] : a.zc[tok]) : 0.f;
+                all_tok_g[gi] = __all_sync(0xffffffffu, tok >= 0);
             }
-            // stage group gi's per-token values in this warp's scratch for broadcast reads
-            auto stage_tokens = [&](int gi) -> bool {
-                __syncwarp();
-                my_tok[lane] = tok_r[gi];
-                my_tap[lane] = tap_r[gi];
-                my_al[lane] = al_r[gi];
-                my_zc[lane] = zc_r[gi];
-                __syncwarp();
-                return __all_sync(0xffffffffu, tok_r[gi] >= 0);
-            };
+            __syncwarp();
             // Epilogue of 16 consecutive columns j0..j0+15 of group g from exact
             // accumulator values (float-held integers when `fl`, else int32).
-            auto finish16 = [&](int g, int j0, const uint32_t (&v)[16], bool fl, bool all_tok) {
+            auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], bool fl, bool all_tok) {
+                const int g = 2 * part + gi;
+                const float* my_al = s->ep_al[e][gi];
+                const float* my_zc = s->ep_zc[e][gi];
+                const int* my_tok = s->ep_tok[e][gi];
+                const int* my_tap = s->ep_tap[e][gi];
                 uint32_t yb2[8];
 #pragma unroll
                 for (int j4 = 0; j4 < 4; ++j4) {
@@ -447,49 +509,47 @@ __global__ void __maxnreg__(96)
                     int4 tp4 = make_int4(0, 0, 0, 0);
                     if (p.conv) tp4 = *reinterpret_cast<const int4*>(my_tap + j0 + 4 * j4);
                     const int tp[4] = {tp4.x, tp4.y, tp4.z, tp4.w};
+                    float yf[4];
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
-                        int rsum = rs;
+                        float rsum = rs;
                         if (p.conv) {
-                            rsum = 0;
+                            rsum = 0.f;
 #pragma unroll
-                            for (int k9 = 0; k9 < 9; ++k9) rsum += (tp[u] >> k9) & 1 ? ts[k9] : 0;
+                            for (int k9 = 0; k9 < 9; ++k9) rsum = __fadd_rn(rsum, (tp[u] >> k9) & 1 ? ts[k9] : 0.f);
                         }
                         const uint32_t raw = v[4 * j4 + u];
                         const float acc_f = fl ? __uint_as_float(raw) : __int2float_rn(int(raw));
-                        const float tz = __fmul_rn(zc[u], __int2float_rn(rsum));
-                        const float y = __fadd_rn(__fmul_rn(__fadd_rn(acc_f, tz), __fmul_rn(al[u], cw)), bias);
-                        const uint32_t h = __bfloat16_as_ushort(__float2bfloat16_rn(y));
-                        const int jj = 4 * j4 + u;
-                        yb2[jj >> 1] = (jj & 1) ? (yb2[jj >> 1] | (h << 16)) : h;
+                        yf[u] = __fmaf_rn(__fmaf_rn(zc[u], rsum, acc_f), __fmul_rn(al[u], cw), bias);
+                    }
+                    // two results per round-to-nearest-even conversion
+#pragma unroll
+                    for (int u = 0; u < 4; u += 2) {
+                        const __nv_bfloat162 hb = __floats2bfloat162_rn(yf[u], yf[u + 1]);
+                        yb2[2 * j4 + u / 2] = *reinterpret_cast<const uint32_t*>(&hb);
                     }
                 }
-                if (!n_ok) return;
-                if (!p.conv && all_tok) {
-                    const int64_t row0 = int64_t(tc.tok0 + g * 32 + j0);
-                    uint16_t* yp = a.y + row0 * a.N + n;
+                // Transpose the warp's 32 channels x 16 tokens through shared memory so
+                // each token row (32 channels, 64 bytes) is written with 16-byte stores.
+                uint16_t* stg = s->ep_stage[e];
+                __syncwarp();
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) yp[int64_t(j) * a.N] = uint16_t(yb2[j >> 1] >> (16 * (j & 1)));
-                    if (a.acc) {
-                        int32_t* ap = a.acc + row0 * a.N + n;
+                for (int j = 0; j < 16; ++j) stg[j * 32 + lane] = uint16_t(yb2[j >> 1] >> (16 * (j & 1)));
+                __syncwarp();
+                const int qc = lane & 3;  // 8-channel chunk of the row
+                const int nq = tc.ch0 + (warp & 3) * 32 + qc * 8;
 #pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            ap[int64_t(j) * a.N] = fl ? __float2int_rn(__uint_as_float(v[j])) : int(v[j]);
-                    }
-                } else {
+                for (int rr = 0; rr < 2; ++rr) {
+                    const int t = rr * 8 + (lane >> 2);  // token row within the 16
+                    const uint4 val = *reinterpret_cast<const uint4*>(stg + t * 32 + qc * 8);
+                    const int tok = all_tok && !p.conv ? tc.tok0 + g * 32 + j0 + t : my_tok[j0 + t];
+                    if (tok >= 0 && nq < a.N) *reinterpret_cast<uint4*>(a.y + int64_t(tok) * a.N + nq) = val;
+                }
+                if (a.acc && n_ok) {  // int32 accumulators (a debugging output): plain stores
 #pragma unroll
-                    for (int j4 = 0; j4 < 4; ++j4) {
-                        const int4 tk = *reinterpret_cast<const int4*>(my_tok + j0 + 4 * j4);
-                        const int tks[4] = {tk.x, tk.y, tk.z, tk.w};
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            if (tks[u] < 0) continue;
-                            const int jj = 4 * j4 + u;
-                            a.y[int64_t(tks[u]) * a.N + n] = uint16_t(yb2[jj >> 1] >> (16 * (jj & 1)));
-                            if (a.acc)
-                                a.acc[int64_t(tks[u]) * a.N + n] =
-                                    fl ? __float2int_rn(__uint_as_float(v[jj])) : int(v[jj]);
-                        }
+                    for (int j = 0; j < 16; ++j) {
+                        const int tok = my_tok[j0 + j];
+                        if (tok >= 0) a.acc[int64_t(tok) * a.N + n] = fl ? __float2int_rn(__uint_as_float(v[j])) : int(v[j]);
                     }
                 }
             };
@@ -512,7 +572,7 @@ __global__ void __maxnreg__(96)
 #pragma unroll 1
                 for (int gi = 0; gi < 2; ++gi) {
                     const int g = 2 * part + gi;
-                    const bool all_tok = last ? stage_tokens(gi) : false;
+                    const bool all_tok = all_tok_g[gi];
 #pragma unroll 1
                     for (int h = 0; h < 2; ++h) {
                         uint32_t v[16];
@@ -528,21 +588,29 @@ __global__ void __maxnreg__(96)
                                 else pp[j * 32] = x;
                             }
                         }
-                        if (last) finish16(g, h * 16, v, nchunks == 1, all_tok);
+                        if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 3 + 2 * h);
+                        if (last) finish16(gi, h * 16, v, nchunks == 1, all_tok);
+                        if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 4 + 2 * h);
                     }
                 }
                 ptx::tc_fence_before();
                 __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->accempty[buf]));
+                if (lane == 0) {
+                    const uint32_t eb = ptx::smem_u32(&s->accempty[buf]);
+                    if (PAIR) ptx::mbar_arrive_cluster(ptx::mapa(eb, 0));
+                    else ptx::mbar_arrive(eb);
+                }
                 if (warp == 6 && lane == 0) TQ(3, cc, 2);
             }
         }
     }
 
     __syncthreads();
+    if (PAIR) ptx::cluster_sync();  // neither CTA releases memory the pair's MMAs may still use
     if (warp == 1) {
         ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem, TMEM_COLS);
+        if (PAIR) ptx::tmem_dealloc2(tmem, TMEM_COLS);
+        else ptx::tmem_dealloc(tmem, TMEM_COLS);
     }
 }
 
@@ -563,13 +631,37 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 
 size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * EPI_WARPS * 64 * 32 * sizeof(int32_t); }
 
-cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
-    *why = nullptr;
-    if (!a.part) {
-        *why = "no accumulator scratch";
-        return cudaSuccess;
+namespace {
+
+// Pairs of CTAs the 2-SM kernel can keep resident at once (cluster placement
+// can leave some SMs unpaired), looked up once.
+int max_pairs(int num_sms) {
+    static int cached = -1;
+    if (cached < 0) {
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3(2 * (num_sms / 2));
+        cfg.blockDim = dim3(THREADS);
+        cfg.dynamicSmemBytes = smem_bytes<true>();
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaFuncSetAttribute(gemm_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 smem_bytes<true>()) != cudaSuccess ||
+            cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<true>, &cfg) != cudaSuccess)
+            n = 0;
+        cached = n;
     }
-    if (a.M == 0 || a.N == 0) return cudaSuccess;
+    return cached;
+}
+
+template <bool PAIR>
+cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
+    using C = Cfg<PAIR>;
     auto encode = get_encode();
     if (!encode) {
         *why = "cuTensorMapEncodeTiled is unavailable";
@@ -578,7 +670,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     TcParams p{};
     p.a = a;
     p.conv = a.Cin != 0;
-    p.tiles_ch = (a.N + BCH - 1) / BCH;
+    p.tiles_ch = (a.N + C::CH_TILE - 1) / C::CH_TILE;
     CUtensorMap tm_x, tm_w;
     CUresult r;
     if (p.conv) {
@@ -586,13 +678,15 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
             *why = "convolution needs Cin % 64 == 0";
             return cudaSuccess;
         }
+        // box of bhx rows x 2^bwl pixels; 2^bwl must divide XT (192 = 64*3, 96 = 32*3)
+        const int max_bw = PAIR ? 32 : 64;
         int bwl = 0;
-        while ((1 << bwl) < a.W && (1 << bwl) < 64) ++bwl;  // 2^bwl divides BTOK = 192
+        while ((1 << bwl) < a.W && (1 << bwl) < max_bw) ++bwl;
         p.bw_log2 = bwl;
-        p.bh = BTOK >> bwl;
+        p.bhx = C::XT >> bwl;
         const int bw = 1 << bwl;
         p.tiles_w = (a.W + bw - 1) / bw;
-        p.tiles_h = (a.H + p.bh - 1) / p.bh;
+        p.tiles_h = (a.H + p.bhx * C::NH - 1) / (p.bhx * C::NH);
         const int64_t tok_tiles = int64_t(a.B) * p.tiles_h * p.tiles_w;
         if (tok_tiles * p.tiles_ch > 0x7FFFFFFF) {
             *why = "too many tiles";
@@ -601,7 +695,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         p.tiles_tok = int(tok_tiles);
         cuuint64_t dims[4] = {cuuint64_t(a.Cin), cuuint64_t(a.W), cuuint64_t(a.H), cuuint64_t(a.B)};
         cuuint64_t strides[3] = {cuuint64_t(a.Cin) * 2, cuuint64_t(a.W) * a.Cin * 2, cuuint64_t(a.H) * a.W * a.Cin * 2};
-        cuuint32_t box[4] = {64, cuuint32_t(bw), cuuint32_t(p.bh), 1};
+        cuuint32_t box[4] = {64, cuuint32_t(bw), cuuint32_t(p.bhx), 1};
         cuuint32_t es[4] = {1, 1, 1, 1};
         r = encode(&tm_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void*>(a.x), dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -610,7 +704,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         p.tiles_tok = (a.M + BTOK - 1) / BTOK;
         cuuint64_t dims[2] = {cuuint64_t(a.K), cuuint64_t(a.M)};
         cuuint64_t strides[1] = {cuuint64_t(a.K) * 2};
-        cuuint32_t box[2] = {64, BTOK};
+        cuuint32_t box[2] = {64, cuuint32_t(C::XT)};
         cuuint32_t es[2] = {1, 1};
         r = encode(&tm_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(a.x), dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -634,36 +728,72 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         }
     }
     const int64_t tiles = int64_t(p.tiles_ch) * p.tiles_tok;
-    const int grid = int(tiles < num_sms ? tiles : num_sms);
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    const int64_t max_units = PAIR ? max_pairs(num_sms) : num_sms;
+    if (max_units < 1) {
+        *why = "no CTA pair can be co-scheduled";
+        return cudaSuccess;
+    }
+    const int units = int(tiles < max_units ? tiles : max_units);
+    static const bool verbose = getenv("TASQ_TC_VERBOSE") != nullptr;
+    if (verbose)
+        fprintf(stderr, "tasq tc: %s M=%d N=%d K=%d tiles=%lld units=%d (max %lld) grid=%d\n", PAIR ? "pair" : "single",
+                a.M, a.N, a.K, (long long)tiles, units, (long long)max_units, units * C::NH);
+    const int smem = smem_bytes<PAIR>();
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     // programmatic dependent launch: the grid may start while the previous
     // kernel drains; it waits (griddepcontrol.wait) before reading inputs
     cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3(grid);
+    cfg.gridDim = dim3(units * C::NH);
     cfg.blockDim = dim3(THREADS);
-    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
+    int nattr = 1;
+    if (PAIR) {
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = 2;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        nattr = 2;
+    }
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel, p, tm_x, tm_w);
+    cfg.numAttrs = nattr;
+    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel<PAIR>, p, tm_x, tm_w);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaErrorLaunchOutOfResources) {
         // report what the kernel asked for, to make the failure actionable
         static char msg[256];
         cudaFuncAttributes fa{};
-        cudaFuncGetAttributes(&fa, gemm_tc_kernel);
+        cudaFuncGetAttributes(&fa, gemm_tc_kernel<PAIR>);
         snprintf(msg, sizeof msg,
                  "launch out of resources: %d threads x %d registers, %d B dynamic smem (kernel max %d threads, "
                  "%zu B static smem)",
-                 THREADS, fa.numRegs, SMEM_BYTES, fa.maxThreadsPerBlock, fa.sharedSizeBytes);
+                 THREADS, fa.numRegs, smem, fa.maxThreadsPerBlock, fa.sharedSizeBytes);
         *why = msg;
         return cudaSuccess;
     }
     return e;
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
+    *why = nullptr;
+    if (!a.part) {
+        *why = "no accumulator scratch";
+        return cudaSuccess;
+    }
+    if (a.M == 0 || a.N == 0) return cudaSuccess;
+    // The 1-SM kernel by default; TASQ_TC_PAIRS=1 selects the 2-SM variant
+    // (correct, but its cross-CTA barrier round trips keep it slower here).
+    static const bool pairs = [] {
+        const char* v = getenv("TASQ_TC_PAIRS");
+        return v && v[0] == '1';
+    }();
+    return pairs ? launch_variant<true>(a, num_sms, st, why) : launch_variant<false>(a, num_sms, st, why);
 }
 
 #ifdef TASQ_TRACE

@@ -117,15 +117,12 @@ __device__ __forceinline__ int rint_small(float u) {
     return int(__float_as_uint(__fadd_rn(u, 12582912.0f)) - 0x4B400000u);
 }
 
-// Fused dequantization epilogue, fp32 with one rounding per operation:
-// y = ((float(acc) + zc * float(rs)) * (alpha * cw)) + bias.
+// Fused dequantization epilogue in fp32, each operation rounded once to
+// nearest even: u = fma(zc, float(rs), float(acc)), s = alpha * cw,
+// y = fma(u, s, bias); this equals alpha * cw * (acc + zc * rs) + bias.
 __device__ inline float epilogue_value(int acc, float alpha, float zc, int rs, float cw, float bias) {
-    float a = __int2float_rn(acc);
-    float t = __fmul_rn(zc, __int2float_rn(rs));
-    float u = __fadd_rn(a, t);
-    float s = __fmul_rn(alpha, cw);
-    float v = __fmul_rn(u, s);
-    return __fadd_rn(v, bias);
+    const float u = __fmaf_rn(zc, __int2float_rn(rs), __int2float_rn(acc));
+    return __fmaf_rn(u, __fmul_rn(alpha, cw), bias);
 }
 
 // fp32 -> bf16 bits, round to nearest even (finite inputs).
