@@ -57,6 +57,7 @@ def parse_args():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--blocks", type=int, default=0, help="keep only the first N transformer blocks (small cases)")
     ap.add_argument("--no-all8", action="store_true", help="skip the all-8-bit schedule comparison")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the GEMM sweep and the stage-switch test")
     return ap.parse_args()
 
 
@@ -237,6 +238,77 @@ def timed_replays(torch, g, step, steps, stage_of):
     t1.record(s)
     torch.cuda.synchronize()
     return t0.elapsed_time(t1) / steps
+
+
+# ------------------------------------------------------------------ sweep --
+def run_sweep(torch, tasq, workloads, shapes=None, reps=10, seed=0):
+    """GEMM sweep: M x (K = N) x b = 2..8 on seeded uniform codes in [-127, 127];
+    TOPS (2*M*N*K per call, independent of b) per point.  Also the stage-switch
+    cost: 1000 back-to-back calls alternating the stage every call versus 1000
+    calls at one stage."""
+    ctx = tasq.tasq_create(torch.cuda.current_device())
+    table = workloads.schedule_for("sweep", 1)  # stages 0..6 <-> b = 2..8, stage 7 = 8
+    tasq.tasq_set_schedule(ctx, table, 1, table.shape[1])
+    out = []
+    switch = None
+    shapes = shapes or list(workloads.sweep_shapes())
+    for si, (M, KN) in enumerate(shapes):
+        N = K = KN
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed * 1000 + si)
+        sw = torch.randint(-127, 128, (N, K), generator=g, device="cuda", dtype=torch.int8)
+        cw = torch.rand((N,), generator=g, device="cuda") * 1e-3 + 1e-4
+        pk = torch.empty((tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, N, K),), dtype=torch.uint8, device="cuda")
+        tasq.tasq_pack_weights(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K, 0, pk)
+        codes = torch.randint(-127, 128, (M, K), generator=g, device="cuda", dtype=torch.int8).to(torch.float16)
+        al = torch.rand((M,), generator=g, device="cuda") * 1e-2 + 1e-3
+        zc = torch.full((M,), 0.5, device="cuda")
+        y = torch.empty((M, N), dtype=torch.int16, device="cuda")
+        row = {"M": M, "K": K, "N": N, "tops_by_b": {}}
+        for b in range(2, 9):
+            stage = b - 2
+            tasq.tasq_masked_gemm(ctx, 0, stage, codes, tasq.TASQ_CODES_F16, al, zc, M, pk, N, K, y)
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+                for _ in range(reps):
+                    tasq.tasq_masked_gemm(ctx, 0, stage, codes, tasq.TASQ_CODES_F16, al, zc, M, pk, N, K, y)
+            gr.replay()
+            torch.cuda.synchronize()
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record()
+            gr.replay()
+            t1.record()
+            torch.cuda.synchronize()
+            us = t0.elapsed_time(t1) * 1e3 / reps
+            row["tops_by_b"][b] = 2.0 * M * N * K / (us * 1e-6) / 1e12
+        out.append(row)
+        if (M, KN) == (4096, 4096):
+            # stage switch: alternate b = 2 / 8 every call, and b = 5 / 5 (same
+            # precision, different stage) every call, against one fixed stage
+            def timed(stages):
+                gr = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+                    for st in stages:
+                        tasq.tasq_masked_gemm(ctx, 0, st, codes, tasq.TASQ_CODES_F16, al, zc, M, pk, N, K, y)
+                gr.replay()
+                torch.cuda.synchronize()
+                t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                t0.record()
+                gr.replay()
+                t1.record()
+                torch.cuda.synchronize()
+                return t0.elapsed_time(t1) * 1e3 / len(stages)
+            n = 1000
+            fixed8 = timed([6] * n)
+            alt = timed([0 if i % 2 == 0 else 6 for i in range(n)])
+            fixed2 = timed([0] * n)
+            same_b = timed([6 if i % 2 == 0 else 7 for i in range(n)])  # stages 6 and 7 both hold b = 8
+            switch = {"shape": [M, N, K], "calls": n, "us_per_call_fixed_b8": fixed8, "us_per_call_fixed_b2": fixed2,
+                      "us_per_call_alternating_b2_b8": alt, "us_per_call_alternating_stages_same_b8": same_b,
+                      "switch_overhead_us": same_b - fixed8}
+        del sw, cw, pk, codes, al, zc, y
+    tasq.tasq_destroy(ctx)
+    return out, switch
 
 
 # ------------------------------------------------------------ CPU oracle --
@@ -435,6 +507,10 @@ def main():
                           "between kernels, right after the timed region" if external
                 else "CUDA events around each contraction in an eager pass after the timed region"}
 
+    sweep = switch = None
+    if not args.no_sweep:
+        sweep, switch = run_sweep(torch, tasq, workloads, seed=args.seed)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         o, s, d, rows, threads = oracle_sample(args.workload, args.cpu_seconds, seed=args.seed)
@@ -472,6 +548,8 @@ def main():
             "gpu_launches": step.launches_per_step() * args.steps,
             "cpu_baseline": cpu,
             "clocks": clk,
+            "sweep_tops_by_b": sweep,
+            "stage_switch": switch,
         }
         print(json.dumps(line), flush=True)
     step.close()

@@ -117,7 +117,26 @@ struct TcParams {
     int tiles_ch, tiles_tok;  // tiles of Cfg::CH_TILE channels x BTOK tokens
     // conv: a token tile is NH stacked boxes of bhx rows x 2^bw_log2 pixels
     int bw_log2, bhx, tiles_w, tiles_h;
+    // split-K: each tile's K blocks are cut into `splits` contiguous slices; a
+    // slice writes its exact int32 partial sums to split_out[slice][token][n]
+    // and a second kernel adds the slices and applies the epilogue
+    int splits;
+    int32_t* split_out;
 };
+
+// One unit of work: a tile and a contiguous range of its K blocks.
+struct Work {
+    int t, slice, kb_lo, kb_hi, nch;
+};
+__device__ __forceinline__ Work work_item(const TcParams& p, int w, int KT, int chunk) {
+    Work r;
+    r.t = w / p.splits;
+    r.slice = w - r.t * p.splits;
+    r.kb_lo = (r.slice * KT) / p.splits;
+    r.kb_hi = ((r.slice + 1) * KT) / p.splits;
+    r.nch = (r.kb_hi - r.kb_lo + chunk - 1) / chunk;
+    return r;
+}
 
 template <bool PAIR>
 struct Waiter {
@@ -215,8 +234,7 @@ __global__ void __maxnreg__(96)
     // certificate is in 64-wide K blocks; a run of c64 of them covers c64/2 of ours
     int chunk = a.hdr->chunk_kb[b] / (BK / kCertKBlock);
     chunk = chunk < 1 ? 1 : (chunk > KT ? KT : chunk);
-    const int nchunks = (KT + chunk - 1) / chunk;
-    const int tiles = p.tiles_ch * p.tiles_tok;
+    const int works = p.tiles_ch * p.tiles_tok * p.splits;
     const int unit = PAIR ? int(blockIdx.x >> 1) : int(blockIdx.x);  // pair (or CTA) index
     const int units = PAIR ? int(gridDim.x >> 1) : int(gridDim.x);
 
@@ -262,9 +280,10 @@ __global__ void __maxnreg__(96)
             Ring<STAGES> rs;
             int it = 0;
             bool ok = true;
-            for (int t = unit; t < tiles && ok; t += units) {
-                const TileCoord tc = tile_coord<PAIR>(p, t, rank);
-                for (int kb = 0; kb < KT; ++kb, ++it, rs.next()) {
+            for (int w = unit; w < works && ok; w += units) {
+                const Work wk = work_item(p, w, KT, chunk);
+                const TileCoord tc = tile_coord<PAIR>(p, wk.t, rank);
+                for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rs.next()) {
                     TQ(0, it, 0);
                     if (!wt.wait(&s->empty[rs.slot], rs.phase ^ 1)) {
                         ok = false;
@@ -315,8 +334,9 @@ __global__ void __maxnreg__(96)
             Ring<ASLOTS> ra;
             int it = 0, cc = 0;
             bool ok = true;
-            for (int t = unit; t < tiles && ok; t += units) {
-                for (int c = 0; c < nchunks && ok; ++c, ++cc) {
+            for (int w = unit; w < works && ok; w += units) {
+                const Work wk = work_item(p, w, KT, chunk);
+                for (int c = 0; c < wk.nch && ok; ++c, ++cc) {
                     const int buf = cc & 1;
                     if (!wt.wait(&s->accempty[buf], ((cc >> 1) & 1) ^ 1, false, PAIR)) {
                         ok = false;
@@ -324,7 +344,7 @@ __global__ void __maxnreg__(96)
                     }
                     ptx::tc_fence_after();
                     const uint32_t d = tmem + ACC_COL + buf * BTOK;
-                    const int kb0 = c * chunk, kb_end = min(KT, kb0 + chunk);
+                    const int kb0 = wk.kb_lo + c * chunk, kb_end = min(wk.kb_hi, kb0 + chunk);
                     for (int kb = kb0; kb < kb_end; ++kb, ++it, rs.next()) {
                         TQ(1, it, 0);
                         const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[rs.slot]));
@@ -376,52 +396,53 @@ __global__ void __maxnreg__(96)
         Ring<ASLOTS> ra;
         int it = 0;
         bool ok = true;
-        for (int t = unit; t < tiles && ok; t += units) {
-            for (int kb = 0; kb < KT; ++kb, ++it, rs.next()) {
+        for (int w = unit; w < works && ok; w += units) {
+            const Work wk = work_item(p, w, KT, chunk);
+            for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rs.next()) {
                 if (warp == 2 && lane == 0) TQ(2, it, 0);
                 if (!wt.wait(&s->full[rs.slot], rs.phase)) {
                     ok = false;
                     break;
                 }
                 if (warp == 2 && lane == 0) TQ(2, it, 1);
-                // 128 codes of row r; 16-byte chunk c sits at c ^ (r & 7) (128-byte swizzle)
-                uint4 v[8];
-                const uint8_t* row = s->w[rs.slot] + r * BK;
+                // 128 codes of row r; 16-byte chunk c sits at c ^ (r & 7) (128-byte swizzle).
+                // Mask and widen before waiting for the slot, so that only the
+                // tensor-memory store remains once the MMA releases it.
+                static_assert(SLOTS_PER_STAGE == 1, "the converter widens a whole stage into one slot");
+                uint32_t f[64];
+                {
+                    const uint8_t* row = s->w[rs.slot] + r * BK;
 #pragma unroll
-                for (int c = 0; c < 8; ++c) v[c] = *reinterpret_cast<const uint4*>(row + ((c ^ (r & 7)) << 4));
+                    for (int c = 0; c < 8; ++c) {
+                        const uint4 u = *reinterpret_cast<const uint4*>(row + ((c ^ (r & 7)) << 4));
+                        widen4(u.x, m, f[8 * c + 0], f[8 * c + 1]);
+                        widen4(u.y, m, f[8 * c + 2], f[8 * c + 3]);
+                        widen4(u.z, m, f[8 * c + 4], f[8 * c + 5]);
+                        widen4(u.w, m, f[8 * c + 6], f[8 * c + 7]);
+                    }
+                }
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->empty[rs.slot]));
                 if (warp == 2 && lane == 0) TQ(2, it, 2);
-#pragma unroll
-                for (int hh = 0; hh < SLOTS_PER_STAGE; ++hh) {
-                    if (!wt.wait(&s->aempty[ra.slot], ra.phase ^ 1)) {
-                        ok = false;
-                        break;
-                    }
-                    if (warp == 2 && lane == 0 && hh == 0) TQ(2, it, 3);
-#pragma unroll
-                    for (int q32 = 0; q32 < SLOT_K / 64; ++q32) {  // 32 columns (64 K) per store
-                        uint32_t f[32];
-#pragma unroll
-                        for (int c = 0; c < 4; ++c) {
-                            const uint4 u = v[(hh * SLOT_K / 64 + q32) * 4 + c];
-                            widen4(u.x, m, f[8 * c + 0], f[8 * c + 1]);
-                            widen4(u.y, m, f[8 * c + 2], f[8 * c + 3]);
-                            widen4(u.z, m, f[8 * c + 4], f[8 * c + 5]);
-                            widen4(u.w, m, f[8 * c + 6], f[8 * c + 7]);
-                        }
-                        ptx::tmem_st32(lane_base + A_COL + ra.slot * A_SLOT_COLS + q32 * 32, f);
-                    }
-                    ptx::tmem_wait_st();
-                    ptx::tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) {
-                        const uint32_t ab = ptx::smem_u32(&s->afull[ra.slot]);
-                        if (PAIR) ptx::mbar_arrive_cluster(ptx::mapa(ab, 0));
-                        else ptx::mbar_arrive(ab);
-                    }
-                    ra.next();
+                if (!wt.wait(&s->aempty[ra.slot], ra.phase ^ 1)) {
+                    ok = false;
+                    break;
                 }
+                if (warp == 2 && lane == 0) TQ(2, it, 3);
+                {
+                    const uint32_t dst = lane_base + A_COL + ra.slot * A_SLOT_COLS;
+                    ptx::tmem_st32(dst, *reinterpret_cast<const uint32_t(*)[32]>(&f[0]));
+                    ptx::tmem_st32(dst + 32, *reinterpret_cast<const uint32_t(*)[32]>(&f[32]));
+                }
+                ptx::tmem_wait_st();
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    const uint32_t ab = ptx::smem_u32(&s->afull[ra.slot]);
+                    if (PAIR) ptx::mbar_arrive_cluster(ptx::mapa(ab, 0));
+                    else ptx::mbar_arrive(ab);
+                }
+                ra.next();
                 if (!ok) break;
                 if (warp == 2 && lane == 0) TQ(2, it, 5);
             }
@@ -437,8 +458,10 @@ __global__ void __maxnreg__(96)
         const int32_t* ts_b = p.conv ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
         int cc = 0;
         bool ok = true;
-        for (int t = unit; t < tiles && ok; t += units) {
-            const TileCoord tc = tile_coord<PAIR>(p, t, rank);
+        for (int w = unit; w < works && ok; w += units) {
+            const Work wk = work_item(p, w, KT, chunk);
+            const int nchunks = wk.nch;
+            const TileCoord tc = tile_coord<PAIR>(p, wk.t, rank);
             const int n = tc.ch0 + r;
             const bool n_ok = n < a.N;
             // row sums as fp32: |sum| < 2^24, so the values and every partial sum
@@ -589,7 +612,22 @@ __global__ void __maxnreg__(96)
                             }
                         }
                         if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 3 + 2 * h);
-                        if (last) finish16(gi, h * 16, v, nchunks == 1, all_tok);
+                        if (last && p.splits > 1) {
+                            // exact int32 partial sums of this K slice, one coalesced
+                            // 128-byte row per token
+                            if (n_ok) {
+                                int32_t* po = p.split_out + int64_t(wk.slice) * a.M * a.N + n;
+#pragma unroll
+                                for (int j = 0; j < 16; ++j) {
+                                    const int tok = s->ep_tok[e][gi][h * 16 + j];
+                                    if (tok >= 0)
+                                        po[int64_t(tok) * a.N] =
+                                            nchunks == 1 ? __float2int_rn(__uint_as_float(v[j])) : int(v[j]);
+                                }
+                            }
+                        } else if (last) {
+                            finish16(gi, h * 16, v, nchunks == 1, all_tok);
+                        }
                         if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 4 + 2 * h);
                     }
                 }
@@ -612,6 +650,70 @@ __global__ void __maxnreg__(96)
         if (PAIR) ptx::tmem_dealloc2(tmem, TMEM_COLS);
         else ptx::tmem_dealloc(tmem, TMEM_COLS);
     }
+}
+
+// Split-K second half: adds the slices' exact int32 partial sums in slice
+// order and applies the same fused epilogue as the contraction kernel, four
+// channels per thread (16-byte loads, 8-byte bf16 stores).
+__global__ void __launch_bounds__(256) splitk_epilogue_kernel(const GemmArgs a, const int32_t* __restrict__ parts,
+                                                              int S) {
+    ptx::grid_dependency_wait();
+    const int b = resolve_bits(a);
+    if (b == 0) return;
+    const int N4 = a.N / 4;
+    const int64_t total = int64_t(a.M) * N4;
+    const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
+    const int32_t* ts_b = a.Cin ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < total; i += int64_t(gridDim.x) * blockDim.x) {
+        const int m = int(i / N4);
+        const int n = int(i - int64_t(m) * N4) * 4;
+        int4 acc = make_int4(0, 0, 0, 0);
+        for (int sl = 0; sl < S; ++sl) {
+            const int4 v = __ldcg(reinterpret_cast<const int4*>(parts + (int64_t(sl) * a.M + m) * a.N + n));
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+        }
+        const float al = a.per_tensor ? a.alpha[0] : a.alpha[m];
+        const float zc = a.per_tensor ? a.zc[0] : a.zc[m];
+        int tap = 0x1FF;
+        if (a.Cin) {
+            const int ww = m % a.W, hh = (m / a.W) % a.H;
+            tap = 0;
+#pragma unroll
+            for (int dh = 0; dh < 3; ++dh)
+#pragma unroll
+                for (int dw = 0; dw < 3; ++dw) {
+                    const int ih = hh + dh - 1, iw = ww + dw - 1;
+                    if (ih >= 0 && ih < a.H && iw >= 0 && iw < a.W) tap |= 1 << (dh * 3 + dw);
+                }
+        }
+        const int accs[4] = {acc.x, acc.y, acc.z, acc.w};
+        float y[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            float rsum;
+            if (a.Cin) {
+                rsum = 0.f;
+#pragma unroll
+                for (int k9 = 0; k9 < 9; ++k9)
+                    rsum = __fadd_rn(rsum, (tap >> k9) & 1 ? __int2float_rn(ts_b[int64_t(n + q) * 9 + k9]) : 0.f);
+            } else {
+                rsum = __int2float_rn(rs_b[n + q]);
+            }
+            const float u = __fmaf_rn(zc, rsum, __int2float_rn(accs[q]));
+            y[q] = __fmaf_rn(u, __fmul_rn(al, a.cw[n + q]), a.bias[n + q]);
+        }
+        const __nv_bfloat162 h0 = __floats2bfloat162_rn(y[0], y[1]);
+        const __nv_bfloat162 h1 = __floats2bfloat162_rn(y[2], y[3]);
+        uint2 pk;
+        pk.x = *reinterpret_cast<const uint32_t*>(&h0);
+        pk.y = *reinterpret_cast<const uint32_t*>(&h1);
+        *reinterpret_cast<uint2*>(a.y + int64_t(m) * a.N + n) = pk;
+        if (a.acc) *reinterpret_cast<int4*>(a.acc + int64_t(m) * a.N + n) = acc;
+    }
+    ptx::grid_launch_dependents();
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
@@ -728,16 +830,39 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         }
     }
     const int64_t tiles = int64_t(p.tiles_ch) * p.tiles_tok;
+    // Split K when the tiles alone would leave most SMs idle and each slice keeps
+    // at least 8 K blocks: a tile's fixed latency (pipeline fill, epilogue) is
+    // not reduced by splitting, only its K loop is.
+    p.splits = 1;
+    p.split_out = nullptr;
+    if (!PAIR && a.split_buf && tiles * 2 <= num_sms) {
+        const int KT = (a.K + BK - 1) / BK;
+        int64_t S = num_sms / tiles;
+        S = S < KT / 8 ? S : KT / 8;
+        static const int max_splits = [] {
+            const char* v = getenv("TASQ_TC_MAX_SPLITS");  // tuning knob; default 16
+            return v ? atoi(v) : 16;
+        }();
+        S = S < max_splits ? S : max_splits;
+        const int64_t fit = a.split_cap / (int64_t(a.M) * a.N);
+        S = S < fit ? S : fit;
+        if (S >= 2) {
+            p.splits = int(S);
+            p.split_out = a.split_buf;
+        }
+    }
     const int64_t max_units = PAIR ? max_pairs(num_sms) : num_sms;
     if (max_units < 1) {
         *why = "no CTA pair can be co-scheduled";
         return cudaSuccess;
     }
-    const int units = int(tiles < max_units ? tiles : max_units);
+    const int64_t works = tiles * p.splits;
+    const int units = int(works < max_units ? works : max_units);
     static const bool verbose = getenv("TASQ_TC_VERBOSE") != nullptr;
     if (verbose)
-        fprintf(stderr, "tasq tc: %s M=%d N=%d K=%d tiles=%lld units=%d (max %lld) grid=%d\n", PAIR ? "pair" : "single",
-                a.M, a.N, a.K, (long long)tiles, units, (long long)max_units, units * C::NH);
+        fprintf(stderr, "tasq tc: %s M=%d N=%d K=%d tiles=%lld splits=%d units=%d (max %lld) grid=%d\n",
+                PAIR ? "pair" : "single", a.M, a.N, a.K, (long long)tiles, p.splits, units, (long long)max_units,
+                units * C::NH);
     const int smem = smem_bytes<PAIR>();
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
@@ -763,6 +888,18 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     cfg.numAttrs = nattr;
     e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel<PAIR>, p, tm_x, tm_w);
     if (e == cudaSuccess) e = cudaGetLastError();
+    if (e == cudaSuccess && p.splits > 1) {
+        const int64_t total = int64_t(a.M) * (a.N / 4);
+        const int64_t blocks = (total + 255) / 256;
+        cudaLaunchConfig_t rc{};
+        rc.gridDim = dim3(unsigned(blocks < 8 * num_sms ? blocks : 8 * num_sms));
+        rc.blockDim = dim3(256);
+        rc.stream = st;
+        rc.attrs = attr;  // programmatic dependent launch only
+        rc.numAttrs = 1;
+        e = cudaLaunchKernelEx(&rc, splitk_epilogue_kernel, a, static_cast<const int32_t*>(p.split_out), p.splits);
+        if (e == cudaSuccess) e = cudaGetLastError();
+    }
     if (e == cudaErrorLaunchOutOfResources) {
         // report what the kernel asked for, to make the failure actionable
         static char msg[256];

@@ -14,6 +14,7 @@ struct tasq_ctx_s {
     int num_sms = 0;
     int* d_words = nullptr;  // [0] status, [16..19] reduction scratch
     int32_t* d_part = nullptr;  // tensor-core route: int32 running sums of multi-chunk tiles
+    int32_t* d_split = nullptr;  // tensor-core route: split-K partial sums
     uint8_t* d_table = nullptr;
     size_t table_cap = 0;
     int L = 0, S = 0;
@@ -93,10 +94,12 @@ TASQ_API int tasq_create(tasq_ctx* out, int device) {
     e = cudaMalloc(&ctx->d_words, 256);
     if (e == cudaSuccess) e = cudaMemset(ctx->d_words, 0, 256);
     if (e == cudaSuccess) e = cudaMalloc(&ctx->d_part, tasq::gemm_tc_part_bytes(ctx->num_sms));
+    if (e == cudaSuccess) e = cudaMalloc(&ctx->d_split, tasq::kSplitBufBytes);
     cudaSetDevice(prev);
     if (e != cudaSuccess) {
         cudaFree(ctx->d_words);
         cudaFree(ctx->d_part);
+        cudaFree(ctx->d_split);
         delete ctx;
         return fail(nullptr, TASQ_ERR_CUDA, "allocating context buffers: %s", cudaGetErrorString(e));
     }
@@ -112,6 +115,7 @@ TASQ_API void tasq_destroy(tasq_ctx ctx) {
     cudaDeviceSynchronize();
     cudaFree(ctx->d_words);
     cudaFree(ctx->d_part);
+    cudaFree(ctx->d_split);
     cudaFree(ctx->d_table);
     cudaSetDevice(prev);
     delete ctx;
@@ -307,6 +311,8 @@ int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void*
     a.y = d_y;
     a.acc = d_acc;
     a.part = ctx->d_part;
+    a.split_buf = ctx->d_split;
+    a.split_cap = tasq::kSplitBufBytes / int64_t(sizeof(int32_t));
     a.status = ctx->d_words;
     a.timeout_ns = ctx->timeout_ns;
     cudaError_t e;

@@ -78,6 +78,8 @@ struct GemmArgs {
     uint16_t* y;              // bf16 bits
     int32_t* acc;             // optional int32 accumulators
     int32_t* part;            // TC route: per-CTA int32 running sums of multi-chunk tiles
+    int32_t* split_buf;       // TC route: int32 partial sums of split-K slices
+    int64_t split_cap;        // elements of split_buf
     int* status;
     unsigned long long timeout_ns;
 };
@@ -163,6 +165,7 @@ cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float
 cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why);
 size_t gemm_tc_part_bytes(int num_sms);  // scratch the TC route needs for `num_sms` persistent CTAs
+constexpr int64_t kSplitBufBytes = int64_t(32) << 20;  // split-K partial sums (context scratch)
 cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, cudaStream_t st);
 void set_noctx_error(const char* msg);
 cudaError_t launch_selftest_quotients(const float* x, int nx, const float* a, int na, unsigned long long* mismatches,
