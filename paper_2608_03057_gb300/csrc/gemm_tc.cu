@@ -7,11 +7,12 @@
 // each operating precision b, a certificate: the number of 64-wide K blocks
 // over which 128 * sum_k |mask_b(w)| <= 2^24 holds for every channel.  The
 // accumulator in tensor memory is restarted after each such chunk and
-// drained into an int32 running sum (also kept in tensor memory), so the
-// final int32 accumulator equals the exact integer result.
+// drained into an int32 running sum (kept by each epilogue thread in the
+// context's per-CTA scratch), so the final int32 accumulator equals the
+// exact integer result.
 //
 // Operand roles (D = A * B^T with the output channels on the MMA's M side):
-//   A: the weight tile, 128 channels x 64 K.  TMA brings the stored int8 codes
+//   A: the weight tile, 128 channels x 128 K.  TMA brings the stored int8 codes
 //      into shared memory; a converter warpgroup applies the operating-
 //      precision mask (Eq. hw_rightshift: clear the low 8-b planes, one AND
 //      per four codes), widens to fp16 and writes the tile straight into
@@ -23,9 +24,9 @@
 //   D: fp32 accumulators in tensor memory, double-buffered so the epilogue
 //      of one chunk overlaps the MMAs of the next.
 //
-// Warp roles (320 threads): warp 0 issues TMA; warp 1 allocates tensor
+// Warp roles (576 threads): warp 0 issues TMA; warp 1 allocates tensor
 // memory and issues the MMAs (one thread); warps 2..5 convert weights; warps
-// 6..9 drain accumulators and run the fused dequantization epilogue.  The
+// 6..17 drain accumulators and run the fused dequantization epilogue.  The
 // grid is persistent: one CTA per SM walks the output tiles.  Every wait is
 // bounded by the context's time limit; a wait that gives up records
 // TASQ_ERR_DEVICE_TIMEOUT, the CTA drains its copies in flight, frees its
@@ -42,80 +43,96 @@
 
 // Optional per-role timestamps of CTA 0 (build with -DTASQ_TRACE; compiled
 // out otherwise): role 0 producer, 1 MMA, 2 converter warp, 3 epilogue warp.
+// TE(ev) records, for every CTA, the global time (ns) and SM clock of one
+// event of its timeline: 0 entry, 1 set-up done, 2 inputs released (producer),
+// 3 first stage landed (converter), 4 first MMA issued, 5 last MMA committed,
+// 6 first accumulator ready, 7 last accumulator ready, 8 epilogue done,
+// 9 producer done, 10 exit.
 #ifdef TASQ_TRACE
 __device__ unsigned long long g_tasq_trace[4][256][8];
+__device__ unsigned long long g_tasq_ev[512][12][2];
 #define TQ(role, it, k)                                                          \
     do {                                                                         \
         if (blockIdx.x == 0 && (it) < 256) g_tasq_trace[role][it][k] = clock64(); \
     } while (0)
+#define TE(ev)                                                    \
+    do {                                                          \
+        if (blockIdx.x < 512) {                                   \
+            g_tasq_ev[blockIdx.x][ev][0] = ptx::globaltimer();    \
+            g_tasq_ev[blockIdx.x][ev][1] = clock64();             \
+        }                                                         \
+    } while (0)
 #else
 #define TQ(role, it, k) \
     do {                \
+    } while (0)
+#define TE(ev) \
+    do {       \
     } while (0)
 #endif
 
 namespace tasq {
 namespace {
 
-constexpr int BCH = 128;          // output channels per CTA (MMA M per CTA)
+constexpr int BCH = 128;          // output channels per tile (MMA M)
 constexpr int BTOK = 192;         // tokens / output pixels per tile (MMA N)
-constexpr int BK = 128;           // K per pipeline stage (two 64-wide swizzle atoms)
-constexpr int SLOT_K = 128;       // K covered by one tensor-memory slot of converted weights
-constexpr int SLOTS_PER_STAGE = BK / SLOT_K;
-constexpr int ASLOTS = 2 * SLOTS_PER_STAGE;  // converted-weight slots in tensor memory
+constexpr int BK = 128;           // K per weight stage and per tensor-memory slot of converted weights
+constexpr int XK = 64;            // K per activation TMA box (one 128-byte swizzle atom of fp16 codes)
+constexpr int X_STAGES = 3;       // activation stages of BK
+constexpr int W_STAGES = 3;
+constexpr int ASLOTS = 2;         // converted-weight slots in tensor memory
+constexpr int KDONE = 6;          // K-block completion barriers (a multiple of X_STAGES and ASLOTS)
+constexpr int EPI_WARP0 = 6;      // first epilogue warp
 constexpr int EPI_WARPS = 12;     // three per tensor-memory lane quadrant
-constexpr int THREADS = (6 + EPI_WARPS) * 32;
+constexpr int WPROD_WARP = EPI_WARP0 + EPI_WARPS;  // weight-tile producer
+constexpr int THREADS = (WPROD_WARP + 1) * 32;
+constexpr int X_HALF = BTOK * XK * 2;   // 24 KB of fp16 codes, 128-byte rows
+constexpr int X_STAGE = 2 * X_HALF;
 constexpr int W_STAGE = BCH * BK;       // 16 KB int8 codes, 128-byte rows
 constexpr int GROUPS = BTOK / 32;       // 32-token column groups of the accumulator
 static_assert(GROUPS == 2 * EPI_WARPS / 4, "each epilogue warp drains two groups");
+static_assert(BK == 2 * XK, "a stage is two 64-wide swizzle atoms");
+static_assert(KDONE % X_STAGES == 0 && KDONE % ASLOTS == 0, "completion ring covers both reuse distances");
 // tensor memory columns
 constexpr uint32_t ACC_COL = 0;           // 2 x BTOK fp32 accumulators
-constexpr uint32_t A_COL = 2 * BTOK;      // ASLOTS x SLOT_K/2 columns (fp16 pairs)
-constexpr uint32_t A_SLOT_COLS = SLOT_K / 2;
+constexpr uint32_t A_COL = 2 * BTOK;      // ASLOTS x BK/2 columns (fp16 pairs)
+constexpr uint32_t A_SLOT_COLS = BK / 2;
 constexpr uint32_t TMEM_COLS = 512;
 static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
+constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BTOK);
 
-// PAIR = false: one CTA computes a 128-channel x 192-token tile.
-// PAIR = true : a cluster of two CTAs computes a 256 x 192 tile with the 2-SM
-// MMA; each CTA converts its own 128 weight rows into its own tensor memory
-// and holds half of the activation tile (96 tokens) in shared memory, so a
-// stage is 40 KB instead of 64 KB and five stages fit.
-template <bool PAIR>
-struct Cfg {
-    static constexpr int NH = PAIR ? 2 : 1;           // CTAs sharing the token tile
-    static constexpr int XT = BTOK / NH;              // tokens of the tile in this CTA's shared memory
-    static constexpr int X_HALF = XT * 64 * 2;        // one 64-wide K atom of fp16 codes
-    static constexpr int X_STAGE = 2 * X_HALF;
-    static constexpr int STAGES = PAIR ? 5 : 3;
-    static constexpr int CH_TILE = BCH * NH;          // channels per tile
-    static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH * NH, BTOK);
-};
-
-template <bool PAIR>
+// Synchronisation is arranged so that the single MMA-issuing thread, whose
+// per-instruction cost bounds the K loop, does one wait and one commit per K
+// block:
+//   xfull[j % 3]  completes when the activation stage of K block j has landed
+//                 (TMA transaction bytes) AND the four converter warps have
+//                 written its weights into tensor-memory slot j % 2;
+//   kdone[j % 6]  completes when the MMAs of K block j have finished; the
+//                 activation producer waits on it before refilling stage j % 3
+//                 with block j + 3, the converters before overwriting slot j % 2
+//                 with block j + 2.
+// The weight ring is separate: a weight stage is released as soon as the
+// converters have read it, so weight tiles run several K blocks ahead.
 struct Smem {
-    static constexpr int STAGES = Cfg<PAIR>::STAGES;
-    uint8_t x[STAGES][Cfg<PAIR>::X_STAGE];  // 1024-aligned (128B swizzle atoms)
-    uint8_t w[STAGES][W_STAGE];
+    uint8_t x[X_STAGES][X_STAGE];  // 1024-aligned (128-byte swizzle atoms)
+    uint8_t w[W_STAGES][W_STAGE];
     float ep_al[EPI_WARPS][2][32], ep_zc[EPI_WARPS][2][32];  // per warp, per group, per column
     int ep_tok[EPI_WARPS][2][32], ep_tap[EPI_WARPS][2][32];
     alignas(16) uint16_t ep_stage[EPI_WARPS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
-    uint64_t full[STAGES], empty[STAGES];
-    uint64_t afull[ASLOTS], aempty[ASLOTS];
+    uint64_t xfull[X_STAGES], kdone[KDONE];
+    uint64_t wfull[W_STAGES], wempty[W_STAGES];
     uint64_t accfull[2], accempty[2];
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
 };
-template <bool PAIR>
-constexpr int smem_bytes() {
-    return int(sizeof(Smem<PAIR>)) + 1024;
-}
+constexpr int smem_bytes() { return int(sizeof(Smem)) + 1024; }
 
 struct TcParams {
     GemmArgs a;
     int conv;
-    int tiles_ch, tiles_tok;  // tiles of Cfg::CH_TILE channels x BTOK tokens
-    // conv: a token tile is NH stacked boxes of bhx rows x 2^bw_log2 pixels
+    int tiles_ch, tiles_tok;  // tiles of BCH channels x BTOK tokens
+    // conv: a token tile is a box of bhx rows x 2^bw_log2 pixels
     int bw_log2, bhx, tiles_w, tiles_h;
     // split-K: each tile's K blocks are cut into `splits` contiguous slices; a
     // slice writes its exact int32 partial sums to split_out[slice][token][n]
@@ -138,21 +155,17 @@ __device__ __forceinline__ Work work_item(const TcParams& p, int w, int KT, int 
     return r;
 }
 
-template <bool PAIR>
 struct Waiter {
-    Smem<PAIR>* s;
+    Smem* s;
     const GemmArgs* a;
     // Bounded wait on phase `parity` of an mbarrier; false after a timeout or
-    // when another role has aborted the CTA.  `cluster` acquires arrivals
-    // released by the peer CTA.
-    __device__ __forceinline__ bool wait(uint64_t* bar, uint32_t parity, bool ignore_abort = false,
-                                         bool cluster = false) const {
+    // when another role has aborted the CTA.
+    __device__ __forceinline__ bool wait(uint64_t* bar, uint32_t parity, bool ignore_abort = false) const {
         const uint32_t addr = ptx::smem_u32(bar);
-        auto probe = [&]() { return cluster ? ptx::mbar_try_wait_cluster(addr, parity) : ptx::mbar_try_wait(addr, parity); };
-        if (probe()) return true;
+        if (ptx::mbar_try_wait(addr, parity)) return true;
         const uint64_t t0 = ptx::globaltimer();
         for (uint32_t it = 1;; ++it) {
-            if (probe()) return true;
+            if (ptx::mbar_try_wait(addr, parity)) return true;
             if ((it & 63) == 0) {
                 if (!ignore_abort && *(volatile int*)&s->abort) return false;
                 if (ptx::globaltimer() - t0 > a->timeout_ns) {
@@ -193,20 +206,19 @@ __device__ __forceinline__ void widen4(uint32_t w, uint32_t m, uint32_t& lo, uin
 }
 
 struct TileCoord {
-    int ch0;             // first channel of this CTA's 128 rows
+    int ch0;  // first channel of the tile's 128 rows
     int tok0, img, h0, w0;
 };
 
-template <bool PAIR>
-__device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t, int rank) {
+__device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
     TileCoord c;
-    c.ch0 = (t % p.tiles_ch) * Cfg<PAIR>::CH_TILE + rank * BCH;
+    c.ch0 = (t % p.tiles_ch) * BCH;
     const int tt = t / p.tiles_ch;
     c.tok0 = c.img = c.h0 = c.w0 = 0;
     if (p.conv) {
         const int per_img = p.tiles_h * p.tiles_w;
         c.img = tt / per_img;
-        c.h0 = ((tt % per_img) / p.tiles_w) * (p.bhx * Cfg<PAIR>::NH);
+        c.h0 = ((tt % per_img) / p.tiles_w) * p.bhx;
         c.w0 = (tt % p.tiles_w) << p.bw_log2;
     } else {
         c.tok0 = tt * BTOK;
@@ -214,19 +226,15 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t, int ra
     return c;
 }
 
-template <bool PAIR>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w) {
-    using C = Cfg<PAIR>;
-    constexpr int STAGES = C::STAGES;
+    if (threadIdx.x == 0) TE(0);
     extern __shared__ uint8_t smem_raw[];
-    Smem<PAIR>* s = reinterpret_cast<Smem<PAIR>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    Smem* s = reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const GemmArgs& a = p.a;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const Waiter<PAIR> wt{s, &a};
-    const uint32_t rank = PAIR ? ptx::cluster_rank() : 0u;
-    const bool leader = rank == 0;
+    const Waiter wt{s, &a};
 
     const int b = resolve_bits(a);
     if (b == 0) return;  // uniform across the grid (a launch-wide check): nothing allocated yet
@@ -235,21 +243,19 @@ __global__ void __maxnreg__(96)
     int chunk = a.hdr->chunk_kb[b] / (BK / kCertKBlock);
     chunk = chunk < 1 ? 1 : (chunk > KT ? KT : chunk);
     const int works = p.tiles_ch * p.tiles_tok * p.splits;
-    const int unit = PAIR ? int(blockIdx.x >> 1) : int(blockIdx.x);  // pair (or CTA) index
-    const int units = PAIR ? int(gridDim.x >> 1) : int(gridDim.x);
+    const int unit = int(blockIdx.x), units = int(gridDim.x);
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < STAGES; ++i) {
-            ptx::mbar_init(ptx::smem_u32(&s->full[i]), 1);
-            ptx::mbar_init(ptx::smem_u32(&s->empty[i]), 4 + 1);  // 4 converter warps + the MMA commit
-        }
-        for (int i = 0; i < ASLOTS; ++i) {
-            ptx::mbar_init(ptx::smem_u32(&s->afull[i]), 4 * C::NH);  // converter warps of every CTA
-            ptx::mbar_init(ptx::smem_u32(&s->aempty[i]), 1);
+        for (int i = 0; i < X_STAGES; ++i)
+            ptx::mbar_init(ptx::smem_u32(&s->xfull[i]), 1 + 4);  // producer's expect_tx + 4 converter warps
+        for (int i = 0; i < KDONE; ++i) ptx::mbar_init(ptx::smem_u32(&s->kdone[i]), 1);  // the MMA commit
+        for (int i = 0; i < W_STAGES; ++i) {
+            ptx::mbar_init(ptx::smem_u32(&s->wfull[i]), 1);
+            ptx::mbar_init(ptx::smem_u32(&s->wempty[i]), 4);  // the 4 converter warps
         }
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(ptx::smem_u32(&s->accfull[i]), 1);
-            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS * C::NH);
+            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS);
         }
         ptx::mbar_init(ptx::smem_u32(&s->drain), 1);
         s->abort = 0;
@@ -258,160 +264,163 @@ __global__ void __maxnreg__(96)
         ptx::prefetch_tmap(&tm_w);
     }
     if (warp == 1) {
-        if (PAIR) {
-            ptx::tmem_alloc2(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
-            ptx::tmem_relinquish2();
-        } else {
-            ptx::tmem_alloc(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
-            ptx::tmem_relinquish();
-        }
+        ptx::tmem_alloc(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
+        ptx::tmem_relinquish();
         ptx::tc_fence_before();
     }
-    if (PAIR) ptx::cluster_sync();  // barriers of both CTAs exist before any cross-CTA use
-    else __syncthreads();
+    __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem_base;
+    if (threadIdx.x == 0) TE(1);
+    if (warp == WPROD_WARP && lane == 0 && unit < works) {
+        // The packed weights are not written by the kernel this one may overlap,
+        // so their first tiles can be pulled into L2 before the wait below (a
+        // prefetch only: nothing reaches shared memory before the wait).
+        const Work wk = work_item(p, unit, KT, chunk);
+        const int ch0 = tile_coord(p, wk.t).ch0;
+        for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * BK, ch0);
+    }
     // the prologue above overlaps the previous kernel; inputs are read only after it
     ptx::grid_dependency_wait();
+    if (threadIdx.x == 0) TE(2);
 
     if (warp == 0) {
-        // ------------------------------------------------------ TMA producer
+        // --------------------------------------------- activation producer
         if (lane == 0) {
-            Ring<STAGES> rs;
-            int it = 0;
+            int j = 0;  // K blocks issued by this CTA
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
-                const TileCoord tc = tile_coord<PAIR>(p, wk.t, rank);
-                for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rs.next()) {
-                    TQ(0, it, 0);
-                    if (!wt.wait(&s->empty[rs.slot], rs.phase ^ 1)) {
+                const TileCoord tc = tile_coord(p, wk.t);
+                for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++j) {
+                    TQ(0, j, 0);
+                    if (j >= X_STAGES && !wt.wait(&s->kdone[(j - X_STAGES) % KDONE], ((j - X_STAGES) / KDONE) & 1)) {
                         ok = false;
                         break;
                     }
-                    TQ(0, it, 1);
-                    const uint32_t fb = ptx::smem_u32(&s->full[rs.slot]);
-                    // the leader's barrier counts both CTAs' activation halves
-                    const uint32_t xbar = PAIR ? ptx::mapa(fb, 0) : fb;
-                    ptx::mbar_arrive_expect_tx(fb, (leader ? C::NH * C::X_STAGE : 0) + W_STAGE);
-                    const uint32_t xdst = ptx::smem_u32(s->x[rs.slot]);
-                    const int k0 = kb * BK;
+                    TQ(0, j, 1);
+                    const uint32_t fb = ptx::smem_u32(&s->xfull[j % X_STAGES]);
+                    ptx::mbar_arrive_expect_tx(fb, X_STAGE);
+                    const uint32_t dst = ptx::smem_u32(s->x[j % X_STAGES]);
 #pragma unroll
                     for (int hh = 0; hh < 2; ++hh) {
-                        const int kh = k0 + 64 * hh;
+                        const int kh = kb * BK + hh * XK;
                         if (p.conv) {
                             // a 128-wide K block may straddle two taps when Cin % 128 == 64
                             const int tap = kh / a.Cin, c0 = kh - tap * a.Cin;
-                            const int c1 = tc.w0 + tap % 3 - 1, c2 = tc.h0 + int(rank) * p.bhx + tap / 3 - 1;
-                            if (PAIR)
-                                ptx::tma2_load_4d(xdst + hh * C::X_HALF, &tm_x, xbar, c0, c1, c2, tc.img);
-                            else
-                                ptx::tma_load_4d(xdst + hh * C::X_HALF, &tm_x, fb, c0, c1, c2, tc.img);
+                            ptx::tma_load_4d(dst + hh * X_HALF, &tm_x, fb, c0, tc.w0 + tap % 3 - 1, tc.h0 + tap / 3 - 1,
+                                             tc.img);
                         } else {
-                            const int c1 = tc.tok0 + int(rank) * C::XT;
-                            if (PAIR)
-                                ptx::tma2_load_2d(xdst + hh * C::X_HALF, &tm_x, xbar, kh, c1);
-                            else
-                                ptx::tma_load_2d(xdst + hh * C::X_HALF, &tm_x, fb, kh, c1);
+                            ptx::tma_load_2d(dst + hh * X_HALF, &tm_x, fb, kh, tc.tok0);
                         }
                     }
-                    ptx::tma_load_2d(ptx::smem_u32(s->w[rs.slot]), &tm_w, fb, k0, tc.ch0);
                 }
             }
+            TE(9);
             // the next kernel may be launched while this grid drains
             ptx::grid_launch_dependents();
-            // copies still in flight must land before the CTA may exit
-            for (int j = 0; j < STAGES && j < it; ++j) {
-                const int jj = it - STAGES + j;  // the last STAGES stages issued, oldest first
-                if (jj < 0) continue;
-                wt.wait(&s->full[jj % STAGES], (jj / STAGES) & 1, true);
+            // copies still in flight must land before the CTA may exit: the MMAs
+            // of the last K blocks consumed them (or the CTA is aborting)
+            for (int i = j - X_STAGES < 0 ? 0 : j - X_STAGES; i < j; ++i)
+                wt.wait(&s->kdone[i % KDONE], (i / KDONE) & 1, true);
+        }
+    } else if (warp == WPROD_WARP) {
+        // ------------------------------------------------ weight producer
+        if (lane == 0) {
+            Ring<W_STAGES> rw;
+            int nw = 0;
+            bool ok = true;
+            for (int w = unit; w < works && ok; w += units) {
+                const Work wk = work_item(p, w, KT, chunk);
+                const int ch0 = tile_coord(p, wk.t).ch0;
+                for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++nw, rw.next()) {
+                    if (!wt.wait(&s->wempty[rw.slot], rw.phase ^ 1)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t fb = ptx::smem_u32(&s->wfull[rw.slot]);
+                    ptx::mbar_arrive_expect_tx(fb, W_STAGE);
+                    ptx::tma_load_2d(ptx::smem_u32(s->w[rw.slot]), &tm_w, fb, kb * BK, ch0);
+                }
             }
+            for (int j = nw - W_STAGES < 0 ? 0 : nw - W_STAGES; j < nw; ++j)
+                wt.wait(&s->wfull[j % W_STAGES], (j / W_STAGES) & 1, true);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
-        if (lane == 0 && leader) {
-            Ring<STAGES> rs;
-            Ring<ASLOTS> ra;
+        if (lane == 0) {
+            // B descriptors differ only in their start-address field (address >> 4)
+            const uint64_t bdesc0 = ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[0]));
             int it = 0, cc = 0;
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
                 for (int c = 0; c < wk.nch && ok; ++c, ++cc) {
                     const int buf = cc & 1;
-                    if (!wt.wait(&s->accempty[buf], ((cc >> 1) & 1) ^ 1, false, PAIR)) {
+                    if (!wt.wait(&s->accempty[buf], ((cc >> 1) & 1) ^ 1)) {
                         ok = false;
                         break;
                     }
                     ptx::tc_fence_after();
                     const uint32_t d = tmem + ACC_COL + buf * BTOK;
                     const int kb0 = wk.kb_lo + c * chunk, kb_end = min(wk.kb_hi, kb0 + chunk);
-                    for (int kb = kb0; kb < kb_end; ++kb, ++it, rs.next()) {
+                    for (int kb = kb0; kb < kb_end; ++kb, ++it) {
                         TQ(1, it, 0);
-                        const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[rs.slot]));
-#pragma unroll
-                        for (int hh = 0; hh < SLOTS_PER_STAGE; ++hh) {
-                            // the converters of every CTA have passed this stage's full
-                            // barrier (activations landed) and written this weight slot
-                            if (!wt.wait(&s->afull[ra.slot], ra.phase, false, PAIR)) {
-                                ok = false;
-                                break;
-                            }
-                            ptx::tc_fence_after();
-                            const uint32_t acol = tmem + A_COL + ra.slot * A_SLOT_COLS;
-#pragma unroll
-                            for (int kk = 0; kk < SLOT_K / 16; ++kk) {
-                                const int k = hh * (SLOT_K / 16) + kk;  // K step of 16 within the stage
-                                const uint64_t bk = bdesc + uint64_t(((k >> 2) * C::X_HALF + (k & 3) * 32) >> 4);
-                                const uint32_t accum = (kb > kb0 || k > 0) ? 1u : 0u;
-                                if (PAIR) ptx::mma2_f16_ts(d, acol + kk * 8, bk, C::IDESC, accum);
-                                else ptx::mma_f16_ts(d, acol + kk * 8, bk, C::IDESC, accum);
-                            }
-                            if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->aempty[ra.slot]), 0x3);
-                            else ptx::mma_commit(ptx::smem_u32(&s->aempty[ra.slot]));
-                            ra.next();
+                        // activations landed and the converters wrote weight slot it % 2
+                        if (!wt.wait(&s->xfull[it % X_STAGES], (it / X_STAGES) & 1)) {
+                            ok = false;
+                            break;
                         }
-                        if (!ok) break;
-                        if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->empty[rs.slot]), 0x3);
-                        else ptx::mma_commit(ptx::smem_u32(&s->empty[rs.slot]));
+                        ptx::tc_fence_after();
+                        TQ(1, it, 1);
+                        if (it == 0) TE(4);
+                        const uint32_t acol = tmem + A_COL + (it % ASLOTS) * A_SLOT_COLS;
+                        const uint64_t bdesc = bdesc0 + uint64_t((it % X_STAGES) * (X_STAGE >> 4));
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k) {
+                            // K step of 16 codes: 32 bytes along the swizzled 128-byte row, the
+                            // second 64-wide atom X_HALF further on
+                            const uint64_t bk = bdesc + uint64_t(((k >> 2) * X_HALF + (k & 3) * 32) >> 4);
+                            if (k == 0 && kb == kb0) ptx::mma_f16_ts(d, acol, bk, IDESC, 0u);
+                            else ptx::mma_f16_ts(d, acol + k * 8, bk, IDESC, 1u);
+                        }
+                        TQ(1, it, 2);
+                        ptx::mma_commit(ptx::smem_u32(&s->kdone[it % KDONE]));
                         TQ(1, it, 3);
                     }
-                    if (ok) {
-                        if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->accfull[buf]), 0x3);
-                        else ptx::mma_commit(ptx::smem_u32(&s->accfull[buf]));
-                    }
+                    if (ok) ptx::mma_commit(ptx::smem_u32(&s->accfull[buf]));
                 }
             }
+            TE(5);
             // every MMA issued must finish before tensor memory is released
-            if (PAIR) ptx::mma2_commit_mc(ptx::smem_u32(&s->drain), 0x1);
-            else ptx::mma_commit(ptx::smem_u32(&s->drain));
+            ptx::mma_commit(ptx::smem_u32(&s->drain));
             wt.wait(&s->drain, 0, true);
         }
-    } else if (warp < 6) {
+    } else if (warp < EPI_WARP0) {
         // ------------------------------------------- weight mask + convert
         const int q = warp & 3;             // tensor-memory lane quadrant
-        const int r = q * 32 + lane;        // channel row within this CTA's 128
+        const int r = q * 32 + lane;        // channel row within the tile
         const uint32_t m = mask_word(b);
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
-        Ring<STAGES> rs;
-        Ring<ASLOTS> ra;
+        Ring<W_STAGES> rw;
         int it = 0;
         bool ok = true;
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
-            for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rs.next()) {
+            for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rw.next()) {
                 if (warp == 2 && lane == 0) TQ(2, it, 0);
-                if (!wt.wait(&s->full[rs.slot], rs.phase)) {
+                if (!wt.wait(&s->wfull[rw.slot], rw.phase)) {
                     ok = false;
                     break;
                 }
                 if (warp == 2 && lane == 0) TQ(2, it, 1);
+                if (warp == 2 && lane == 0 && it == 0) TE(3);
                 // 128 codes of row r; 16-byte chunk c sits at c ^ (r & 7) (128-byte swizzle).
                 // Mask and widen before waiting for the slot, so that only the
                 // tensor-memory store remains once the MMA releases it.
-                static_assert(SLOTS_PER_STAGE == 1, "the converter widens a whole stage into one slot");
                 uint32_t f[64];
                 {
-                    const uint8_t* row = s->w[rs.slot] + r * BK;
+                    const uint8_t* row = s->w[rw.slot] + r * BK;
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
                         const uint4 u = *reinterpret_cast<const uint4*>(row + ((c ^ (r & 7)) << 4));
@@ -422,34 +431,29 @@ __global__ void __maxnreg__(96)
                     }
                 }
                 __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->empty[rs.slot]));
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->wempty[rw.slot]));
                 if (warp == 2 && lane == 0) TQ(2, it, 2);
-                if (!wt.wait(&s->aempty[ra.slot], ra.phase ^ 1)) {
+                // slot it % 2 last held K block it - 2: its MMAs must have finished
+                if (it >= ASLOTS && !wt.wait(&s->kdone[(it - ASLOTS) % KDONE], ((it - ASLOTS) / KDONE) & 1)) {
                     ok = false;
                     break;
                 }
                 if (warp == 2 && lane == 0) TQ(2, it, 3);
                 {
-                    const uint32_t dst = lane_base + A_COL + ra.slot * A_SLOT_COLS;
+                    const uint32_t dst = lane_base + A_COL + (it % ASLOTS) * A_SLOT_COLS;
                     ptx::tmem_st32(dst, *reinterpret_cast<const uint32_t(*)[32]>(&f[0]));
                     ptx::tmem_st32(dst + 32, *reinterpret_cast<const uint32_t(*)[32]>(&f[32]));
                 }
                 ptx::tmem_wait_st();
                 ptx::tc_fence_before();
                 __syncwarp();
-                if (lane == 0) {
-                    const uint32_t ab = ptx::smem_u32(&s->afull[ra.slot]);
-                    if (PAIR) ptx::mbar_arrive_cluster(ptx::mapa(ab, 0));
-                    else ptx::mbar_arrive(ab);
-                }
-                ra.next();
-                if (!ok) break;
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->xfull[it % X_STAGES]));
                 if (warp == 2 && lane == 0) TQ(2, it, 5);
             }
         }
     } else {
         // ------------------------------------- accumulator drain + epilogue
-        const int e = warp - 6;              // 0..EPI_WARPS-1
+        const int e = warp - EPI_WARP0;      // 0..EPI_WARPS-1
         const int q = warp & 3;              // lane quadrant: channels q*32 .. q*32+31
         const int part = e >> 2;             // which pair of 32-token groups
         const int r = q * 32 + lane;
@@ -461,7 +465,7 @@ __global__ void __maxnreg__(96)
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
             const int nchunks = wk.nch;
-            const TileCoord tc = tile_coord<PAIR>(p, wk.t, rank);
+            const TileCoord tc = tile_coord(p, wk.t);
             const int n = tc.ch0 + r;
             const bool n_ok = n < a.N;
             // row sums as fp32: |sum| < 2^24, so the values and every partial sum
@@ -491,9 +495,7 @@ __global__ void __maxnreg__(96)
                 const int jt = (2 * part + gi) * 32 + lane;
                 int tok = -1, tap = 0;
                 if (p.conv) {
-                    // column jt came from box jt / XT (stacked bhx-row boxes of the tile)
-                    const int jb = jt / C::XT, jj = jt - jb * C::XT;
-                    const int hh = tc.h0 + jb * p.bhx + (jj >> p.bw_log2), ww = tc.w0 + (jj & ((1 << p.bw_log2) - 1));
+                    const int hh = tc.h0 + (jt >> p.bw_log2), ww = tc.w0 + (jt & ((1 << p.bw_log2) - 1));
                     if (hh < a.H && ww < a.W) {
                         tok = (tc.img * a.H + hh) * a.W + ww;
 #pragma unroll
@@ -589,6 +591,8 @@ __global__ void __maxnreg__(96)
                     break;
                 }
                 if (warp == 6 && lane == 0) TQ(3, cc, 1);
+                if (warp == 6 && lane == 0 && cc == 0) TE(6);
+                if (warp == 6 && lane == 0) TE(7);
                 ptx::tc_fence_after();
                 const uint32_t acc_base = lane_base + ACC_COL + buf * BTOK;
                 const bool last = c == nchunks - 1;
@@ -633,22 +637,18 @@ __global__ void __maxnreg__(96)
                 }
                 ptx::tc_fence_before();
                 __syncwarp();
-                if (lane == 0) {
-                    const uint32_t eb = ptx::smem_u32(&s->accempty[buf]);
-                    if (PAIR) ptx::mbar_arrive_cluster(ptx::mapa(eb, 0));
-                    else ptx::mbar_arrive(eb);
-                }
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->accempty[buf]));
                 if (warp == 6 && lane == 0) TQ(3, cc, 2);
             }
         }
     }
 
+    if (warp == 6 && lane == 0) TE(8);
     __syncthreads();
-    if (PAIR) ptx::cluster_sync();  // neither CTA releases memory the pair's MMAs may still use
+    if (threadIdx.x == 0) TE(10);
     if (warp == 1) {
         ptx::tc_fence_after();
-        if (PAIR) ptx::tmem_dealloc2(tmem, TMEM_COLS);
-        else ptx::tmem_dealloc(tmem, TMEM_COLS);
+        ptx::tmem_dealloc(tmem, TMEM_COLS);
     }
 }
 
@@ -735,35 +735,7 @@ size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * EPI_WARPS * 64
 
 namespace {
 
-// Pairs of CTAs the 2-SM kernel can keep resident at once (cluster placement
-// can leave some SMs unpaired), looked up once.
-int max_pairs(int num_sms) {
-    static int cached = -1;
-    if (cached < 0) {
-        cudaLaunchConfig_t cfg{};
-        cfg.gridDim = dim3(2 * (num_sms / 2));
-        cfg.blockDim = dim3(THREADS);
-        cfg.dynamicSmemBytes = smem_bytes<true>();
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = 2;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        int n = 0;
-        if (cudaFuncSetAttribute(gemm_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 smem_bytes<true>()) != cudaSuccess ||
-            cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<true>, &cfg) != cudaSuccess)
-            n = 0;
-        cached = n;
-    }
-    return cached;
-}
-
-template <bool PAIR>
-cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
-    using C = Cfg<PAIR>;
+cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
     auto encode = get_encode();
     if (!encode) {
         *why = "cuTensorMapEncodeTiled is unavailable";
@@ -772,7 +744,7 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     TcParams p{};
     p.a = a;
     p.conv = a.Cin != 0;
-    p.tiles_ch = (a.N + C::CH_TILE - 1) / C::CH_TILE;
+    p.tiles_ch = (a.N + BCH - 1) / BCH;
     CUtensorMap tm_x, tm_w;
     CUresult r;
     if (p.conv) {
@@ -780,15 +752,14 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
             *why = "convolution needs Cin % 64 == 0";
             return cudaSuccess;
         }
-        // box of bhx rows x 2^bwl pixels; 2^bwl must divide XT (192 = 64*3, 96 = 32*3)
-        const int max_bw = PAIR ? 32 : 64;
+        // box of bhx rows x 2^bwl pixels; 2^bwl must divide BTOK (192 = 64 * 3)
         int bwl = 0;
-        while ((1 << bwl) < a.W && (1 << bwl) < max_bw) ++bwl;
+        while ((1 << bwl) < a.W && (1 << bwl) < 64) ++bwl;
         p.bw_log2 = bwl;
-        p.bhx = C::XT >> bwl;
+        p.bhx = BTOK >> bwl;
         const int bw = 1 << bwl;
         p.tiles_w = (a.W + bw - 1) / bw;
-        p.tiles_h = (a.H + p.bhx * C::NH - 1) / (p.bhx * C::NH);
+        p.tiles_h = (a.H + p.bhx - 1) / p.bhx;
         const int64_t tok_tiles = int64_t(a.B) * p.tiles_h * p.tiles_w;
         if (tok_tiles * p.tiles_ch > 0x7FFFFFFF) {
             *why = "too many tiles";
@@ -797,7 +768,7 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         p.tiles_tok = int(tok_tiles);
         cuuint64_t dims[4] = {cuuint64_t(a.Cin), cuuint64_t(a.W), cuuint64_t(a.H), cuuint64_t(a.B)};
         cuuint64_t strides[3] = {cuuint64_t(a.Cin) * 2, cuuint64_t(a.W) * a.Cin * 2, cuuint64_t(a.H) * a.W * a.Cin * 2};
-        cuuint32_t box[4] = {64, cuuint32_t(bw), cuuint32_t(p.bhx), 1};
+        cuuint32_t box[4] = {XK, cuuint32_t(bw), cuuint32_t(p.bhx), 1};
         cuuint32_t es[4] = {1, 1, 1, 1};
         r = encode(&tm_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void*>(a.x), dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -806,7 +777,7 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         p.tiles_tok = (a.M + BTOK - 1) / BTOK;
         cuuint64_t dims[2] = {cuuint64_t(a.K), cuuint64_t(a.M)};
         cuuint64_t strides[1] = {cuuint64_t(a.K) * 2};
-        cuuint32_t box[2] = {64, cuuint32_t(C::XT)};
+        cuuint32_t box[2] = {XK, cuuint32_t(BTOK)};
         cuuint32_t es[2] = {1, 1};
         r = encode(&tm_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(a.x), dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -835,7 +806,7 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     // not reduced by splitting, only its K loop is.
     p.splits = 1;
     p.split_out = nullptr;
-    if (!PAIR && a.split_buf && tiles * 2 <= num_sms) {
+    if (a.split_buf && tiles * 2 <= num_sms) {
         const int KT = (a.K + BK - 1) / BK;
         int64_t S = num_sms / tiles;
         S = S < KT / 8 ? S : KT / 8;
@@ -851,42 +822,28 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
             p.split_out = a.split_buf;
         }
     }
-    const int64_t max_units = PAIR ? max_pairs(num_sms) : num_sms;
-    if (max_units < 1) {
-        *why = "no CTA pair can be co-scheduled";
-        return cudaSuccess;
-    }
     const int64_t works = tiles * p.splits;
-    const int units = int(works < max_units ? works : max_units);
+    const int units = int(works < num_sms ? works : num_sms);
     static const bool verbose = getenv("TASQ_TC_VERBOSE") != nullptr;
     if (verbose)
-        fprintf(stderr, "tasq tc: %s M=%d N=%d K=%d tiles=%lld splits=%d units=%d (max %lld) grid=%d\n",
-                PAIR ? "pair" : "single", a.M, a.N, a.K, (long long)tiles, p.splits, units, (long long)max_units,
-                units * C::NH);
-    const int smem = smem_bytes<PAIR>();
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        fprintf(stderr, "tasq tc: M=%d N=%d K=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, (long long)tiles,
+                p.splits, units);
+    const int smem = smem_bytes();
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     // programmatic dependent launch: the grid may start while the previous
     // kernel drains; it waits (griddepcontrol.wait) before reading inputs
     cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3(units * C::NH);
+    cfg.gridDim = dim3(units);
     cfg.blockDim = dim3(THREADS);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[2];
+    cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
-    int nattr = 1;
-    if (PAIR) {
-        attr[1].id = cudaLaunchAttributeClusterDimension;
-        attr[1].val.clusterDim.x = 2;
-        attr[1].val.clusterDim.y = 1;
-        attr[1].val.clusterDim.z = 1;
-        nattr = 2;
-    }
     cfg.attrs = attr;
-    cfg.numAttrs = nattr;
-    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel<PAIR>, p, tm_x, tm_w);
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel, p, tm_x, tm_w);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaSuccess && p.splits > 1) {
         const int64_t total = int64_t(a.M) * (a.N / 4);
@@ -895,7 +852,7 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         rc.gridDim = dim3(unsigned(blocks < 8 * num_sms ? blocks : 8 * num_sms));
         rc.blockDim = dim3(256);
         rc.stream = st;
-        rc.attrs = attr;  // programmatic dependent launch only
+        rc.attrs = attr;  // programmatic dependent launch
         rc.numAttrs = 1;
         e = cudaLaunchKernelEx(&rc, splitk_epilogue_kernel, a, static_cast<const int32_t*>(p.split_out), p.splits);
         if (e == cudaSuccess) e = cudaGetLastError();
@@ -904,7 +861,7 @@ cudaError_t launch_variant(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         // report what the kernel asked for, to make the failure actionable
         static char msg[256];
         cudaFuncAttributes fa{};
-        cudaFuncGetAttributes(&fa, gemm_tc_kernel<PAIR>);
+        cudaFuncGetAttributes(&fa, gemm_tc_kernel);
         snprintf(msg, sizeof msg,
                  "launch out of resources: %d threads x %d registers, %d B dynamic smem (kernel max %d threads, "
                  "%zu B static smem)",
@@ -924,18 +881,15 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         return cudaSuccess;
     }
     if (a.M == 0 || a.N == 0) return cudaSuccess;
-    // The 1-SM kernel by default; TASQ_TC_PAIRS=1 selects the 2-SM variant
-    // (correct, but its cross-CTA barrier round trips keep it slower here).
-    static const bool pairs = [] {
-        const char* v = getenv("TASQ_TC_PAIRS");
-        return v && v[0] == '1';
-    }();
-    return pairs ? launch_variant<true>(a, num_sms, st, why) : launch_variant<false>(a, num_sms, st, why);
+    return launch_tc(a, num_sms, st, why);
 }
 
 #ifdef TASQ_TRACE
 extern "C" __attribute__((visibility("default"))) int tasq_debug_trace(void* host, size_t bytes) {
     return (int)cudaMemcpyFromSymbol(host, g_tasq_trace, bytes < sizeof(g_tasq_trace) ? bytes : sizeof(g_tasq_trace));
+}
+extern "C" __attribute__((visibility("default"))) int tasq_debug_events(void* host, size_t bytes) {
+    return (int)cudaMemcpyFromSymbol(host, g_tasq_ev, bytes < sizeof(g_tasq_ev) ? bytes : sizeof(g_tasq_ev));
 }
 #endif
 

@@ -428,18 +428,3 @@ def test_quotient_routine_matches_ieee_division(ctx):
     torch.cuda.synchronize()
     assert int(mism.item()) == 0
 
-
-def test_pair_variant_parity_subprocess():
-    """The 2-SM (cta_group::2) variant of the tensor-core kernel is selected
-    per process (TASQ_TC_PAIRS=1); run a representative subset of the
-    tensor-core parity tests under it in a child process."""
-    import os
-    import subprocess
-    import sys
-    env = dict(os.environ, TASQ_TC_PAIRS="1")
-    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-m", "gpu", "-p", "no:cacheprovider",
-                        os.path.join(root, "tests", "test_gpu_parity.py"), "-k",
-                        "tc and (single_linear or ragged or extreme or uniform_codes or conv_small or stage_from)"],
-                       cwd=root, env=env, capture_output=True, text=True, timeout=600)
-    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-2000:]
