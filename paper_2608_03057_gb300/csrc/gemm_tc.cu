@@ -33,6 +33,7 @@
 // tensor memory and returns.
 #include <cstdio>
 #include <cstdlib>
+#include <type_traits>
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -210,12 +211,13 @@ struct TileCoord {
     int tok0, img, h0, w0;
 };
 
+template <bool CONV>
 __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
     TileCoord c;
     c.ch0 = (t % p.tiles_ch) * BCH;
     const int tt = t / p.tiles_ch;
     c.tok0 = c.img = c.h0 = c.w0 = 0;
-    if (p.conv) {
+    if constexpr (CONV) {
         const int per_img = p.tiles_h * p.tiles_w;
         c.img = tt / per_img;
         c.h0 = ((tt % per_img) / p.tiles_w) * p.bhx;
@@ -226,6 +228,9 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
     return c;
 }
 
+// CONV selects the implicit-GEMM 3x3 convolution (one instantiation per
+// operand layout, so neither pays for the other's index arithmetic).
+template <bool CONV>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w) {
@@ -277,7 +282,7 @@ __global__ void __maxnreg__(96)
         // so their first tiles can be pulled into L2 before the wait below (a
         // prefetch only: nothing reaches shared memory before the wait).
         const Work wk = work_item(p, unit, KT, chunk);
-        const int ch0 = tile_coord(p, wk.t).ch0;
+        const int ch0 = tile_coord<CONV>(p, wk.t).ch0;
         for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * BK, ch0);
     }
     // the prologue above overlaps the previous kernel; inputs are read only after it
@@ -291,7 +296,7 @@ __global__ void __maxnreg__(96)
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
-                const TileCoord tc = tile_coord(p, wk.t);
+                const TileCoord tc = tile_coord<CONV>(p, wk.t);
                 for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++j) {
                     TQ(0, j, 0);
                     if (j >= X_STAGES && !wt.wait(&s->kdone[(j - X_STAGES) % KDONE], ((j - X_STAGES) / KDONE) & 1)) {
@@ -305,7 +310,7 @@ __global__ void __maxnreg__(96)
 #pragma unroll
                     for (int hh = 0; hh < 2; ++hh) {
                         const int kh = kb * BK + hh * XK;
-                        if (p.conv) {
+                        if constexpr (CONV) {
                             // a 128-wide K block may straddle two taps when Cin % 128 == 64
                             const int tap = kh / a.Cin, c0 = kh - tap * a.Cin;
                             ptx::tma_load_4d(dst + hh * X_HALF, &tm_x, fb, c0, tc.w0 + tap % 3 - 1, tc.h0 + tap / 3 - 1,
@@ -332,7 +337,7 @@ __global__ void __maxnreg__(96)
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
-                const int ch0 = tile_coord(p, wk.t).ch0;
+                const int ch0 = tile_coord<CONV>(p, wk.t).ch0;
                 for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++nw, rw.next()) {
                     if (!wt.wait(&s->wempty[rw.slot], rw.phase ^ 1)) {
                         ok = false;
@@ -459,13 +464,13 @@ __global__ void __maxnreg__(96)
         const int r = q * 32 + lane;
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
-        const int32_t* ts_b = p.conv ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
+        const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
         int cc = 0;
         bool ok = true;
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
             const int nchunks = wk.nch;
-            const TileCoord tc = tile_coord(p, wk.t);
+            const TileCoord tc = tile_coord<CONV>(p, wk.t);
             const int n = tc.ch0 + r;
             const bool n_ok = n < a.N;
             // row sums as fp32: |sum| < 2^24, so the values and every partial sum
@@ -477,7 +482,7 @@ __global__ void __maxnreg__(96)
             if (n_ok) {
                 cw = a.cw[n];
                 bias = a.bias[n];
-                if (p.conv) {
+                if constexpr (CONV) {
 #pragma unroll
                     for (int i = 0; i < 9; ++i) ts[i] = __int2float_rn(ts_b[int64_t(n) * 9 + i]);
                 } else {
@@ -494,7 +499,7 @@ __global__ void __maxnreg__(96)
             for (int gi = 0; gi < 2; ++gi) {
                 const int jt = (2 * part + gi) * 32 + lane;
                 int tok = -1, tap = 0;
-                if (p.conv) {
+                if constexpr (CONV) {
                     const int hh = tc.h0 + (jt >> p.bw_log2), ww = tc.w0 + (jt & ((1 << p.bw_log2) - 1));
                     if (hh < a.H && ww < a.W) {
                         tok = (tc.img * a.H + hh) * a.W + ww;
@@ -518,12 +523,14 @@ __global__ void __maxnreg__(96)
             __syncwarp();
             // Epilogue of 16 consecutive columns j0..j0+15 of group g from exact
             // accumulator values (float-held integers when `fl`, else int32).
-            auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], bool fl, bool all_tok) {
+            // FL: the accumulator values are float-held integers (single-chunk tiles), else int32
+            auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag, bool all_tok) {
+                constexpr bool fl = decltype(fl_tag)::value;
                 const int g = 2 * part + gi;
                 const float* my_al = s->ep_al[e][gi];
                 const float* my_zc = s->ep_zc[e][gi];
                 const int* my_tok = s->ep_tok[e][gi];
-                const int* my_tap = s->ep_tap[e][gi];
+                [[maybe_unused]] const int* my_tap = s->ep_tap[e][gi];
                 uint32_t yb2[8];
 #pragma unroll
                 for (int j4 = 0; j4 < 4; ++j4) {
@@ -532,19 +539,21 @@ __global__ void __maxnreg__(96)
                     const float al[4] = {al4.x, al4.y, al4.z, al4.w};
                     const float zc[4] = {zc4.x, zc4.y, zc4.z, zc4.w};
                     int4 tp4 = make_int4(0, 0, 0, 0);
-                    if (p.conv) tp4 = *reinterpret_cast<const int4*>(my_tap + j0 + 4 * j4);
-                    const int tp[4] = {tp4.x, tp4.y, tp4.z, tp4.w};
+                    if constexpr (CONV) tp4 = *reinterpret_cast<const int4*>(my_tap + j0 + 4 * j4);
+                    [[maybe_unused]] const int tp[4] = {tp4.x, tp4.y, tp4.z, tp4.w};
                     float yf[4];
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
                         float rsum = rs;
-                        if (p.conv) {
+                        if constexpr (CONV) {
                             rsum = 0.f;
 #pragma unroll
                             for (int k9 = 0; k9 < 9; ++k9) rsum = __fadd_rn(rsum, (tp[u] >> k9) & 1 ? ts[k9] : 0.f);
                         }
                         const uint32_t raw = v[4 * j4 + u];
-                        const float acc_f = fl ? __uint_as_float(raw) : __int2float_rn(int(raw));
+                        float acc_f;
+                        if constexpr (fl) acc_f = __uint_as_float(raw);
+                        else acc_f = __int2float_rn(int(raw));
                         yf[u] = __fmaf_rn(__fmaf_rn(zc[u], rsum, acc_f), __fmul_rn(al[u], cw), bias);
                     }
                     // two results per round-to-nearest-even conversion
@@ -567,7 +576,7 @@ __global__ void __maxnreg__(96)
                 for (int rr = 0; rr < 2; ++rr) {
                     const int t = rr * 8 + (lane >> 2);  // token row within the 16
                     const uint4 val = *reinterpret_cast<const uint4*>(stg + t * 32 + qc * 8);
-                    const int tok = all_tok && !p.conv ? tc.tok0 + g * 32 + j0 + t : my_tok[j0 + t];
+                    const int tok = all_tok && !CONV ? tc.tok0 + g * 32 + j0 + t : my_tok[j0 + t];
                     if (tok >= 0 && nq < a.N) *reinterpret_cast<uint4*>(a.y + int64_t(tok) * a.N + nq) = val;
                 }
                 if (a.acc && n_ok) {  // int32 accumulators (a debugging output): plain stores
@@ -630,7 +639,8 @@ __global__ void __maxnreg__(96)
                                 }
                             }
                         } else if (last) {
-                            finish16(gi, h * 16, v, nchunks == 1, all_tok);
+                            if (nchunks == 1) finish16(gi, h * 16, v, std::true_type{}, all_tok);
+                            else finish16(gi, h * 16, v, std::false_type{}, all_tok);
                         }
                         if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 4 + 2 * h);
                     }
@@ -829,7 +839,8 @@ cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const cha
         fprintf(stderr, "tasq tc: M=%d N=%d K=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, (long long)tiles,
                 p.splits, units);
     const int smem = smem_bytes();
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    auto kernel = p.conv ? gemm_tc_kernel<true> : gemm_tc_kernel<false>;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     // programmatic dependent launch: the grid may start while the previous
     // kernel drains; it waits (griddepcontrol.wait) before reading inputs
@@ -843,7 +854,7 @@ cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const cha
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel, p, tm_x, tm_w);
+    e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaSuccess && p.splits > 1) {
         const int64_t total = int64_t(a.M) * (a.N / 4);
@@ -861,7 +872,7 @@ cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const cha
         // report what the kernel asked for, to make the failure actionable
         static char msg[256];
         cudaFuncAttributes fa{};
-        cudaFuncGetAttributes(&fa, gemm_tc_kernel);
+        cudaFuncGetAttributes(&fa, kernel);
         snprintf(msg, sizeof msg,
                  "launch out of resources: %d threads x %d registers, %d B dynamic smem (kernel max %d threads, "
                  "%zu B static smem)",

@@ -47,6 +47,30 @@ def test_quant_weights_bitexact(ctx, oracle, dtype):
     assert np.array_equal(al.cpu().numpy(), ref["alpha"])
 
 
+def _near_boundary_rows(x, r0, n_bits, mode, nrows=8):
+    """Rows whose values sit within a few ulps of the rounding boundaries
+    x / alpha + z = k + 1/2 (scale and offset computed as the quantizer does,
+    in fp32), so that any shortcut in the division or the rounding shows up."""
+    K = x.shape[1]
+    qmax = np.float32((1 << n_bits) - 1)
+    f = np.float32
+    for i in range(nrows):
+        A = f(0.37 + 0.61 * i)
+        row = x[r0 + i]
+        row[0], row[1] = A, -A if mode == tasq.TASQ_SYMRANGE else -f(0.5) * A
+        lo, hi = (-A, A) if mode == tasq.TASQ_SYMRANGE else (row[1], A)
+        alpha = f(f(hi - lo) / qmax)
+        z = f(f(-lo) / alpha)
+        k = np.arange(K - 2) % int(qmax)
+        base = ((k + f(0.5) - z).astype(np.float32) * alpha).astype(np.float32)
+        steps = (np.arange(K - 2) % 7) - 3
+        v = base.copy()
+        for _ in range(3):
+            v = np.where(steps > 0, np.nextafter(v, np.float32(np.inf)), np.where(steps < 0, np.nextafter(v, np.float32(-np.inf)), v))
+            steps = steps - np.sign(steps)
+        row[2:] = np.clip(v, lo, hi)
+
+
 @pytest.mark.parametrize("code_fmt", [tasq.TASQ_CODES_S8, tasq.TASQ_CODES_F16])
 @pytest.mark.parametrize("mode", [tasq.TASQ_SYMRANGE, tasq.TASQ_ASYM])
 @pytest.mark.parametrize("n_bits", [8, 4])
@@ -58,6 +82,8 @@ def test_quant_act_per_token_bitexact(ctx, oracle, code_fmt, mode, n_bits, dtype
     x[9] = np.abs(x[9]) + 0.5  # one-signed row
     x[11, :] = 3.0
     x[11, 5] = 2.5      # exact ties of the rounding
+    _near_boundary_rows(x, 13, n_bits, mode)
+    x[21] = 1000.0 + workloads.uniform((K,), seed=4, lo=0.0, hi=1.0)  # far from zero: large quotients, small range
     if dtype == tasq.TASQ_BF16:
         xd, x = G.to_bf16(x)
     else:
