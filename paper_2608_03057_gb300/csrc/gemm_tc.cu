@@ -63,12 +63,21 @@ __device__ unsigned long long g_tasq_ev[512][12][2];
             g_tasq_ev[blockIdx.x][ev][1] = clock64();             \
         }                                                         \
     } while (0)
+// TF(call, k): steps of the epilogue's 16-column finishing of CTA 0, warp 6
+__device__ unsigned long long g_tasq_fin[64][8];
+#define TF(call, k)                                                                      \
+    do {                                                                                 \
+        if (blockIdx.x == 0 && warp == 6 && lane == 0 && (call) < 64) g_tasq_fin[call][k] = clock64(); \
+    } while (0)
 #else
 #define TQ(role, it, k) \
     do {                \
     } while (0)
 #define TE(ev) \
     do {       \
+    } while (0)
+#define TF(call, k) \
+    do {            \
     } while (0)
 #endif
 
@@ -354,8 +363,6 @@ __global__ void __maxnreg__(96)
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
         if (lane == 0) {
-            // B descriptors differ only in their start-address field (address >> 4)
-            const uint64_t bdesc0 = ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[0]));
             int it = 0, cc = 0;
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
@@ -380,14 +387,13 @@ __global__ void __maxnreg__(96)
                         TQ(1, it, 1);
                         if (it == 0) TE(4);
                         const uint32_t acol = tmem + A_COL + (it % ASLOTS) * A_SLOT_COLS;
-                        const uint64_t bdesc = bdesc0 + uint64_t((it % X_STAGES) * (X_STAGE >> 4));
-#pragma unroll
-                        for (int k = 0; k < BK / 16; ++k) {
-                            // K step of 16 codes: 32 bytes along the swizzled 128-byte row, the
-                            // second 64-wide atom X_HALF further on
-                            const uint64_t bk = bdesc + uint64_t(((k >> 2) * X_HALF + (k & 3) * 32) >> 4);
-                            if (k == 0 && kb == kb0) ptx::mma_f16_ts(d, acol, bk, IDESC, 0u);
-                            else ptx::mma_f16_ts(d, acol + k * 8, bk, IDESC, 1u);
+                        for (int hh = 0; hh < BK / XK; ++hh) {
+                            // one 64-wide swizzle atom; a K step of 16 codes is 32 bytes along its rows
+                            const uint64_t bdesc =
+                                ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[it % X_STAGES] + hh * X_HALF));
+                            for (int kk = 0; kk < XK / 16; ++kk)
+                                ptx::mma_f16_ts(d, acol + (hh * (XK / 16) + kk) * 8, bdesc + uint64_t((kk * 32) >> 4),
+                                                IDESC, (kb > kb0 || hh > 0 || kk > 0) ? 1u : 0u);
                         }
                         TQ(1, it, 2);
                         ptx::mma_commit(ptx::smem_u32(&s->kdone[it % KDONE]));
@@ -466,6 +472,9 @@ __global__ void __maxnreg__(96)
         const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
         const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
         int cc = 0;
+#ifdef TASQ_TRACE
+        int fcall = 0;
+#endif
         bool ok = true;
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
@@ -526,6 +535,7 @@ __global__ void __maxnreg__(96)
             // FL: the accumulator values are float-held integers (single-chunk tiles), else int32
             auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag, bool all_tok) {
                 constexpr bool fl = decltype(fl_tag)::value;
+                TF(fcall, 0);
                 const int g = 2 * part + gi;
                 const float* my_al = s->ep_al[e][gi];
                 const float* my_zc = s->ep_zc[e][gi];
@@ -563,13 +573,16 @@ __global__ void __maxnreg__(96)
                         yb2[2 * j4 + u / 2] = *reinterpret_cast<const uint32_t*>(&hb);
                     }
                 }
+                TF(fcall, 1);
                 // Transpose the warp's 32 channels x 16 tokens through shared memory so
                 // each token row (32 channels, 64 bytes) is written with 16-byte stores.
                 uint16_t* stg = s->ep_stage[e];
                 __syncwarp();
+                TF(fcall, 2);
 #pragma unroll
                 for (int j = 0; j < 16; ++j) stg[j * 32 + lane] = uint16_t(yb2[j >> 1] >> (16 * (j & 1)));
                 __syncwarp();
+                TF(fcall, 3);
                 const int qc = lane & 3;  // 8-channel chunk of the row
                 const int nq = tc.ch0 + (warp & 3) * 32 + qc * 8;
 #pragma unroll
@@ -579,6 +592,10 @@ __global__ void __maxnreg__(96)
                     const int tok = all_tok && !CONV ? tc.tok0 + g * 32 + j0 + t : my_tok[j0 + t];
                     if (tok >= 0 && nq < a.N) *reinterpret_cast<uint4*>(a.y + int64_t(tok) * a.N + nq) = val;
                 }
+                TF(fcall, 4);
+#ifdef TASQ_TRACE
+                ++fcall;
+#endif
                 if (a.acc && n_ok) {  // int32 accumulators (a debugging output): plain stores
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
@@ -898,6 +915,9 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
 #ifdef TASQ_TRACE
 extern "C" __attribute__((visibility("default"))) int tasq_debug_trace(void* host, size_t bytes) {
     return (int)cudaMemcpyFromSymbol(host, g_tasq_trace, bytes < sizeof(g_tasq_trace) ? bytes : sizeof(g_tasq_trace));
+}
+extern "C" __attribute__((visibility("default"))) int tasq_debug_fin(void* host, size_t bytes) {
+    return (int)cudaMemcpyFromSymbol(host, g_tasq_fin, bytes < sizeof(g_tasq_fin) ? bytes : sizeof(g_tasq_fin));
 }
 extern "C" __attribute__((visibility("default"))) int tasq_debug_events(void* host, size_t bytes) {
     return (int)cudaMemcpyFromSymbol(host, g_tasq_ev, bytes < sizeof(g_tasq_ev) ? bytes : sizeof(g_tasq_ev));
