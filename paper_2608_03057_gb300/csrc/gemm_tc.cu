@@ -85,31 +85,45 @@ namespace tasq {
 namespace {
 
 constexpr int BCH = 128;          // output channels per tile (MMA M)
-constexpr int BTOK = 192;         // tokens / output pixels per tile (MMA N)
 constexpr int BK = 128;           // K per weight stage and per tensor-memory slot of converted weights
 constexpr int XK = 64;            // K per activation TMA box (one 128-byte swizzle atom of fp16 codes)
-constexpr int X_STAGES = 3;       // activation stages of BK
 constexpr int W_STAGES = 3;
 constexpr int ASLOTS = 2;         // converted-weight slots in tensor memory
 constexpr int KDONE = 6;          // K-block completion barriers (a multiple of X_STAGES and ASLOTS)
 constexpr int EPI_WARP0 = 6;      // first epilogue warp
 constexpr int EPI_WARPS = 12;     // three per tensor-memory lane quadrant
+constexpr int EPI_PARTS = EPI_WARPS / 4;           // epilogue warps per lane quadrant
 constexpr int WPROD_WARP = EPI_WARP0 + EPI_WARPS;  // weight-tile producer
 constexpr int THREADS = (WPROD_WARP + 1) * 32;
-constexpr int X_HALF = BTOK * XK * 2;   // 24 KB of fp16 codes, 128-byte rows
-constexpr int X_STAGE = 2 * X_HALF;
 constexpr int W_STAGE = BCH * BK;       // 16 KB int8 codes, 128-byte rows
-constexpr int GROUPS = BTOK / 32;       // 32-token column groups of the accumulator
-static_assert(GROUPS == 2 * EPI_WARPS / 4, "each epilogue warp drains two groups");
-static_assert(BK == 2 * XK, "a stage is two 64-wide swizzle atoms");
-static_assert(KDONE % X_STAGES == 0 && KDONE % ASLOTS == 0, "completion ring covers both reuse distances");
-// tensor memory columns
-constexpr uint32_t ACC_COL = 0;           // 2 x BTOK fp32 accumulators
-constexpr uint32_t A_COL = 2 * BTOK;      // ASLOTS x BK/2 columns (fp16 pairs)
 constexpr uint32_t A_SLOT_COLS = BK / 2;
 constexpr uint32_t TMEM_COLS = 512;
-static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
-constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BTOK);
+constexpr int MAX_GPW = 3;              // most 32-token groups one epilogue warp drains
+static_assert(BK == 2 * XK, "a stage is two 64-wide swizzle atoms");
+
+// Tile configuration.  BT tokens per tile (MMA N); NACC accumulator buffers in
+// tensor memory.  <192, 2>: the epilogue of one tile overlaps the next tile's
+// MMAs.  <256, 1>: a wider MMA (the tensor pipe rather than the issuing thread
+// bounds N = 256) for launches where every CTA gets a single tile; the
+// accumulator then only has to wait for the drain between certified chunks.
+template <int BT_, int NACC_>
+struct Cfg {
+    static constexpr int BT = BT_;
+    static constexpr int NACC = NACC_;
+    static constexpr int X_STAGES = NACC == 2 ? 3 : 2;  // activation stages of BK
+    static constexpr int X_HALF = BT * XK * 2;           // one 64-wide TMA box of fp16 codes
+    static constexpr int X_STAGE = 2 * X_HALF;
+    static constexpr int GROUPS = BT / 32;               // 32-token column groups of the accumulator
+    static constexpr int GPW = (GROUPS + EPI_PARTS - 1) / EPI_PARTS;  // groups per epilogue warp
+    static constexpr uint32_t ACC_COL = 0;               // NACC x BT fp32 accumulators
+    static constexpr uint32_t A_COL = NACC * BT;         // ASLOTS x BK/2 columns (fp16 pairs)
+    static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BT);
+    static_assert(KDONE % X_STAGES == 0 && KDONE % ASLOTS == 0, "completion ring covers both reuse distances");
+    static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
+    static_assert(GPW <= MAX_GPW && BT <= 256 && BT % 32 == 0, "tile shape");
+};
+using CfgStd = Cfg<192, 2>;
+using CfgWide = Cfg<256, 1>;
 
 // Synchronisation is arranged so that the single MMA-issuing thread, whose
 // per-instruction cost bounds the K loop, does one wait and one commit per K
@@ -123,25 +137,27 @@ constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BTOK);
 //                 with block j + 2.
 // The weight ring is separate: a weight stage is released as soon as the
 // converters have read it, so weight tiles run several K blocks ahead.
+template <class C>
 struct Smem {
-    uint8_t x[X_STAGES][X_STAGE];  // 1024-aligned (128-byte swizzle atoms)
+    uint8_t x[C::X_STAGES][C::X_STAGE];  // 1024-aligned (128-byte swizzle atoms)
     uint8_t w[W_STAGES][W_STAGE];
-    float ep_al[EPI_WARPS][2][32], ep_zc[EPI_WARPS][2][32];  // per warp, per group, per column
-    int ep_tok[EPI_WARPS][2][32], ep_tap[EPI_WARPS][2][32];
+    float ep_al[EPI_WARPS][C::GPW][32], ep_zc[EPI_WARPS][C::GPW][32];  // per warp, per group, per column
+    int ep_tok[EPI_WARPS][C::GPW][32], ep_tap[EPI_WARPS][C::GPW][32];
     alignas(16) uint16_t ep_stage[EPI_WARPS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
-    uint64_t xfull[X_STAGES], kdone[KDONE];
+    uint64_t xfull[C::X_STAGES], kdone[KDONE];
     uint64_t wfull[W_STAGES], wempty[W_STAGES];
-    uint64_t accfull[2], accempty[2];
+    uint64_t accfull[C::NACC], accempty[C::NACC];
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
 };
-constexpr int smem_bytes() { return int(sizeof(Smem)) + 1024; }
+template <class C>
+constexpr int smem_bytes() { return int(sizeof(Smem<C>)) + 1024; }
 
 struct TcParams {
     GemmArgs a;
     int conv;
-    int tiles_ch, tiles_tok;  // tiles of BCH channels x BTOK tokens
+    int tiles_ch, tiles_tok;  // tiles of BCH channels x BT tokens
     // conv: a token tile is a box of bhx rows x 2^bw_log2 pixels
     int bw_log2, bhx, tiles_w, tiles_h;
     // split-K: each tile's K blocks are cut into `splits` contiguous slices; a
@@ -165,8 +181,9 @@ __device__ __forceinline__ Work work_item(const TcParams& p, int w, int KT, int 
     return r;
 }
 
+template <class C>
 struct Waiter {
-    Smem* s;
+    Smem<C>* s;
     const GemmArgs* a;
     // Bounded wait on phase `parity` of an mbarrier; false after a timeout or
     // when another role has aborted the CTA.
@@ -220,7 +237,7 @@ struct TileCoord {
     int tok0, img, h0, w0;
 };
 
-template <bool CONV>
+template <bool CONV, int BT>
 __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
     TileCoord c;
     c.ch0 = (t % p.tiles_ch) * BCH;
@@ -232,23 +249,25 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
         c.h0 = ((tt % per_img) / p.tiles_w) * p.bhx;
         c.w0 = (tt % p.tiles_w) << p.bw_log2;
     } else {
-        c.tok0 = tt * BTOK;
+        c.tok0 = tt * BT;
     }
     return c;
 }
 
 // CONV selects the implicit-GEMM 3x3 convolution (one instantiation per
 // operand layout, so neither pays for the other's index arithmetic).
-template <bool CONV>
+template <bool CONV, class C>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w) {
+    constexpr int X_STAGES = C::X_STAGES, X_HALF = C::X_HALF, X_STAGE = C::X_STAGE, NACC = C::NACC;
+    constexpr int BT = C::BT, GPW = C::GPW;
     if (threadIdx.x == 0) TE(0);
     extern __shared__ uint8_t smem_raw[];
-    Smem* s = reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    Smem<C>* s = reinterpret_cast<Smem<C>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const GemmArgs& a = p.a;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const Waiter wt{s, &a};
+    const Waiter<C> wt{s, &a};
 
     const int b = resolve_bits(a);
     if (b == 0) return;  // uniform across the grid (a launch-wide check): nothing allocated yet
@@ -267,7 +286,7 @@ __global__ void __maxnreg__(96)
             ptx::mbar_init(ptx::smem_u32(&s->wfull[i]), 1);
             ptx::mbar_init(ptx::smem_u32(&s->wempty[i]), 4);  // the 4 converter warps
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < NACC; ++i) {
             ptx::mbar_init(ptx::smem_u32(&s->accfull[i]), 1);
             ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS);
         }
@@ -291,7 +310,7 @@ __global__ void __maxnreg__(96)
         // so their first tiles can be pulled into L2 before the wait below (a
         // prefetch only: nothing reaches shared memory before the wait).
         const Work wk = work_item(p, unit, KT, chunk);
-        const int ch0 = tile_coord<CONV>(p, wk.t).ch0;
+        const int ch0 = tile_coord<CONV, BT>(p, wk.t).ch0;
         for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * BK, ch0);
     }
     // the prologue above overlaps the previous kernel; inputs are read only after it
@@ -305,7 +324,7 @@ __global__ void __maxnreg__(96)
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
-                const TileCoord tc = tile_coord<CONV>(p, wk.t);
+                const TileCoord tc = tile_coord<CONV, BT>(p, wk.t);
                 for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++j) {
                     TQ(0, j, 0);
                     if (j >= X_STAGES && !wt.wait(&s->kdone[(j - X_STAGES) % KDONE], ((j - X_STAGES) / KDONE) & 1)) {
@@ -346,7 +365,7 @@ __global__ void __maxnreg__(96)
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
-                const int ch0 = tile_coord<CONV>(p, wk.t).ch0;
+                const int ch0 = tile_coord<CONV, BT>(p, wk.t).ch0;
                 for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++nw, rw.next()) {
                     if (!wt.wait(&s->wempty[rw.slot], rw.phase ^ 1)) {
                         ok = false;
@@ -368,13 +387,13 @@ __global__ void __maxnreg__(96)
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
                 for (int c = 0; c < wk.nch && ok; ++c, ++cc) {
-                    const int buf = cc & 1;
-                    if (!wt.wait(&s->accempty[buf], ((cc >> 1) & 1) ^ 1)) {
+                    const int buf = cc % NACC;
+                    if (!wt.wait(&s->accempty[buf], ((cc / NACC) & 1) ^ 1)) {
                         ok = false;
                         break;
                     }
                     ptx::tc_fence_after();
-                    const uint32_t d = tmem + ACC_COL + buf * BTOK;
+                    const uint32_t d = tmem + C::ACC_COL + buf * BT;
                     const int kb0 = wk.kb_lo + c * chunk, kb_end = min(wk.kb_hi, kb0 + chunk);
                     for (int kb = kb0; kb < kb_end; ++kb, ++it) {
                         TQ(1, it, 0);
@@ -386,14 +405,14 @@ __global__ void __maxnreg__(96)
                         ptx::tc_fence_after();
                         TQ(1, it, 1);
                         if (it == 0) TE(4);
-                        const uint32_t acol = tmem + A_COL + (it % ASLOTS) * A_SLOT_COLS;
+                        const uint32_t acol = tmem + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
                         for (int hh = 0; hh < BK / XK; ++hh) {
                             // one 64-wide swizzle atom; a K step of 16 codes is 32 bytes along its rows
                             const uint64_t bdesc =
                                 ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[it % X_STAGES] + hh * X_HALF));
                             for (int kk = 0; kk < XK / 16; ++kk)
                                 ptx::mma_f16_ts(d, acol + (hh * (XK / 16) + kk) * 8, bdesc + uint64_t((kk * 32) >> 4),
-                                                IDESC, (kb > kb0 || hh > 0 || kk > 0) ? 1u : 0u);
+                                                C::IDESC, (kb > kb0 || hh > 0 || kk > 0) ? 1u : 0u);
                         }
                         TQ(1, it, 2);
                         ptx::mma_commit(ptx::smem_u32(&s->kdone[it % KDONE]));
@@ -451,7 +470,7 @@ __global__ void __maxnreg__(96)
                 }
                 if (warp == 2 && lane == 0) TQ(2, it, 3);
                 {
-                    const uint32_t dst = lane_base + A_COL + (it % ASLOTS) * A_SLOT_COLS;
+                    const uint32_t dst = lane_base + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
                     ptx::tmem_st32(dst, *reinterpret_cast<const uint32_t(*)[32]>(&f[0]));
                     ptx::tmem_st32(dst + 32, *reinterpret_cast<const uint32_t(*)[32]>(&f[32]));
                 }
@@ -479,7 +498,7 @@ __global__ void __maxnreg__(96)
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
             const int nchunks = wk.nch;
-            const TileCoord tc = tile_coord<CONV>(p, wk.t);
+            const TileCoord tc = tile_coord<CONV, BT>(p, wk.t);
             const int n = tc.ch0 + r;
             const bool n_ok = n < a.N;
             // row sums as fp32: |sum| < 2^24, so the values and every partial sum
@@ -502,11 +521,11 @@ __global__ void __maxnreg__(96)
             // Token index, (conv) in-bounds taps and per-token scales of column j = lane of
             // each of this warp's two groups, written to this warp's shared scratch before
             // the accumulator wait, so the global loads' latency hides under the MMAs.
-            bool all_tok_g[2];
+            bool all_tok_g[GPW];
             __syncwarp();  // the previous tile's reads of the scratch are done
 #pragma unroll
-            for (int gi = 0; gi < 2; ++gi) {
-                const int jt = (2 * part + gi) * 32 + lane;
+            for (int gi = 0; gi < GPW; ++gi) {
+                const int jt = (part * GPW + gi) * 32 + lane;  // beyond the tile when part * GPW + gi >= GROUPS
                 int tok = -1, tap = 0;
                 if constexpr (CONV) {
                     const int hh = tc.h0 + (jt >> p.bw_log2), ww = tc.w0 + (jt & ((1 << p.bw_log2) - 1));
@@ -521,7 +540,10 @@ __global__ void __maxnreg__(96)
                             }
                     }
                 } else {
-                    tok = tc.tok0 + jt < a.M ? tc.tok0 + jt : -1;
+                    tok = jt < BT && tc.tok0 + jt < a.M ? tc.tok0 + jt : -1;
+                }
+                if constexpr (CONV) {
+                    if (jt >= BT) tok = -1;
                 }
                 s->ep_tok[e][gi][lane] = tok;
                 s->ep_tap[e][gi][lane] = tap;
@@ -536,7 +558,7 @@ __global__ void __maxnreg__(96)
             auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag, bool all_tok) {
                 constexpr bool fl = decltype(fl_tag)::value;
                 TF(fcall, 0);
-                const int g = 2 * part + gi;
+                const int g = part * GPW + gi;
                 const float* my_al = s->ep_al[e][gi];
                 const float* my_zc = s->ep_zc[e][gi];
                 const int* my_tok = s->ep_tok[e][gi];
@@ -606,13 +628,13 @@ __global__ void __maxnreg__(96)
             };
 
             // Multi-chunk tiles keep their int32 running sums in this warp's slice of the
-            // per-CTA scratch (32 channels x 64 tokens); each value is only re-read by
-            // the thread that wrote it.
-            int32_t* my_part = a.part + (int64_t(blockIdx.x) * EPI_WARPS + e) * (64 * 32) + lane;
+            // per-CTA scratch (32 channels x 32 * MAX_GPW tokens); each value is only
+            // re-read by the thread that wrote it.
+            int32_t* my_part = a.part + (int64_t(blockIdx.x) * EPI_WARPS + e) * (MAX_GPW * 32 * 32) + lane;
             for (int c = 0; c < nchunks; ++c, ++cc) {
-                const int buf = cc & 1;
+                const int buf = cc % NACC;
                 if (warp == 6 && lane == 0) TQ(3, cc, 0);
-                if (!wt.wait(&s->accfull[buf], (cc >> 1) & 1)) {
+                if (!wt.wait(&s->accfull[buf], (cc / NACC) & 1)) {
                     ok = false;
                     break;
                 }
@@ -620,11 +642,12 @@ __global__ void __maxnreg__(96)
                 if (warp == 6 && lane == 0 && cc == 0) TE(6);
                 if (warp == 6 && lane == 0) TE(7);
                 ptx::tc_fence_after();
-                const uint32_t acc_base = lane_base + ACC_COL + buf * BTOK;
+                const uint32_t acc_base = lane_base + C::ACC_COL + buf * BT;
                 const bool last = c == nchunks - 1;
 #pragma unroll 1
-                for (int gi = 0; gi < 2; ++gi) {
-                    const int g = 2 * part + gi;
+                for (int gi = 0; gi < GPW; ++gi) {
+                    const int g = part * GPW + gi;
+                    if (g >= C::GROUPS) break;
                     const bool all_tok = all_tok_g[gi];
 #pragma unroll 1
                     for (int h = 0; h < 2; ++h) {
@@ -758,11 +781,36 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 
 }  // namespace
 
-size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * EPI_WARPS * 64 * 32 * sizeof(int32_t); }
+size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * EPI_WARPS * MAX_GPW * 32 * 32 * sizeof(int32_t); }
 
 namespace {
 
-cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
+// Token tiles of a launch with BT-token tiles (conv: boxes of bhx rows x 2^bwl
+// pixels, 2^bwl dividing BT).
+struct TokTiling {
+    int64_t tiles;
+    int bw_log2, bhx, tiles_w, tiles_h;
+};
+TokTiling token_tiling(const GemmArgs& a, int BT) {
+    TokTiling t{};
+    if (a.Cin) {
+        int bwl = 0;
+        while ((1 << bwl) < a.W && (1 << bwl) < 64) ++bwl;
+        t.bw_log2 = bwl;
+        t.bhx = BT >> bwl;
+        const int bw = 1 << bwl;
+        t.tiles_w = (a.W + bw - 1) / bw;
+        t.tiles_h = (a.H + t.bhx - 1) / t.bhx;
+        t.tiles = int64_t(a.B) * t.tiles_h * t.tiles_w;
+    } else {
+        t.tiles = (a.M + BT - 1) / BT;
+    }
+    return t;
+}
+
+template <class C>
+cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
+    constexpr int BTOK = C::BT;
     auto encode = get_encode();
     if (!encode) {
         *why = "cuTensorMapEncodeTiled is unavailable";
@@ -779,15 +827,14 @@ cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const cha
             *why = "convolution needs Cin % 64 == 0";
             return cudaSuccess;
         }
-        // box of bhx rows x 2^bwl pixels; 2^bwl must divide BTOK (192 = 64 * 3)
-        int bwl = 0;
-        while ((1 << bwl) < a.W && (1 << bwl) < 64) ++bwl;
-        p.bw_log2 = bwl;
-        p.bhx = BTOK >> bwl;
-        const int bw = 1 << bwl;
-        p.tiles_w = (a.W + bw - 1) / bw;
-        p.tiles_h = (a.H + p.bhx - 1) / p.bhx;
-        const int64_t tok_tiles = int64_t(a.B) * p.tiles_h * p.tiles_w;
+        // box of bhx rows x 2^bwl pixels; 2^bwl divides BTOK (192 = 64 * 3, 256)
+        const TokTiling tt = token_tiling(a, BTOK);
+        p.bw_log2 = tt.bw_log2;
+        p.bhx = tt.bhx;
+        const int bw = 1 << tt.bw_log2;
+        p.tiles_w = tt.tiles_w;
+        p.tiles_h = tt.tiles_h;
+        const int64_t tok_tiles = tt.tiles;
         if (tok_tiles * p.tiles_ch > 0x7FFFFFFF) {
             *why = "too many tiles";
             return cudaSuccess;
@@ -833,7 +880,7 @@ cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const cha
     // not reduced by splitting, only its K loop is.
     p.splits = 1;
     p.split_out = nullptr;
-    if (a.split_buf && tiles * 2 <= num_sms) {
+    if (C::NACC == 2 && a.split_buf && tiles * 2 <= num_sms) {
         const int KT = (a.K + BK - 1) / BK;
         int64_t S = num_sms / tiles;
         S = S < KT / 8 ? S : KT / 8;
@@ -855,8 +902,8 @@ cudaError_t launch_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const cha
     if (verbose)
         fprintf(stderr, "tasq tc: M=%d N=%d K=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, (long long)tiles,
                 p.splits, units);
-    const int smem = smem_bytes();
-    auto kernel = p.conv ? gemm_tc_kernel<true> : gemm_tc_kernel<false>;
+    const int smem = smem_bytes<C>();
+    auto kernel = p.conv ? gemm_tc_kernel<true, C> : gemm_tc_kernel<false, C>;
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     // programmatic dependent launch: the grid may start while the previous
@@ -909,7 +956,13 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         return cudaSuccess;
     }
     if (a.M == 0 || a.N == 0) return cudaSuccess;
-    return launch_tc(a, num_sms, st, why);
+    // The wide single-tile configuration when it covers the output in one wave
+    // of CTAs and the standard one would need more than one.
+    const int64_t tiles_ch = (a.N + BCH - 1) / BCH;
+    const int64_t std_tiles = tiles_ch * token_tiling(a, CfgStd::BT).tiles;
+    const int64_t wide_tiles = tiles_ch * token_tiling(a, CfgWide::BT).tiles;
+    if (std_tiles > num_sms && wide_tiles <= num_sms) return launch_cfg<CfgWide>(a, num_sms, st, why);
+    return launch_cfg<CfgStd>(a, num_sms, st, why);
 }
 
 #ifdef TASQ_TRACE

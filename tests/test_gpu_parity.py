@@ -205,6 +205,19 @@ def test_ragged_shapes(ctx, oracle, code_fmt, M, N, K):
 
 
 @pytest.mark.parametrize("code_fmt", ROUTES)
+def test_wide_tiles_ragged_full(ctx, oracle, code_fmt):
+    """A launch whose 256-token tiles fit one wave of CTAs (the wide, single-
+    accumulator configuration of the tensor-core route), with a ragged last
+    token tile and a ragged last channel tile, checked in full."""
+    M, N, K = 4000, 1096, 384
+    bits = [8, 3]
+    st = _setup_linear(ctx, oracle, M, N, K, bits, seed=7, code_fmt=code_fmt)
+    for stage, b in enumerate(bits):
+        y, acc = G.gemm(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+        _check_layer(oracle, st, b, y, acc)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
 def test_output_without_acc(ctx, oracle, code_fmt):
     M, N, K = 200, 128, 256
     st = _setup_linear(ctx, oracle, M, N, K, [6], code_fmt=code_fmt)
@@ -287,7 +300,8 @@ def test_stage_from_device_int(ctx, oracle, code_fmt):
 
 
 @pytest.mark.parametrize("code_fmt", ROUTES)
-@pytest.mark.parametrize("M,N,K", [(4096, 3456, 1152), (4096, 1152, 4608), (1200, 2240, 2240), (77, 1280, 2048)])
+@pytest.mark.parametrize("M,N,K", [(4096, 3456, 1152), (4096, 1152, 4608), (4096, 1152, 1152), (1200, 2240, 2240),
+                                   (77, 1280, 2048)])
 def test_full_size_sampled_rows(ctx, oracle, code_fmt, M, N, K):
     """Full-size layer shapes of the backbones, checked on sampled token rows
     (the oracle computes those rows one by one)."""
@@ -371,13 +385,15 @@ def test_conv_narrow_channels(ctx, oracle, B, H, W, Cin, Cout):
 
 
 @pytest.mark.parametrize("code_fmt", ROUTES)
-@pytest.mark.parametrize("C,HW", [(320, 64), (640, 32), (1280, 16)])
-def test_conv_full_size_sampled(ctx, oracle, code_fmt, C, HW):
+@pytest.mark.parametrize("C,HW,Cout", [(320, 64, 320), (640, 32, 640), (1280, 16, 1280), (64, 64, 1024)])
+def test_conv_full_size_sampled(ctx, oracle, code_fmt, C, HW, Cout):
+    """Full-size convolutions on sampled output pixels (borders included); the
+    64-channel, 1024-output case runs the wide single-tile configuration."""
     rng = workloads.rng(C)
     P = HW * HW
     border = [0, HW - 1, HW * (HW - 1), P - 1, HW // 2, HW * (HW // 2)]
     rows = np.unique(np.concatenate([border, rng.integers(0, P, 24)]))
-    _run_conv(ctx, oracle, 1, HW, HW, C, C, [5, 8], code_fmt, seed=C, rows=rows)
+    _run_conv(ctx, oracle, 1, HW, HW, C, Cout, [5, 8], code_fmt, seed=C, rows=rows)
 
 
 # ------------------------------------------------------ failure handling --
