@@ -89,7 +89,6 @@ constexpr int BK = 128;           // K per weight stage and per tensor-memory sl
 constexpr int XK = 64;            // K per activation TMA box (one 128-byte swizzle atom of fp16 codes)
 constexpr int W_STAGES = 3;
 constexpr int ASLOTS = 2;         // converted-weight slots in tensor memory
-constexpr int KDONE = 6;          // K-block completion barriers (a multiple of X_STAGES and ASLOTS)
 constexpr int EPI_WARP0 = 6;      // first epilogue warp
 constexpr int EPI_WARPS = 12;     // three per tensor-memory lane quadrant
 constexpr int EPI_PARTS = EPI_WARPS / 4;           // epilogue warps per lane quadrant
@@ -110,15 +109,21 @@ template <int BT_, int NACC_>
 struct Cfg {
     static constexpr int BT = BT_;
     static constexpr int NACC = NACC_;
-    static constexpr int X_STAGES = NACC == 2 ? 3 : 2;  // activation stages of BK
+    // Q activation stages per K block: 1 (a 128-K stage, one wait per K block on
+    // the MMA thread) or 2 (64-K stages released half a block earlier, for the
+    // N = 256 tile, whose MMAs leave the issuing thread time for a second wait)
+    static constexpr int Q = NACC == 2 ? 1 : 2;
+    static constexpr int X_STAGES = NACC == 2 ? 3 : 4;  // activation stages in the ring
     static constexpr int X_HALF = BT * XK * 2;           // one 64-wide TMA box of fp16 codes
-    static constexpr int X_STAGE = 2 * X_HALF;
+    static constexpr int X_STAGE = (2 / Q) * X_HALF;
+    static constexpr int DONE = 2 * X_STAGES;            // stage-completion barriers (ring of MMA commits)
     static constexpr int GROUPS = BT / 32;               // 32-token column groups of the accumulator
     static constexpr int GPW = (GROUPS + EPI_PARTS - 1) / EPI_PARTS;  // groups per epilogue warp
     static constexpr uint32_t ACC_COL = 0;               // NACC x BT fp32 accumulators
     static constexpr uint32_t A_COL = NACC * BT;         // ASLOTS x BK/2 columns (fp16 pairs)
     static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BT);
-    static_assert(KDONE % X_STAGES == 0 && KDONE % ASLOTS == 0, "completion ring covers both reuse distances");
+    static_assert(DONE % X_STAGES == 0 && DONE >= (ASLOTS + 1) * Q, "completion ring covers both reuse distances");
+    static_assert(Q == 1 || X_STAGES % 2 == 0, "first-half stages must keep their parity");
     static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
     static_assert(GPW <= MAX_GPW && BT <= 256 && BT % 32 == 0, "tile shape");
 };
@@ -126,15 +131,16 @@ using CfgStd = Cfg<192, 2>;
 using CfgWide = Cfg<256, 1>;
 
 // Synchronisation is arranged so that the single MMA-issuing thread, whose
-// per-instruction cost bounds the K loop, does one wait and one commit per K
-// block:
-//   xfull[j % 3]  completes when the activation stage of K block j has landed
-//                 (TMA transaction bytes) AND the four converter warps have
-//                 written its weights into tensor-memory slot j % 2;
-//   kdone[j % 6]  completes when the MMAs of K block j have finished; the
-//                 activation producer waits on it before refilling stage j % 3
-//                 with block j + 3, the converters before overwriting slot j % 2
-//                 with block j + 2.
+// per-instruction cost bounds the K loop, does one wait and one commit per
+// activation stage.  Stage u (u = Q j + i for part i of K block j):
+//   xfull[u % X_STAGES]  completes when its activation bytes have landed (TMA
+//                 transaction bytes) and, for the first stage of a K block,
+//                 when the four converter warps have written the block's
+//                 weights into tensor-memory slot j % 2;
+//   done[u % DONE]  completes when the MMAs reading stage u have finished; the
+//                 activation producer waits on it before refilling the stage
+//                 with u + X_STAGES, the converters (on the last stage of block
+//                 j) before overwriting slot j % 2 with block j + 2.
 // The weight ring is separate: a weight stage is released as soon as the
 // converters have read it, so weight tiles run several K blocks ahead.
 template <class C>
@@ -144,7 +150,7 @@ struct Smem {
     float ep_al[EPI_WARPS][C::GPW][32], ep_zc[EPI_WARPS][C::GPW][32];  // per warp, per group, per column
     int ep_tok[EPI_WARPS][C::GPW][32], ep_tap[EPI_WARPS][C::GPW][32];
     alignas(16) uint16_t ep_stage[EPI_WARPS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
-    uint64_t xfull[C::X_STAGES], kdone[KDONE];
+    uint64_t xfull[C::X_STAGES], done[C::DONE];
     uint64_t wfull[W_STAGES], wempty[W_STAGES];
     uint64_t accfull[C::NACC], accempty[C::NACC];
     uint64_t drain;
@@ -261,6 +267,7 @@ __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w) {
     constexpr int X_STAGES = C::X_STAGES, X_HALF = C::X_HALF, X_STAGE = C::X_STAGE, NACC = C::NACC;
+    constexpr int Q = C::Q, DONE = C::DONE;
     constexpr int BT = C::BT, GPW = C::GPW;
     if (threadIdx.x == 0) TE(0);
     extern __shared__ uint8_t smem_raw[];
@@ -279,9 +286,9 @@ __global__ void __maxnreg__(96)
     const int unit = int(blockIdx.x), units = int(gridDim.x);
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < X_STAGES; ++i)
-            ptx::mbar_init(ptx::smem_u32(&s->xfull[i]), 1 + 4);  // producer's expect_tx + 4 converter warps
-        for (int i = 0; i < KDONE; ++i) ptx::mbar_init(ptx::smem_u32(&s->kdone[i]), 1);  // the MMA commit
+        for (int i = 0; i < X_STAGES; ++i)  // producer's expect_tx (+ the 4 converter warps on first stages)
+            ptx::mbar_init(ptx::smem_u32(&s->xfull[i]), i % Q == 0 ? 1 + 4 : 1);
+        for (int i = 0; i < DONE; ++i) ptx::mbar_init(ptx::smem_u32(&s->done[i]), 1);  // the MMA commit
         for (int i = 0; i < W_STAGES; ++i) {
             ptx::mbar_init(ptx::smem_u32(&s->wfull[i]), 1);
             ptx::mbar_init(ptx::smem_u32(&s->wempty[i]), 4);  // the 4 converter warps
@@ -320,24 +327,24 @@ __global__ void __maxnreg__(96)
     if (warp == 0) {
         // --------------------------------------------- activation producer
         if (lane == 0) {
-            int j = 0;  // K blocks issued by this CTA
+            int u = 0;  // activation stages issued by this CTA
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
                 const TileCoord tc = tile_coord<CONV, BT>(p, wk.t);
-                for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++j) {
-                    TQ(0, j, 0);
-                    if (j >= X_STAGES && !wt.wait(&s->kdone[(j - X_STAGES) % KDONE], ((j - X_STAGES) / KDONE) & 1)) {
+                for (int kq = wk.kb_lo * Q; kq < wk.kb_hi * Q; ++kq, ++u) {
+                    TQ(0, u, 0);
+                    if (u >= X_STAGES && !wt.wait(&s->done[(u - X_STAGES) % DONE], ((u - X_STAGES) / DONE) & 1)) {
                         ok = false;
                         break;
                     }
-                    TQ(0, j, 1);
-                    const uint32_t fb = ptx::smem_u32(&s->xfull[j % X_STAGES]);
+                    TQ(0, u, 1);
+                    const uint32_t fb = ptx::smem_u32(&s->xfull[u % X_STAGES]);
                     ptx::mbar_arrive_expect_tx(fb, X_STAGE);
-                    const uint32_t dst = ptx::smem_u32(s->x[j % X_STAGES]);
+                    const uint32_t dst = ptx::smem_u32(s->x[u % X_STAGES]);
 #pragma unroll
-                    for (int hh = 0; hh < 2; ++hh) {
-                        const int kh = kb * BK + hh * XK;
+                    for (int hh = 0; hh < 2 / Q; ++hh) {
+                        const int kh = kq * (BK / Q) + hh * XK;
                         if constexpr (CONV) {
                             // a 128-wide K block may straddle two taps when Cin % 128 == 64
                             const int tap = kh / a.Cin, c0 = kh - tap * a.Cin;
@@ -353,9 +360,9 @@ __global__ void __maxnreg__(96)
             // the next kernel may be launched while this grid drains
             ptx::grid_launch_dependents();
             // copies still in flight must land before the CTA may exit: the MMAs
-            // of the last K blocks consumed them (or the CTA is aborting)
-            for (int i = j - X_STAGES < 0 ? 0 : j - X_STAGES; i < j; ++i)
-                wt.wait(&s->kdone[i % KDONE], (i / KDONE) & 1, true);
+            // of the last stages consumed them (or the CTA is aborting)
+            for (int i = u - X_STAGES < 0 ? 0 : u - X_STAGES; i < u; ++i)
+                wt.wait(&s->done[i % DONE], (i / DONE) & 1, true);
         }
     } else if (warp == WPROD_WARP) {
         // ------------------------------------------------ weight producer
@@ -395,27 +402,31 @@ __global__ void __maxnreg__(96)
                     ptx::tc_fence_after();
                     const uint32_t d = tmem + C::ACC_COL + buf * BT;
                     const int kb0 = wk.kb_lo + c * chunk, kb_end = min(wk.kb_hi, kb0 + chunk);
-                    for (int kb = kb0; kb < kb_end; ++kb, ++it) {
+                    for (int kb = kb0; kb < kb_end && ok; ++kb, ++it) {
                         TQ(1, it, 0);
-                        // activations landed and the converters wrote weight slot it % 2
-                        if (!wt.wait(&s->xfull[it % X_STAGES], (it / X_STAGES) & 1)) {
-                            ok = false;
-                            break;
-                        }
-                        ptx::tc_fence_after();
-                        TQ(1, it, 1);
-                        if (it == 0) TE(4);
                         const uint32_t acol = tmem + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
-                        for (int hh = 0; hh < BK / XK; ++hh) {
-                            // one 64-wide swizzle atom; a K step of 16 codes is 32 bytes along its rows
-                            const uint64_t bdesc =
-                                ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[it % X_STAGES] + hh * X_HALF));
-                            for (int kk = 0; kk < XK / 16; ++kk)
-                                ptx::mma_f16_ts(d, acol + (hh * (XK / 16) + kk) * 8, bdesc + uint64_t((kk * 32) >> 4),
-                                                C::IDESC, (kb > kb0 || hh > 0 || kk > 0) ? 1u : 0u);
+                        for (int i = 0; i < Q; ++i) {
+                            const int u = it * Q + i;
+                            // activations landed (and, for i == 0, the converters wrote slot it % 2)
+                            if (!wt.wait(&s->xfull[u % X_STAGES], (u / X_STAGES) & 1)) {
+                                ok = false;
+                                break;
+                            }
+                            ptx::tc_fence_after();
+                            if (i == 0) TQ(1, it, 1);
+                            if (it == 0 && i == 0) TE(4);
+                            for (int hh = 0; hh < 2 / Q; ++hh) {
+                                // one 64-wide swizzle atom; a K step of 16 codes is 32 bytes along its rows
+                                const uint64_t bdesc =
+                                    ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[u % X_STAGES] + hh * X_HALF));
+                                const int k0 = (i * (2 / Q) + hh) * (XK / 16);  // K step of 16 within the block
+                                for (int kk = 0; kk < XK / 16; ++kk)
+                                    ptx::mma_f16_ts(d, acol + (k0 + kk) * 8, bdesc + uint64_t((kk * 32) >> 4), C::IDESC,
+                                                    (kb > kb0 || k0 + kk > 0) ? 1u : 0u);
+                            }
+                            ptx::mma_commit(ptx::smem_u32(&s->done[u % DONE]));
                         }
                         TQ(1, it, 2);
-                        ptx::mma_commit(ptx::smem_u32(&s->kdone[it % KDONE]));
                         TQ(1, it, 3);
                     }
                     if (ok) ptx::mma_commit(ptx::smem_u32(&s->accfull[buf]));
@@ -464,7 +475,9 @@ __global__ void __maxnreg__(96)
                 if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->wempty[rw.slot]));
                 if (warp == 2 && lane == 0) TQ(2, it, 2);
                 // slot it % 2 last held K block it - 2: its MMAs must have finished
-                if (it >= ASLOTS && !wt.wait(&s->kdone[(it - ASLOTS) % KDONE], ((it - ASLOTS) / KDONE) & 1)) {
+                // (the last activation stage of block it - 2 completes after all its MMAs)
+                if (it >= ASLOTS && !wt.wait(&s->done[((it - ASLOTS) * Q + Q - 1) % DONE],
+                                             (((it - ASLOTS) * Q + Q - 1) / DONE) & 1)) {
                     ok = false;
                     break;
                 }
@@ -477,7 +490,7 @@ __global__ void __maxnreg__(96)
                 ptx::tmem_wait_st();
                 ptx::tc_fence_before();
                 __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->xfull[it % X_STAGES]));
+                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->xfull[(it * Q) % X_STAGES]));
                 if (warp == 2 && lane == 0) TQ(2, it, 5);
             }
         }
