@@ -187,6 +187,9 @@ __global__ void __launch_bounds__(256) quant_act_rowreg_kernel(const void* __res
     // launched with programmatic dependent launch: wait for the previous kernel
     // (which may still read the code buffer) before touching memory
     ptx::grid_dependency_wait();
+    // let the next kernel's CTAs start their prologue on SMs this grid vacates;
+    // they still wait for this grid's completion before reading its output
+    ptx::grid_launch_dependents();
     if (m >= M) return;
     const int chunks = K / EPC;
     const uint4* row = reinterpret_cast<const uint4*>(x) + int64_t(m) * chunks;
@@ -271,7 +274,6 @@ __global__ void __launch_bounds__(256) quant_act_rowreg_kernel(const void* __res
         alpha_out[m] = alpha;
         zc_out[m] = __fsub_rn(float(half), z);
     }
-    ptx::grid_launch_dependents();
 }
 
 template <int NPL, int DTYPE>
