@@ -105,6 +105,8 @@ static_assert(BK == 2 * XK, "a stage is two 64-wide swizzle atoms");
 // MMAs.  <256, 1>: a wider MMA (the tensor pipe rather than the issuing thread
 // bounds N = 256) for launches where every CTA gets a single tile; the
 // accumulator then only has to wait for the drain between certified chunks.
+// <64, 2>: for launches with few tokens, three times as many CTAs as <192, 2>
+// and a third of its per-tile epilogue.
 template <int BT_, int NACC_>
 struct Cfg {
     static constexpr int BT = BT_;
@@ -129,6 +131,7 @@ struct Cfg {
 };
 using CfgStd = Cfg<192, 2>;
 using CfgWide = Cfg<256, 1>;
+using CfgNarrow = Cfg<64, 2>;  // few tokens (cross-attention keys and values): more CTAs, shorter epilogue
 
 // Synchronisation is arranged so that the single MMA-issuing thread, whose
 // per-instruction cost bounds the K loop, does one wait and one commit per
@@ -970,11 +973,13 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     }
     if (a.M == 0 || a.N == 0) return cudaSuccess;
     // The wide single-tile configuration when it covers the output in one wave
-    // of CTAs and the standard one would need more than one.
+    // of CTAs and the standard one would need more than one; the narrow one when
+    // the standard tiles would leave most SMs idle.
     const int64_t tiles_ch = (a.N + BCH - 1) / BCH;
     const int64_t std_tiles = tiles_ch * token_tiling(a, CfgStd::BT).tiles;
     const int64_t wide_tiles = tiles_ch * token_tiling(a, CfgWide::BT).tiles;
     if (std_tiles > num_sms && wide_tiles <= num_sms) return launch_cfg<CfgWide>(a, num_sms, st, why);
+    if (std_tiles * 2 <= num_sms) return launch_cfg<CfgNarrow>(a, num_sms, st, why);
     return launch_cfg<CfgStd>(a, num_sms, st, why);
 }
 
