@@ -152,7 +152,7 @@ struct Smem {
     uint8_t w[W_STAGES][W_STAGE];
     float ep_al[EPI_WARPS][C::GPW][32], ep_zc[EPI_WARPS][C::GPW][32];  // per warp, per group, per column
     int ep_tok[EPI_WARPS][C::GPW][32], ep_tap[EPI_WARPS][C::GPW][32];
-    alignas(16) uint16_t ep_stage[EPI_WARPS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
+    alignas(128) uint16_t ep_stage[EPI_WARPS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
     uint64_t xfull[C::X_STAGES], done[C::DONE];
     uint64_t wfull[W_STAGES], wempty[W_STAGES];
     uint64_t accfull[C::NACC], accempty[C::NACC];
@@ -268,7 +268,7 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
 template <bool CONV, class C>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
-                   const __grid_constant__ CUtensorMap tm_w) {
+                   const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_y) {
     constexpr int X_STAGES = C::X_STAGES, X_HALF = C::X_HALF, X_STAGE = C::X_STAGE, NACC = C::NACC;
     constexpr int Q = C::Q, DONE = C::DONE;
     constexpr int BT = C::BT, GPW = C::GPW;
@@ -305,6 +305,7 @@ __global__ void __maxnreg__(96)
         ptx::fence_mbar_init();
         ptx::prefetch_tmap(&tm_x);
         ptx::prefetch_tmap(&tm_w);
+        if constexpr (!CONV) ptx::prefetch_tmap(&tm_y);
     }
     if (warp == 1) {
         ptx::tmem_alloc(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
@@ -612,23 +613,41 @@ __global__ void __maxnreg__(96)
                     }
                 }
                 TF(fcall, 1);
-                // Transpose the warp's 32 channels x 16 tokens through shared memory so
-                // each token row (32 channels, 64 bytes) is written with 16-byte stores.
+                // Transpose the warp's 32 channels x 16 tokens through shared memory:
+                // a [16 tokens][32 channels] bf16 box (64-byte rows).
                 uint16_t* stg = s->ep_stage[e];
+                if constexpr (!CONV) {
+                    if (lane == 0) ptx::bulk_wait_read0();  // the previous box has left the buffer
+                }
                 __syncwarp();
                 TF(fcall, 2);
 #pragma unroll
                 for (int j = 0; j < 16; ++j) stg[j * 32 + lane] = uint16_t(yb2[j >> 1] >> (16 * (j & 1)));
-                __syncwarp();
-                TF(fcall, 3);
-                const int qc = lane & 3;  // 8-channel chunk of the row
-                const int nq = tc.ch0 + (warp & 3) * 32 + qc * 8;
+                if constexpr (!CONV) {
+                    // linear layer: consecutive tokens are consecutive rows of y, so one TMA
+                    // store writes the box (rows past M and channels past N are clipped)
+                    ptx::fence_proxy_async_smem();
+                    __syncwarp();
+                    TF(fcall, 3);
+                    const int xc = tc.ch0 + (warp & 3) * 32, yt = tc.tok0 + g * 32 + j0;
+                    if (lane == 0 && xc < a.N && yt < a.M) {
+                        ptx::tma_store_2d(&tm_y, ptx::smem_u32(stg), xc, yt);
+                        ptx::bulk_commit();
+                    }
+                } else {
+                    // convolution: the box's pixels need not be consecutive rows; 16-byte stores
+                    __syncwarp();
+                    TF(fcall, 3);
+                    const int qc = lane & 3;  // 8-channel chunk of the row
+                    const int nq = tc.ch0 + (warp & 3) * 32 + qc * 8;
 #pragma unroll
-                for (int rr = 0; rr < 2; ++rr) {
-                    const int t = rr * 8 + (lane >> 2);  // token row within the 16
-                    const uint4 val = *reinterpret_cast<const uint4*>(stg + t * 32 + qc * 8);
-                    const int tok = all_tok && !CONV ? tc.tok0 + g * 32 + j0 + t : my_tok[j0 + t];
-                    if (tok >= 0 && nq < a.N) *reinterpret_cast<uint4*>(a.y + int64_t(tok) * a.N + nq) = val;
+                    for (int rr = 0; rr < 2; ++rr) {
+                        const int t = rr * 8 + (lane >> 2);  // token row within the 16
+                        const uint4 val = *reinterpret_cast<const uint4*>(stg + t * 32 + qc * 8);
+                        const int tok = my_tok[j0 + t];
+                        if (tok >= 0 && nq < a.N) *reinterpret_cast<uint4*>(a.y + int64_t(tok) * a.N + nq) = val;
+                    }
+                    __syncwarp();  // the box is read before the next one is written
                 }
                 TF(fcall, 4);
 #ifdef TASQ_TRACE
@@ -710,6 +729,8 @@ __global__ void __maxnreg__(96)
     }
 
     if (warp == 6 && lane == 0) TE(8);
+    // epilogue TMA stores complete before the CTA exits
+    if (!CONV && warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS && lane == 0) ptx::bulk_wait0();
     __syncthreads();
     if (threadIdx.x == 0) TE(10);
     if (warp == 1) {
@@ -836,7 +857,7 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
     p.a = a;
     p.conv = a.Cin != 0;
     p.tiles_ch = (a.N + BCH - 1) / BCH;
-    CUtensorMap tm_x, tm_w;
+    CUtensorMap tm_x, tm_w, tm_y;
     CUresult r;
     if (p.conv) {
         if (a.Cin % 64) {
@@ -890,6 +911,21 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
             return cudaSuccess;
         }
     }
+    if (!p.conv) {
+        // output y [M][N] bf16: the epilogue stores [16 tokens][32 channels] boxes
+        cuuint64_t dims[2] = {cuuint64_t(a.N), cuuint64_t(a.M)};
+        cuuint64_t strides[1] = {cuuint64_t(a.N) * 2};
+        cuuint32_t box[2] = {32, 16};
+        cuuint32_t es[2] = {1, 1};
+        r = encode(&tm_y, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, a.y, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) {
+            *why = "output tensor map rejected";
+            return cudaSuccess;
+        }
+    } else {
+        tm_y = tm_x;  // unused by the convolution instantiation
+    }
     const int64_t tiles = int64_t(p.tiles_ch) * p.tiles_tok;
     // Split K when the tiles alone would leave most SMs idle and each slice keeps
     // at least 8 K blocks: a tile's fixed latency (pipeline fill, epilogue) is
@@ -934,7 +970,7 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w);
+    e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w, tm_y);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaSuccess && p.splits > 1) {
         const int64_t total = int64_t(a.M) * (a.N / 4);
