@@ -60,6 +60,14 @@ __device__ inline void scale_of_range(float lo, float hi, float denom, float hal
     }
 }
 
+// Activation code Q = clamp(rint(x / alpha + z), 0, qmax) as the low 16 bits of
+// the returned fp32 bits (Q + 1.5 * 2^23).  Clamping u to the integer bounds
+// before rounding gives the same Q as rounding first.
+__device__ __forceinline__ uint32_t act_qbits(float x, float alpha, float ralpha, float z, float qmaxf) {
+    const float u = __fadd_rn(div_rn_by(x, alpha, ralpha), z);
+    return __float_as_uint(__fadd_rn(fminf(fmaxf(u, 0.0f), qmaxf), 12582912.0f));
+}
+
 // Activation code: Q = clamp(rint(x / alpha + z), 0, qmax), s = Q - half.
 // ralpha = RN(1 / alpha); x / alpha is still rounded exactly as IEEE division.
 __device__ inline int act_code(float x, float alpha, float ralpha, float z, int qmax, int half) {
@@ -205,14 +213,33 @@ __global__ void __launch_bounds__(256) quant_act_rowreg_kernel(const void* __res
         return __uint_as_float((j & 1) ? (w[j >> 1] & 0xFFFF0000u) : (w[j >> 1] << 16));
     };
     float lo = INFINITY, hi = -INFINITY;
+    if constexpr (DTYPE == TASQ_BF16) {
+        // bf16 pairs compared as bf16 (exact), one instruction per two elements
+        __nv_bfloat162 mn = __float2bfloat162_rn(INFINITY), mx = __float2bfloat162_rn(-INFINITY);
 #pragma unroll
-    for (int k = 0; k < NPL; ++k) {
-        if (lane + 32 * k < chunks) {
+        for (int k = 0; k < NPL; ++k) {
+            if (lane + 32 * k < chunks) {
+                const uint32_t w[4] = {d[k].x, d[k].y, d[k].z, d[k].w};
 #pragma unroll
-            for (int j = 0; j < EPC; ++j) {
-                const float f = elem(d[k], j);
-                lo = fminf(lo, f);
-                hi = fmaxf(hi, f);
+                for (int j = 0; j < 4; ++j) {
+                    const __nv_bfloat162 p = *reinterpret_cast<const __nv_bfloat162*>(&w[j]);
+                    mn = __hmin2(mn, p);
+                    mx = __hmax2(mx, p);
+                }
+            }
+        }
+        lo = fminf(__low2float(mn), __high2float(mn));
+        hi = fmaxf(__low2float(mx), __high2float(mx));
+    } else {
+#pragma unroll
+        for (int k = 0; k < NPL; ++k) {
+            if (lane + 32 * k < chunks) {
+#pragma unroll
+                for (int j = 0; j < EPC; ++j) {
+                    const float f = elem(d[k], j);
+                    lo = fminf(lo, f);
+                    hi = fmaxf(hi, f);
+                }
             }
         }
     }
@@ -231,9 +258,13 @@ __global__ void __launch_bounds__(256) quant_act_rowreg_kernel(const void* __res
     for (int k = 0; k < NPL; ++k) {
         const int c = lane + 32 * k;
         if (c >= chunks) continue;
+        // vb[j]: fp32 bits of Q + 1.5 * 2^23, the code Q in the low 16 bits
+        uint32_t vb[EPC];
+#pragma unroll
+        for (int j = 0; j < EPC; ++j) vb[j] = act_qbits(elem(d[k], j), alpha, ralpha, z, float(qmax));
         int q[EPC];
 #pragma unroll
-        for (int j = 0; j < EPC; ++j) q[j] = act_code(elem(d[k], j), alpha, ralpha, z, qmax, half);
+        for (int j = 0; j < EPC; ++j) q[j] = int(vb[j] & 0xFFFFu) - half;
         if (CODES == TASQ_CODES_S8) {
             if (EPC == 8) {
                 uint2 pk;
@@ -248,16 +279,17 @@ __global__ void __launch_bounds__(256) quant_act_rowreg_kernel(const void* __res
         } else {
             // fp16 of a small integer s: the bits 0x6400 + (s + half) hold 1024 + s + half
             // exactly; one packed subtraction of 1024 + half leaves s
-            uint32_t h[EPC];
-#pragma unroll
-            for (int j = 0; j < EPC; ++j) h[j] = 0x6400u + uint32_t(q[j] + half);
             const uint32_t off = 0x6400u + uint32_t(half);
             const __half2 bias2 = __halves2half2(__ushort_as_half(uint16_t(off)), __ushort_as_half(uint16_t(off)));
-            auto sub2 = [&](uint32_t lo16, uint32_t hi16) -> uint32_t {
-                uint32_t w = lo16 | (hi16 << 16);
+            // the low halves of two vb words, Q0 | Q1 << 16, with 0x6400 in each half
+            // are the fp16 values 1024 + Q; one packed subtraction of 1024 + half
+            // leaves the codes s = Q - half
+            auto sub2 = [&](uint32_t v0, uint32_t v1) -> uint32_t {
+                uint32_t w = __byte_perm(v0, v1, 0x5410) | 0x64006400u;
                 __half2 r = __hsub2(*reinterpret_cast<__half2*>(&w), bias2);
                 return *reinterpret_cast<uint32_t*>(&r);
             };
+            const uint32_t* h = vb;
             if (EPC == 8) {
                 uint4 pk;
                 pk.x = sub2(h[0], h[1]);

@@ -101,15 +101,14 @@ __device__ inline int resolve_bits(const GemmArgs& a) {
 }
 
 // x / a rounded to nearest even, from ra = RN(1/a): the quotient estimate
-// q = RN(x * ra) is refined twice by the exact FMA remainder r = x - q * a
-// (Markstein's correction, q <- RN(q + r * ra)), which reaches the correctly
-// rounded quotient for normal operands.  Checked against IEEE division by
-// tasq_selftest_quotients over every finite bf16 input.
+// q = RN(x * ra) lies within one ulp of x / a, and one correction by the exact
+// FMA remainder r = x - q * a, q <- RN(q + r * ra), gives the correctly rounded
+// quotient for normal operands (Markstein's theorem: ra within half an ulp of
+// 1/a and q within one ulp of x/a suffice).  Checked against IEEE division by
+// tasq_selftest_quotients over every finite normal bf16 dividend.
 __device__ __forceinline__ float div_rn_by(float x, float a, float ra) {
-    float q = __fmul_rn(x, ra);
-    float r = __fmaf_rn(-q, a, x);
-    q = __fmaf_rn(r, ra, q);
-    r = __fmaf_rn(-q, a, x);
+    const float q = __fmul_rn(x, ra);
+    const float r = __fmaf_rn(-q, a, x);
     return __fmaf_rn(r, ra, q);
 }
 
