@@ -35,6 +35,25 @@ if ROOT not in sys.path:
 import numpy as np
 
 METRIC = "masked W8A8 GEMM TOPS and % int8 tensor peak vs effective bits b; ms/denoise step"
+
+# DRAM bytes (read + write) per masked-contraction launch, averaged over the 224
+# launches of one PixArt-Sigma step, from one `ncu --metrics dram__bytes_read.sum,
+# dram__bytes_write.sum` capture (profiles/launch_list_pixart_sigma_step.md).  It
+# describes only the kernel sources it was measured on, identified by their SHA-256;
+# after any change to them the field reads null until the capture is repeated.
+TRAFFIC = {"pixart": {"bytes_per_launch": 13556210,
+                      "sources_sha256": "f3c6cd4804eeffcb97c94104d54188ce305afd55db3c4e2368e79dce23a3d347"}}
+KERNEL_SOURCES = ("gemm_tc.cu", "tc_ptx.cuh", "tasq_internal.cuh")
+
+
+def kernel_sources_sha256() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    here = os.path.join(os.path.dirname(os.path.abspath(__file__)), "paper_2608_03057_gb300", "csrc")
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(here, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
 UNIT = "TOPS"
 WORKLOAD_NAMES = {
     "pixart": "pixart_sigma_1024px_denoise_step",
@@ -192,8 +211,14 @@ class Step:
                 events[i][1].record()
 
     def launches_per_step(self):
-        # per-token quant: 1 kernel; per-tensor quant: 2 kernels (+ a memset); contraction: 1 kernel
-        return sum(3 if l.kind == self.conv else 2 for l in self.layers)
+        """Kernels the library enqueues for one step, counted by the library itself
+        (one eager launch of the step, outside any timed region)."""
+        if not hasattr(self, "_launches"):
+            before = self.tasq.tasq_kernel_count(self.ctx)
+            self.launch()
+            self.torch.cuda.synchronize()
+            self._launches = self.tasq.tasq_kernel_count(self.ctx) - before
+        return self._launches
 
     def act_bytes(self):
         """HBM bytes of activation quantization per step (bf16 in, fp16 codes out, scales)."""
@@ -500,8 +525,15 @@ def main():
     gemm_total_ms = sum(gemm_ms)
     achieved = step.ops / (gemm_total_ms * 1e-3) / 1e12
     peak = peaks["bf16_sus"]
+    tr = TRAFFIC.get(args.workload)
+    traffic = tr["bytes_per_launch"] if tr and tr["sources_sha256"] == kernel_sources_sha256() else None
+    alg_bytes = step.gemm_bytes() / len(step.layers)
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                "traffic": None, "kernel": "gemm_tc_kernel",
+                "traffic": traffic, "algorithmic_bytes_per_launch": alg_bytes,
+                "traffic_note": "mean DRAM bytes per contraction launch (ncu); inputs just written by the "
+                                "quantization stay in L2 and outputs leave L2 after the kernel, so traffic sits "
+                                "below the algorithmic bytes",
+                "kernel": "gemm_tc_kernel",
                 "peak_source": f"{peaks['src']} bf16 sustained (fp16 MMA runs at the bf16 rate)",
                 "timing": "CUDA events around each contraction in a replay of the step with event nodes "
                           "between kernels, right after the timed region" if external

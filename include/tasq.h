@@ -109,6 +109,14 @@ const char* tasq_last_error(tasq_ctx ctx);
  * TASQ_ERR_DEVICE) in *out, then clears it.  Set-up call. */
 int tasq_device_status(tasq_ctx ctx, int* out);
 
+/* Number of kernels that tasq_quant_act, tasq_masked_gemm and
+ * tasq_masked_conv3x3 have enqueued on this context since it was created
+ * (a contraction enqueues one, or two when it splits K; per-tensor
+ * quantization enqueues two).  Host-side count, no synchronization; a launch
+ * captured into a CUDA graph counts once, at capture.  Diagnostic only (the
+ * paper has no counterpart). */
+int tasq_kernel_count(tasq_ctx ctx, unsigned long long* out);
+
 /* Route used by tasq_masked_gemm / tasq_masked_conv3x3 (TASQ_ROUTE_*). */
 int tasq_set_route(tasq_ctx ctx, int route);
 

@@ -846,7 +846,7 @@ TokTiling token_tiling(const GemmArgs& a, int BT) {
 }
 
 template <class C>
-cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
+cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why, int* kernels) {
     constexpr int BTOK = C::BT;
     auto encode = get_encode();
     if (!encode) {
@@ -972,6 +972,7 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w, tm_y);
     if (e == cudaSuccess) e = cudaGetLastError();
+    if (e == cudaSuccess) *kernels = 1;
     if (e == cudaSuccess && p.splits > 1) {
         const int64_t total = int64_t(a.M) * (a.N / 4);
         const int64_t blocks = (total + 255) / 256;
@@ -983,6 +984,7 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
         rc.numAttrs = 1;
         e = cudaLaunchKernelEx(&rc, splitk_epilogue_kernel, a, static_cast<const int32_t*>(p.split_out), p.splits);
         if (e == cudaSuccess) e = cudaGetLastError();
+        if (e == cudaSuccess) *kernels = 2;
     }
     if (e == cudaErrorLaunchOutOfResources) {
         // report what the kernel asked for, to make the failure actionable
@@ -1001,8 +1003,9 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
 
 }  // namespace
 
-cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why) {
+cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why, int* kernels) {
     *why = nullptr;
+    *kernels = 0;
     if (!a.part) {
         *why = "no accumulator scratch";
         return cudaSuccess;
@@ -1014,9 +1017,9 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     const int64_t tiles_ch = (a.N + BCH - 1) / BCH;
     const int64_t std_tiles = tiles_ch * token_tiling(a, CfgStd::BT).tiles;
     const int64_t wide_tiles = tiles_ch * token_tiling(a, CfgWide::BT).tiles;
-    if (std_tiles > num_sms && wide_tiles <= num_sms) return launch_cfg<CfgWide>(a, num_sms, st, why);
-    if (std_tiles * 2 <= num_sms) return launch_cfg<CfgNarrow>(a, num_sms, st, why);
-    return launch_cfg<CfgStd>(a, num_sms, st, why);
+    if (std_tiles > num_sms && wide_tiles <= num_sms) return launch_cfg<CfgWide>(a, num_sms, st, why, kernels);
+    if (std_tiles * 2 <= num_sms) return launch_cfg<CfgNarrow>(a, num_sms, st, why, kernels);
+    return launch_cfg<CfgStd>(a, num_sms, st, why, kernels);
 }
 
 #ifdef TASQ_TRACE

@@ -21,6 +21,7 @@ struct tasq_ctx_s {
     const int32_t* d_stage = nullptr;
     int route = TASQ_ROUTE_AUTO;
     unsigned long long timeout_ns = 2000000000ull;
+    unsigned long long kernels = 0;  // kernels enqueued by quant_act / masked_gemm / masked_conv3x3
     std::string err;
 };
 
@@ -141,6 +142,13 @@ TASQ_API int tasq_device_status(tasq_ctx ctx, int* out) {
     return TASQ_OK;
 }
 
+TASQ_API int tasq_kernel_count(tasq_ctx ctx, unsigned long long* out) {
+    CHECK_CTX(ctx);
+    REQUIRE(out, TASQ_ERR_INVALID_ARG, "out is NULL");
+    *out = ctx->kernels;
+    return TASQ_OK;
+}
+
 TASQ_API int tasq_set_route(tasq_ctx ctx, int route) {
     CHECK_CTX(ctx);
     REQUIRE(route >= TASQ_ROUTE_AUTO && route <= TASQ_ROUTE_MMA_S8, TASQ_ERR_INVALID_ARG, "route %d", route);
@@ -258,7 +266,9 @@ TASQ_API int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int
     else
         e = tasq::launch_quant_act_tensor(d_x, dtype, (int64_t)M * K, n_bits, mode, d_codes, code_fmt, d_alpha, d_zc,
                                           reinterpret_cast<unsigned int*>(ctx->d_words + 16), (cudaStream_t)stream);
-    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "quant_act launch");
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "quant_act launch");
+    ctx->kernels += gran == TASQ_PER_TOKEN ? 1 : 2;
+    return TASQ_OK;
 }
 
 namespace {
@@ -316,14 +326,18 @@ int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void*
     a.status = ctx->d_words;
     a.timeout_ns = ctx->timeout_ns;
     cudaError_t e;
+    int kernels = 0;
     if (route == TASQ_ROUTE_TC) {
         const char* why = nullptr;
-        e = tasq::launch_gemm_tc(a, ctx->num_sms, (cudaStream_t)stream, &why);
+        e = tasq::launch_gemm_tc(a, ctx->num_sms, (cudaStream_t)stream, &why, &kernels);
         if (why) return fail(ctx, TASQ_ERR_UNSUPPORTED, "tensor-core route: %s", why);
     } else {
         e = tasq::launch_gemm_s8(a, ctx->num_sms, (cudaStream_t)stream);
+        kernels = 1;
     }
-    return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "masked contraction launch");
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "masked contraction launch");
+    ctx->kernels += kernels;
+    return TASQ_OK;
 }
 
 }  // namespace

@@ -162,7 +162,9 @@ cudaError_t launch_quant_act_tensor(const void* x, int dtype, int64_t count, int
 cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* bias, int N, int K, int Cin,
                         void* packed, cudaStream_t st);
 cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
-cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why);
+// *kernels: how many kernels the call enqueued (the contraction, plus the split-K
+// reduction when K is split).
+cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why, int* kernels);
 size_t gemm_tc_part_bytes(int num_sms);  // scratch the TC route needs for `num_sms` persistent CTAs
 constexpr int64_t kSplitBufBytes = int64_t(32) << 20;  // split-K partial sums (context scratch)
 cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, cudaStream_t st);

@@ -54,6 +54,7 @@ def lib():
                 "tasq_destroy": ([P], None),
                 "tasq_last_error": ([P], ctypes.c_char_p),
                 "tasq_device_status": ([P, ctypes.POINTER(I)], I),
+                "tasq_kernel_count": ([P, ctypes.POINTER(ctypes.c_ulonglong)], I),
                 "tasq_set_route": ([P, I], I),
                 "tasq_set_timeout_ns": ([P, U64], I),
                 "tasq_selftest_timeout": ([P, U64, P], I),
@@ -126,6 +127,12 @@ def tasq_last_error(ctx) -> str:
 def tasq_device_status(ctx) -> int:
     v = ctypes.c_int()
     _check(ctx, lib().tasq_device_status(ctx, ctypes.byref(v)))
+    return v.value
+
+
+def tasq_kernel_count(ctx) -> int:
+    v = ctypes.c_ulonglong()
+    _check(ctx, lib().tasq_kernel_count(ctx, ctypes.byref(v)))
     return v.value
 
 
