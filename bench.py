@@ -187,28 +187,33 @@ class Step:
 
     def launch(self, events=None):
         """Enqueue one step on the current stream (stage read from d_stage)."""
+        for i in range(len(self.layers)):
+            self.launch_layer(i, events)
+
+    def launch_layer(self, i, events=None):
+        """Enqueue layer i (quantization + masked contraction) on the current stream."""
         t = self.tasq
-        for i, l in enumerate(self.layers):
-            if l.kind == self.conv:
-                if events:
-                    events[i][2].record()
-                t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.Cin, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TENSOR,
-                                 self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
-                if events:
-                    events[i][0].record()
-                t.tasq_masked_conv3x3(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B, l.H,
-                                      l.W, l.Cin, self.packed[i], l.N, self.y[i], None)
-            else:
-                if events:
-                    events[i][2].record()
-                t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.K, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TOKEN,
-                                 self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
-                if events:
-                    events[i][0].record()
-                t.tasq_masked_gemm(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
-                                   self.packed[i], l.N, l.K, self.y[i], None)
+        l = self.layers[i]
+        if l.kind == self.conv:
             if events:
-                events[i][1].record()
+                events[i][2].record()
+            t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.Cin, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TENSOR,
+                             self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
+            if events:
+                events[i][0].record()
+            t.tasq_masked_conv3x3(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B, l.H,
+                                  l.W, l.Cin, self.packed[i], l.N, self.y[i], None)
+        else:
+            if events:
+                events[i][2].record()
+            t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.K, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TOKEN,
+                             self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
+            if events:
+                events[i][0].record()
+            t.tasq_masked_gemm(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
+                               self.packed[i], l.N, l.K, self.y[i], None)
+        if events:
+            events[i][1].record()
 
     def launches_per_step(self):
         """Kernels the library enqueues for one step, counted by the library itself
@@ -493,18 +498,37 @@ def main():
         ms8 = timed_replays(torch, g, step, max(10, args.steps // 2), stage_of)
         tasq.tasq_set_schedule(step.ctx, step.table, L, S)
 
-    # end to end through the C ABI with host buffers
+    # end to end through the C ABI with host buffers: each layer's input is copied in
+    # on one stream, its output copied out on another, the layers run in order on the
+    # compute stream, so the copies of other layers overlap the kernels
     e2e = None
     if not args.no_e2e:
         xh = [x.cpu().pin_memory() for x in step.x]
         yh = [torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for y in step.y]
         s = torch.cuda.current_stream()
+        sh, sd = torch.cuda.Stream(), torch.cuda.Stream()
+        evx = [torch.cuda.Event() for _ in range(L)]
+        evy = [torch.cuda.Event() for _ in range(L)]
+        fork, join_h, join_d = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
+
         def e2e_step():
+            fork.record(s)
+            sh.wait_event(fork)
+            sd.wait_event(fork)
             for i in range(L):
-                step.x[i].copy_(xh[i], non_blocking=True)
-            step.launch()
-            for i in range(L):
-                yh[i].copy_(step.y[i], non_blocking=True)
+                with torch.cuda.stream(sh):
+                    step.x[i].copy_(xh[i], non_blocking=True)
+                    evx[i].record(sh)
+                s.wait_event(evx[i])
+                step.launch_layer(i)
+                evy[i].record(s)
+                with torch.cuda.stream(sd):
+                    sd.wait_event(evy[i])
+                    yh[i].copy_(step.y[i], non_blocking=True)
+            join_h.record(sh)
+            join_d.record(sd)
+            s.wait_event(join_h)
+            s.wait_event(join_d)
         e2e_step()
         torch.cuda.synchronize()
         ge = torch.cuda.CUDAGraph()
