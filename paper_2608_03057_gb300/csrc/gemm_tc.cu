@@ -535,6 +535,20 @@ __global__ void __maxnreg__(96)
                 }
             }
 
+            // Linear layers drain the accumulator in the mma-fragment layout (see
+            // finish16f): this thread's channels are lane/4 + 8k, k = 0..3.
+            [[maybe_unused]] float cwf[4], biasf[4], rsf[4];
+            if constexpr (!CONV) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int nk = tc.ch0 + q * 32 + (lane >> 2) + 8 * k;
+                    const bool ok_k = nk < a.N;
+                    cwf[k] = ok_k ? a.cw[nk] : 0.f;
+                    biasf[k] = ok_k ? a.bias[nk] : 0.f;
+                    rsf[k] = ok_k ? __int2float_rn(rs_b[nk]) : 0.f;
+                }
+            }
+
             // Token index, (conv) in-bounds taps and per-token scales of column j = lane of
             // each of this warp's two groups, written to this warp's shared scratch before
             // the accumulator wait, so the global loads' latency hides under the MMAs.
@@ -662,6 +676,73 @@ __global__ void __maxnreg__(96)
                 }
             };
 
+            // Linear-layer epilogue of 16 consecutive columns j0..j0+15 of group g from
+            // values in the mma-fragment layout: with s = lane % 4, v[(k>>1)*8 + (k&1)*2
+            // + 4*tp + e] is channel lane/4 + 8k, token j0 + 8*tp + 2s + e.  Four 8x8
+            // transposed matrix stores build the [16 tokens][32 channels] box.
+            [[maybe_unused]] auto finish16f = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag) {
+                constexpr bool fl = decltype(fl_tag)::value;
+                const int g = part * GPW + gi;
+                const int s4 = lane & 3;
+                const float2 al0 = *reinterpret_cast<const float2*>(s->ep_al[e][gi] + j0 + 2 * s4);
+                const float2 al1 = *reinterpret_cast<const float2*>(s->ep_al[e][gi] + j0 + 8 + 2 * s4);
+                const float2 zc0 = *reinterpret_cast<const float2*>(s->ep_zc[e][gi] + j0 + 2 * s4);
+                const float2 zc1 = *reinterpret_cast<const float2*>(s->ep_zc[e][gi] + j0 + 8 + 2 * s4);
+                const float alv[4] = {al0.x, al0.y, al1.x, al1.y}, zcv[4] = {zc0.x, zc0.y, zc1.x, zc1.y};
+                uint32_t pk[4][2];  // [channel k][token pair tp]
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+#pragma unroll
+                    for (int tp = 0; tp < 2; ++tp) {
+                        float yf[2];
+#pragma unroll
+                        for (int ee = 0; ee < 2; ++ee) {
+                            const uint32_t raw = v[(k >> 1) * 8 + (k & 1) * 2 + 4 * tp + ee];
+                            float acc_f;
+                            if constexpr (fl) acc_f = __uint_as_float(raw);
+                            else acc_f = __int2float_rn(int(raw));
+                            const float alj = alv[2 * tp + ee], zcj = zcv[2 * tp + ee];
+                            yf[ee] = __fmaf_rn(__fmaf_rn(zcj, rsf[k], acc_f), __fmul_rn(alj, cwf[k]), biasf[k]);
+                        }
+                        const __nv_bfloat162 hb = __floats2bfloat162_rn(yf[0], yf[1]);
+                        pk[k][tp] = *reinterpret_cast<const uint32_t*>(&hb);
+                    }
+                }
+                uint16_t* stg = s->ep_stage[e];
+                if (lane == 0) ptx::bulk_wait_read0();  // the previous box has left the buffer
+                __syncwarp();
+                {
+                    // stored matrix i = lane / 8: (channel block, token block) = (i & 1, i >> 1), plus
+                    // two channel blocks for the second store; row k = lane % 8 is token 8 * tb + k
+                    const int i = lane >> 3, kr = lane & 7;
+                    const uint32_t row = ptx::smem_u32(stg) + uint32_t((((i >> 1) * 8 + kr) * 32 + (i & 1) * 8) * 2);
+                    ptx::stmatrix_x4_trans(row, pk[0][0], pk[1][0], pk[0][1], pk[1][1]);
+                    ptx::stmatrix_x4_trans(row + 16 * 2, pk[2][0], pk[3][0], pk[2][1], pk[3][1]);
+                }
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+                const int xc = tc.ch0 + q * 32, yt = tc.tok0 + g * 32 + j0;
+                if (lane == 0 && xc < a.N && yt < a.M) {
+                    ptx::tma_store_2d(&tm_y, ptx::smem_u32(stg), xc, yt);
+                    ptx::bulk_commit();
+                }
+                if (a.acc) {  // int32 accumulators (a debugging output): plain stores
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int nk = tc.ch0 + q * 32 + (lane >> 2) + 8 * k;
+#pragma unroll
+                        for (int tp = 0; tp < 2; ++tp)
+#pragma unroll
+                            for (int ee = 0; ee < 2; ++ee) {
+                                const int tok = yt + 8 * tp + 2 * s4 + ee;
+                                const uint32_t raw = v[(k >> 1) * 8 + (k & 1) * 2 + 4 * tp + ee];
+                                if (tok < a.M && nk < a.N)
+                                    a.acc[int64_t(tok) * a.N + nk] = fl ? __float2int_rn(__uint_as_float(raw)) : int(raw);
+                            }
+                    }
+                }
+            };
+
             // Multi-chunk tiles keep their int32 running sums in this warp's slice of the
             // per-CTA scratch (32 channels x 32 * MAX_GPW tokens); each value is only
             // re-read by the thread that wrote it.
@@ -687,7 +768,14 @@ __global__ void __maxnreg__(96)
 #pragma unroll 1
                     for (int h = 0; h < 2; ++h) {
                         uint32_t v[16];
-                        ptx::tmem_ld16(acc_base + g * 32 + h * 16, v);
+                        const bool frag = !CONV && p.splits == 1;  // linear, not split: fragment layout
+                        if (frag) {
+                            // lanes q*32 .. +15 and +16 .. +31 of the quadrant, 16 columns each
+                            ptx::tmem_ld16x256b_x2(acc_base + g * 32 + h * 16, v);
+                            ptx::tmem_ld16x256b_x2(acc_base + (16u << 16) + g * 32 + h * 16, v + 8);
+                        } else {
+                            ptx::tmem_ld16(acc_base + g * 32 + h * 16, v);
+                        }
                         ptx::tmem_wait_ld();
                         if (nchunks > 1) {
                             int32_t* pp = my_part + (gi * 32 + h * 16) * 32;
@@ -714,8 +802,13 @@ __global__ void __maxnreg__(96)
                                 }
                             }
                         } else if (last) {
-                            if (nchunks == 1) finish16(gi, h * 16, v, std::true_type{}, all_tok);
-                            else finish16(gi, h * 16, v, std::false_type{}, all_tok);
+                            if constexpr (!CONV) {
+                                if (nchunks == 1) finish16f(gi, h * 16, v, std::true_type{});
+                                else finish16f(gi, h * 16, v, std::false_type{});
+                            } else {
+                                if (nchunks == 1) finish16(gi, h * 16, v, std::true_type{}, all_tok);
+                                else finish16(gi, h * 16, v, std::false_type{}, all_tok);
+                            }
                         }
                         if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 4 + 2 * h);
                     }
