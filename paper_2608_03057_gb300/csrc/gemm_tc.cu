@@ -694,17 +694,20 @@ __global__ void __maxnreg__(96)
                 for (int k = 0; k < 4; ++k) {
 #pragma unroll
                     for (int tp = 0; tp < 2; ++tp) {
-                        float yf[2];
-#pragma unroll
-                        for (int ee = 0; ee < 2; ++ee) {
-                            const uint32_t raw = v[(k >> 1) * 8 + (k & 1) * 2 + 4 * tp + ee];
-                            float acc_f;
-                            if constexpr (fl) acc_f = __uint_as_float(raw);
-                            else acc_f = __int2float_rn(int(raw));
-                            const float alj = alv[2 * tp + ee], zcj = zcv[2 * tp + ee];
-                            yf[ee] = __fmaf_rn(__fmaf_rn(zcj, rsf[k], acc_f), __fmul_rn(alj, cwf[k]), biasf[k]);
+                        // two tokens of channel k at once, each lane rounded as the scalar
+                        // sequence u = fma(zc, rs, acc), s = alpha * cw, y = fma(u, s, bias)
+                        const int i0 = (k >> 1) * 8 + (k & 1) * 2 + 4 * tp;
+                        float2 acc2;
+                        if constexpr (fl) {
+                            acc2 = make_float2(__uint_as_float(v[i0]), __uint_as_float(v[i0 + 1]));
+                        } else {
+                            acc2 = make_float2(__int2float_rn(int(v[i0])), __int2float_rn(int(v[i0 + 1])));
                         }
-                        const __nv_bfloat162 hb = __floats2bfloat162_rn(yf[0], yf[1]);
+                        const float2 u2 = ptx::ffma2(make_float2(zcv[2 * tp], zcv[2 * tp + 1]),
+                                                     make_float2(rsf[k], rsf[k]), acc2);
+                        const float2 s2 = ptx::fmul2(make_float2(alv[2 * tp], alv[2 * tp + 1]), make_float2(cwf[k], cwf[k]));
+                        const float2 y2 = ptx::ffma2(u2, s2, make_float2(biasf[k], biasf[k]));
+                        const __nv_bfloat162 hb = __floats2bfloat162_rn(y2.x, y2.y);
                         pk[k][tp] = *reinterpret_cast<const uint32_t*>(&hb);
                     }
                 }

@@ -162,6 +162,25 @@ __device__ __forceinline__ void stmatrix_x4_trans(uint32_t saddr, uint32_t a, ui
                  "r"(c), "r"(d)
                  : "memory");
 }
+// Packed fp32 pairs (each lane rounded to nearest even, as fma.rn.f32 / mul.rn.f32).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+    float2 d;
+    asm("{\n.reg .b64 A, B, C, D;\n"
+        "mov.b64 A, {%2, %3};\nmov.b64 B, {%4, %5};\nmov.b64 C, {%6, %7};\n"
+        "fma.rn.f32x2 D, A, B, C;\nmov.b64 {%0, %1}, D;\n}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n.reg .b64 A, B, D;\n"
+        "mov.b64 A, {%2, %3};\nmov.b64 B, {%4, %5};\n"
+        "mul.rn.f32x2 D, A, B;\nmov.b64 {%0, %1}, D;\n}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
