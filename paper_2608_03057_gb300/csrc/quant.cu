@@ -14,6 +14,9 @@ namespace tasq {
 namespace {
 
 constexpr int kRowWarps = 8;  // rows per 256-thread block
+// Rows per block of the single-pass per-token kernel: small blocks spread the
+// one wave of rows evenly over the SMs (blocks, not warps, are what get placed).
+constexpr int kRegRowWarps = 2;
 
 // Eight consecutive input floats (as fp32) from a 16-byte (bf16) or two
 // 16-byte (fp32) chunks.  `i` counts 8-element groups along the row.
@@ -185,13 +188,13 @@ __global__ void __launch_bounds__(256) quant_act_token_kernel(const void* __rest
 // registers as NPL 16-byte chunks per lane (chunk c of the row is lane c % 32,
 // slot c / 32), so every load is issued before the min/max reduction.
 template <int NPL, int DTYPE, int CODES>
-__global__ void __launch_bounds__(256) quant_act_rowreg_kernel(const void* __restrict__ x, int M, int K, int n_bits,
+__global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(const void* __restrict__ x, int M, int K, int n_bits,
                                                                int mode, void* __restrict__ codes,
                                                                float* __restrict__ alpha_out,
                                                                float* __restrict__ zc_out) {
     constexpr int EPC = DTYPE == TASQ_F32 ? 4 : 8;  // elements per 16-byte chunk
     const int lane = threadIdx.x & 31;
-    const int m = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    const int m = blockIdx.x * kRegRowWarps + (threadIdx.x >> 5);
     // launched with programmatic dependent launch: wait for the previous kernel
     // (which may still read the code buffer) before touching memory
     ptx::grid_dependency_wait();
@@ -312,8 +315,8 @@ template <int NPL, int DTYPE>
 cudaError_t launch_rowreg(const void* x, int M, int K, int n_bits, int mode, void* codes, int code_fmt, float* alpha,
                           float* zc, cudaStream_t st) {
     cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3((M + kRowWarps - 1) / kRowWarps);
-    cfg.blockDim = dim3(256);
+    cfg.gridDim = dim3((M + kRegRowWarps - 1) / kRegRowWarps);
+    cfg.blockDim = dim3(kRegRowWarps * 32);
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
