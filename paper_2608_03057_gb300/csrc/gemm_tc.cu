@@ -121,6 +121,9 @@ struct Cfg {
     static constexpr int DONE = 2 * X_STAGES;            // stage-completion barriers (ring of MMA commits)
     static constexpr int GROUPS = BT / 32;               // 32-token column groups of the accumulator
     static constexpr int GPW = (GROUPS + EPI_PARTS - 1) / EPI_PARTS;  // groups per epilogue warp
+    // the single-tile configuration lets the 4 converter warps, idle once the last K
+    // block is converted, drain a fourth share of the tile's groups
+    static constexpr int EPI_SLOTS = EPI_WARPS + (NACC == 1 ? 4 : 0);
     static constexpr uint32_t ACC_COL = 0;               // NACC x BT fp32 accumulators
     static constexpr uint32_t A_COL = NACC * BT;         // ASLOTS x BK/2 columns (fp16 pairs)
     static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BT);
@@ -150,9 +153,9 @@ template <class C>
 struct Smem {
     uint8_t x[C::X_STAGES][C::X_STAGE];  // 1024-aligned (128-byte swizzle atoms)
     uint8_t w[W_STAGES][W_STAGE];
-    float ep_al[EPI_WARPS][C::GPW][32], ep_zc[EPI_WARPS][C::GPW][32];  // per warp, per group, per column
-    int ep_tok[EPI_WARPS][C::GPW][32], ep_tap[EPI_WARPS][C::GPW][32];
-    alignas(128) uint16_t ep_stage[EPI_WARPS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
+    float ep_al[C::EPI_SLOTS][C::GPW][32], ep_zc[C::EPI_SLOTS][C::GPW][32];  // per warp, per group, per column
+    int ep_tok[C::EPI_SLOTS][C::GPW][32], ep_tap[C::EPI_SLOTS][C::GPW][32];
+    alignas(128) uint16_t ep_stage[C::EPI_SLOTS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
     uint64_t xfull[C::X_STAGES], done[C::DONE];
     uint64_t wfull[W_STAGES], wempty[W_STAGES];
     uint64_t accfull[C::NACC], accempty[C::NACC];
@@ -162,6 +165,9 @@ struct Smem {
 };
 template <class C>
 constexpr int smem_bytes() { return int(sizeof(Smem<C>)) + 1024; }
+static_assert(smem_bytes<CfgStd>() <= 227 * 1024 && smem_bytes<CfgWide>() <= 227 * 1024 &&
+                  smem_bytes<CfgNarrow>() <= 227 * 1024,
+              "shared memory per CTA");
 
 struct TcParams {
     GemmArgs a;
@@ -498,11 +504,19 @@ __global__ void __maxnreg__(96)
                 if (warp == 2 && lane == 0) TQ(2, it, 5);
             }
         }
-    } else {
+    }
+    // Helper mode (uniform over the CTA): a single-tile CTA whose tile is one
+    // certified chunk (linear layers) drains it with the converter warps too,
+    // four warps per lane quadrant instead of three.
+    const bool helpers = !CONV && C::NACC == 1 && unit < works && works <= units &&
+                         work_item(p, unit, KT, chunk).nch == 1;
+    if ((warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS) || (helpers && warp >= 2 && warp < EPI_WARP0)) {
         // ------------------------------------- accumulator drain + epilogue
-        const int e = warp - EPI_WARP0;      // 0..EPI_WARPS-1
+        // shared-scratch slot: epilogue warps 0..11, converter warps 12..15
+        const int e = warp >= EPI_WARP0 ? warp - EPI_WARP0 : EPI_WARPS + (warp - 2);
         const int q = warp & 3;              // lane quadrant: channels q*32 .. q*32+31
-        const int part = e >> 2;             // which pair of 32-token groups
+        const int part = e >> 2;             // which share of the tile's 32-token groups
+        const int gpw = helpers ? (C::GROUPS + EPI_PARTS) / (EPI_PARTS + 1) : GPW;  // groups per share
         const int r = q * 32 + lane;
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
@@ -556,7 +570,8 @@ __global__ void __maxnreg__(96)
             __syncwarp();  // the previous tile's reads of the scratch are done
 #pragma unroll
             for (int gi = 0; gi < GPW; ++gi) {
-                const int jt = (part * GPW + gi) * 32 + lane;  // beyond the tile when part * GPW + gi >= GROUPS
+                // beyond the tile (no token) when part * gpw + gi >= GROUPS or gi >= gpw
+                const int jt = gi < gpw ? (part * gpw + gi) * 32 + lane : BT;
                 int tok = -1, tap = 0;
                 if constexpr (CONV) {
                     const int hh = tc.h0 + (jt >> p.bw_log2), ww = tc.w0 + (jt & ((1 << p.bw_log2) - 1));
@@ -589,7 +604,7 @@ __global__ void __maxnreg__(96)
             auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag, bool all_tok) {
                 constexpr bool fl = decltype(fl_tag)::value;
                 TF(fcall, 0);
-                const int g = part * GPW + gi;
+                const int g = part * gpw + gi;
                 const float* my_al = s->ep_al[e][gi];
                 const float* my_zc = s->ep_zc[e][gi];
                 const int* my_tok = s->ep_tok[e][gi];
@@ -682,7 +697,7 @@ __global__ void __maxnreg__(96)
             // transposed matrix stores build the [16 tokens][32 channels] box.
             [[maybe_unused]] auto finish16f = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag) {
                 constexpr bool fl = decltype(fl_tag)::value;
-                const int g = part * GPW + gi;
+                const int g = part * gpw + gi;
                 const int s4 = lane & 3;
                 const float2 al0 = *reinterpret_cast<const float2*>(s->ep_al[e][gi] + j0 + 2 * s4);
                 const float2 al1 = *reinterpret_cast<const float2*>(s->ep_al[e][gi] + j0 + 8 + 2 * s4);
@@ -749,7 +764,8 @@ __global__ void __maxnreg__(96)
             // Multi-chunk tiles keep their int32 running sums in this warp's slice of the
             // per-CTA scratch (32 channels x 32 * MAX_GPW tokens); each value is only
             // re-read by the thread that wrote it.
-            int32_t* my_part = a.part + (int64_t(blockIdx.x) * EPI_WARPS + e) * (MAX_GPW * 32 * 32) + lane;
+            // (helper converter warps, e >= EPI_WARPS, only run single-chunk tiles and never touch it)
+            int32_t* my_part = a.part + (int64_t(blockIdx.x) * EPI_WARPS + (e < EPI_WARPS ? e : 0)) * (MAX_GPW * 32 * 32) + lane;
             for (int c = 0; c < nchunks; ++c, ++cc) {
                 const int buf = cc % NACC;
                 if (warp == 6 && lane == 0) TQ(3, cc, 0);
@@ -764,8 +780,8 @@ __global__ void __maxnreg__(96)
                 const uint32_t acc_base = lane_base + C::ACC_COL + buf * BT;
                 const bool last = c == nchunks - 1;
 #pragma unroll 1
-                for (int gi = 0; gi < GPW; ++gi) {
-                    const int g = part * GPW + gi;
+                for (int gi = 0; gi < gpw; ++gi) {
+                    const int g = part * gpw + gi;
                     if (g >= C::GROUPS) break;
                     const bool all_tok = all_tok_g[gi];
 #pragma unroll 1
@@ -818,7 +834,8 @@ __global__ void __maxnreg__(96)
                 }
                 ptx::tc_fence_before();
                 __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->accempty[buf]));
+                // (helper converter warps only join the tile's single chunk: nothing waits for them)
+                if (lane == 0 && e < EPI_WARPS) ptx::mbar_arrive(ptx::smem_u32(&s->accempty[buf]));
                 if (warp == 6 && lane == 0) TQ(3, cc, 2);
             }
         }
@@ -826,7 +843,9 @@ __global__ void __maxnreg__(96)
 
     if (warp == 6 && lane == 0) TE(8);
     // epilogue TMA stores complete before the CTA exits
-    if (!CONV && warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS && lane == 0) ptx::bulk_wait0();
+    if (!CONV && lane == 0 &&
+        ((warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS) || (helpers && warp >= 2 && warp < EPI_WARP0)))
+        ptx::bulk_wait0();
     __syncthreads();
     if (threadIdx.x == 0) TE(10);
     if (warp == 1) {
