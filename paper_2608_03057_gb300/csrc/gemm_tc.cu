@@ -323,20 +323,23 @@ __global__ void __maxnreg__(96)
     const uint32_t tmem = s->tmem_base;
     if (threadIdx.x == 0) TE(1);
     if (warp == WPROD_WARP && lane == 0 && unit < works) {
-        // The packed weights are not written by the kernel this one may overlap,
-        // so their first tiles can be pulled into L2 before the wait below (a
-        // prefetch only: nothing reaches shared memory before the wait).
+        // pull the first weight tiles into L2 ahead of the weight ring
         const Work wk = work_item(p, unit, KT, chunk);
         const int ch0 = tile_coord<CONV, BT>(p, wk.t).ch0;
         for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * BK, ch0);
     }
-    // the prologue above overlaps the previous kernel; inputs are read only after it
-    ptx::grid_dependency_wait();
-    if (threadIdx.x == 0) TE(2);
+    // Programmatic dependent launch: this grid may start while the previous kernel
+    // (normally the quantization of this layer's activations) still runs.  Only the
+    // activation codes and the per-token scales come from it, so only the warps that
+    // read those (the activation producer and the epilogue) wait for it; the packed
+    // weights, the bit table and the stage were complete before that kernel began,
+    // so the weight ring, the converters and the MMA issuer start at once.
 
     if (warp == 0) {
         // --------------------------------------------- activation producer
         if (lane == 0) {
+            ptx::grid_dependency_wait();
+            TE(2);
             int u = 0;  // activation stages issued by this CTA
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
@@ -512,6 +515,7 @@ __global__ void __maxnreg__(96)
                          work_item(p, unit, KT, chunk).nch == 1;
     if ((warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS) || (helpers && warp >= 2 && warp < EPI_WARP0)) {
         // ------------------------------------- accumulator drain + epilogue
+        ptx::grid_dependency_wait();  // per-token scales come from the previous kernel
         // shared-scratch slot: epilogue warps 0..11, converter warps 12..15
         const int e = warp >= EPI_WARP0 ? warp - EPI_WARP0 : EPI_WARPS + (warp - 2);
         const int q = warp & 3;              // lane quadrant: channels q*32 .. q*32+31
