@@ -17,6 +17,10 @@ constexpr int kRowWarps = 8;  // rows per 256-thread block
 // Rows per block of the single-pass per-token kernel: small blocks spread the
 // one wave of rows evenly over the SMs (blocks, not warps, are what get placed).
 constexpr int kRegRowWarps = 2;
+// L2 prefetch of the input ahead of the dependency wait: the first kPrefetchBlocks
+// blocks take one slice each, for inputs up to half of the 129 MB L2
+constexpr int kPrefetchBlocks = 128;
+constexpr uint64_t kPrefetchMaxBytes = 64ull << 20;
 
 // Eight consecutive input floats (as fp32) from a 16-byte (bf16) or two
 // 16-byte (fp32) chunks.  `i` counts 8-element groups along the row.
@@ -195,8 +199,21 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
     constexpr int EPC = DTYPE == TASQ_F32 ? 4 : 8;  // elements per 16-byte chunk
     const int lane = threadIdx.x & 31;
     const int m = blockIdx.x * kRegRowWarps + (threadIdx.x >> 5);
-    // launched with programmatic dependent launch: wait for the previous kernel
-    // (which may still read the code buffer) before touching memory
+    // Launched with programmatic dependent launch, so the first blocks may run beside
+    // the previous kernel's last CTAs.  They pull the whole input into L2 meanwhile,
+    // one slice each: L2 is the GPU's point of coherence, so if the previous kernel
+    // writes x after this, its stores update the lines and the loads below (issued
+    // after the wait) see them.  Nothing else is read or written before the wait
+    // (the previous kernel may still read the code buffer).
+    if (threadIdx.x == 0 && blockIdx.x < kPrefetchBlocks) {
+        const uint64_t total = uint64_t(M) * uint64_t(K) * (DTYPE == TASQ_F32 ? 4u : 2u);  // K % 8 == 0: 16-byte rows
+        const uint64_t slice = ((total + kPrefetchBlocks - 1) / kPrefetchBlocks + 15) & ~uint64_t(15);
+        const uint64_t lo = uint64_t(blockIdx.x) * slice;
+        if (lo < total && total <= kPrefetchMaxBytes) {
+            const uint64_t n = total - lo < slice ? total - lo : slice;
+            ptx::prefetch_l2_bulk(reinterpret_cast<const char*>(x) + lo, uint32_t(n));
+        }
+    }
     ptx::grid_dependency_wait();
     // let the next kernel's CTAs start their prologue on SMs this grid vacates;
     // they still wait for this grid's completion before reading its output
