@@ -65,6 +65,10 @@ def _lib():
             lib.oq_linear_def_f64.argtypes = [P, P, P, i32, P, P, P, i32, i32, i32, P]
             lib.oq_conv3x3.argtypes = [P, i32, i32, i32, i32, P, i32, i32, P, P]
             lib.oq_conv3x3_def_f64.argtypes = [P, f32, f32, i32, i32, i32, i32, P, P, P, i32, i32, P]
+            lib.oq_weight_zero_offsets.argtypes = [P, i32, i32, P]
+            lib.oq_code_sums.argtypes = [P, i32, i32, P]
+            lib.oq_epilogue_zp_f32.argtypes = [P, i32, i32, i32, P, P, P, P, P, P, P, P, P]
+            lib.oq_linear_zp_def_f64.argtypes = [P, P, P, i32, P, P, P, P, i32, i32, i32, P]
             _LIB = lib
     return _LIB
 
@@ -90,7 +94,9 @@ def bf16_bits_to_f32(b):
 
 
 def quant_weight(w, n_bits=8, mode=SYMRANGE):
-    """App. A.1.1, per output channel.  Returns dict(q, s, alpha, z, c)."""
+    """App. A.1.1, per output channel.  Returns dict(q, s, alpha, z, c, zcw);
+    zcw = RN(2^(n-1) - z) is the weight zero offset of Eq. weight_dequant on the
+    stored signed code (0 for the symmetric range)."""
     w = _c(w, np.float32)
     N, K = w.shape
     q = np.empty((N, K), np.int32)
@@ -99,7 +105,9 @@ def quant_weight(w, n_bits=8, mode=SYMRANGE):
     z = np.empty(N, np.float32)
     c = np.empty(N, np.float32)
     _lib().oq_quant_weight(_p(w), N, K, n_bits, mode, _p(q), _p(s) if n_bits <= 8 else None, _p(alpha), _p(z), _p(c))
-    return dict(q=q, s=s if n_bits <= 8 else None, alpha=alpha, z=z, c=c)
+    zcw = np.empty(N, np.float32)
+    _lib().oq_weight_zero_offsets(_p(z), N, n_bits, _p(zcw))
+    return dict(q=q, s=s if n_bits <= 8 else None, alpha=alpha, z=z, c=c, zcw=zcw)
 
 
 def quant_act(x, n_bits=8, mode=SYMRANGE, gran=PER_TOKEN):
@@ -162,6 +170,43 @@ def epilogue_f32(acc, alpha, zc, rs, c_w, bias=None, per_tensor=False, rs_per_ro
     _lib().oq_epilogue_f32(_p(acc), M, N, _p(alpha), _p(zc), int(per_tensor), _p(rs), N if rs_per_row else 0,
                            _p(c_w), _p(bias), _p(y), _p(yb))
     return y, yb
+
+
+def code_sums(s_x):
+    """sx[m] = sum_k s_x[m][k], int32."""
+    s_x = _c(s_x, np.int8)
+    M, K = s_x.shape
+    sx = np.empty(M, np.int32)
+    _lib().oq_code_sums(_p(s_x), M, K, _p(sx))
+    return sx
+
+
+def epilogue_zp_f32(acc, alpha, zc, sx, rs, c_w, zcw, bias, K):
+    """Four-term dequant epilogue (asymmetric weights, per token) in the kernel's
+    fp32 order.  Returns (y_f32, y_bf16_bits)."""
+    acc = _c(acc, np.int32)
+    M, N = acc.shape
+    args = [_c(alpha, np.float32), _c(zc, np.float32), _c(sx, np.int32), _c(rs, np.int32), _c(c_w, np.float32),
+            _c(zcw, np.float32)]
+    bias = None if bias is None else _c(bias, np.float32)
+    y = np.empty((M, N), np.float32)
+    yb = np.empty((M, N), np.uint16)
+    _lib().oq_epilogue_zp_f32(_p(acc), M, N, int(K), *[_p(a) for a in args], _p(bias), _p(y), _p(yb))
+    return y, yb
+
+
+def linear_zp_def_f64(s_x, alpha, zc, s_w, c_w, z, bias, b):
+    """The dequantized linear layer with asymmetric weights (zero point z per
+    channel) by definition, fp64."""
+    s_x = _c(s_x, np.int8)
+    s_w = _c(s_w, np.int8)
+    M, K = s_x.shape
+    N = s_w.shape[0]
+    bias = None if bias is None else _c(bias, np.float32)
+    y = np.empty((M, N), np.float64)
+    _lib().oq_linear_zp_def_f64(_p(s_x), _p(_c(alpha, np.float32)), _p(_c(zc, np.float32)), M, _p(s_w),
+                                _p(_c(c_w, np.float32)), _p(_c(z, np.float32)), _p(bias), N, K, int(b), _p(y))
+    return y
 
 
 def linear_def_f64(s_x, alpha, zc, s_w, c_w, bias, b):

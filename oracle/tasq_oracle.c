@@ -334,3 +334,78 @@ void oq_conv3x3_def_f64(const int8_t* s_x, float alpha, float zc, int B, int H, 
         }
     }
 }
+
+/* ------------------------------------------------------------------------
+ * Asymmetric weights: the App. A.1.1 quantizer on each channel's true
+ * [min, max] (oq_quant_weight with OQ_ASYM) leaves a real-valued zero point
+ * z, and Eq. weight_dequant on the masked code reads
+ *   w_hat = c * (Q_b - z) = c * (mask_b(s_w) + zcw),   zcw = 2^(n-1) - z,
+ * (Q_b = mask_b(s_w) + 2^(n-1) on the stored grid).  The dequantized
+ * contraction then has four integer-carried terms:
+ *   sum_k x_hat * w_hat = alpha * c * (acc + zc * rs_b + zcw * sx + K * zc * zcw),
+ *   sx[m] = sum_k s_x[m][k].
+ * ------------------------------------------------------------------------ */
+
+/* zcw[n] = RN(2^(n-1) - z[n]). */
+void oq_weight_zero_offsets(const float* z, int N, int n_bits, float* zcw) {
+    const float half = (float)(1 << (n_bits - 1));
+    for (int n = 0; n < N; ++n) zcw[n] = half - z[n];
+}
+
+/* sx[m] = sum_k s_x[m][k] (int32: |sx| <= 128 K). */
+void oq_code_sums(const int8_t* s_x, int M, int K, int32_t* sx) {
+    for (int m = 0; m < M; ++m) {
+        int64_t sum = 0;
+        for (int k = 0; k < K; ++k) sum += s_x[(int64_t)m * K + k];
+        sx[m] = (int32_t)sum;
+    }
+}
+
+/*
+ * The four-term dequantization in fp32, per token (linear layers), each
+ * fused multiply-add rounded once:
+ *   u1 = RN(zc * float(rs) + float(acc)),   u2 = RN(zcw * float(sx) + u1),
+ *   kz = RN(float(K) * zc),                 u3 = RN(kz * zcw + u2),
+ *   s  = RN(alpha * c),                     y  = RN(u3 * s + bias),   bf16_rne(y).
+ * With zcw = 0 (symmetric weights) u3 = u1 and this is oq_epilogue_f32.
+ */
+void oq_epilogue_zp_f32(const int32_t* acc, int M, int N, int K, const float* alpha, const float* zc,
+                        const int32_t* sx, const int32_t* rs, const float* c_w, const float* zcw, const float* bias,
+                        float* y_f32, uint16_t* y_bf16) {
+    for (int m = 0; m < M; ++m) {
+        const float kz = (float)K * zc[m];
+        for (int n = 0; n < N; ++n) {
+            float a = (float)acc[(int64_t)m * N + n];
+            float u1 = fmaf(zc[m], (float)rs[n], a);
+            float u2 = fmaf(zcw[n], (float)sx[m], u1);
+            float u3 = fmaf(kz, zcw[n], u2);
+            float s = alpha[m] * c_w[n];
+            float y = fmaf(u3, s, bias ? bias[n] : 0.0f);
+            if (y_f32) y_f32[(int64_t)m * N + n] = y;
+            if (y_bf16) y_bf16[(int64_t)m * N + n] = oq_bf16_rne(y);
+        }
+    }
+}
+
+/*
+ * The linear layer with asymmetric weights by its definition, in fp64:
+ * x_hat = alpha * (s_x + zc) (Eq. act_dequant), w_hat = c * (Q_b - z) with
+ * Q_b = mask_b(s_w) + 128 and the quantizer's own z (Eq. weight_dequant),
+ * summed product by product.  No term is factored out.
+ */
+void oq_linear_zp_def_f64(const int8_t* s_x, const float* alpha, const float* zc, int M, const int8_t* s_w,
+                          const float* c_w, const float* z, const float* bias, int N, int K, int b, double* y) {
+#pragma omp parallel for schedule(static)
+    for (int m = 0; m < M; ++m) {
+        for (int n = 0; n < N; ++n) {
+            double sum = 0.0;
+            for (int k = 0; k < K; ++k) {
+                double xh = (double)alpha[m] * ((double)s_x[(int64_t)m * K + k] + (double)zc[m]);
+                double qb = (double)oq_mask(s_w[(int64_t)n * K + k], b) + 128.0;
+                double wh = (double)c_w[n] * (qb - (double)z[n]);
+                sum += xh * wh;
+            }
+            y[(int64_t)m * N + n] = sum + (bias ? (double)bias[n] : 0.0);
+        }
+    }
+}

@@ -218,6 +218,25 @@ def test_wide_tiles_ragged_full(ctx, oracle, code_fmt):
 
 
 @pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("M,N,K", [(300, 1152, 1168), (77, 640, 2048), (64, 128, 4096)])
+def test_split_k_repeated_launches(ctx, oracle, code_fmt, M, N, K):
+    """Few tiles and a long K (ragged last K block): where the tensor-core route
+    cuts K into slices, their exact partial sums are added by a second kernel.
+    Each stage runs twice on the same context (shared split scratch) and must
+    give identical, exact results."""
+    bits = [8, 3]
+    st = _setup_linear(ctx, oracle, M, N, K, bits, seed=M + 3, code_fmt=code_fmt)
+    for stage, b in enumerate(bits):
+        outs = []
+        for _ in range(2):
+            y, acc = G.gemm(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+            _check_layer(oracle, st, b, y, acc)
+            outs.append(G.bf16_bits_host(y))
+        assert np.array_equal(outs[0], outs[1])
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
 def test_output_without_acc(ctx, oracle, code_fmt):
     M, N, K = 200, 128, 256
     st = _setup_linear(ctx, oracle, M, N, K, [6], code_fmt=code_fmt)

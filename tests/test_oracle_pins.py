@@ -289,6 +289,110 @@ def test_epilogue_real_domain_error_is_quantization_sized(oracle):
     assert rel < 0.02
 
 
+# ------------------------------------------- asymmetric weights (zero point) --
+
+def test_asym_weight_quant_closed_form(oracle):
+    # App. A.1.1 on each channel's true [min, max]: alpha = (max - min) / 2^n,
+    # z = -min / alpha (real valued), Q = clamp(floor(w / alpha + z), 0, 2^n - 1).
+    w = workloads.normal((24, 1152), seed=41, std=0.02)
+    w[::3] += 0.03  # skewed channels: min and max of different magnitude
+    d = oracle.quant_weight(w, 8, 1)
+    lo, hi = w.min(1), w.max(1)
+    assert np.array_equal(d["alpha"], ((hi - lo).astype(np.float32) / np.float32(256)).astype(np.float32))
+    assert np.array_equal(d["z"], (-lo / d["alpha"]).astype(np.float32))
+    assert np.array_equal(d["zcw"], (np.float32(128) - d["z"]).astype(np.float32))
+    # the channel minimum is code 0 and the maximum the top code (clamped from 2^n)
+    assert np.all(d["q"][np.arange(24), np.argmin(w, 1)] == 0)
+    assert np.all(d["q"][np.arange(24), np.argmax(w, 1)] == 255)
+    # floor quantizer: alpha (Q - z) lies in (w - alpha, w] up to the fp32 rounding of
+    # w / alpha + z (ulp <= 2^-15 below 256), except at the clamped top code
+    rec = d["alpha"][:, None].astype(np.float64) * (d["q"] - d["z"][:, None].astype(np.float64))
+    err = w.astype(np.float64) - rec
+    a = np.broadcast_to(d["alpha"][:, None].astype(np.float64), w.shape)
+    top = d["q"] == 255
+    slack = 2.0 ** -14 * a
+    assert np.all((err[~top] > -slack[~top]) & (err[~top] < a[~top] + slack[~top]))
+    assert np.all(np.abs(err[top]) <= a[top] + slack[top])
+
+
+def test_asym_weight_quant_on_a_symmetric_channel_is_the_symmetric_one(oracle):
+    # a channel whose minimum is exactly -max: both readings give z = 128, zcw = 0
+    w = workloads.normal((6, 300), seed=42, std=0.02)
+    for n in range(6):
+        w[n, 7] = -np.abs(w[n]).max()
+        w[n, 9] = -w[n, 7]
+    ds, da = oracle.quant_weight(w, 8, 0), oracle.quant_weight(w, 8, 1)
+    assert np.array_equal(ds["q"], da["q"]) and np.all(da["z"] == 128.0) and np.all(da["zcw"] == 0.0)
+
+
+def test_code_sums(oracle):
+    s_x = workloads.uniform_codes((9, 1000), seed=43)
+    assert np.array_equal(oracle.code_sums(s_x), s_x.astype(np.int64).sum(1))
+
+
+def test_epilogue_zp_with_zero_offsets_is_the_symmetric_epilogue(oracle):
+    M, N, K = 20, 36, 640
+    s_x, alpha, zc = oracle.quant_act(workloads.normal((M, K), seed=44), 8, 1, 0)
+    wq = oracle.quant_weight(workloads.normal((N, K), seed=45, std=0.02), 8, 0)
+    acc = oracle.gemm(s_x, wq["s"], 5)
+    rs = oracle.row_sums(wq["s"], 5)
+    bias = workloads.normal((N,), seed=46, std=0.02)
+    y0, yb0 = oracle.epilogue_f32(acc, alpha, zc, rs, wq["c"], bias)
+    y1, yb1 = oracle.epilogue_zp_f32(acc, alpha, zc, oracle.code_sums(s_x), rs, wq["c"], wq["zcw"], bias, K)
+    assert np.all(wq["zcw"] == 0.0)
+    assert np.array_equal(y0.view(np.uint32), y1.view(np.uint32)) and np.array_equal(yb0, yb1)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("b", [8, 5, 3, 2])
+def test_epilogue_zp_matches_definition(oracle, mode, b):
+    # The factored four-term fp32 sequence against the element-by-element fp64
+    # definition with the quantizer's own zero point: a dropped term, a wrong sign
+    # or a wrong zero offset is off by far more than fp32 rounding.
+    M, N, K = 40, 48, 1152
+    x = workloads.normal((M, K), seed=47)
+    w = workloads.normal((N, K), seed=48, std=0.02)
+    w[::2] += 0.02
+    bias = workloads.normal((N,), seed=49, std=0.02)
+    wq = oracle.quant_weight(w, 8, 1)
+    s_x, alpha, zc = oracle.quant_act(x, 8, mode, 0)
+    acc = oracle.gemm(s_x, wq["s"], b)
+    rs = oracle.row_sums(wq["s"], b)
+    sx = oracle.code_sums(s_x)
+    y32, ybf = oracle.epilogue_zp_f32(acc, alpha, zc, sx, rs, wq["c"], wq["zcw"], bias, K)
+    y64 = oracle.linear_zp_def_f64(s_x, alpha, zc, wq["s"], wq["c"], wq["z"], bias, b)
+    terms = (np.abs(acc) + np.abs(zc)[:, None] * np.abs(rs)[None, :] + np.abs(wq["zcw"])[None, :] * np.abs(sx)[:, None]
+             + K * np.abs(zc)[:, None] * np.abs(wq["zcw"])[None, :])
+    scale = np.abs(alpha)[:, None] * np.abs(wq["c"])[None, :] * terms
+    assert np.all(np.abs(y32 - y64) <= 16 * 2.0 ** -24 * (scale + np.abs(y64)) + 1e-9)
+    # and the zero-offset terms are not negligible here (the check has teeth)
+    dropped = np.abs(alpha)[:, None] * np.abs(wq["c"])[None, :] * np.abs(
+        wq["zcw"][None, :] * sx[:, None] + K * zc[:, None] * wq["zcw"][None, :])
+    assert np.median(dropped) > 1e3 * np.median(16 * 2.0 ** -24 * (scale + np.abs(y64)))
+
+
+def test_asym_weights_fit_skewed_channels_better(oracle):
+    # The reason for a weight zero point: on channels whose values are not centred
+    # at 0 the asymmetric grid is finer (here about half the step), so the weight
+    # grid alpha (Q - z) is closer to w and the dequantized layer closer to x w^T.
+    # (Both layers also carry the 2^n / (2^n - 1) factor of Eq. weight_dequant, a
+    # common 0.4 % scale that the comparison of weight grids leaves out.)
+    M, N, K = 16, 32, 512
+    x = workloads.normal((M, K), seed=50)
+    w = workloads.normal((N, K), seed=51, std=0.02) + 0.05
+    ref = x.astype(np.float64) @ w.astype(np.float64).T
+    s_x, alpha, zc = oracle.quant_act(x, 8, 1, 0)
+    grid_err, layer_err = [], []
+    for mode in (0, 1):
+        wq = oracle.quant_weight(w, 8, mode)
+        grid = wq["alpha"][:, None].astype(np.float64) * (wq["q"] - wq["z"][:, None].astype(np.float64))
+        grid_err.append(np.sqrt(np.mean((grid - w) ** 2)))
+        y = oracle.linear_zp_def_f64(s_x, alpha, zc, wq["s"], wq["c"], wq["z"], None, 8)
+        layer_err.append(np.linalg.norm(y - ref) / np.linalg.norm(ref))
+    assert grid_err[1] < 0.7 * grid_err[0], grid_err
+    assert layer_err[1] < layer_err[0], layer_err
+
+
 def test_bf16_rounding_ties_to_even(oracle):
     # 1 + 2^-8 is halfway between bf16 neighbours 1 and 1 + 2^-7: ties go to even (1.0)
     v = np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -(1.0 + 2 ** -8), 1.0 + 2 ** -8 + 2 ** -20], np.float32)
