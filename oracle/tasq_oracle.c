@@ -362,25 +362,27 @@ void oq_code_sums(const int8_t* s_x, int M, int K, int32_t* sx) {
 }
 
 /*
- * The four-term dequantization in fp32, per token (linear layers), each
- * fused multiply-add rounded once:
- *   u1 = RN(zc * float(rs) + float(acc)),   u2 = RN(zcw * float(sx) + u1),
- *   kz = RN(float(K) * zc),                 u3 = RN(kz * zcw + u2),
- *   s  = RN(alpha * c),                     y  = RN(u3 * s + bias),   bf16_rne(y).
- * With zcw = 0 (symmetric weights) u3 = u1 and this is oq_epilogue_f32.
+ * The four-term dequantization in fp32, per token (linear layers).  The two
+ * zero-offset terms share the factor zcw: zcw * sx + K * zc * zcw =
+ * zcw * t with t[m] = sx[m] + K * zc[m] = sum_k (s_x[m][k] + zc[m]), the
+ * token's dequantized activation sum over alpha.  Each step rounded once:
+ *   t  = RN(float(sx) + RN(float(K) * zc))                    (per token)
+ *   u1 = RN(zc * float(rs) + float(acc)),  u2 = RN(zcw * t + u1),
+ *   s  = RN(alpha * c),                    y  = RN(u2 * s + bias),  bf16_rne(y).
+ * With zcw = 0 (symmetric weights) u2 = u1 and this is oq_epilogue_f32.
  */
 void oq_epilogue_zp_f32(const int32_t* acc, int M, int N, int K, const float* alpha, const float* zc,
                         const int32_t* sx, const int32_t* rs, const float* c_w, const float* zcw, const float* bias,
                         float* y_f32, uint16_t* y_bf16) {
     for (int m = 0; m < M; ++m) {
         const float kz = (float)K * zc[m];
+        const float t = (float)sx[m] + kz;
         for (int n = 0; n < N; ++n) {
             float a = (float)acc[(int64_t)m * N + n];
             float u1 = fmaf(zc[m], (float)rs[n], a);
-            float u2 = fmaf(zcw[n], (float)sx[m], u1);
-            float u3 = fmaf(kz, zcw[n], u2);
+            float u2 = fmaf(zcw[n], t, u1);
             float s = alpha[m] * c_w[n];
-            float y = fmaf(u3, s, bias ? bias[n] : 0.0f);
+            float y = fmaf(u2, s, bias ? bias[n] : 0.0f);
             if (y_f32) y_f32[(int64_t)m * N + n] = y;
             if (y_bf16) y_bf16[(int64_t)m * N + n] = oq_bf16_rne(y);
         }
