@@ -341,6 +341,71 @@ def run_sweep(torch, tasq, workloads, shapes=None, reps=10, seed=0):
     return out, switch
 
 
+def run_zero_point(torch, tasq, workloads, shapes=((4096, 1152, 1152), (4096, 3456, 1152), (300, 1152, 1152)),
+                   reps=20, seed=0):
+    """Asymmetric weights (App. A.1.1 on each channel's [min, max], a real zero
+    point per channel) against the symmetric reading on the same layer shapes:
+    per-call time of the activation quantization (with / without the per-token
+    code sums) and of the contraction (four-term / two-term epilogue), CUDA
+    graphs of `reps` back-to-back calls, b = 5."""
+    ctx = tasq.tasq_create(torch.cuda.current_device())
+    table = workloads.schedule_for("sweep", 1)  # stage 3 <-> b = 5
+    tasq.tasq_set_schedule(ctx, table, 1, table.shape[1])
+    stage = 3
+
+    def graph_us(fn):
+        fn()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+            for _ in range(reps):
+                fn()
+        gr.replay()
+        torch.cuda.synchronize()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record()
+        gr.replay()
+        t1.record()
+        torch.cuda.synchronize()
+        return t0.elapsed_time(t1) * 1e3 / reps
+
+    out = []
+    for si, (M, N, K) in enumerate(shapes):
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed * 1000 + 500 + si)
+        w = torch.randn((N, K), generator=g, device="cuda") * 0.02
+        w[::2] += 0.02  # skewed channels
+        x = torch.randn((M, K), generator=g, device="cuda").to(torch.bfloat16)
+        sw = torch.empty((N, K), dtype=torch.int8, device="cuda")
+        cw = torch.empty((N,), device="cuda")
+        zcw = torch.empty((N,), device="cuda")
+        nbytes = tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, N, K)
+        pk_sym = torch.empty((nbytes,), dtype=torch.uint8, device="cuda")
+        pk_zp = torch.empty((nbytes,), dtype=torch.uint8, device="cuda")
+        tasq.tasq_quant_weights(ctx, w, tasq.TASQ_F32, N, K, sw, cw)
+        tasq.tasq_pack_weights(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K, 0, pk_sym)
+        tasq.tasq_quant_weights_asym(ctx, w, tasq.TASQ_F32, N, K, sw, cw, zcw)
+        tasq.tasq_pack_weights_zp(ctx, sw, cw, zcw, None, N, K, pk_zp)
+        codes = torch.empty((M, K), dtype=torch.float16, device="cuda")
+        al = torch.empty((M,), device="cuda")
+        zc = torch.empty((M,), device="cuda")
+        sums = torch.empty((M,), dtype=torch.int32, device="cuda")
+        y = torch.empty((M, N), dtype=torch.int16, device="cuda")
+        q_sym = graph_us(lambda: tasq.tasq_quant_act(ctx, x, tasq.TASQ_BF16, M, K, 8, tasq.TASQ_SYMRANGE,
+                                                     tasq.TASQ_PER_TOKEN, codes, tasq.TASQ_CODES_F16, al, zc))
+        q_zp = graph_us(lambda: tasq.tasq_quant_act_sums(ctx, x, tasq.TASQ_BF16, M, K, 8, tasq.TASQ_SYMRANGE, codes,
+                                                         tasq.TASQ_CODES_F16, al, zc, sums))
+        g_sym = graph_us(lambda: tasq.tasq_masked_gemm(ctx, 0, stage, codes, tasq.TASQ_CODES_F16, al, zc, M, pk_sym,
+                                                       N, K, y))
+        g_zp = graph_us(lambda: tasq.tasq_masked_gemm_zp(ctx, 0, stage, codes, tasq.TASQ_CODES_F16, al, zc, sums, M,
+                                                         pk_zp, N, K, y))
+        out.append({"M": M, "N": N, "K": K, "b": 5, "quant_us_symmetric": q_sym, "quant_us_with_code_sums": q_zp,
+                    "contraction_us_symmetric": g_sym, "contraction_us_zero_point": g_zp,
+                    "contraction_tops_zero_point": 2.0 * M * N * K / (g_zp * 1e-6) / 1e12})
+        del w, x, sw, cw, zcw, pk_sym, pk_zp, codes, al, zc, sums, y
+    tasq.tasq_destroy(ctx)
+    return out
+
+
 # ------------------------------------------------------------ CPU oracle --
 def oracle_sample(workload: str, budget_s: float, rows: int = 32, seed: int = 0, max_layers=None):
     """Time the CPU oracle (act quant, int32 contraction, row sums, fp32
@@ -563,9 +628,10 @@ def main():
                           "between kernels, right after the timed region" if external
                 else "CUDA events around each contraction in an eager pass after the timed region"}
 
-    sweep = switch = None
+    sweep = switch = zp = None
     if not args.no_sweep:
         sweep, switch = run_sweep(torch, tasq, workloads, seed=args.seed)
+        zp = run_zero_point(torch, tasq, workloads, seed=args.seed)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -606,6 +672,7 @@ def main():
             "clocks": clk,
             "sweep_tops_by_b": sweep,
             "stage_switch": switch,
+            "asym_weights": zp,
         }
         print(json.dumps(line), flush=True)
     step.close()

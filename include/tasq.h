@@ -56,7 +56,7 @@
 extern "C" {
 #endif
 
-#define TASQ_ABI_VERSION 1
+#define TASQ_ABI_VERSION 2
 
 /* Return codes. */
 enum {
@@ -156,6 +156,23 @@ int tasq_quant_weights(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, i
                        float* d_alpha, tasq_stream stream);
 
 /*
+ * Weight quantization with a weight zero point: App. A.1.1 (Eqs. weight_quant,
+ * weight_scale, weight_dequant) applied as written, on each output channel's
+ * true range [min(w), max(w)]:
+ *   alpha = (max - min) / 256,  z = -min / alpha  (real valued),
+ *   Q = clamp(floor(w / alpha + z), 0, 255),  stored s_w = Q - 128 (int8),
+ *   c_w = (256/255) * alpha,  zcw = 128 - z,
+ * so that w_hat = c_w * (Q - z) = c_w * (s_w + zcw), and at operating
+ * precision b, w_hat_b = c_w * (mask_b(s_w) + zcw).  Same fp32 operation order
+ * as tasq_quant_weights, then zcw = 128 - z rounded once.  A constant channel
+ * gets alpha = 1, z = -min.  Outputs d_sw [N][K] int8, d_cw [N], d_zcw [N]
+ * fp32, d_alpha [N] (may be NULL).  Pack the result with
+ * tasq_pack_weights_zp.  Enqueue call.
+ */
+int tasq_quant_weights_asym(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, int8_t* d_sw, float* d_cw,
+                            float* d_zcw, float* d_alpha, tasq_stream stream);
+
+/*
  * Bytes of the packed form of one layer (see tasq_pack_weights), for
  * kind TASQ_LINEAR (K = in features) or TASQ_CONV3X3 (K = 9*Cin).
  * Returns 0 for invalid shapes.
@@ -182,6 +199,17 @@ size_t tasq_packed_bytes(int kind, int N, int K);
  */
 int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_bias, int N,
                       int K, int Cin, void* d_packed, tasq_stream stream);
+
+/*
+ * tasq_pack_weights for a linear layer quantized with a weight zero point
+ * (tasq_quant_weights_asym): also stores zcw [N] and marks the buffer, so
+ * that the contraction must be given the activations' code sums
+ * (tasq_masked_gemm_zp).  tasq_masked_gemm on such a buffer records
+ * TASQ_ERR_DEVICE and writes nothing.  Same buffer size (tasq_packed_bytes
+ * with TASQ_LINEAR).  Enqueue call.
+ */
+int tasq_pack_weights_zp(tasq_ctx ctx, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
+                         const float* d_bias, int N, int K, void* d_packed, tasq_stream stream);
 
 /*
  * Bit-allocation map (App. F.1): h_bits [L][S] uint8, each value in 2..8,
@@ -221,6 +249,15 @@ int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n
                    void* d_codes, int code_fmt, float* d_alpha, float* d_zc, tasq_stream stream);
 
 /*
+ * tasq_quant_act per token, also writing d_code_sums [M] int32, the sum over
+ * k of the stored codes s[m][k] (exact).  The four-term epilogue of
+ * asymmetric weights needs it (tasq_masked_gemm_zp).  Enqueue call.
+ */
+int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode,
+                        void* d_codes, int code_fmt, float* d_alpha, float* d_zc, int32_t* d_code_sums,
+                        tasq_stream stream);
+
+/*
  * Masked linear layer (Eq. qalora with the Temporal-Spatial LSB mask of
  * Eq. lsb_masking at operating precision b = table[layer][stage]):
  *   acc[m][n] = sum_k s_x[m][k] * mask_b(s_w[n][k])            (exact int32)
@@ -239,6 +276,23 @@ int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n
 int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt, const float* d_alpha,
                      const float* d_zc, int M, const void* d_packed, int N, int K, uint16_t* d_y, int32_t* d_acc,
                      tasq_stream stream);
+
+/*
+ * Masked linear layer with asymmetric weights (Eq. weight_dequant with the
+ * zero point of tasq_quant_weights_asym, Eq. act_dequant):
+ *   sum_k x_hat w_hat_b = alpha * c_w * (acc + zc * rs_b + zcw * t),
+ *   t[m] = sum_k (s_x[m][k] + zc[m]) = sx[m] + K * zc[m],
+ * in fp32 with each step rounded once, in this order:
+ *   t = sx + K * zc (per token; K * zc rounded first), u = fma(zc, rs_b, acc),
+ *   u = fma(zcw, t, u), s = alpha * c_w, y = bf16(fma(u, s, bias)).
+ * d_code_sums: [M] from tasq_quant_act_sums.  d_packed: from
+ * tasq_pack_weights_zp (zcw stored) or tasq_pack_weights (zcw = 0: the
+ * result equals tasq_masked_gemm's).  Other arguments as tasq_masked_gemm.
+ * Enqueue call.
+ */
+int tasq_masked_gemm_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt, const float* d_alpha,
+                        const float* d_zc, const int32_t* d_code_sums, int M, const void* d_packed, int N, int K,
+                        uint16_t* d_y, int32_t* d_acc, tasq_stream stream);
 
 /*
  * Masked 3x3 convolution, stride 1, padding 1, as an implicit GEMM over

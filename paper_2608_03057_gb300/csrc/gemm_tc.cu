@@ -270,8 +270,9 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
 }
 
 // CONV selects the implicit-GEMM 3x3 convolution (one instantiation per
-// operand layout, so neither pays for the other's index arithmetic).
-template <bool CONV, class C>
+// operand layout, so neither pays for the other's index arithmetic); ZP the
+// four-term epilogue of asymmetric weights (linear layers only).
+template <bool CONV, bool ZP, class C>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_y) {
@@ -525,6 +526,7 @@ __global__ void __maxnreg__(96)
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
         const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
+        constexpr bool zp = !CONV && ZP;  // asymmetric weights: the four-term epilogue
         int cc = 0;
 #ifdef TASQ_TRACE
         int fcall = 0;
@@ -555,7 +557,7 @@ __global__ void __maxnreg__(96)
 
             // Linear layers drain the accumulator in the mma-fragment layout (see
             // finish16f): this thread's channels are lane/4 + 8k, k = 0..3.
-            [[maybe_unused]] float cwf[4], biasf[4], rsf[4];
+            [[maybe_unused]] float cwf[4], biasf[4], rsf[4], zcwf[4];
             if constexpr (!CONV) {
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
@@ -564,6 +566,7 @@ __global__ void __maxnreg__(96)
                     cwf[k] = ok_k ? a.cw[nk] : 0.f;
                     biasf[k] = ok_k ? a.bias[nk] : 0.f;
                     rsf[k] = ok_k ? __int2float_rn(rs_b[nk]) : 0.f;
+                    zcwf[k] = ok_k && zp ? a.zcw[nk] : 0.f;
                 }
             }
 
@@ -595,6 +598,10 @@ __global__ void __maxnreg__(96)
                 if constexpr (CONV) {
                     if (jt >= BT) tok = -1;
                 }
+                if constexpr (!CONV) {
+                    // asymmetric weights: the token's activation sum t, kept in the tap slot
+                    if (zp && tok >= 0) tap = __float_as_int(token_zero_sum(a.code_sums[tok], a.K, a.zc[tok]));
+                }
                 s->ep_tok[e][gi][lane] = tok;
                 s->ep_tap[e][gi][lane] = tap;
                 s->ep_al[e][gi][lane] = tok >= 0 ? (a.per_tensor ? a.alpha[0] : a.alpha[tok]) : 0.f;
@@ -608,7 +615,7 @@ __global__ void __maxnreg__(96)
             auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag, bool all_tok) {
                 constexpr bool fl = decltype(fl_tag)::value;
                 TF(fcall, 0);
-                const int g = part * gpw + gi;
+                [[maybe_unused]] const int g = part * gpw + gi;
                 const float* my_al = s->ep_al[e][gi];
                 const float* my_zc = s->ep_zc[e][gi];
                 const int* my_tok = s->ep_tok[e][gi];
@@ -708,6 +715,12 @@ __global__ void __maxnreg__(96)
                 const float2 zc0 = *reinterpret_cast<const float2*>(s->ep_zc[e][gi] + j0 + 2 * s4);
                 const float2 zc1 = *reinterpret_cast<const float2*>(s->ep_zc[e][gi] + j0 + 8 + 2 * s4);
                 const float alv[4] = {al0.x, al0.y, al1.x, al1.y}, zcv[4] = {zc0.x, zc0.y, zc1.x, zc1.y};
+                [[maybe_unused]] float tv[4] = {0.f, 0.f, 0.f, 0.f};  // asymmetric weights: token sums
+                if constexpr (zp) {
+                    const float2 t0 = *reinterpret_cast<const float2*>(s->ep_tap[e][gi] + j0 + 2 * s4);
+                    const float2 t1 = *reinterpret_cast<const float2*>(s->ep_tap[e][gi] + j0 + 8 + 2 * s4);
+                    tv[0] = t0.x, tv[1] = t0.y, tv[2] = t1.x, tv[3] = t1.y;
+                }
                 uint32_t pk[4][2];  // [channel k][token pair tp]
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
@@ -722,8 +735,10 @@ __global__ void __maxnreg__(96)
                         } else {
                             acc2 = make_float2(__int2float_rn(int(v[i0])), __int2float_rn(int(v[i0 + 1])));
                         }
-                        const float2 u2 = ptx::ffma2(make_float2(zcv[2 * tp], zcv[2 * tp + 1]),
-                                                     make_float2(rsf[k], rsf[k]), acc2);
+                        float2 u2 = ptx::ffma2(make_float2(zcv[2 * tp], zcv[2 * tp + 1]), make_float2(rsf[k], rsf[k]),
+                                               acc2);
+                        // asymmetric weights: u = fma(zcw, t, u)
+                        if constexpr (zp) u2 = ptx::ffma2(make_float2(zcwf[k], zcwf[k]), make_float2(tv[2 * tp], tv[2 * tp + 1]), u2);
                         const float2 s2 = ptx::fmul2(make_float2(alv[2 * tp], alv[2 * tp + 1]), make_float2(cwf[k], cwf[k]));
                         const float2 y2 = ptx::ffma2(u2, s2, make_float2(biasf[k], biasf[k]));
                         const __nv_bfloat162 hb = __floats2bfloat162_rn(y2.x, y2.y);
@@ -883,6 +898,8 @@ __global__ void __launch_bounds__(256) splitk_epilogue_kernel(const GemmArgs a, 
         }
         const float al = a.per_tensor ? a.alpha[0] : a.alpha[m];
         const float zc = a.per_tensor ? a.zc[0] : a.zc[m];
+        const bool zp = !a.Cin && a.code_sums;  // asymmetric weights (linear)
+        const float t = zp ? token_zero_sum(a.code_sums[m], a.K, zc) : 0.f;
         int tap = 0x1FF;
         if (a.Cin) {
             const int ww = m % a.W, hh = (m / a.W) % a.H;
@@ -908,7 +925,8 @@ __global__ void __launch_bounds__(256) splitk_epilogue_kernel(const GemmArgs a, 
             } else {
                 rsum = __int2float_rn(rs_b[n + q]);
             }
-            const float u = __fmaf_rn(zc, rsum, __int2float_rn(accs[q]));
+            float u = __fmaf_rn(zc, rsum, __int2float_rn(accs[q]));
+            if (zp) u = __fmaf_rn(a.zcw[n + q], t, u);
             y[q] = __fmaf_rn(u, __fmul_rn(al, a.cw[n + q]), a.bias[n + q]);
         }
         const __nv_bfloat162 h0 = __floats2bfloat162_rn(y[0], y[1]);
@@ -1074,7 +1092,8 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
         fprintf(stderr, "tasq tc: M=%d N=%d K=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, (long long)tiles,
                 p.splits, units);
     const int smem = smem_bytes<C>();
-    auto kernel = p.conv ? gemm_tc_kernel<true, C> : gemm_tc_kernel<false, C>;
+    auto kernel = p.conv ? gemm_tc_kernel<true, false, C>
+                         : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     // programmatic dependent launch: the grid may start while the previous

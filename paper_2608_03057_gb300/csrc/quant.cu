@@ -51,6 +51,11 @@ __device__ inline float warp_min(float v) {
     for (int o = 16; o; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
     return v;
 }
+__device__ inline int warp_sum(int v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
 
 // Quantization range of a group: [lo, hi] -> (alpha, z) in the fp32 order
 // alpha = (hi - lo) / denom, z = -lo / alpha; a constant group gets alpha = 1
@@ -105,24 +110,38 @@ __device__ inline void store8_codes(void* out, int code_fmt, int64_t i, const in
 }
 
 // ---------------------------------------------------------------- weights --
+// mode TASQ_SYMRANGE: range [-max|w|, max|w|] (z = 128); TASQ_ASYM: the channel's
+// [min, max] and a real zero point, zcw_out[n] = 128 - z.
 __global__ void __launch_bounds__(256) quant_weights_kernel(const void* __restrict__ w, int dtype, int N, int K,
-                                                            int8_t* __restrict__ sw, float* __restrict__ cw,
+                                                            int mode, int8_t* __restrict__ sw, float* __restrict__ cw,
+                                                            float* __restrict__ zcw_out,
                                                             float* __restrict__ alpha_out) {
     int lane = threadIdx.x & 31;
     int n = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
     if (n >= N) return;
     const char* row = reinterpret_cast<const char*>(w) + int64_t(n) * K * (dtype == TASQ_F32 ? 4 : 2);
     int groups = K / 8;
-    float amax = 0.0f;
+    float amax = 0.0f, lo = INFINITY, hi = -INFINITY;
     for (int i = lane; i < groups; i += 32) {
         float v[8];
         load8(row, dtype, i, v);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) amax = fmaxf(amax, fabsf(v[j]));
+        for (int j = 0; j < 8; ++j) {
+            amax = fmaxf(amax, fabsf(v[j]));
+            lo = fminf(lo, v[j]);
+            hi = fmaxf(hi, v[j]);
+        }
     }
-    amax = warp_max(amax);
+    if (mode == TASQ_ASYM) {
+        lo = warp_min(lo);
+        hi = warp_max(hi);
+    } else {
+        amax = warp_max(amax);
+        lo = -amax;
+        hi = amax;
+    }
     float alpha, z;
-    scale_of_range(-amax, amax, 256.0f, 128.0f, TASQ_SYMRANGE, &alpha, &z);
+    scale_of_range(lo, hi, 256.0f, 128.0f, mode, &alpha, &z);
     int8_t* srow = sw + int64_t(n) * K;
     for (int i = lane; i < groups; i += 32) {
         float v[8];
@@ -139,6 +158,7 @@ __global__ void __launch_bounds__(256) quant_weights_kernel(const void* __restri
     }
     if (lane == 0) {
         cw[n] = __fmul_rn(alpha, __fdiv_rn(256.0f, 255.0f));
+        if (zcw_out) zcw_out[n] = __fsub_rn(128.0f, z);
         if (alpha_out) alpha_out[n] = alpha;
     }
 }
@@ -147,7 +167,8 @@ __global__ void __launch_bounds__(256) quant_weights_kernel(const void* __restri
 __global__ void __launch_bounds__(256) quant_act_token_kernel(const void* __restrict__ x, int dtype, int M, int K,
                                                               int n_bits, int mode, void* __restrict__ codes,
                                                               int code_fmt, float* __restrict__ alpha_out,
-                                                              float* __restrict__ zc_out) {
+                                                              float* __restrict__ zc_out,
+                                                              int32_t* __restrict__ code_sums) {
     int lane = threadIdx.x & 31;
     int m = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
     if (m >= M) return;
@@ -174,28 +195,36 @@ __global__ void __launch_bounds__(256) quant_act_token_kernel(const void* __rest
     scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
     const float ralpha = __frcp_rn(alpha);
     char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (code_fmt == TASQ_CODES_S8 ? 1 : 2);
+    int csum = 0;
     for (int i = lane; i < groups; i += 32) {
         float v[8];
         load8(row, dtype, i, v);
         int s[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, ralpha, z, qmax, half);
+        for (int j = 0; j < 8; ++j) {
+            s[j] = act_code(v[j], alpha, ralpha, z, qmax, half);
+            csum += s[j];
+        }
         store8_codes(out, code_fmt, i, s);
     }
+    if (code_sums) csum = warp_sum(csum);
     if (lane == 0) {
         alpha_out[m] = alpha;
         zc_out[m] = __fsub_rn(float(half), z);
+        if (code_sums) code_sums[m] = csum;
     }
 }
 
 // Single-pass per-token quantization: one warp per row, the whole row held in
 // registers as NPL 16-byte chunks per lane (chunk c of the row is lane c % 32,
-// slot c / 32), so every load is issued before the min/max reduction.
-template <int NPL, int DTYPE, int CODES>
+// slot c / 32), so every load is issued before the min/max reduction.  SUMS:
+// also write the row's code sum (asymmetric weights need it).
+template <int NPL, int DTYPE, int CODES, bool SUMS>
 __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(const void* __restrict__ x, int M, int K, int n_bits,
                                                                int mode, void* __restrict__ codes,
                                                                float* __restrict__ alpha_out,
-                                                               float* __restrict__ zc_out) {
+                                                               float* __restrict__ zc_out,
+                                                               int32_t* __restrict__ code_sums) {
     constexpr int EPC = DTYPE == TASQ_F32 ? 4 : 8;  // elements per 16-byte chunk
     const int lane = threadIdx.x & 31;
     const int m = blockIdx.x * kRegRowWarps + (threadIdx.x >> 5);
@@ -274,6 +303,7 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
     scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
     const float ralpha = __frcp_rn(alpha);
     char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (CODES == TASQ_CODES_S8 ? 1 : 2);
+    int csum = 0;  // sum of this lane's codes Q - half (kept only when code_sums is set)
 #pragma unroll
     for (int k = 0; k < NPL; ++k) {
         const int c = lane + 32 * k;
@@ -285,6 +315,10 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
         int q[EPC];
 #pragma unroll
         for (int j = 0; j < EPC; ++j) q[j] = int(vb[j] & 0xFFFFu) - half;
+        if constexpr (SUMS) {
+#pragma unroll
+            for (int j = 0; j < EPC; ++j) csum += q[j];
+        }
         if (CODES == TASQ_CODES_S8) {
             if (EPC == 8) {
                 uint2 pk;
@@ -322,15 +356,17 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
             }
         }
     }
+    if constexpr (SUMS) csum = warp_sum(csum);
     if (lane == 0) {
         alpha_out[m] = alpha;
         zc_out[m] = __fsub_rn(float(half), z);
+        if constexpr (SUMS) code_sums[m] = csum;
     }
 }
 
 template <int NPL, int DTYPE>
 cudaError_t launch_rowreg(const void* x, int M, int K, int n_bits, int mode, void* codes, int code_fmt, float* alpha,
-                          float* zc, cudaStream_t st) {
+                          float* zc, int32_t* sums, cudaStream_t st) {
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3((M + kRegRowWarps - 1) / kRegRowWarps);
     cfg.blockDim = dim3(kRegRowWarps * 32);
@@ -340,22 +376,25 @@ cudaError_t launch_rowreg(const void* x, int M, int K, int n_bits, int mode, voi
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = code_fmt == TASQ_CODES_S8
-                        ? cudaLaunchKernelEx(&cfg, quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_S8>, x, M, K, n_bits,
-                                             mode, codes, alpha, zc)
-                        : cudaLaunchKernelEx(&cfg, quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16>, x, M, K, n_bits,
-                                             mode, codes, alpha, zc);
+    auto kernel = code_fmt == TASQ_CODES_S8
+                      ? (sums ? quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_S8, true>
+                              : quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_S8, false>)
+                      : (sums ? quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16, true>
+                              : quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16, false>);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, x, M, K, n_bits, mode, codes, alpha, zc, sums);
     return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 template <int DTYPE>
 bool dispatch_rowreg(int chunks_per_lane, const void* x, int M, int K, int n_bits, int mode, void* codes, int code_fmt,
-                     float* alpha, float* zc, cudaStream_t st, cudaError_t* e) {
-    if (chunks_per_lane <= 2) *e = launch_rowreg<2, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
-    else if (chunks_per_lane <= 5) *e = launch_rowreg<5, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
-    else if (chunks_per_lane <= 9) *e = launch_rowreg<9, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
-    else if (chunks_per_lane <= 18) *e = launch_rowreg<18, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
-    else if (chunks_per_lane <= 24) *e = launch_rowreg<24, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st);
+                     float* alpha, float* zc, int32_t* sums, cudaStream_t st, cudaError_t* e) {
+    if (chunks_per_lane <= 2) *e = launch_rowreg<2, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, sums, st);
+    else if (chunks_per_lane <= 5) *e = launch_rowreg<5, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, sums, st);
+    else if (chunks_per_lane <= 9) *e = launch_rowreg<9, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, sums, st);
+    else if (chunks_per_lane <= 18)
+        *e = launch_rowreg<18, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, sums, st);
+    else if (chunks_per_lane <= 24)
+        *e = launch_rowreg<24, DTYPE>(x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, sums, st);
     else return false;
     return true;
 }
@@ -434,8 +473,9 @@ __global__ void __launch_bounds__(256) quant_act_tensor_kernel(const void* __res
 }
 
 // -------------------------------------------------------------------- pack --
-__global__ void pack_header_kernel(int kind, int N, int K, PackedHeader* hdr) {
+__global__ void pack_header_kernel(int kind, int N, int K, int has_zp, PackedHeader* hdr) {
     PackedHeader h = packed_layout(kind, N, K);
+    h.has_zp = has_zp;
     for (int b = 0; b <= kBMax; ++b) h.chunk_kb[b] = (b >= kBMin) ? 0x7FFFFFFF : 0;
     *hdr = h;
 }
@@ -568,26 +608,27 @@ cudaError_t launch_selftest_quotients(const float* x, int nx, const float* a, in
     return cudaGetLastError();
 }
 
-cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int8_t* sw, float* cw, float* alpha,
-                                 cudaStream_t st) {
+cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int mode, int8_t* sw, float* cw,
+                                 float* zcw, float* alpha, cudaStream_t st) {
     if (N == 0) return cudaSuccess;
-    quant_weights_kernel<<<(N + kRowWarps - 1) / kRowWarps, 256, 0, st>>>(w, dtype, N, K, sw, cw, alpha);
+    quant_weights_kernel<<<(N + kRowWarps - 1) / kRowWarps, 256, 0, st>>>(w, dtype, N, K, mode, sw, cw, zcw, alpha);
     return cudaGetLastError();
 }
 
 cudaError_t launch_quant_act_token(const void* x, int dtype, int M, int K, int n_bits, int mode, void* codes,
-                                   int code_fmt, float* alpha, float* zc, cudaStream_t st) {
+                                   int code_fmt, float* alpha, float* zc, int32_t* code_sums, cudaStream_t st) {
     if (M == 0) return cudaSuccess;
     // rows that fit in registers: one pass over HBM
     const int chunks = K * (dtype == TASQ_F32 ? 4 : 2) / 16;
     const int per_lane = (chunks + 31) / 32;
     cudaError_t e = cudaSuccess;
-    if (dtype == TASQ_F32 ? dispatch_rowreg<TASQ_F32>(per_lane, x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st, &e)
-                          : dispatch_rowreg<TASQ_BF16>(per_lane, x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, st, &e))
+    if (dtype == TASQ_F32
+            ? dispatch_rowreg<TASQ_F32>(per_lane, x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, code_sums, st, &e)
+            : dispatch_rowreg<TASQ_BF16>(per_lane, x, M, K, n_bits, mode, codes, code_fmt, alpha, zc, code_sums, st, &e))
         return e;
     // longer rows: two passes (the second mostly from L2)
     quant_act_token_kernel<<<(M + kRowWarps - 1) / kRowWarps, 256, 0, st>>>(x, dtype, M, K, n_bits, mode, codes,
-                                                                            code_fmt, alpha, zc);
+                                                                            code_fmt, alpha, zc, code_sums);
     return cudaGetLastError();
 }
 
@@ -609,18 +650,20 @@ cudaError_t launch_quant_act_tensor(const void* x, int dtype, int64_t count, int
     return cudaGetLastError();
 }
 
-cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* bias, int N, int K, int Cin,
-                        void* packed, cudaStream_t st) {
+cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* zcw, const float* bias, int N, int K,
+                        int Cin, void* packed, cudaStream_t st) {
     const PackedHeader lay = packed_layout(kind, N, K);
     char* p = reinterpret_cast<char*>(packed);
     cudaError_t e = cudaMemsetAsync(p, 0, lay.total, st);
     if (e != cudaSuccess) return e;
-    pack_header_kernel<<<1, 1, 0, st>>>(kind, N, K, reinterpret_cast<PackedHeader*>(p));
+    pack_header_kernel<<<1, 1, 0, st>>>(kind, N, K, zcw ? 1 : 0, reinterpret_cast<PackedHeader*>(p));
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (N == 0) return cudaSuccess;
     if ((e = cudaMemcpyAsync(p + lay.off_w, sw, size_t(N) * K, cudaMemcpyDeviceToDevice, st)) != cudaSuccess) return e;
     if ((e = cudaMemcpyAsync(p + lay.off_cw, cw, size_t(N) * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess) return e;
     if (bias && (e = cudaMemcpyAsync(p + lay.off_bias, bias, size_t(N) * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+        return e;
+    if (zcw && (e = cudaMemcpyAsync(p + lay.off_zcw, zcw, size_t(N) * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
         return e;
     int KB = (K + kCertKBlock - 1) / kCertKBlock;
     size_t smem = size_t(kNumB) * KB * sizeof(int);

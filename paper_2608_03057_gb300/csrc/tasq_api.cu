@@ -177,17 +177,33 @@ TASQ_API int tasq_selftest_quotients(tasq_ctx ctx, const float* d_x, int nx, con
     return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "selftest launch");
 }
 
-TASQ_API int tasq_quant_weights(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, int8_t* d_sw, float* d_cw,
-                                float* d_alpha, tasq_stream stream) {
-    CHECK_CTX(ctx);
+namespace {
+
+int quant_weights(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, int mode, int8_t* d_sw, float* d_cw,
+                  float* d_zcw, float* d_alpha, tasq_stream stream) {
     REQUIRE(dtype == TASQ_F32 || dtype == TASQ_BF16, TASQ_ERR_INVALID_ARG, "dtype %d", dtype);
     REQUIRE(N >= 0 && K > 0, TASQ_ERR_INVALID_ARG, "N=%d K=%d", N, K);
     REQUIRE(K % 16 == 0, TASQ_ERR_UNSUPPORTED, "K=%d must be a multiple of 16", K);
-    REQUIRE(N == 0 || (d_w && d_sw && d_cw), TASQ_ERR_INVALID_ARG, "NULL pointer");
-    REQUIRE(aligned16(d_w) && aligned16(d_sw) && aligned16(d_cw) && aligned16(d_alpha), TASQ_ERR_UNSUPPORTED,
-            "pointers must be 16-byte aligned");
-    cudaError_t e = tasq::launch_quant_weights(d_w, dtype, N, K, d_sw, d_cw, d_alpha, (cudaStream_t)stream);
+    REQUIRE(N == 0 || (d_w && d_sw && d_cw && (mode == TASQ_SYMRANGE || d_zcw)), TASQ_ERR_INVALID_ARG,
+            "NULL pointer");
+    REQUIRE(aligned16(d_w) && aligned16(d_sw) && aligned16(d_cw) && aligned16(d_alpha) && aligned16(d_zcw),
+            TASQ_ERR_UNSUPPORTED, "pointers must be 16-byte aligned");
+    cudaError_t e = tasq::launch_quant_weights(d_w, dtype, N, K, mode, d_sw, d_cw, d_zcw, d_alpha, (cudaStream_t)stream);
     return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "quant_weights launch");
+}
+
+}  // namespace
+
+TASQ_API int tasq_quant_weights(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, int8_t* d_sw, float* d_cw,
+                                float* d_alpha, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    return quant_weights(ctx, d_w, dtype, N, K, TASQ_SYMRANGE, d_sw, d_cw, nullptr, d_alpha, stream);
+}
+
+TASQ_API int tasq_quant_weights_asym(tasq_ctx ctx, const void* d_w, int dtype, int N, int K, int8_t* d_sw,
+                                     float* d_cw, float* d_zcw, float* d_alpha, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    return quant_weights(ctx, d_w, dtype, N, K, TASQ_ASYM, d_sw, d_cw, d_zcw, d_alpha, stream);
 }
 
 TASQ_API size_t tasq_packed_bytes(int kind, int N, int K) {
@@ -196,10 +212,12 @@ TASQ_API size_t tasq_packed_bytes(int kind, int N, int K) {
     return (size_t)tasq::packed_layout(kind, N, K).total;
 }
 
-TASQ_API int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_bias,
-                               int N, int K, int Cin, void* d_packed, tasq_stream stream) {
-    CHECK_CTX(ctx);
+namespace {
+
+int pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
+                 const float* d_bias, int N, int K, int Cin, void* d_packed, tasq_stream stream) {
     REQUIRE(kind == TASQ_LINEAR || kind == TASQ_CONV3X3, TASQ_ERR_INVALID_ARG, "kind %d", kind);
+    REQUIRE(!d_zcw || kind == TASQ_LINEAR, TASQ_ERR_UNSUPPORTED, "weight zero offsets: linear layers only");
     REQUIRE(N > 0 && K > 0, TASQ_ERR_INVALID_ARG, "N=%d K=%d", N, K);
     REQUIRE(K % 16 == 0 && N % 8 == 0, TASQ_ERR_UNSUPPORTED, "need K %% 16 == 0 and N %% 8 == 0 (N=%d K=%d)", N, K);
     if (kind == TASQ_CONV3X3) {
@@ -208,11 +226,26 @@ TASQ_API int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const
     }
     REQUIRE(d_sw && d_cw && d_packed, TASQ_ERR_INVALID_ARG, "NULL pointer");
     REQUIRE((reinterpret_cast<uintptr_t>(d_packed) & 255u) == 0, TASQ_ERR_UNSUPPORTED, "d_packed must be 256-byte aligned");
-    REQUIRE(aligned16(d_sw) && aligned16(d_cw) && aligned16(d_bias), TASQ_ERR_UNSUPPORTED,
+    REQUIRE(aligned16(d_sw) && aligned16(d_cw) && aligned16(d_bias) && aligned16(d_zcw), TASQ_ERR_UNSUPPORTED,
             "pointers must be 16-byte aligned");
-    cudaError_t e = tasq::launch_pack(kind, d_sw, d_cw, d_bias, N, K, kind == TASQ_CONV3X3 ? Cin : 0, d_packed,
+    cudaError_t e = tasq::launch_pack(kind, d_sw, d_cw, d_zcw, d_bias, N, K, kind == TASQ_CONV3X3 ? Cin : 0, d_packed,
                                       (cudaStream_t)stream);
     return e == cudaSuccess ? TASQ_OK : cuda_fail(ctx, e, "pack launch");
+}
+
+}  // namespace
+
+TASQ_API int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_bias,
+                               int N, int K, int Cin, void* d_packed, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    return pack_weights(ctx, kind, d_sw, d_cw, nullptr, d_bias, N, K, Cin, d_packed, stream);
+}
+
+TASQ_API int tasq_pack_weights_zp(tasq_ctx ctx, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
+                                  const float* d_bias, int N, int K, void* d_packed, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(d_zcw, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    return pack_weights(ctx, TASQ_LINEAR, d_sw, d_cw, d_zcw, d_bias, N, K, 0, d_packed, stream);
 }
 
 TASQ_API int tasq_set_schedule(tasq_ctx ctx, const uint8_t* h_bits, int L, int S) {
@@ -246,9 +279,10 @@ TASQ_API int tasq_set_stage_device(tasq_ctx ctx, const int32_t* d_stage) {
     return TASQ_OK;
 }
 
-TASQ_API int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode, int gran,
-                            void* d_codes, int code_fmt, float* d_alpha, float* d_zc, tasq_stream stream) {
-    CHECK_CTX(ctx);
+namespace {
+
+int quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode, int gran, void* d_codes,
+              int code_fmt, float* d_alpha, float* d_zc, int32_t* d_code_sums, tasq_stream stream) {
     REQUIRE(dtype == TASQ_F32 || dtype == TASQ_BF16, TASQ_ERR_INVALID_ARG, "dtype %d", dtype);
     REQUIRE(mode == TASQ_SYMRANGE || mode == TASQ_ASYM, TASQ_ERR_INVALID_ARG, "mode %d", mode);
     REQUIRE(gran == TASQ_PER_TOKEN || gran == TASQ_PER_TENSOR, TASQ_ERR_INVALID_ARG, "gran %d", gran);
@@ -261,7 +295,7 @@ TASQ_API int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int
     REQUIRE(aligned16(d_x) && aligned16(d_codes), TASQ_ERR_UNSUPPORTED, "pointers must be 16-byte aligned");
     cudaError_t e;
     if (gran == TASQ_PER_TOKEN)
-        e = tasq::launch_quant_act_token(d_x, dtype, M, K, n_bits, mode, d_codes, code_fmt, d_alpha, d_zc,
+        e = tasq::launch_quant_act_token(d_x, dtype, M, K, n_bits, mode, d_codes, code_fmt, d_alpha, d_zc, d_code_sums,
                                          (cudaStream_t)stream);
     else
         e = tasq::launch_quant_act_tensor(d_x, dtype, (int64_t)M * K, n_bits, mode, d_codes, code_fmt, d_alpha, d_zc,
@@ -271,11 +305,29 @@ TASQ_API int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int
     return TASQ_OK;
 }
 
+}  // namespace
+
+TASQ_API int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode, int gran,
+                            void* d_codes, int code_fmt, float* d_alpha, float* d_zc, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    return quant_act(ctx, d_x, dtype, M, K, n_bits, mode, gran, d_codes, code_fmt, d_alpha, d_zc, nullptr, stream);
+}
+
+TASQ_API int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode,
+                                 void* d_codes, int code_fmt, float* d_alpha, float* d_zc, int32_t* d_code_sums,
+                                 tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(M == 0 || d_code_sums, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    return quant_act(ctx, d_x, dtype, M, K, n_bits, mode, TASQ_PER_TOKEN, d_codes, code_fmt, d_alpha, d_zc,
+                     d_code_sums, stream);
+}
+
 namespace {
 
 int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void* d_codes, int code_fmt,
-                       const float* d_alpha, const float* d_zc, int M, const void* d_packed, int N, int K, int B,
-                       int H, int W, int Cin, uint16_t* d_y, int32_t* d_acc, tasq_stream stream) {
+                       const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int M,
+                       const void* d_packed, int N, int K, int B, int H, int W, int Cin, uint16_t* d_y,
+                       int32_t* d_acc, tasq_stream stream) {
     REQUIRE(ctx->d_table, TASQ_ERR_INVALID_ARG, "no schedule: call tasq_set_schedule first");
     REQUIRE(layer >= 0 && layer < ctx->L, TASQ_ERR_INVALID_ARG, "layer %d outside 0..%d", layer, ctx->L - 1);
     REQUIRE(stage >= -1 && stage < ctx->S, TASQ_ERR_INVALID_ARG, "stage %d outside -1..%d", stage, ctx->S - 1);
@@ -325,6 +377,8 @@ int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void*
     a.split_cap = tasq::kSplitBufBytes / int64_t(sizeof(int32_t));
     a.status = ctx->d_words;
     a.timeout_ns = ctx->timeout_ns;
+    a.zcw = reinterpret_cast<const float*>(p + lay.off_zcw);
+    a.code_sums = d_code_sums;
     cudaError_t e;
     int kernels = 0;
     if (route == TASQ_ROUTE_TC) {
@@ -346,8 +400,18 @@ TASQ_API int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_
                               const float* d_alpha, const float* d_zc, int M, const void* d_packed, int N, int K,
                               uint16_t* d_y, int32_t* d_acc, tasq_stream stream) {
     CHECK_CTX(ctx);
-    return masked_contraction(ctx, TASQ_LINEAR, layer, stage, d_codes, code_fmt, d_alpha, d_zc, M, d_packed, N, K, 1,
-                              0, 0, 0, d_y, d_acc, stream);
+    return masked_contraction(ctx, TASQ_LINEAR, layer, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, M, d_packed,
+                              N, K, 1, 0, 0, 0, d_y, d_acc, stream);
+}
+
+TASQ_API int tasq_masked_gemm_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
+                                 const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int M,
+                                 const void* d_packed, int N, int K, uint16_t* d_y, int32_t* d_acc,
+                                 tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(M == 0 || d_code_sums, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    return masked_contraction(ctx, TASQ_LINEAR, layer, stage, d_codes, code_fmt, d_alpha, d_zc, d_code_sums, M,
+                              d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream);
 }
 
 TASQ_API int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
@@ -357,6 +421,6 @@ TASQ_API int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void*
     REQUIRE(B >= 0 && H > 0 && W > 0 && Cin > 0, TASQ_ERR_INVALID_ARG, "B=%d H=%d W=%d Cin=%d", B, H, W, Cin);
     REQUIRE(Cin % 16 == 0, TASQ_ERR_UNSUPPORTED, "conv: Cin=%d must be a multiple of 16", Cin);
     REQUIRE((int64_t)B * H * W <= 0x7FFFFFFF && (int64_t)9 * Cin <= 0x7FFFFFFF, TASQ_ERR_UNSUPPORTED, "too large");
-    return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, B * H * W, d_packed,
-                              Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
+    return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, B * H * W,
+                              d_packed, Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
 }

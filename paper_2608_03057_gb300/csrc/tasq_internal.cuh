@@ -22,6 +22,8 @@ struct PackedHeader {
     int32_t kind, N, K, Cin;
     int32_t chunk_kb[kBMax + 1];  // TC route: K blocks per exact fp32 chunk, indexed by b
     int64_t off_w, off_cw, off_bias, off_rs, off_ts, total;
+    int64_t off_zcw;  // fp32 [N] weight zero offsets zcw = 128 - z (zeros unless has_zp)
+    int32_t has_zp;   // packed with zero offsets: the four-term epilogue applies
 };
 static_assert(sizeof(PackedHeader) <= 256, "header must fit in 256 bytes");
 
@@ -39,7 +41,8 @@ __host__ __device__ inline PackedHeader packed_layout(int kind, int N, int K) {
     h.off_bias = align_up(h.off_cw + 4 * int64_t(N), 256);
     h.off_rs = align_up(h.off_bias + 4 * int64_t(N), 256);          // int32 [kNumB][N]
     h.off_ts = align_up(h.off_rs + 4 * int64_t(kNumB) * N, 256);     // int32 [kNumB][N][9] (conv)
-    h.total = align_up(h.off_ts + (kind == TASQ_CONV3X3 ? 4 * int64_t(kNumB) * N * 9 : 0), 256);
+    h.off_zcw = align_up(h.off_ts + (kind == TASQ_CONV3X3 ? 4 * int64_t(kNumB) * N * 9 : 0), 256);  // fp32 [N]
+    h.total = align_up(h.off_zcw + 4 * int64_t(N), 256);
     return h;
 }
 
@@ -82,6 +85,11 @@ struct GemmArgs {
     int64_t split_cap;        // elements of split_buf
     int* status;
     unsigned long long timeout_ns;
+    // Asymmetric weights (App. A.1.1 on the true per-channel range, Eq.
+    // weight_dequant with a real zero point): w_hat = c_w * (mask_b(s_w) + zcw).
+    // With code_sums set the epilogue adds zcw[n] * t[m], t = sum_k (s_x + zc).
+    const float* zcw;          // [N] from the packed buffer (zeros for a symmetric pack)
+    const int32_t* code_sums;  // [M] sum_k s_x[m][k], or NULL (two-term epilogue)
 };
 
 // Resolves b for this launch on the device; returns 0 (and records an error)
@@ -93,7 +101,9 @@ __device__ inline int resolve_bits(const GemmArgs& a) {
         return 0;
     }
     int b = a.table[a.layer * a.S + stage];
-    if (b < kBMin || b > kBMax || a.hdr->magic != kPackedMagic || a.hdr->N != a.N || a.hdr->K != a.K) {
+    // a buffer packed with zero offsets needs the code sums of the four-term epilogue
+    if (b < kBMin || b > kBMax || a.hdr->magic != kPackedMagic || a.hdr->N != a.N || a.hdr->K != a.K ||
+        (a.hdr->has_zp && !a.code_sums)) {
         set_status(a.status, TASQ_ERR_DEVICE);
         return 0;
     }
@@ -126,6 +136,21 @@ __device__ inline float epilogue_value(int acc, float alpha, float zc, int rs, f
     return __fmaf_rn(u, __fmul_rn(alpha, cw), bias);
 }
 
+// Asymmetric weights: t = RN(float(sx) + RN(float(K) * zc)), the token's
+// activation sum sum_k (s_x + zc) (exact integer sx, |sx| <= 128 K < 2^24),
+// and the epilogue with the weight zero-offset term, each step rounded once:
+// u1 = fma(zc, float(rs), float(acc)), u2 = fma(zcw, t, u1), y = fma(u2, alpha*cw, bias),
+// i.e. y = alpha * cw * (acc + zc * rs + zcw * (sx + K * zc)) + bias.
+__device__ __forceinline__ float token_zero_sum(int sx, int K, float zc) {
+    return __fadd_rn(__int2float_rn(sx), __fmul_rn(__int2float_rn(K), zc));
+}
+__device__ inline float epilogue_value_zp(int acc, float alpha, float zc, float t, int rs, float cw, float zcw,
+                                          float bias) {
+    const float u1 = __fmaf_rn(zc, __int2float_rn(rs), __int2float_rn(acc));
+    const float u2 = __fmaf_rn(zcw, t, u1);
+    return __fmaf_rn(u2, __fmul_rn(alpha, cw), bias);
+}
+
 // fp32 -> bf16 bits, round to nearest even (finite inputs).
 __device__ inline uint16_t bf16_bits(float f) {
     uint32_t u = __float_as_uint(f);
@@ -153,14 +178,17 @@ __device__ inline int conv_row_sum(const int32_t* ts_n, int h, int w, int H, int
 // ---------------------------------------------------------------------------
 // Host-side launchers implemented in the kernel translation units.
 // ---------------------------------------------------------------------------
-cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int8_t* sw, float* cw, float* alpha,
-                                 cudaStream_t st);
+// mode: TASQ_SYMRANGE or TASQ_ASYM (then zcw [N] receives 128 - z; may be NULL otherwise)
+cudaError_t launch_quant_weights(const void* w, int dtype, int N, int K, int mode, int8_t* sw, float* cw,
+                                 float* zcw, float* alpha, cudaStream_t st);
+// code_sums: [M] int32 sum_k s[m][k], or NULL
 cudaError_t launch_quant_act_token(const void* x, int dtype, int M, int K, int n_bits, int mode, void* codes,
-                                   int code_fmt, float* alpha, float* zc, cudaStream_t st);
+                                   int code_fmt, float* alpha, float* zc, int32_t* code_sums, cudaStream_t st);
 cudaError_t launch_quant_act_tensor(const void* x, int dtype, int64_t count, int n_bits, int mode, void* codes,
                                     int code_fmt, float* alpha, float* zc, unsigned int* scratch, cudaStream_t st);
-cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* bias, int N, int K, int Cin,
-                        void* packed, cudaStream_t st);
+// zcw: [N] weight zero offsets (linear only), or NULL for a symmetric pack
+cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* zcw, const float* bias, int N, int K,
+                        int Cin, void* packed, cudaStream_t st);
 cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
 // *kernels: how many kernels the call enqueued (the contraction, plus the split-K
 // reduction when K is split).

@@ -60,12 +60,16 @@ def lib():
                 "tasq_selftest_timeout": ([P, U64, P], I),
                 "tasq_selftest_quotients": ([P, P, I, P, I, P, P], I),
                 "tasq_quant_weights": ([P, P, I, I, I, P, P, P, P], I),
+                "tasq_quant_weights_asym": ([P, P, I, I, I, P, P, P, P, P], I),
                 "tasq_packed_bytes": ([I, I, I], SZ),
                 "tasq_pack_weights": ([P, I, P, P, P, I, I, I, P, P], I),
+                "tasq_pack_weights_zp": ([P, P, P, P, P, I, I, P, P], I),
                 "tasq_set_schedule": ([P, P, I, I], I),
                 "tasq_set_stage_device": ([P, P], I),
                 "tasq_quant_act": ([P, P, I, I, I, I, I, I, P, I, P, P, P], I),
+                "tasq_quant_act_sums": ([P, P, I, I, I, I, I, P, I, P, P, P, P], I),
                 "tasq_masked_gemm": ([P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
+                "tasq_masked_gemm_zp": ([P, I, I, P, I, P, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_conv3x3": ([P, I, I, P, I, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_quant_act_tensor_noalloc": ([P, I, I, I, I, I, P, I, P, P, P], I),
             }
@@ -158,6 +162,11 @@ def tasq_quant_weights(ctx, w, dtype, N, K, sw, cw, alpha=None, stream=None) -> 
                                          _stream(stream)))
 
 
+def tasq_quant_weights_asym(ctx, w, dtype, N, K, sw, cw, zcw, alpha=None, stream=None) -> None:
+    _check(ctx, lib().tasq_quant_weights_asym(ctx, _ptr(w), int(dtype), int(N), int(K), _ptr(sw), _ptr(cw), _ptr(zcw),
+                                              _ptr(alpha), _stream(stream)))
+
+
 def tasq_packed_bytes(kind, N, K) -> int:
     return int(lib().tasq_packed_bytes(int(kind), int(N), int(K)))
 
@@ -165,6 +174,11 @@ def tasq_packed_bytes(kind, N, K) -> int:
 def tasq_pack_weights(ctx, kind, sw, cw, bias, N, K, Cin, packed, stream=None) -> None:
     _check(ctx, lib().tasq_pack_weights(ctx, int(kind), _ptr(sw), _ptr(cw), _ptr(bias), int(N), int(K), int(Cin),
                                         _ptr(packed), _stream(stream)))
+
+
+def tasq_pack_weights_zp(ctx, sw, cw, zcw, bias, N, K, packed, stream=None) -> None:
+    _check(ctx, lib().tasq_pack_weights_zp(ctx, _ptr(sw), _ptr(cw), _ptr(zcw), _ptr(bias), int(N), int(K),
+                                           _ptr(packed), _stream(stream)))
 
 
 def tasq_set_schedule(ctx, h_bits, L, S) -> None:
@@ -179,6 +193,18 @@ def tasq_set_stage_device(ctx, d_stage) -> None:
 def tasq_quant_act(ctx, x, dtype, M, K, n_bits, mode, gran, codes, code_fmt, alpha, zc, stream=None) -> None:
     _check(ctx, lib().tasq_quant_act(ctx, _ptr(x), int(dtype), int(M), int(K), int(n_bits), int(mode), int(gran),
                                      _ptr(codes), int(code_fmt), _ptr(alpha), _ptr(zc), _stream(stream)))
+
+
+def tasq_quant_act_sums(ctx, x, dtype, M, K, n_bits, mode, codes, code_fmt, alpha, zc, code_sums, stream=None) -> None:
+    _check(ctx, lib().tasq_quant_act_sums(ctx, _ptr(x), int(dtype), int(M), int(K), int(n_bits), int(mode), _ptr(codes),
+                                          int(code_fmt), _ptr(alpha), _ptr(zc), _ptr(code_sums), _stream(stream)))
+
+
+def tasq_masked_gemm_zp(ctx, layer, stage, codes, code_fmt, alpha, zc, code_sums, M, packed, N, K, y, acc=None,
+                        stream=None) -> None:
+    _check(ctx, lib().tasq_masked_gemm_zp(ctx, int(layer), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
+                                          _ptr(zc), _ptr(code_sums), int(M), _ptr(packed), int(N), int(K), _ptr(y),
+                                          _ptr(acc), _stream(stream)))
 
 
 def tasq_masked_gemm(ctx, layer, stage, codes, code_fmt, alpha, zc, M, packed, N, K, y, acc=None, stream=None) -> None:

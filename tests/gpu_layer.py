@@ -49,6 +49,41 @@ def quant_weights(ctx, w_dev, dtype, N, K):
     return sw, cw, al
 
 
+def quant_weights_asym(ctx, w_dev, dtype, N, K):
+    t = torch()
+    sw = empty((N, K), t.int8)
+    cw = empty((N,), t.float32)
+    zcw = empty((N,), t.float32)
+    al = empty((N,), t.float32)
+    tasq.tasq_quant_weights_asym(ctx.h, w_dev, dtype, N, K, sw, cw, zcw, al)
+    return sw, cw, zcw, al
+
+
+def pack_zp(ctx, sw, cw, zcw, bias, N, K):
+    t = torch()
+    packed = empty((tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, N, K),), t.uint8)
+    tasq.tasq_pack_weights_zp(ctx.h, sw, cw, zcw, bias, N, K, packed)
+    return packed
+
+
+def quant_act_sums(ctx, x_dev, dtype, M, K, n_bits=8, mode=tasq.TASQ_SYMRANGE, code_fmt=tasq.TASQ_CODES_S8):
+    t = torch()
+    codes = empty((M, K), t.int8 if code_fmt == tasq.TASQ_CODES_S8 else t.float16)
+    alpha = empty((max(M, 1),), t.float32)
+    zc = empty((max(M, 1),), t.float32)
+    sums = empty((max(M, 1),), t.int32)
+    tasq.tasq_quant_act_sums(ctx.h, x_dev, dtype, M, K, n_bits, mode, codes, code_fmt, alpha, zc, sums)
+    return codes, alpha, zc, sums
+
+
+def gemm_zp(ctx, layer, stage, codes, code_fmt, alpha, zc, sums, M, packed, N, K, want_acc=True):
+    t = torch()
+    y = empty((M, N), t.int16)
+    acc = empty((M, N), t.int32) if want_acc else None
+    tasq.tasq_masked_gemm_zp(ctx.h, layer, stage, codes, code_fmt, alpha, zc, sums, M, packed, N, K, y, acc)
+    return y, acc
+
+
 def pack(ctx, kind, sw, cw, bias, N, K, Cin=0):
     t = torch()
     nbytes = tasq.tasq_packed_bytes(kind, N, K)

@@ -59,8 +59,8 @@ def test_packed_bytes_layout(built_lib):
     from paper_2608_03057_gb300 import tasq
     n, k = 1152, 1152
     b = tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, n, k)
-    # 1 KB header, int8 weights, scale, bias, 7 row-sum vectors, 256-byte aligned
-    assert b % 256 == 0 and b >= 1024 + n * k + 4 * n * 2 + 7 * 4 * n
+    # 1 KB header, int8 weights, scale, bias, 7 row-sum vectors, weight zero offsets, 256-byte aligned
+    assert b % 256 == 0 and b >= 1024 + n * k + 4 * n * 2 + 7 * 4 * n + 4 * n
     c = tasq.tasq_packed_bytes(tasq.TASQ_CONV3X3, 320, 9 * 320)
     assert c >= 1024 + 320 * 2880 + 7 * 4 * 320 * 10
     assert tasq.tasq_packed_bytes(tasq.TASQ_CONV3X3, 320, 100) == 0  # K not 9*Cin

@@ -332,6 +332,126 @@ def test_full_size_sampled_rows(ctx, oracle, code_fmt, M, N, K):
         _check_layer(oracle, st, b, y, acc, rows=rows)
 
 
+# ---------------------------------------------- asymmetric weights (zp) --
+
+@pytest.mark.parametrize("dtype", [tasq.TASQ_F32, tasq.TASQ_BF16])
+def test_quant_weights_asym_bitexact(ctx, oracle, dtype):
+    N, K = 136, 1168
+    w = workloads.normal((N, K), seed=71, std=0.02)
+    w[::3] += 0.03  # skewed channels
+    w[5] = 0.25     # constant channel: alpha = 1, z = -min
+    if dtype == tasq.TASQ_BF16:
+        wd, w = G.to_bf16(w)
+    else:
+        wd = G.dev(w)
+    sw, cw, zcw, al = G.quant_weights_asym(ctx, wd, dtype, N, K)
+    ref = oracle.quant_weight(w, 8, oracle.ASYM)
+    assert np.array_equal(sw.cpu().numpy(), ref["s"])
+    assert np.array_equal(cw.cpu().numpy(), ref["c"])
+    assert np.array_equal(zcw.cpu().numpy(), ref["zcw"])
+    assert np.array_equal(al.cpu().numpy(), ref["alpha"])
+
+
+@pytest.mark.parametrize("code_fmt", [tasq.TASQ_CODES_S8, tasq.TASQ_CODES_F16])
+@pytest.mark.parametrize("mode", [tasq.TASQ_SYMRANGE, tasq.TASQ_ASYM])
+@pytest.mark.parametrize("M,K", [(70, 1152), (33, 8192)])
+def test_quant_act_code_sums_bitexact(ctx, oracle, code_fmt, mode, M, K):
+    """Per-token codes with their sums, from the one-pass (rows in registers)
+    and the two-pass (K = 8192) kernels."""
+    x = workloads.normal((M, K), seed=72)
+    x[3] += 2.0
+    codes, alpha, zc, sums = G.quant_act_sums(ctx, G.dev(x), tasq.TASQ_F32, M, K, 8, mode, code_fmt)
+    s_x, a_ref, z_ref = oracle.quant_act(x, 8, mode, oracle.PER_TOKEN)
+    assert np.array_equal(G.codes_to_int8(codes), s_x)
+    assert np.array_equal(alpha.cpu().numpy(), a_ref) and np.array_equal(zc.cpu().numpy(), z_ref)
+    assert np.array_equal(sums.cpu().numpy(), oracle.code_sums(s_x))
+
+
+def _setup_linear_zp(ctx, oracle, M, N, K, bits, seed, code_fmt, mode=tasq.TASQ_SYMRANGE, dtype=tasq.TASQ_F32):
+    w = workloads.normal((N, K), seed + 1, 0.02)
+    w[::2] += 0.02  # half the channels skewed: their zero offsets are far from 0
+    bias = workloads.normal((N,), seed + 2, 0.02)
+    x = workloads.normal((M, K), seed, 1.0)
+    if dtype == tasq.TASQ_BF16:
+        xd, x = G.to_bf16(x)
+    else:
+        xd = G.dev(x)
+    sw, cw, zcw, _ = G.quant_weights_asym(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+    packed = G.pack_zp(ctx, sw, cw, zcw, G.dev(bias), N, K)
+    tasq.tasq_set_schedule(ctx.h, np.asarray([bits], np.uint8), 1, len(bits))
+    codes, alpha, zc, sums = G.quant_act_sums(ctx, xd, dtype, M, K, 8, mode, code_fmt)
+    wq = oracle.quant_weight(w, 8, oracle.ASYM)
+    s_x, a_ref, z_ref = oracle.quant_act(x, 8, mode, oracle.PER_TOKEN)
+    return dict(packed=packed, codes=codes, alpha=alpha, zc=zc, sums=sums, wq=wq, s_x=s_x, a=a_ref, z=z_ref,
+                bias=bias, K=K)
+
+
+def _check_layer_zp(oracle, st, b, y, acc, rows=None):
+    s_x, a, z = st["s_x"], st["a"], st["z"]
+    if rows is not None:
+        s_x, a, z = s_x[rows], a[rows], z[rows]
+    ref_acc = oracle.gemm(s_x, st["wq"]["s"], b)
+    got_acc = acc.cpu().numpy() if rows is None else acc.cpu().numpy()[rows]
+    assert np.array_equal(got_acc, ref_acc), f"b={b}: {(got_acc != ref_acc).sum()} int32 mismatches"
+    rs = oracle.row_sums(st["wq"]["s"], b)
+    _, yb = oracle.epilogue_zp_f32(ref_acc, a, z, oracle.code_sums(s_x), rs, st["wq"]["c"], st["wq"]["zcw"],
+                                   st["bias"], st["K"])
+    got_y = G.bf16_bits_host(y) if rows is None else G.bf16_bits_host(y)[rows]
+    same = G.assert_bf16_close(got_y, yb)
+    assert same == yb.size, f"b={b}: {yb.size - same} bf16 outputs differ in the last bit"
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("M,N,K", [(256, 1152, 1152), (300, 136, 1168), (64, 128, 4096), (4000, 1096, 384),
+                                   (1, 8, 16)])
+def test_zp_linear_parity(ctx, oracle, code_fmt, M, N, K):
+    """Four-term epilogue (asymmetric weights) on every tile configuration of
+    the tensor-core route (192-, 256- and 64-token tiles, split K) and on the
+    mma.sync route: exact int32 sums and bit-exact bf16 outputs."""
+    bits = [8, 5, 3, 2]
+    st = _setup_linear_zp(ctx, oracle, M, N, K, bits, seed=M + 5, code_fmt=code_fmt, mode=tasq.TASQ_ASYM)
+    for stage, b in enumerate(bits):
+        y, acc = G.gemm_zp(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], st["sums"], M, st["packed"],
+                           N, K)
+        _check_layer_zp(oracle, st, b, y, acc)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_zp_full_size_sampled_rows(ctx, oracle, code_fmt):
+    M, N, K = 4096, 3456, 1152
+    bits = [4, 8]
+    st = _setup_linear_zp(ctx, oracle, M, N, K, bits, seed=9, code_fmt=code_fmt, dtype=tasq.TASQ_BF16)
+    rows = np.unique(np.concatenate([np.arange(0, M, max(1, M // 40)), [M - 1]]))
+    for stage, b in enumerate(bits):
+        y, acc = G.gemm_zp(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], st["sums"], M, st["packed"],
+                           N, K)
+        _check_layer_zp(oracle, st, b, y, acc, rows=rows)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_zp_call_on_a_symmetric_pack_equals_the_plain_call(ctx, oracle, code_fmt):
+    # a symmetric pack stores zcw = 0: the four-term epilogue gives the two-term result
+    M, N, K = 200, 264, 640
+    st = _setup_linear(ctx, oracle, M, N, K, [6], code_fmt=code_fmt)
+    _, _, _, sums = G.quant_act_sums(ctx, G.dev(workloads.normal((M, K), 0, 1.0)), tasq.TASQ_F32, M, K, 8,
+                                     tasq.TASQ_SYMRANGE, code_fmt)
+    y0, _ = G.gemm(ctx, 0, 0, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K)
+    y1, _ = G.gemm_zp(ctx, 0, 0, st["codes"], code_fmt, st["alpha"], st["zc"], sums, M, st["packed"], N, K)
+    assert np.array_equal(G.bf16_bits_host(y0), G.bf16_bits_host(y1))
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_zp_pack_without_code_sums_is_caught_on_device(ctx, oracle, code_fmt):
+    torch = G.torch()
+    M, N, K = 128, 128, 256
+    st = _setup_linear_zp(ctx, oracle, M, N, K, [8], seed=3, code_fmt=code_fmt)
+    y = torch.full((M, N), 0x1234, dtype=torch.int16, device="cuda")
+    tasq.tasq_masked_gemm(ctx.h, 0, 0, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K, y, None)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_ERR_DEVICE
+    assert bool((y == 0x1234).all())  # nothing written
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
 # ------------------------------------------------------------------ conv --
 
 def _run_conv(ctx, oracle, B, H, W, Cin, Cout, bits, code_fmt, seed=0, rows=None):
