@@ -417,6 +417,45 @@ def test_zp_linear_parity(ctx, oracle, code_fmt, M, N, K):
 
 
 @pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("zero_point", [False, True])
+def test_a4_activations(ctx, oracle, code_fmt, zero_point):
+    """4-bit activations (App. A.1.2 with n = 4: codes in [-8, 7], zc = 8 - z)
+    through the same contraction, with symmetric or asymmetric weights."""
+    M, N, K = 300, 264, 1152
+    bits = [8, 4, 2]
+    x = workloads.normal((M, K), 81)
+    w = workloads.normal((N, K), 82, 0.02)
+    w[::2] += 0.02
+    bias = workloads.normal((N,), 83, 0.02)
+    if zero_point:
+        sw, cw, zcw, _ = G.quant_weights_asym(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+        packed = G.pack_zp(ctx, sw, cw, zcw, G.dev(bias), N, K)
+        wq = oracle.quant_weight(w, 8, oracle.ASYM)
+    else:
+        sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+        packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, G.dev(bias), N, K)
+        wq = oracle.quant_weight(w, 8, oracle.SYMRANGE)
+    tasq.tasq_set_schedule(ctx.h, np.asarray([bits], np.uint8), 1, len(bits))
+    codes, alpha, zc, sums = G.quant_act_sums(ctx, G.dev(x), tasq.TASQ_F32, M, K, 4, tasq.TASQ_ASYM, code_fmt)
+    s_x, a_ref, z_ref = oracle.quant_act(x, 4, oracle.ASYM, oracle.PER_TOKEN)
+    assert np.array_equal(G.codes_to_int8(codes), s_x) and s_x.min() >= -8 and s_x.max() <= 7
+    for stage, b in enumerate(bits):
+        if zero_point:
+            y, acc = G.gemm_zp(ctx, 0, stage, codes, code_fmt, alpha, zc, sums, M, packed, N, K)
+        else:
+            y, acc = G.gemm(ctx, 0, stage, codes, code_fmt, alpha, zc, M, packed, N, K)
+        ref_acc = oracle.gemm(s_x, wq["s"], b)
+        assert np.array_equal(acc.cpu().numpy(), ref_acc)
+        rs = oracle.row_sums(wq["s"], b)
+        if zero_point:
+            _, yb = oracle.epilogue_zp_f32(ref_acc, a_ref, z_ref, oracle.code_sums(s_x), rs, wq["c"], wq["zcw"],
+                                           bias, K)
+        else:
+            _, yb = oracle.epilogue_f32(ref_acc, a_ref, z_ref, rs, wq["c"], bias)
+        assert G.assert_bf16_close(G.bf16_bits_host(y), yb) == yb.size
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
 def test_zp_full_size_sampled_rows(ctx, oracle, code_fmt):
     M, N, K = 4096, 3456, 1152
     bits = [4, 8]
