@@ -69,6 +69,9 @@ def _lib():
             lib.oq_code_sums.argtypes = [P, i32, i32, P]
             lib.oq_epilogue_zp_f32.argtypes = [P, i32, i32, i32, P, P, P, P, P, P, P, P, P]
             lib.oq_linear_zp_def_f64.argtypes = [P, P, P, i32, P, P, P, P, i32, i32, i32, P]
+            lib.oq_conv3x3_code_sums.argtypes = [P, i32, i32, i32, i32, P, P]
+            lib.oq_conv_epilogue_zp_f32.argtypes = [P, i64, i32, f32, f32, P, P, P, P, P, P, P, P]
+            lib.oq_conv3x3_zp_def_f64.argtypes = [P, f32, f32, i32, i32, i32, i32, P, P, P, P, i32, i32, P]
             _LIB = lib
     return _LIB
 
@@ -264,3 +267,40 @@ def stage_of_step(step, n_steps, n_stages):
     """Contiguous partition of the trajectory into stages (Sec. 3.2, stage-wise
     sharing): stage = floor(step * S / T), stage 0 = the noisiest steps."""
     return (step * n_stages) // n_steps
+
+
+def conv3x3_code_sums(s_x_nhwc):
+    """Per output pixel: (sxw, Kv) = (sum of the in-bounds taps' input codes, Cin x in-bounds taps)."""
+    s_x = _c(s_x_nhwc, np.int8)
+    B, H, W, Cin = s_x.shape
+    P = B * H * W
+    sxw = np.empty(P, np.int32)
+    kv = np.empty(P, np.int32)
+    _lib().oq_conv3x3_code_sums(_p(s_x), B, H, W, Cin, _p(sxw), _p(kv))
+    return sxw, kv
+
+
+def conv_epilogue_zp_f32(acc, alpha, zc, sxw, kv, rs, c_w, zcw, bias):
+    """Four-term conv epilogue (asymmetric weights, one activation scale) in the
+    kernel's fp32 order.  acc, rs: [P, N].  Returns (y_f32, y_bf16_bits)."""
+    acc = _c(acc, np.int32)
+    P, N = acc.shape
+    bias = None if bias is None else _c(bias, np.float32)
+    y = np.empty((P, N), np.float32)
+    yb = np.empty((P, N), np.uint16)
+    _lib().oq_conv_epilogue_zp_f32(_p(acc), P, N, float(np.float32(alpha)), float(np.float32(zc)),
+                                   _p(_c(sxw, np.int32)), _p(_c(kv, np.int32)), _p(_c(rs, np.int32)),
+                                   _p(_c(c_w, np.float32)), _p(_c(zcw, np.float32)), _p(bias), _p(y), _p(yb))
+    return y, yb
+
+
+def conv3x3_zp_def_f64(s_x_nhwc, alpha, zc, s_w, c_w, z, bias, b):
+    s_x = _c(s_x_nhwc, np.int8)
+    B, H, W, Cin = s_x.shape
+    s_w = _c(s_w, np.int8).reshape(s_w.shape[0], -1)
+    Cout = s_w.shape[0]
+    bias = None if bias is None else _c(bias, np.float32)
+    y = np.empty((B * H * W, Cout), np.float64)
+    _lib().oq_conv3x3_zp_def_f64(_p(s_x), float(alpha), float(zc), B, H, W, Cin, _p(s_w), _p(_c(c_w, np.float32)),
+                                 _p(_c(z, np.float32)), _p(bias), Cout, int(b), _p(y))
+    return y

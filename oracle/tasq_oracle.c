@@ -411,3 +411,96 @@ void oq_linear_zp_def_f64(const int8_t* s_x, const float* alpha, const float* zc
         }
     }
 }
+
+/*
+ * 3x3 convolution with asymmetric weights.  The padded taps are zero in the
+ * real domain, so over output pixel p only the in-bounds taps carry terms:
+ *   sum x_hat * w_hat_b = alpha * c * (acc + zc * rs[p] + zcw * t[p]),
+ *   t[p] = sxw[p] + Kv[p] * zc,
+ * with sxw[p] the sum of the codes of the in-bounds taps' input pixels (all
+ * Cin channels) and Kv[p] = Cin * (number of in-bounds taps).  Outputs sxw
+ * and Kv per output pixel p = (b*H + h)*W + w.
+ */
+void oq_conv3x3_code_sums(const int8_t* s_x, int B, int H, int W, int Cin, int32_t* sxw, int32_t* kv) {
+    int64_t P = (int64_t)B * H * W;
+    for (int64_t p = 0; p < P; ++p) {
+        int bb = (int)(p / ((int64_t)H * W));
+        int h = (int)((p / W) % H);
+        int w = (int)(p % W);
+        int64_t sum = 0;
+        int taps = 0;
+        for (int kh = 0; kh < 3; ++kh) {
+            int ih = h + kh - 1;
+            if (ih < 0 || ih >= H) continue;
+            for (int kw = 0; kw < 3; ++kw) {
+                int iw = w + kw - 1;
+                if (iw < 0 || iw >= W) continue;
+                const int8_t* xr = s_x + (((int64_t)bb * H + ih) * W + iw) * Cin;
+                for (int c = 0; c < Cin; ++c) sum += xr[c];
+                ++taps;
+            }
+        }
+        sxw[p] = (int32_t)sum;
+        kv[p] = taps * Cin;
+    }
+}
+
+/*
+ * The conv four-term dequantization in fp32, one activation scale for the
+ * tensor (alpha, zc), rs[p][n] the in-bounds row sums of oq_conv3x3:
+ *   t  = RN(float(sxw[p]) + RN(float(Kv[p]) * zc)),
+ *   u1 = RN(zc * float(rs) + float(acc)),  u2 = RN(zcw * t + u1),
+ *   y  = RN(u2 * RN(alpha * c) + bias),    bf16_rne(y).
+ */
+void oq_conv_epilogue_zp_f32(const int32_t* acc, int64_t P, int N, float alpha, float zc, const int32_t* sxw,
+                             const int32_t* kv, const int32_t* rs, const float* c_w, const float* zcw,
+                             const float* bias, float* y_f32, uint16_t* y_bf16) {
+    for (int64_t p = 0; p < P; ++p) {
+        const float t = (float)sxw[p] + (float)kv[p] * zc;
+        for (int n = 0; n < N; ++n) {
+            float a = (float)acc[p * N + n];
+            float u1 = fmaf(zc, (float)rs[p * N + n], a);
+            float u2 = fmaf(zcw[n], t, u1);
+            float s = alpha * c_w[n];
+            float y = fmaf(u2, s, bias ? bias[n] : 0.0f);
+            if (y_f32) y_f32[p * N + n] = y;
+            if (y_bf16) y_bf16[p * N + n] = oq_bf16_rne(y);
+        }
+    }
+}
+
+/*
+ * The 3x3 convolution with asymmetric weights by its definition, in fp64:
+ * x_hat = alpha * (s_x + zc) inside the image and 0 in the padding,
+ * w_hat = c * (Q_b - z) with Q_b = mask_b(s_w) + 128 and the quantizer's z.
+ */
+void oq_conv3x3_zp_def_f64(const int8_t* s_x, float alpha, float zc, int B, int H, int W, int Cin,
+                           const int8_t* s_w, const float* c_w, const float* z, const float* bias, int Cout, int b,
+                           double* y) {
+    int64_t P = (int64_t)B * H * W;
+    int K = 9 * Cin;
+#pragma omp parallel for schedule(static)
+    for (int64_t p = 0; p < P; ++p) {
+        int bb = (int)(p / ((int64_t)H * W));
+        int h = (int)((p / W) % H);
+        int w = (int)(p % W);
+        for (int n = 0; n < Cout; ++n) {
+            double sum = 0.0;
+            for (int kh = 0; kh < 3; ++kh) {
+                for (int kw = 0; kw < 3; ++kw) {
+                    int ih = h + kh - 1, iw = w + kw - 1;
+                    for (int c = 0; c < Cin; ++c) {
+                        double xh = 0.0;
+                        if (ih >= 0 && ih < H && iw >= 0 && iw < W)
+                            xh = (double)alpha *
+                                 ((double)s_x[(((int64_t)bb * H + ih) * W + iw) * Cin + c] + (double)zc);
+                        double qb = (double)oq_mask(s_w[(int64_t)n * K + (kh * 3 + kw) * Cin + c], b) + 128.0;
+                        double wh = (double)c_w[n] * (qb - (double)z[n]);
+                        sum += xh * wh;
+                    }
+                }
+            }
+            y[p * Cout + n] = sum + (bias ? (double)bias[n] : 0.0);
+        }
+    }
+}

@@ -446,6 +446,57 @@ def test_conv_interior_pixel_is_full_im2col_row(oracle):
     assert np.array_equal(rs[h * W + w], oracle.row_sums(s_w, 5))
 
 
+def test_conv_zp_definition_matches_torch_conv2d(oracle):
+    # asymmetric weights in a 3x3 conv: the fp64 definition equals torch's conv2d on
+    # dequantized operands (padding zero in the real domain), and the code-domain
+    # four-term epilogue with windowed code sums reproduces it
+    torch = pytest.importorskip("torch")
+    B, H, W, Cin, Cout = 2, 5, 6, 8, 7
+    x = workloads.normal((B, H, W, Cin), seed=61)
+    w = workloads.normal((Cout, 9 * Cin), seed=62, std=0.05)
+    w[::2] += 0.05
+    bias = workloads.normal((Cout,), seed=63, std=0.02)
+    wq = oracle.quant_weight(w, 8, oracle.ASYM)
+    s_x, alpha, zc = oracle.quant_act(x.reshape(1, -1), 8, 1, 0)
+    s_x = s_x.reshape(B, H, W, Cin)
+    sxw, kv = oracle.conv3x3_code_sums(s_x)
+    for b in (8, 4, 2):
+        y64 = oracle.conv3x3_zp_def_f64(s_x, alpha[0], zc[0], wq["s"], wq["c"], wq["z"], bias, b)
+        xh = torch.tensor(alpha[0], dtype=torch.float64) * (torch.tensor(s_x, dtype=torch.float64) + float(zc[0]))
+        qb = torch.tensor(oracle.mask(wq["s"], b), dtype=torch.float64) + 128.0
+        wh = torch.tensor(wq["c"], dtype=torch.float64)[:, None] * (qb - torch.tensor(wq["z"], dtype=torch.float64)[:, None])
+        wh = wh.reshape(Cout, 3, 3, Cin).permute(0, 3, 1, 2)
+        ref = torch.nn.functional.conv2d(xh.permute(0, 3, 1, 2), wh, torch.tensor(bias, dtype=torch.float64), padding=1)
+        ref = ref.permute(0, 2, 3, 1).reshape(-1, Cout).numpy()
+        np.testing.assert_allclose(y64, ref, rtol=1e-12, atol=1e-12)
+        acc, rs = oracle.conv3x3(s_x, wq["s"], b)
+        y32, _ = oracle.conv_epilogue_zp_f32(acc, alpha[0], zc[0], sxw, kv, rs, wq["c"], wq["zcw"], bias)
+        np.testing.assert_allclose(y32, y64, rtol=1e-5, atol=1e-5)
+
+
+def test_conv_code_sums_interior_and_corner(oracle):
+    B, H, W, Cin = 1, 4, 5, 16
+    s_x = workloads.uniform_codes((B, H, W, Cin), seed=64, lo=-128, hi=127)
+    sxw, kv = oracle.conv3x3_code_sums(s_x)
+    px = s_x.astype(np.int64).sum(3)[0]  # per-pixel sums [H, W]
+    assert sxw[2 * W + 2] == px[1:4, 1:4].sum() and kv[2 * W + 2] == 9 * Cin  # interior
+    assert sxw[0] == px[0:2, 0:2].sum() and kv[0] == 4 * Cin                  # corner
+    assert sxw[W - 2] == px[0:2, W - 3:W].sum() and kv[W - 2] == 6 * Cin      # top edge
+
+
+def test_conv_epilogue_zp_with_zero_offsets_is_the_symmetric_epilogue(oracle):
+    B, H, W, Cin, Cout = 1, 3, 4, 16, 8
+    s_x = workloads.uniform_codes((B, H, W, Cin), seed=65, lo=-128, hi=127)
+    wq = oracle.quant_weight(workloads.normal((Cout, 9 * Cin), seed=66, std=0.02), 8, 0)
+    acc, rs = oracle.conv3x3(s_x, wq["s"], 6)
+    sxw, kv = oracle.conv3x3_code_sums(s_x)
+    alpha, zc = np.float32(0.01), np.float32(0.5)
+    y0, _ = oracle.epilogue_f32(acc, np.array([alpha]), np.array([zc]), rs, wq["c"], None, per_tensor=True,
+                                rs_per_row=True)
+    y1, _ = oracle.conv_epilogue_zp_f32(acc, alpha, zc, sxw, kv, rs, wq["c"], wq["zcw"], None)
+    assert np.array_equal(y0.view(np.uint32), y1.view(np.uint32))
+
+
 # --------------------------------------------------------------- schedule --
 
 def _golden_rows(name):
