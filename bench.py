@@ -384,7 +384,7 @@ def run_zero_point(torch, tasq, workloads, shapes=((4096, 1152, 1152), (4096, 34
         tasq.tasq_quant_weights(ctx, w, tasq.TASQ_F32, N, K, sw, cw)
         tasq.tasq_pack_weights(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K, 0, pk_sym)
         tasq.tasq_quant_weights_asym(ctx, w, tasq.TASQ_F32, N, K, sw, cw, zcw)
-        tasq.tasq_pack_weights_zp(ctx, sw, cw, zcw, None, N, K, pk_zp)
+        tasq.tasq_pack_weights_zp(ctx, tasq.TASQ_LINEAR, sw, cw, zcw, None, N, K, 0, pk_zp)
         codes = torch.empty((M, K), dtype=torch.float16, device="cuda")
         al = torch.empty((M,), device="cuda")
         zc = torch.empty((M,), device="cuda")
@@ -392,8 +392,8 @@ def run_zero_point(torch, tasq, workloads, shapes=((4096, 1152, 1152), (4096, 34
         y = torch.empty((M, N), dtype=torch.int16, device="cuda")
         q_sym = graph_us(lambda: tasq.tasq_quant_act(ctx, x, tasq.TASQ_BF16, M, K, 8, tasq.TASQ_SYMRANGE,
                                                      tasq.TASQ_PER_TOKEN, codes, tasq.TASQ_CODES_F16, al, zc))
-        q_zp = graph_us(lambda: tasq.tasq_quant_act_sums(ctx, x, tasq.TASQ_BF16, M, K, 8, tasq.TASQ_SYMRANGE, codes,
-                                                         tasq.TASQ_CODES_F16, al, zc, sums))
+        q_zp = graph_us(lambda: tasq.tasq_quant_act_sums(ctx, x, tasq.TASQ_BF16, M, K, 8, tasq.TASQ_SYMRANGE,
+                                                         tasq.TASQ_PER_TOKEN, codes, tasq.TASQ_CODES_F16, al, zc, sums))
         g_sym = graph_us(lambda: tasq.tasq_masked_gemm(ctx, 0, stage, codes, tasq.TASQ_CODES_F16, al, zc, M, pk_sym,
                                                        N, K, y))
         g_zp = graph_us(lambda: tasq.tasq_masked_gemm_zp(ctx, 0, stage, codes, tasq.TASQ_CODES_F16, al, zc, sums, M,

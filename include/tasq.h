@@ -201,15 +201,16 @@ int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d
                       int K, int Cin, void* d_packed, tasq_stream stream);
 
 /*
- * tasq_pack_weights for a linear layer quantized with a weight zero point
- * (tasq_quant_weights_asym): also stores zcw [N] and marks the buffer, so
- * that the contraction must be given the activations' code sums
- * (tasq_masked_gemm_zp).  tasq_masked_gemm on such a buffer records
- * TASQ_ERR_DEVICE and writes nothing.  Same buffer size (tasq_packed_bytes
- * with TASQ_LINEAR).  Enqueue call.
+ * tasq_pack_weights for a layer quantized with a weight zero point
+ * (tasq_quant_weights_asym; a conv's weights as rows [Cout][9*Cin]): also
+ * stores zcw [N] and marks the buffer, so that the contraction must be given
+ * the activations' code sums (tasq_masked_gemm_zp, tasq_masked_conv3x3_zp).
+ * tasq_masked_gemm / tasq_masked_conv3x3 on such a buffer record
+ * TASQ_ERR_DEVICE and write nothing.  Same buffer size (tasq_packed_bytes).
+ * Other arguments as tasq_pack_weights.  Enqueue call.
  */
-int tasq_pack_weights_zp(tasq_ctx ctx, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
-                         const float* d_bias, int N, int K, void* d_packed, tasq_stream stream);
+int tasq_pack_weights_zp(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
+                         const float* d_bias, int N, int K, int Cin, void* d_packed, tasq_stream stream);
 
 /*
  * Bit-allocation map (App. F.1): h_bits [L][S] uint8, each value in 2..8,
@@ -249,11 +250,13 @@ int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n
                    void* d_codes, int code_fmt, float* d_alpha, float* d_zc, tasq_stream stream);
 
 /*
- * tasq_quant_act per token, also writing d_code_sums [M] int32, the sum over
- * k of the stored codes s[m][k] (exact).  The four-term epilogue of
- * asymmetric weights needs it (tasq_masked_gemm_zp).  Enqueue call.
+ * tasq_quant_act that also writes d_code_sums [M] int32, the sum over k of
+ * the stored codes s[m][k] of each row of d_x (exact; per tensor the rows are
+ * still summed one by one: for NHWC activations, one sum per pixel).  The
+ * four-term epilogue of asymmetric weights needs it (tasq_masked_gemm_zp,
+ * tasq_masked_conv3x3_zp).  Enqueue call (per tensor: one more kernel).
  */
-int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode,
+int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode, int gran,
                         void* d_codes, int code_fmt, float* d_alpha, float* d_zc, int32_t* d_code_sums,
                         tasq_stream stream);
 
@@ -308,6 +311,25 @@ int tasq_masked_gemm_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes,
 int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt, const float* d_alpha,
                         const float* d_zc, int B, int H, int W, int Cin, const void* d_packed, int Cout, uint16_t* d_y,
                         int32_t* d_acc, tasq_stream stream);
+
+/*
+ * Masked 3x3 convolution with asymmetric weights.  Padding is zero in the
+ * real domain, so for output pixel p only its in-bounds taps carry zero-point
+ * terms:
+ *   y = alpha * c_w * (acc + zc * rs_b[p] + zcw * t[p]) + bias,
+ *   t[p] = sxw[p] + Kv[p] * zc,
+ * sxw[p] = sum of d_code_sums over the in-bounds taps' input pixels,
+ * Kv[p] = Cin * (number of in-bounds taps), rs_b[p] as in tasq_masked_conv3x3.
+ * fp32 order: t = sxw + (Kv * zc), u = fma(zc, rs_b, acc), u = fma(zcw, t, u),
+ * y = bf16(fma(u, alpha * c_w, bias)).  d_code_sums: [B*H*W] per-pixel code
+ * sums from tasq_quant_act_sums with TASQ_PER_TENSOR.  d_packed: from
+ * tasq_pack_weights_zp with kind TASQ_CONV3X3.  Other arguments as
+ * tasq_masked_conv3x3.  Enqueue call.
+ */
+int tasq_masked_conv3x3_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
+                           const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int B, int H, int W,
+                           int Cin, const void* d_packed, int Cout, uint16_t* d_y, int32_t* d_acc,
+                           tasq_stream stream);
 
 /*
  * Per-tensor activation quantization without any allocation (no context).

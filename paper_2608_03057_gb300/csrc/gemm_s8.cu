@@ -40,7 +40,7 @@ __device__ inline void mma_s8(int (&d)[4], const uint32_t (&a)[4], uint32_t b0, 
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-// ZP: the four-term epilogue of asymmetric weights (linear layers only)
+// ZP: the four-term epilogue of asymmetric weights
 template <bool CONV, bool ZP>
 __global__ void __launch_bounds__(THREADS) gemm_s8_kernel(const GemmArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -160,8 +160,8 @@ __global__ void __launch_bounds__(THREADS) gemm_s8_kernel(const GemmArgs a) {
         const float cw0 = a.cw[n], cw1 = a.cw[n + 1];
         const float bi0 = a.bias[n], bi1 = a.bias[n + 1];
         const int rsl0 = CONV ? 0 : rs_b[n], rsl1 = CONV ? 0 : rs_b[n + 1];
-        // asymmetric weights (linear): zero offsets per channel, activation sums per token
-        constexpr bool zp = !CONV && ZP;
+        // asymmetric weights: zero offsets per channel, activation sums per token
+        constexpr bool zp = ZP;
         const float zw0 = zp ? a.zcw[n] : 0.f, zw1 = zp ? a.zcw[n + 1] : 0.f;
 #pragma unroll
         for (int mi = 0; mi < 4; ++mi)
@@ -180,7 +180,8 @@ __global__ void __launch_bounds__(THREADS) gemm_s8_kernel(const GemmArgs a) {
                 const int v0 = acc[mi][ni][2 * hh], v1 = acc[mi][ni][2 * hh + 1];
                 uint32_t y0, y1;
                 if constexpr (zp) {
-                    const float t = token_zero_sum(a.code_sums[m], a.K, z);
+                    const float t = CONV ? conv_token_zero_sum(a.code_sums, m, a.H, a.W, a.Cin, z)
+                                         : token_zero_sum(a.code_sums[m], a.K, z);
                     y0 = bf16_bits(epilogue_value_zp(v0, al, z, t, rs0, cw0, zw0, bi0));
                     y1 = bf16_bits(epilogue_value_zp(v1, al, z, t, rs1, cw1, zw1, bi1));
                 } else {
@@ -200,7 +201,8 @@ cudaError_t launch_gemm_s8(const GemmArgs& a, int /*num_sms*/, cudaStream_t st) 
     dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM);
     if (grid.y > 65535) return cudaErrorInvalidConfiguration;
     cudaError_t e;
-    auto kernel = a.Cin ? gemm_s8_kernel<true, false> : (a.code_sums ? gemm_s8_kernel<false, true> : gemm_s8_kernel<false, false>);
+    auto kernel = a.Cin ? (a.code_sums ? gemm_s8_kernel<true, true> : gemm_s8_kernel<true, false>)
+                        : (a.code_sums ? gemm_s8_kernel<false, true> : gemm_s8_kernel<false, false>);
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (e != cudaSuccess) return e;
     kernel<<<grid, THREADS, SMEM_BYTES, st>>>(a);

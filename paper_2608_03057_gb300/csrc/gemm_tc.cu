@@ -155,6 +155,7 @@ struct Smem {
     uint8_t w[W_STAGES][W_STAGE];
     float ep_al[C::EPI_SLOTS][C::GPW][32], ep_zc[C::EPI_SLOTS][C::GPW][32];  // per warp, per group, per column
     int ep_tok[C::EPI_SLOTS][C::GPW][32], ep_tap[C::EPI_SLOTS][C::GPW][32];
+    float ep_t[C::EPI_SLOTS][C::GPW][32];  // asymmetric weights: per-column activation sums t
     alignas(128) uint16_t ep_stage[C::EPI_SLOTS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
     uint64_t xfull[C::X_STAGES], done[C::DONE];
     uint64_t wfull[W_STAGES], wempty[W_STAGES];
@@ -271,7 +272,7 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
 
 // CONV selects the implicit-GEMM 3x3 convolution (one instantiation per
 // operand layout, so neither pays for the other's index arithmetic); ZP the
-// four-term epilogue of asymmetric weights (linear layers only).
+// four-term epilogue of asymmetric weights.
 template <bool CONV, bool ZP, class C>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
@@ -526,7 +527,7 @@ __global__ void __maxnreg__(96)
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
         const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
-        constexpr bool zp = !CONV && ZP;  // asymmetric weights: the four-term epilogue
+        constexpr bool zp = ZP;  // asymmetric weights: the four-term epilogue
         int cc = 0;
 #ifdef TASQ_TRACE
         int fcall = 0;
@@ -541,12 +542,14 @@ __global__ void __maxnreg__(96)
             // row sums as fp32: |sum| < 2^24, so the values and every partial sum
             // of in-bounds taps below are exact, equal to float(int sum)
             float cw = 0.f, bias = 0.f, rs = 0.f;
+            [[maybe_unused]] float zcw_l = 0.f;  // asymmetric weights: this lane's channel zero offset
             float ts[9];
 #pragma unroll
             for (int i = 0; i < 9; ++i) ts[i] = 0.f;
             if (n_ok) {
                 cw = a.cw[n];
                 bias = a.bias[n];
+                if constexpr (zp) zcw_l = a.zcw[n];
                 if constexpr (CONV) {
 #pragma unroll
                     for (int i = 0; i < 9; ++i) ts[i] = __int2float_rn(ts_b[int64_t(n) * 9 + i]);
@@ -598,9 +601,13 @@ __global__ void __maxnreg__(96)
                 if constexpr (CONV) {
                     if (jt >= BT) tok = -1;
                 }
-                if constexpr (!CONV) {
-                    // asymmetric weights: the token's activation sum t, kept in the tap slot
-                    if (zp && tok >= 0) tap = __float_as_int(token_zero_sum(a.code_sums[tok], a.K, a.zc[tok]));
+                if constexpr (zp) {
+                    // asymmetric weights: the column's activation sum t (conv: over in-bounds taps)
+                    float t = 0.f;
+                    if (tok >= 0)
+                        t = CONV ? conv_token_zero_sum(a.code_sums, tok, a.H, a.W, a.Cin, a.zc[0])
+                                 : token_zero_sum(a.code_sums[tok], a.K, a.zc[tok]);
+                    s->ep_t[e][gi][lane] = t;
                 }
                 s->ep_tok[e][gi][lane] = tok;
                 s->ep_tap[e][gi][lane] = tap;
@@ -630,6 +637,9 @@ __global__ void __maxnreg__(96)
                     int4 tp4 = make_int4(0, 0, 0, 0);
                     if constexpr (CONV) tp4 = *reinterpret_cast<const int4*>(my_tap + j0 + 4 * j4);
                     [[maybe_unused]] const int tp[4] = {tp4.x, tp4.y, tp4.z, tp4.w};
+                    float4 t4 = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if constexpr (zp) t4 = *reinterpret_cast<const float4*>(s->ep_t[e][gi] + j0 + 4 * j4);
+                    [[maybe_unused]] const float tz[4] = {t4.x, t4.y, t4.z, t4.w};
                     float yf[4];
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
@@ -643,7 +653,9 @@ __global__ void __maxnreg__(96)
                         float acc_f;
                         if constexpr (fl) acc_f = __uint_as_float(raw);
                         else acc_f = __int2float_rn(int(raw));
-                        yf[u] = __fmaf_rn(__fmaf_rn(zc[u], rsum, acc_f), __fmul_rn(al[u], cw), bias);
+                        float uu = __fmaf_rn(zc[u], rsum, acc_f);
+                        if constexpr (zp) uu = __fmaf_rn(zcw_l, tz[u], uu);  // asymmetric weights
+                        yf[u] = __fmaf_rn(uu, __fmul_rn(al[u], cw), bias);
                     }
                     // two results per round-to-nearest-even conversion
 #pragma unroll
@@ -717,8 +729,8 @@ __global__ void __maxnreg__(96)
                 const float alv[4] = {al0.x, al0.y, al1.x, al1.y}, zcv[4] = {zc0.x, zc0.y, zc1.x, zc1.y};
                 [[maybe_unused]] float tv[4] = {0.f, 0.f, 0.f, 0.f};  // asymmetric weights: token sums
                 if constexpr (zp) {
-                    const float2 t0 = *reinterpret_cast<const float2*>(s->ep_tap[e][gi] + j0 + 2 * s4);
-                    const float2 t1 = *reinterpret_cast<const float2*>(s->ep_tap[e][gi] + j0 + 8 + 2 * s4);
+                    const float2 t0 = *reinterpret_cast<const float2*>(s->ep_t[e][gi] + j0 + 2 * s4);
+                    const float2 t1 = *reinterpret_cast<const float2*>(s->ep_t[e][gi] + j0 + 8 + 2 * s4);
                     tv[0] = t0.x, tv[1] = t0.y, tv[2] = t1.x, tv[3] = t1.y;
                 }
                 uint32_t pk[4][2];  // [channel k][token pair tp]
@@ -898,8 +910,10 @@ __global__ void __launch_bounds__(256) splitk_epilogue_kernel(const GemmArgs a, 
         }
         const float al = a.per_tensor ? a.alpha[0] : a.alpha[m];
         const float zc = a.per_tensor ? a.zc[0] : a.zc[m];
-        const bool zp = !a.Cin && a.code_sums;  // asymmetric weights (linear)
-        const float t = zp ? token_zero_sum(a.code_sums[m], a.K, zc) : 0.f;
+        const bool zp = a.code_sums != nullptr;  // asymmetric weights
+        const float t = !zp ? 0.f
+                            : a.Cin ? conv_token_zero_sum(a.code_sums, m, a.H, a.W, a.Cin, zc)
+                                    : token_zero_sum(a.code_sums[m], a.K, zc);
         int tap = 0x1FF;
         if (a.Cin) {
             const int ww = m % a.W, hh = (m / a.W) % a.H;
@@ -1092,7 +1106,7 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
         fprintf(stderr, "tasq tc: M=%d N=%d K=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, (long long)tiles,
                 p.splits, units);
     const int smem = smem_bytes<C>();
-    auto kernel = p.conv ? gemm_tc_kernel<true, false, C>
+    auto kernel = p.conv ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
                          : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;

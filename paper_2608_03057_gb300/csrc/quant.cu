@@ -472,6 +472,31 @@ __global__ void __launch_bounds__(256) quant_act_tensor_kernel(const void* __res
     }
 }
 
+// --------------------------------------------------------- code row sums --
+// One warp per row of codes [M][K] (K % 16 == 0): sums[m] = sum_k codes[m][k].
+__global__ void __launch_bounds__(256) code_row_sums_kernel(const void* __restrict__ codes, int code_fmt, int M, int K,
+                                                            int32_t* __restrict__ sums) {
+    const int lane = threadIdx.x & 31;
+    const int m = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (m >= M) return;
+    int s = 0;
+    if (code_fmt == TASQ_CODES_S8) {
+        const char4* row = reinterpret_cast<const char4*>(codes) + int64_t(m) * (K / 4);
+        for (int i = lane; i < K / 4; i += 32) {
+            const char4 v = row[i];
+            s += v.x + v.y + v.z + v.w;
+        }
+    } else {
+        const __half2* row = reinterpret_cast<const __half2*>(codes) + int64_t(m) * (K / 2);
+        for (int i = lane; i < K / 2; i += 32) {
+            const float2 v = __half22float2(row[i]);
+            s += int(v.x) + int(v.y);
+        }
+    }
+    s = warp_sum(s);
+    if (lane == 0) sums[m] = s;
+}
+
 // -------------------------------------------------------------------- pack --
 __global__ void pack_header_kernel(int kind, int N, int K, int has_zp, PackedHeader* hdr) {
     PackedHeader h = packed_layout(kind, N, K);
@@ -647,6 +672,12 @@ cudaError_t launch_quant_act_tensor(const void* x, int dtype, int64_t count, int
     if (e != cudaSuccess) return e;
     quant_act_tensor_kernel<<<grid, 256, 0, st>>>(x, dtype, groups, n_bits, mode, codes, code_fmt, alpha, zc,
                                                   scratch);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_code_row_sums(const void* codes, int code_fmt, int M, int K, int32_t* sums, cudaStream_t st) {
+    if (M == 0) return cudaSuccess;
+    code_row_sums_kernel<<<(M + kRowWarps - 1) / kRowWarps, 256, 0, st>>>(codes, code_fmt, M, K, sums);
     return cudaGetLastError();
 }
 

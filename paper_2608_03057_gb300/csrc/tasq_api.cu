@@ -217,7 +217,6 @@ namespace {
 int pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
                  const float* d_bias, int N, int K, int Cin, void* d_packed, tasq_stream stream) {
     REQUIRE(kind == TASQ_LINEAR || kind == TASQ_CONV3X3, TASQ_ERR_INVALID_ARG, "kind %d", kind);
-    REQUIRE(!d_zcw || kind == TASQ_LINEAR, TASQ_ERR_UNSUPPORTED, "weight zero offsets: linear layers only");
     REQUIRE(N > 0 && K > 0, TASQ_ERR_INVALID_ARG, "N=%d K=%d", N, K);
     REQUIRE(K % 16 == 0 && N % 8 == 0, TASQ_ERR_UNSUPPORTED, "need K %% 16 == 0 and N %% 8 == 0 (N=%d K=%d)", N, K);
     if (kind == TASQ_CONV3X3) {
@@ -241,11 +240,11 @@ TASQ_API int tasq_pack_weights(tasq_ctx ctx, int kind, const int8_t* d_sw, const
     return pack_weights(ctx, kind, d_sw, d_cw, nullptr, d_bias, N, K, Cin, d_packed, stream);
 }
 
-TASQ_API int tasq_pack_weights_zp(tasq_ctx ctx, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
-                                  const float* d_bias, int N, int K, void* d_packed, tasq_stream stream) {
+TASQ_API int tasq_pack_weights_zp(tasq_ctx ctx, int kind, const int8_t* d_sw, const float* d_cw, const float* d_zcw,
+                                  const float* d_bias, int N, int K, int Cin, void* d_packed, tasq_stream stream) {
     CHECK_CTX(ctx);
     REQUIRE(d_zcw, TASQ_ERR_INVALID_ARG, "NULL pointer");
-    return pack_weights(ctx, TASQ_LINEAR, d_sw, d_cw, d_zcw, d_bias, N, K, 0, d_packed, stream);
+    return pack_weights(ctx, kind, d_sw, d_cw, d_zcw, d_bias, N, K, Cin, d_packed, stream);
 }
 
 TASQ_API int tasq_set_schedule(tasq_ctx ctx, const uint8_t* h_bits, int L, int S) {
@@ -302,6 +301,12 @@ int quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits
                                           reinterpret_cast<unsigned int*>(ctx->d_words + 16), (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "quant_act launch");
     ctx->kernels += gran == TASQ_PER_TOKEN ? 1 : 2;
+    if (gran == TASQ_PER_TENSOR && d_code_sums) {
+        // per-row code sums of a per-tensor quantization (conv: one row per pixel)
+        e = tasq::launch_code_row_sums(d_codes, code_fmt, M, K, d_code_sums, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "code sums launch");
+        ctx->kernels += 1;
+    }
     return TASQ_OK;
 }
 
@@ -314,12 +319,11 @@ TASQ_API int tasq_quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int
 }
 
 TASQ_API int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits, int mode,
-                                 void* d_codes, int code_fmt, float* d_alpha, float* d_zc, int32_t* d_code_sums,
-                                 tasq_stream stream) {
+                                 int gran, void* d_codes, int code_fmt, float* d_alpha, float* d_zc,
+                                 int32_t* d_code_sums, tasq_stream stream) {
     CHECK_CTX(ctx);
     REQUIRE(M == 0 || d_code_sums, TASQ_ERR_INVALID_ARG, "NULL pointer");
-    return quant_act(ctx, d_x, dtype, M, K, n_bits, mode, TASQ_PER_TOKEN, d_codes, code_fmt, d_alpha, d_zc,
-                     d_code_sums, stream);
+    return quant_act(ctx, d_x, dtype, M, K, n_bits, mode, gran, d_codes, code_fmt, d_alpha, d_zc, d_code_sums, stream);
 }
 
 namespace {
@@ -423,4 +427,17 @@ TASQ_API int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void*
     REQUIRE((int64_t)B * H * W <= 0x7FFFFFFF && (int64_t)9 * Cin <= 0x7FFFFFFF, TASQ_ERR_UNSUPPORTED, "too large");
     return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, B * H * W,
                               d_packed, Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
+}
+
+TASQ_API int tasq_masked_conv3x3_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
+                                    const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int B, int H,
+                                    int W, int Cin, const void* d_packed, int Cout, uint16_t* d_y, int32_t* d_acc,
+                                    tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(B >= 0 && H > 0 && W > 0 && Cin > 0, TASQ_ERR_INVALID_ARG, "B=%d H=%d W=%d Cin=%d", B, H, W, Cin);
+    REQUIRE(Cin % 16 == 0, TASQ_ERR_UNSUPPORTED, "conv: Cin=%d must be a multiple of 16", Cin);
+    REQUIRE((int64_t)B * H * W <= 0x7FFFFFFF && (int64_t)9 * Cin <= 0x7FFFFFFF, TASQ_ERR_UNSUPPORTED, "too large");
+    REQUIRE(B == 0 || d_code_sums, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, d_code_sums,
+                              B * H * W, d_packed, Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
 }

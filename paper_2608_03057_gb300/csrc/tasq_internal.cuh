@@ -89,7 +89,7 @@ struct GemmArgs {
     // weight_dequant with a real zero point): w_hat = c_w * (mask_b(s_w) + zcw).
     // With code_sums set the epilogue adds zcw[n] * t[m], t = sum_k (s_x + zc).
     const float* zcw;          // [N] from the packed buffer (zeros for a symmetric pack)
-    const int32_t* code_sums;  // [M] sum_k s_x[m][k], or NULL (two-term epilogue)
+    const int32_t* code_sums;  // [M] sum_k s_x[m][k] (conv: per input pixel), or NULL (two-term epilogue)
 };
 
 // Resolves b for this launch on the device; returns 0 (and records an error)
@@ -158,6 +158,29 @@ __device__ inline uint16_t bf16_bits(float f) {
     return (uint16_t)(u >> 16);
 }
 
+// 3x3 conv with asymmetric weights: for output pixel p, t = RN(float(sxw) +
+// RN(float(Kv) * zc)) with sxw the sum of the per-pixel code sums over its
+// in-bounds taps and Kv = Cin x (in-bounds taps) (padding is zero in the real
+// domain, so a padded tap carries no zero-point term).
+__device__ inline float conv_token_zero_sum(const int32_t* code_sums, int p, int H, int W, int Cin, float zc) {
+    const int w = p % W, h = (p / W) % H;
+    const int base = p - (h * W + w);  // first pixel of the image
+    int sum = 0, taps = 0;
+#pragma unroll
+    for (int dh = -1; dh <= 1; ++dh) {
+        const int ih = h + dh;
+        if (ih < 0 || ih >= H) continue;
+#pragma unroll
+        for (int dw = -1; dw <= 1; ++dw) {
+            const int iw = w + dw;
+            if (iw < 0 || iw >= W) continue;
+            sum += code_sums[base + ih * W + iw];
+            ++taps;
+        }
+    }
+    return __fadd_rn(__int2float_rn(sum), __fmul_rn(__int2float_rn(taps * Cin), zc));
+}
+
 // Sum of the in-bounds taps' per-tap weight sums for output pixel (h, w).
 __device__ inline int conv_row_sum(const int32_t* ts_n, int h, int w, int H, int W) {
     int s = 0;
@@ -186,7 +209,9 @@ cudaError_t launch_quant_act_token(const void* x, int dtype, int M, int K, int n
                                    int code_fmt, float* alpha, float* zc, int32_t* code_sums, cudaStream_t st);
 cudaError_t launch_quant_act_tensor(const void* x, int dtype, int64_t count, int n_bits, int mode, void* codes,
                                     int code_fmt, float* alpha, float* zc, unsigned int* scratch, cudaStream_t st);
-// zcw: [N] weight zero offsets (linear only), or NULL for a symmetric pack
+// sums[m] = sum_k codes[m][k] (int8 or fp16 codes, [M][K])
+cudaError_t launch_code_row_sums(const void* codes, int code_fmt, int M, int K, int32_t* sums, cudaStream_t st);
+// zcw: [N] weight zero offsets, or NULL for a symmetric pack
 cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* zcw, const float* bias, int N, int K,
                         int Cin, void* packed, cudaStream_t st);
 cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);

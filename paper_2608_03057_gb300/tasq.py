@@ -63,14 +63,15 @@ def lib():
                 "tasq_quant_weights_asym": ([P, P, I, I, I, P, P, P, P, P], I),
                 "tasq_packed_bytes": ([I, I, I], SZ),
                 "tasq_pack_weights": ([P, I, P, P, P, I, I, I, P, P], I),
-                "tasq_pack_weights_zp": ([P, P, P, P, P, I, I, P, P], I),
+                "tasq_pack_weights_zp": ([P, I, P, P, P, P, I, I, I, P, P], I),
                 "tasq_set_schedule": ([P, P, I, I], I),
                 "tasq_set_stage_device": ([P, P], I),
                 "tasq_quant_act": ([P, P, I, I, I, I, I, I, P, I, P, P, P], I),
-                "tasq_quant_act_sums": ([P, P, I, I, I, I, I, P, I, P, P, P, P], I),
+                "tasq_quant_act_sums": ([P, P, I, I, I, I, I, I, P, I, P, P, P, P], I),
                 "tasq_masked_gemm": ([P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_gemm_zp": ([P, I, I, P, I, P, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_conv3x3": ([P, I, I, P, I, P, P, I, I, I, I, P, I, P, P, P], I),
+                "tasq_masked_conv3x3_zp": ([P, I, I, P, I, P, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_quant_act_tensor_noalloc": ([P, I, I, I, I, I, P, I, P, P, P], I),
             }
             for name, (args, res) in sigs.items():
@@ -176,9 +177,9 @@ def tasq_pack_weights(ctx, kind, sw, cw, bias, N, K, Cin, packed, stream=None) -
                                         _ptr(packed), _stream(stream)))
 
 
-def tasq_pack_weights_zp(ctx, sw, cw, zcw, bias, N, K, packed, stream=None) -> None:
-    _check(ctx, lib().tasq_pack_weights_zp(ctx, _ptr(sw), _ptr(cw), _ptr(zcw), _ptr(bias), int(N), int(K),
-                                           _ptr(packed), _stream(stream)))
+def tasq_pack_weights_zp(ctx, kind, sw, cw, zcw, bias, N, K, Cin, packed, stream=None) -> None:
+    _check(ctx, lib().tasq_pack_weights_zp(ctx, int(kind), _ptr(sw), _ptr(cw), _ptr(zcw), _ptr(bias), int(N), int(K),
+                                           int(Cin), _ptr(packed), _stream(stream)))
 
 
 def tasq_set_schedule(ctx, h_bits, L, S) -> None:
@@ -195,9 +196,11 @@ def tasq_quant_act(ctx, x, dtype, M, K, n_bits, mode, gran, codes, code_fmt, alp
                                      _ptr(codes), int(code_fmt), _ptr(alpha), _ptr(zc), _stream(stream)))
 
 
-def tasq_quant_act_sums(ctx, x, dtype, M, K, n_bits, mode, codes, code_fmt, alpha, zc, code_sums, stream=None) -> None:
-    _check(ctx, lib().tasq_quant_act_sums(ctx, _ptr(x), int(dtype), int(M), int(K), int(n_bits), int(mode), _ptr(codes),
-                                          int(code_fmt), _ptr(alpha), _ptr(zc), _ptr(code_sums), _stream(stream)))
+def tasq_quant_act_sums(ctx, x, dtype, M, K, n_bits, mode, gran, codes, code_fmt, alpha, zc, code_sums,
+                        stream=None) -> None:
+    _check(ctx, lib().tasq_quant_act_sums(ctx, _ptr(x), int(dtype), int(M), int(K), int(n_bits), int(mode), int(gran),
+                                          _ptr(codes), int(code_fmt), _ptr(alpha), _ptr(zc), _ptr(code_sums),
+                                          _stream(stream)))
 
 
 def tasq_masked_gemm_zp(ctx, layer, stage, codes, code_fmt, alpha, zc, code_sums, M, packed, N, K, y, acc=None,
@@ -217,6 +220,13 @@ def tasq_masked_conv3x3(ctx, layer, stage, codes, code_fmt, alpha, zc, B, H, W, 
     _check(ctx, lib().tasq_masked_conv3x3(ctx, int(layer), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
                                           _ptr(zc), int(B), int(H), int(W), int(Cin), _ptr(packed), int(Cout), _ptr(y),
                                           _ptr(acc), _stream(stream)))
+
+
+def tasq_masked_conv3x3_zp(ctx, layer, stage, codes, code_fmt, alpha, zc, code_sums, B, H, W, Cin, packed, Cout, y,
+                           acc=None, stream=None) -> None:
+    _check(ctx, lib().tasq_masked_conv3x3_zp(ctx, int(layer), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
+                                             _ptr(zc), _ptr(code_sums), int(B), int(H), int(W), int(Cin), _ptr(packed),
+                                             int(Cout), _ptr(y), _ptr(acc), _stream(stream)))
 
 
 def tasq_quant_act_tensor_noalloc(x, dtype, M, K, n_bits, mode, codes, code_fmt, alpha, zc, stream=None) -> None:

@@ -59,20 +59,22 @@ def quant_weights_asym(ctx, w_dev, dtype, N, K):
     return sw, cw, zcw, al
 
 
-def pack_zp(ctx, sw, cw, zcw, bias, N, K):
+def pack_zp(ctx, sw, cw, zcw, bias, N, K, kind=tasq.TASQ_LINEAR, Cin=0):
     t = torch()
-    packed = empty((tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, N, K),), t.uint8)
-    tasq.tasq_pack_weights_zp(ctx.h, sw, cw, zcw, bias, N, K, packed)
+    packed = empty((tasq.tasq_packed_bytes(kind, N, K),), t.uint8)
+    tasq.tasq_pack_weights_zp(ctx.h, kind, sw, cw, zcw, bias, N, K, Cin, packed)
     return packed
 
 
-def quant_act_sums(ctx, x_dev, dtype, M, K, n_bits=8, mode=tasq.TASQ_SYMRANGE, code_fmt=tasq.TASQ_CODES_S8):
+def quant_act_sums(ctx, x_dev, dtype, M, K, n_bits=8, mode=tasq.TASQ_SYMRANGE, code_fmt=tasq.TASQ_CODES_S8,
+                   gran=tasq.TASQ_PER_TOKEN):
     t = torch()
     codes = empty((M, K), t.int8 if code_fmt == tasq.TASQ_CODES_S8 else t.float16)
-    alpha = empty((max(M, 1),), t.float32)
-    zc = empty((max(M, 1),), t.float32)
+    g = 1 if gran == tasq.TASQ_PER_TENSOR else M
+    alpha = empty((max(g, 1),), t.float32)
+    zc = empty((max(g, 1),), t.float32)
     sums = empty((max(M, 1),), t.int32)
-    tasq.tasq_quant_act_sums(ctx.h, x_dev, dtype, M, K, n_bits, mode, codes, code_fmt, alpha, zc, sums)
+    tasq.tasq_quant_act_sums(ctx.h, x_dev, dtype, M, K, n_bits, mode, gran, codes, code_fmt, alpha, zc, sums)
     return codes, alpha, zc, sums
 
 

@@ -523,6 +523,59 @@ def _run_conv(ctx, oracle, B, H, W, Cin, Cout, bits, code_fmt, seed=0, rows=None
         assert same == yb.size
 
 
+def _run_conv_zp(ctx, oracle, B, H, W, Cin, Cout, bits, code_fmt, seed=0, rows=None):
+    """3x3 conv with asymmetric weights (zero offsets) and per-pixel code sums."""
+    K = 9 * Cin
+    x = workloads.normal((B, H, W, Cin), seed)
+    w = workloads.normal((Cout, K), seed + 1, 0.02)
+    w[::2] += 0.02
+    bias = workloads.normal((Cout,), seed + 2, 0.02)
+    sw, cw, zcw, _ = G.quant_weights_asym(ctx, G.dev(w), tasq.TASQ_F32, Cout, K)
+    packed = G.pack_zp(ctx, sw, cw, zcw, G.dev(bias), Cout, K, kind=tasq.TASQ_CONV3X3, Cin=Cin)
+    tasq.tasq_set_schedule(ctx.h, np.asarray([bits], np.uint8), 1, len(bits))
+    codes, alpha, zc, sums = G.quant_act_sums(ctx, G.dev(x), tasq.TASQ_F32, B * H * W, Cin, 8, tasq.TASQ_ASYM,
+                                              code_fmt, gran=tasq.TASQ_PER_TENSOR)
+    wq = oracle.quant_weight(w, 8, oracle.ASYM)
+    s_x, a, z = oracle.quant_act(x.reshape(1, -1), 8, oracle.ASYM, 0)
+    s_x = s_x.reshape(B, H, W, Cin)
+    assert np.array_equal(G.codes_to_int8(codes).reshape(B, H, W, Cin), s_x)
+    assert np.array_equal(sums.cpu().numpy(), s_x.astype(np.int64).sum(3).reshape(-1))
+    sxw, kv = oracle.conv3x3_code_sums(s_x)
+    for stage, b in enumerate(bits):
+        y = G.empty((B * H * W, Cout), G.torch().int16)
+        acc = G.empty((B * H * W, Cout), G.torch().int32)
+        tasq.tasq_masked_conv3x3_zp(ctx.h, 0, stage, codes, code_fmt, alpha, zc, sums, B, H, W, Cin, packed, Cout,
+                                    y, acc)
+        if rows is None:
+            ref_acc, rs = oracle.conv3x3(s_x, wq["s"], b)
+            got_acc, got_y, sx_r, kv_r = acc.cpu().numpy(), G.bf16_bits_host(y), sxw, kv
+        else:
+            ref_acc, rs = _conv_rows(oracle, s_x, wq["s"], b, rows)
+            got_acc, got_y, sx_r, kv_r = acc.cpu().numpy()[rows], G.bf16_bits_host(y)[rows], sxw[rows], kv[rows]
+        assert np.array_equal(got_acc, ref_acc), f"b={b}: {(got_acc != ref_acc).sum()} int32 mismatches"
+        _, yb = oracle.conv_epilogue_zp_f32(ref_acc, a[0], z[0], sx_r, kv_r, rs, wq["c"], wq["zcw"], bias)
+        same = G.assert_bf16_close(got_y, yb)
+        assert same == yb.size, f"b={b}: {yb.size - same} bf16 outputs differ in the last bit"
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("B,H,W,Cin,Cout", [(1, 8, 8, 64, 16), (2, 5, 7, 64, 24), (1, 1, 1, 128, 8),
+                                            (2, 16, 16, 64, 256), (1, 4, 4, 1280, 128)])
+def test_conv_zp_small_full(ctx, oracle, code_fmt, B, H, W, Cin, Cout):
+    """Asymmetric-weight convs checked in full: borders and corners (windowed code
+    sums over in-bounds taps only), a 1x1 image, several tile configurations and a
+    long K (9 * 1280, split K)."""
+    _run_conv_zp(ctx, oracle, B, H, W, Cin, Cout, [8, 5, 2], code_fmt, seed=B * 7 + H)
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_conv_zp_full_size_sampled(ctx, oracle, code_fmt):
+    B, C, HW = 1, 320, 64
+    P = B * HW * HW
+    rows = np.unique(np.concatenate([np.arange(0, P, 97), [0, HW - 1, P - HW, P - 1]]))
+    _run_conv_zp(ctx, oracle, B, HW, HW, C, C, [4, 8], code_fmt, seed=5, rows=rows)
+
+
 def _conv_rows(oracle, s_x, s_w, b, rows):
     """Oracle conv restricted to output pixels `rows`: each pixel's 3x3
     neighbourhood is cut out (zero code padding outside the image) and run
