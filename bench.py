@@ -447,8 +447,7 @@ def oracle_sample(workload: str, budget_s: float, rows: int = 32, seed: int = 0,
 
 
 def run_reference(args):
-    rank = int(os.environ.get("RANK", "0"))
-    if rank != 0:
+    if dist_env()[1] != 0:  # under torchrun only rank 0 times the oracle
         return 0
     # warm-up samples, then K timed samples of one layer-row block each
     per_step = max(0.5, min(5.0, 60.0 / max(1, args.steps + args.warmup)))
@@ -478,6 +477,28 @@ def run_reference(args):
     return 0
 
 
+# ------------------------------------------------- replicas over N GPUs --
+def dist_env():
+    """(world, rank, local_rank) from the launcher's environment (1, 0, 0 alone)."""
+    return (int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(torch, dist, value: float, device) -> float:
+    """The largest of every rank's `value` (each rank calls it; no-op alone)."""
+    if dist is None:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tops(ops_per_rank: float, world: int, ms: float) -> float:
+    """Whole-job throughput: every rank runs an independent replica of the step
+    (weak scaling), so the job does world x the ops in the slowest rank's time."""
+    return world * ops_per_rank / (ms * 1e-3) / 1e12
+
+
 # ------------------------------------------------------------------- main --
 def main():
     args = parse_args()
@@ -488,9 +509,7 @@ def main():
 
     from paper_2608_03057_gb300 import tasq, workloads
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = dist_env()
     torch.cuda.set_device(local)
     dist = None
     if world > 1:
@@ -549,11 +568,8 @@ def main():
     gemm_ms = [events[i][0].elapsed_time(events[i][1]) for i in range(len(step.layers))]
     quant_ms = [events[i][2].elapsed_time(events[i][0]) for i in range(len(step.layers))]
 
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * step.ops / (ms * 1e-3) / 1e12
+    ms = max_over_ranks(torch, dist, ms, "cuda")
+    value = job_tops(step.ops, world, ms)
 
     # the all-8-bit schedule on the same captured graph (same table buffer)
     L = len(step.layers)
@@ -601,11 +617,8 @@ def main():
             e2e_step()
         n_e2e = max(5, args.steps // 10)
         ms_e2e = timed_replays(torch, ge, step, n_e2e, stage_of)
-        if dist:
-            t = torch.tensor([ms_e2e], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms_e2e = float(t.item())
-        e2e = {"value": world * step.ops / (ms_e2e * 1e-3) / 1e12, "unit": UNIT,
+        ms_e2e = max_over_ranks(torch, dist, ms_e2e, "cuda")
+        e2e = {"value": job_tops(step.ops, world, ms_e2e), "unit": UNIT,
                "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in xh)),
                "d2h_bytes_per_step": int(sum(y.numel() * y.element_size() for y in yh)),
                "ms_per_step": ms_e2e}
