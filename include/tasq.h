@@ -36,7 +36,18 @@
  *    (a 16-byte reduction) and tensor-core contractions whose certificate
  *    splits K into several chunks (int32 running sums, 96 KB per SM).  Calls
  *    of either kind on different streams of one context must not overlap;
- *    use one context per concurrent stream.
+ *    use one context per concurrent stream.  Split-K contractions (few
+ *    output tiles, long K) also use the context's 32 MB of partial sums.
+ *  - Kernels are launched with programmatic dependent launch: a contraction
+ *    or quantization may start while the previous kernel in the stream
+ *    drains.  Each one waits for that kernel before it reads the
+ *    activations, codes or scales, or writes any output.  The contraction
+ *    reads the stage (argument or device int), the bit table and the packed
+ *    buffer before that wait, so write those with work that precedes the
+ *    previous kernel (as the library's own calls do), not with the kernel
+ *    launched immediately before the contraction.  The quantization only
+ *    prefetches its input into L2 before the wait, which is safe whoever
+ *    writes it.
  *
  * Data layouts: row-major, innermost index last.  Activations of a linear
  * layer are [M][K] (M tokens); of a conv, NHWC [B][H][W][Cin].  Weights are
