@@ -156,7 +156,10 @@ struct Smem {
     float ep_al[C::EPI_SLOTS][C::GPW][32], ep_zc[C::EPI_SLOTS][C::GPW][32];  // per warp, per group, per column
     int ep_tok[C::EPI_SLOTS][C::GPW][32], ep_tap[C::EPI_SLOTS][C::GPW][32];
     float ep_t[C::EPI_SLOTS][C::GPW][32];  // asymmetric weights: per-column activation sums t
-    alignas(128) uint16_t ep_stage[C::EPI_SLOTS][16 * 32];  // per-warp bf16 transpose tile (16 tokens x 32 channels)
+    // per-warp bf16 transpose tile, 16 tokens x 32 channels (64-byte rows); linear layers
+    // keep it in the output tensor map's 64-byte swizzle (16-byte chunk c of row t at
+    // c ^ ((t >> 1) & 3)), whose pattern repeats every 512 bytes
+    alignas(1024) uint16_t ep_stage[C::EPI_SLOTS][16 * 32];
     uint64_t xfull[C::X_STAGES], done[C::DONE];
     uint64_t wfull[W_STAGES], wempty[W_STAGES];
     uint64_t accfull[C::NACC], accempty[C::NACC];
@@ -667,27 +670,14 @@ __global__ void __maxnreg__(96)
                 TF(fcall, 1);
                 // Transpose the warp's 32 channels x 16 tokens through shared memory:
                 // a [16 tokens][32 channels] bf16 box (64-byte rows).
+                // (convolutions only: linear layers finish in finish16f)
                 uint16_t* stg = s->ep_stage[e];
-                if constexpr (!CONV) {
-                    if (lane == 0) ptx::bulk_wait_read0();  // the previous box has left the buffer
-                }
                 __syncwarp();
                 TF(fcall, 2);
 #pragma unroll
                 for (int j = 0; j < 16; ++j) stg[j * 32 + lane] = uint16_t(yb2[j >> 1] >> (16 * (j & 1)));
-                if constexpr (!CONV) {
-                    // linear layer: consecutive tokens are consecutive rows of y, so one TMA
-                    // store writes the box (rows past M and channels past N are clipped)
-                    ptx::fence_proxy_async_smem();
-                    __syncwarp();
-                    TF(fcall, 3);
-                    const int xc = tc.ch0 + (warp & 3) * 32, yt = tc.tok0 + g * 32 + j0;
-                    if (lane == 0 && xc < a.N && yt < a.M) {
-                        ptx::tma_store_2d(&tm_y, ptx::smem_u32(stg), xc, yt);
-                        ptx::bulk_commit();
-                    }
-                } else {
-                    // convolution: the box's pixels need not be consecutive rows; 16-byte stores
+                {
+                    // the box's pixels need not be consecutive rows of y: 16-byte stores
                     __syncwarp();
                     TF(fcall, 3);
                     const int qc = lane & 3;  // 8-channel chunk of the row
@@ -763,10 +753,14 @@ __global__ void __maxnreg__(96)
                 {
                     // stored matrix i = lane / 8: (channel block, token block) = (i & 1, i >> 1), plus
                     // two channel blocks for the second store; row k = lane % 8 is token 8 * tb + k
+                    // 16-byte chunks placed in the 64-byte swizzle of the output tensor map,
+                    // so the eight rows of each stored matrix fall in eight different bank groups
                     const int i = lane >> 3, kr = lane & 7;
-                    const uint32_t row = ptx::smem_u32(stg) + uint32_t((((i >> 1) * 8 + kr) * 32 + (i & 1) * 8) * 2);
-                    ptx::stmatrix_x4_trans(row, pk[0][0], pk[1][0], pk[0][1], pk[1][1]);
-                    ptx::stmatrix_x4_trans(row + 16 * 2, pk[2][0], pk[3][0], pk[2][1], pk[3][1]);
+                    const int t = (i >> 1) * 8 + kr, sw = (t >> 1) & 3;
+                    const uint32_t row = ptx::smem_u32(stg) + uint32_t(t * 64);
+                    ptx::stmatrix_x4_trans(row + uint32_t((((i & 1)) ^ sw) << 4), pk[0][0], pk[1][0], pk[0][1], pk[1][1]);
+                    ptx::stmatrix_x4_trans(row + uint32_t(((2 + (i & 1)) ^ sw) << 4), pk[2][0], pk[3][0], pk[2][1],
+                                           pk[3][1]);
                 }
                 ptx::fence_proxy_async_smem();
                 __syncwarp();
@@ -1069,7 +1063,7 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
         cuuint32_t box[2] = {32, 16};
         cuuint32_t es[2] = {1, 1};
         r = encode(&tm_y, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, a.y, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                   CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                   CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) {
             *why = "output tensor map rejected";
             return cudaSuccess;
