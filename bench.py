@@ -341,6 +341,59 @@ def run_sweep(torch, tasq, workloads, shapes=None, reps=10, seed=0):
     return out, switch
 
 
+def int8_tensor_peak(torch, n=8192, reps=20):
+    """Measured int8 tensor-core peak of this GPU from the library int8 GEMM
+    (torch._int_mm, cuBLASLt s8 x s8 -> s32) on n^3: 2 n^3 / t in TOPS."""
+    try:
+        a = torch.randint(-127, 128, (n, n), dtype=torch.int8, device="cuda")
+        b = torch.randint(-127, 128, (n, n), dtype=torch.int8, device="cuda")
+        for _ in range(3):
+            torch._int_mm(a, b)
+        torch.cuda.synchronize()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(reps):
+            torch._int_mm(a, b)
+        t1.record()
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1) / reps
+        del a, b
+        return {"tops": 2.0 * n ** 3 / (ms * 1e-3) / 1e12, "shape": [n, n, n],
+                "source": "torch._int_mm (cuBLASLt int8 GEMM), CUDA events, 20 back-to-back calls"}
+    except (RuntimeError, AttributeError) as exc:  # no int8 GEMM in this torch build
+        return {"tops": None, "source": f"unavailable: {exc}"}
+
+
+def s8_route_tops(torch, tasq, workloads, n=4096, reps=10):
+    """The library's own int8 route (warp-level mma.sync s8, TASQ_CODES_S8) on an
+    n^3 masked contraction at b = 8, for comparison with the tensor-core route."""
+    ctx = tasq.tasq_create(torch.cuda.current_device())
+    table = workloads.schedule_for("sweep", 1)
+    tasq.tasq_set_schedule(ctx, table, 1, table.shape[1])
+    g = torch.Generator(device="cuda")
+    g.manual_seed(7)
+    sw = torch.randint(-127, 128, (n, n), generator=g, device="cuda", dtype=torch.int8)
+    cw = torch.rand((n,), generator=g, device="cuda") * 1e-3 + 1e-4
+    pk = torch.empty((tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, n, n),), dtype=torch.uint8, device="cuda")
+    tasq.tasq_pack_weights(ctx, tasq.TASQ_LINEAR, sw, cw, None, n, n, 0, pk)
+    codes = torch.randint(-127, 128, (n, n), generator=g, device="cuda", dtype=torch.int8)
+    al = torch.rand((n,), generator=g, device="cuda") * 1e-2 + 1e-3
+    zc = torch.full((n,), 0.5, device="cuda")
+    y = torch.empty((n, n), dtype=torch.int16, device="cuda")
+    call = lambda: tasq.tasq_masked_gemm(ctx, 0, 6, codes, tasq.TASQ_CODES_S8, al, zc, n, pk, n, n, y)
+    call()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(reps):
+        call()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / reps
+    tasq.tasq_destroy(ctx)
+    return {"shape": [n, n, n], "b": 8, "tops": 2.0 * n ** 3 / (ms * 1e-3) / 1e12}
+
+
 def run_zero_point(torch, tasq, workloads, shapes=((4096, 1152, 1152), (4096, 3456, 1152), (300, 1152, 1152)),
                    reps=20, seed=0):
     """Asymmetric weights (App. A.1.1 on each channel's [min, max], a real zero
@@ -641,10 +694,18 @@ def main():
                           "between kernels, right after the timed region" if external
                 else "CUDA events around each contraction in an eager pass after the timed region"}
 
-    sweep = switch = zp = None
+    sweep = switch = zp = i8 = None
     if not args.no_sweep:
         sweep, switch = run_sweep(torch, tasq, workloads, seed=args.seed)
         zp = run_zero_point(torch, tasq, workloads, seed=args.seed)
+        # int8 tensor reference: the best int8 GEMM measured on this GPU (the library
+        # int8 GEMM, and this library's own mma.sync s8 route)
+        lt = int8_tensor_peak(torch)
+        s8 = s8_route_tops(torch, tasq, workloads)
+        best = max(x for x in (lt["tops"], s8["tops"]) if x)
+        i8 = {"tops": best, "source": "best measured int8 GEMM on this GPU",
+              "cublaslt_int8_gemm": lt, "mma_sync_s8_route": s8,
+              "step_pct": 100.0 * value / best}  # this step's int8-equivalent TOPS against it
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -686,6 +747,7 @@ def main():
             "sweep_tops_by_b": sweep,
             "stage_switch": switch,
             "asym_weights": zp,
+            "int8_tensor_peak": i8,
         }
         print(json.dumps(line), flush=True)
     step.close()
