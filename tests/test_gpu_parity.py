@@ -236,6 +236,71 @@ def test_split_k_repeated_launches(ctx, oracle, code_fmt, M, N, K):
     assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
 
 
+@pytest.mark.parametrize("graph", [False, True])
+def test_two_layer_chain_reads_the_previous_output(ctx, oracle, graph):
+    """Layer 2 quantizes layer 1's bf16 output, so every kernel depends on the one
+    before it: the quantization may start (and prefetch its input into L2) while the
+    first contraction drains, and the second contraction runs its weight pipeline
+    before its dependency wait.  Eager and captured in a CUDA graph, the chain must
+    give the oracle's result on the first layer's actual output."""
+    torch = G.torch()
+    M, K1, N1, N2 = 1000, 1152, 1152, 2304
+    x1 = workloads.normal((M, K1), 91)
+    w1 = workloads.normal((N1, K1), 92, 0.03)
+    w2 = workloads.normal((N2, N1), 93, 0.03)
+    b1 = workloads.normal((N1,), 94, 0.02)
+    b2 = workloads.normal((N2,), 95, 0.02)
+    sw1, cw1, _ = G.quant_weights(ctx, G.dev(w1), tasq.TASQ_F32, N1, K1)
+    sw2, cw2, _ = G.quant_weights(ctx, G.dev(w2), tasq.TASQ_F32, N2, N1)
+    p1 = G.pack(ctx, tasq.TASQ_LINEAR, sw1, cw1, G.dev(b1), N1, K1)
+    p2 = G.pack(ctx, tasq.TASQ_LINEAR, sw2, cw2, G.dev(b2), N2, N1)
+    tasq.tasq_set_schedule(ctx.h, np.array([[5, 8], [3, 6]], np.uint8), 2, 2)
+    x1d, x1h = G.to_bf16(x1)
+    F16 = tasq.TASQ_CODES_F16
+    c1, c2 = G.empty((M, K1), torch.float16), G.empty((M, N1), torch.float16)
+    a1, z1, a2, z2 = (G.empty((M,), torch.float32) for _ in range(4))
+    y1, y2 = G.empty((M, N1), torch.int16), G.empty((M, N2), torch.int16)
+
+    def chain(stage):
+        tasq.tasq_quant_act(ctx.h, x1d, tasq.TASQ_BF16, M, K1, 8, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, c1, F16,
+                            a1, z1)
+        tasq.tasq_masked_gemm(ctx.h, 0, stage, c1, F16, a1, z1, M, p1, N1, K1, y1, None)
+        tasq.tasq_quant_act(ctx.h, y1, tasq.TASQ_BF16, M, N1, 8, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, c2, F16,
+                            a2, z2)
+        tasq.tasq_masked_gemm(ctx.h, 1, stage, c2, F16, a2, z2, M, p2, N2, N1, y2, None)
+
+    wq1, wq2 = oracle.quant_weight(w1), oracle.quant_weight(w2)
+    for stage in (0, 1):
+        y1.fill_(0)
+        y2.fill_(0)
+        if graph:
+            chain(stage)  # first launches set kernel attributes outside the capture
+            torch.cuda.synchronize()
+            y1.fill_(0)
+            y2.fill_(0)
+            s = torch.cuda.Stream()
+            s.wait_stream(torch.cuda.current_stream())
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.stream(s), torch.cuda.graph(g, stream=s):
+                chain(stage)
+            g.replay()
+        else:
+            chain(stage)
+        torch.cuda.synchronize()
+        b1_, b2_ = [(5, 8), (3, 6)][0][stage], [(5, 8), (3, 6)][1][stage]
+        s_x1, ar1, zr1 = oracle.quant_act(x1h)
+        acc1 = oracle.gemm(s_x1, wq1["s"], b1_)
+        _, yb1 = oracle.epilogue_f32(acc1, ar1, zr1, oracle.row_sums(wq1["s"], b1_), wq1["c"], b1)
+        assert np.array_equal(G.bf16_bits_host(y1), yb1)
+        # layer 2 from the GPU's layer-1 output (bit-identical to the oracle's)
+        x2h = oracle.bf16_bits_to_f32(yb1)
+        s_x2, ar2, zr2 = oracle.quant_act(x2h)
+        acc2 = oracle.gemm(s_x2, wq2["s"], b2_)
+        _, yb2 = oracle.epilogue_f32(acc2, ar2, zr2, oracle.row_sums(wq2["s"], b2_), wq2["c"], b2)
+        assert np.array_equal(G.bf16_bits_host(y2), yb2)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
 @pytest.mark.parametrize("code_fmt", ROUTES)
 def test_output_without_acc(ctx, oracle, code_fmt):
     M, N, K = 200, 128, 256
