@@ -275,6 +275,8 @@ int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, 
  * Masked linear layer (Eq. qalora with the Temporal-Spatial LSB mask of
  * Eq. lsb_masking at operating precision b = table[layer][stage]):
  *   acc[m][n] = sum_k s_x[m][k] * mask_b(s_w[n][k])            (exact int32)
+ * (exact whenever the sum fits in int32, which |s| <= 128 guarantees for
+ * K <= 131072; past that, adversarial codes could wrap it)
  *   u = fma(zc[m], float(rs_b[n]), float(acc)),  s = alpha[m] * c_w[n],
  *   y[m][n] = bf16(fma(u, s, bias[n]))
  * with every fp32 operation (and each fused multiply-add) rounded once to
