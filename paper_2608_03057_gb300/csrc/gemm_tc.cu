@@ -290,15 +290,8 @@ __global__ void __maxnreg__(96)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const Waiter<C> wt{s, &a};
 
-    const int b = resolve_bits(a);
-    if (b == 0) return;  // uniform across the grid (a launch-wide check): nothing allocated yet
-    const int KT = (a.K + BK - 1) / BK;
-    // certificate is in 64-wide K blocks; a run of c64 of them covers c64/2 of ours
-    int chunk = a.hdr->chunk_kb[b] / (BK / kCertKBlock);
-    chunk = chunk < 1 ? 1 : (chunk > KT ? KT : chunk);
-    const int works = p.tiles_ch * p.tiles_tok * p.splits;
-    const int unit = int(blockIdx.x), units = int(gridDim.x);
-
+    // Set-up that does not depend on b (barriers, tensor memory, descriptor prefetch)
+    // overlaps the loads that resolve it.
     if (threadIdx.x == 0) {
         for (int i = 0; i < X_STAGES; ++i)  // producer's expect_tx (+ the 4 converter warps on first stages)
             ptx::mbar_init(ptx::smem_u32(&s->xfull[i]), i % Q == 0 ? 1 + 4 : 1);
@@ -323,9 +316,28 @@ __global__ void __maxnreg__(96)
         ptx::tmem_relinquish();
         ptx::tc_fence_before();
     }
+    // the certificate of every b is loaded alongside the stage and table reads
+    int cert[kNumB];
+#pragma unroll
+    for (int i = 0; i < kNumB; ++i) cert[i] = a.hdr->chunk_kb[kBMin + i];
+    const int b = resolve_bits(a);
+    int chunk_kb = 1;
+#pragma unroll
+    for (int i = 0; i < kNumB; ++i)
+        if (b == kBMin + i) chunk_kb = cert[i];
+    const int KT = (a.K + BK - 1) / BK;
+    // certificate is in 64-wide K blocks; a run of c64 of them covers c64/2 of ours
+    int chunk = chunk_kb / (BK / kCertKBlock);
+    chunk = chunk < 1 ? 1 : (chunk > KT ? KT : chunk);
+    const int works = p.tiles_ch * p.tiles_tok * p.splits;
+    const int unit = int(blockIdx.x), units = int(gridDim.x);
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem_base;
+    if (b == 0) {  // uniform across the grid (a launch-wide check, recorded in the status word)
+        if (warp == 1) ptx::tmem_dealloc(tmem, TMEM_COLS);
+        return;
+    }
     if (threadIdx.x == 0) TE(1);
     if (warp == WPROD_WARP && lane == 0 && unit < works) {
         // pull the first weight tiles into L2 ahead of the weight ring

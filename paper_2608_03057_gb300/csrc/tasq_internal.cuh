@@ -95,15 +95,15 @@ struct GemmArgs {
 // Resolves b for this launch on the device; returns 0 (and records an error)
 // when the stage or the table entry is out of range or the header mismatches.
 __device__ inline int resolve_bits(const GemmArgs& a) {
-    int stage = a.stage >= 0 ? a.stage : (a.d_stage ? *a.d_stage : -1);
-    if (stage < 0 || stage >= a.S) {
-        set_status(a.status, TASQ_ERR_DEVICE);
-        return 0;
-    }
-    int b = a.table[a.layer * a.S + stage];
+    // the header fields and the stage do not depend on one another: load them together
+    const uint32_t magic = a.hdr->magic;
+    const int hdr_n = a.hdr->N, hdr_k = a.hdr->K, hdr_zp = a.hdr->has_zp;
+    const int stage = a.stage >= 0 ? a.stage : (a.d_stage ? *a.d_stage : -1);
+    const bool stage_ok = stage >= 0 && stage < a.S;
+    const int b = stage_ok ? a.table[a.layer * a.S + stage] : 0;
     // a buffer packed with zero offsets needs the code sums of the four-term epilogue
-    if (b < kBMin || b > kBMax || a.hdr->magic != kPackedMagic || a.hdr->N != a.N || a.hdr->K != a.K ||
-        (a.hdr->has_zp && !a.code_sums)) {
+    if (!stage_ok || b < kBMin || b > kBMax || magic != kPackedMagic || hdr_n != a.N || hdr_k != a.K ||
+        (hdr_zp && !a.code_sums)) {
         set_status(a.status, TASQ_ERR_DEVICE);
         return 0;
     }
