@@ -72,14 +72,6 @@ __device__ inline void scale_of_range(float lo, float hi, float denom, float hal
     }
 }
 
-// Activation code Q = clamp(rint(x / alpha + z), 0, qmax) as the low 16 bits of
-// the returned fp32 bits (Q + 1.5 * 2^23).  Clamping u to the integer bounds
-// before rounding gives the same Q as rounding first.
-__device__ __forceinline__ uint32_t act_qbits(float x, float alpha, float ralpha, float z, float qmaxf) {
-    const float u = __fadd_rn(div_rn_by(x, alpha, ralpha), z);
-    return __float_as_uint(__fadd_rn(fminf(fmaxf(u, 0.0f), qmaxf), 12582912.0f));
-}
-
 // Activation code: Q = clamp(rint(x / alpha + z), 0, qmax), s = Q - half.
 // ralpha = RN(1 / alpha); x / alpha is still rounded exactly as IEEE division.
 __device__ inline int act_code(float x, float alpha, float ralpha, float z, int qmax, int half) {
@@ -302,16 +294,32 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
     float alpha, z;
     scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
     const float ralpha = __frcp_rn(alpha);
+    const float qmaxf = float(qmax);
+    const float2 ra2 = make_float2(ralpha, ralpha), na2 = make_float2(-alpha, -alpha), z2 = make_float2(z, z);
+    const float2 magic2 = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
     char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (CODES == TASQ_CODES_S8 ? 1 : 2);
     int csum = 0;  // sum of this lane's codes Q - half (kept only when code_sums is set)
 #pragma unroll
     for (int k = 0; k < NPL; ++k) {
         const int c = lane + 32 * k;
         if (c >= chunks) continue;
-        // vb[j]: fp32 bits of Q + 1.5 * 2^23, the code Q in the low 16 bits
+        // vb[j]: fp32 bits of Q + 1.5 * 2^23 with Q = clamp(rint(x / alpha + z), 0, qmax)
+        // in the low 16 bits (clamping u to the integer bounds before rounding gives the
+        // same Q as rounding first); x / alpha as div_rn_by.  Element pairs: every packed
+        // f32x2 operation rounds each lane exactly as the scalar one (the divide's
+        // remainder fma(-q, a, x) is taken as fma(q, -a, x)).
         uint32_t vb[EPC];
 #pragma unroll
-        for (int j = 0; j < EPC; ++j) vb[j] = act_qbits(elem(d[k], j), alpha, ralpha, z, float(qmax));
+        for (int j = 0; j < EPC; j += 2) {
+            const float2 x2 = make_float2(elem(d[k], j), elem(d[k], j + 1));
+            const float2 q2 = ptx::fmul2(x2, ra2);
+            const float2 r2 = ptx::ffma2(q2, na2, x2);
+            const float2 u2 = ptx::fadd2(ptx::ffma2(r2, ra2, q2), z2);
+            const float2 c2 = make_float2(fminf(fmaxf(u2.x, 0.0f), qmaxf), fminf(fmaxf(u2.y, 0.0f), qmaxf));
+            const float2 v2 = ptx::fadd2(c2, magic2);
+            vb[j] = __float_as_uint(v2.x);
+            vb[j + 1] = __float_as_uint(v2.y);
+        }
         int q[EPC];
 #pragma unroll
         for (int j = 0; j < EPC; ++j) q[j] = int(vb[j] & 0xFFFFu) - half;
