@@ -296,16 +296,18 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
     const float ralpha = __frcp_rn(alpha);
     const float qmaxf = float(qmax);
     const float2 ra2 = make_float2(ralpha, ralpha), na2 = make_float2(-alpha, -alpha), z2 = make_float2(z, z);
-    const float2 magic2 = make_float2(12582912.0f, 12582912.0f);  // 1.5 * 2^23
+    // 1.5 * 2^23 + 0x6400: RN(u + this) is the integer rint(u) + this, whose fp32 bits
+    // end in the 16 bits 0x6400 + rint(u) (for 0 <= rint(u) <= 255)
+    const float2 magic2 = make_float2(12608512.0f, 12608512.0f);
     char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (CODES == TASQ_CODES_S8 ? 1 : 2);
     int csum = 0;  // sum of this lane's codes Q - half (kept only when code_sums is set)
 #pragma unroll
     for (int k = 0; k < NPL; ++k) {
         const int c = lane + 32 * k;
         if (c >= chunks) continue;
-        // vb[j]: fp32 bits of Q + 1.5 * 2^23 with Q = clamp(rint(x / alpha + z), 0, qmax)
-        // in the low 16 bits (clamping u to the integer bounds before rounding gives the
-        // same Q as rounding first); x / alpha as div_rn_by.  Element pairs: every packed
+        // vb[j]: fp32 bits of Q + 1.5 * 2^23 + 0x6400 with Q = clamp(rint(x / alpha + z),
+        // 0, qmax), so the low 16 bits are 0x6400 + Q (clamping u to the integer bounds
+        // before rounding gives the same Q as rounding first); x / alpha as div_rn_by.  Element pairs: every packed
         // f32x2 operation rounds each lane exactly as the scalar one (the divide's
         // remainder fma(-q, a, x) is taken as fma(q, -a, x)).
         uint32_t vb[EPC];
@@ -322,7 +324,7 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
         }
         int q[EPC];
 #pragma unroll
-        for (int j = 0; j < EPC; ++j) q[j] = int(vb[j] & 0xFFFFu) - half;
+        for (int j = 0; j < EPC; ++j) q[j] = int(vb[j] & 0xFFFFu) - (0x6400 + half);
         if constexpr (SUMS) {
 #pragma unroll
             for (int j = 0; j < EPC; ++j) csum += q[j];
@@ -343,11 +345,10 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
             // exactly; one packed subtraction of 1024 + half leaves s
             const uint32_t off = 0x6400u + uint32_t(half);
             const __half2 bias2 = __halves2half2(__ushort_as_half(uint16_t(off)), __ushort_as_half(uint16_t(off)));
-            // the low halves of two vb words, Q0 | Q1 << 16, with 0x6400 in each half
-            // are the fp16 values 1024 + Q; one packed subtraction of 1024 + half
-            // leaves the codes s = Q - half
+            // the low halves of two vb words, 0x6400 + Q each, are the fp16 values
+            // 1024 + Q; one packed subtraction of 1024 + half leaves the codes s = Q - half
             auto sub2 = [&](uint32_t v0, uint32_t v1) -> uint32_t {
-                uint32_t w = __byte_perm(v0, v1, 0x5410) | 0x64006400u;
+                uint32_t w = __byte_perm(v0, v1, 0x5410);
                 __half2 r = __hsub2(*reinterpret_cast<__half2*>(&w), bias2);
                 return *reinterpret_cast<uint32_t*>(&r);
             };
