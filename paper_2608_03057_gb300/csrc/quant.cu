@@ -317,7 +317,15 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
             const float2 q2 = ptx::fmul2(x2, ra2);
             const float2 r2 = ptx::ffma2(q2, na2, x2);
             const float2 u2 = ptx::fadd2(ptx::ffma2(r2, ra2, q2), z2);
-            const float2 c2 = make_float2(fminf(fmaxf(u2.x, 0.0f), qmaxf), fminf(fmaxf(u2.y, 0.0f), qmaxf));
+            // For a finite row whose alpha is a normal float, u stays within (-0.5,
+            // qmax + 0.5) (alpha and z come from the row's own range; the error is a few
+            // ulps of qmax), so the clamp never binds and fp16 codes are clamped once,
+            // packed, after the subtraction below instead (which also keeps codes in
+            // range for inputs outside that class).  Integer codes and code sums take Q
+            // from the bits here, so they clamp u first.
+            float2 c2 = u2;
+            if constexpr (CODES == TASQ_CODES_S8 || SUMS)
+                c2 = make_float2(fminf(fmaxf(u2.x, 0.0f), qmaxf), fminf(fmaxf(u2.y, 0.0f), qmaxf));
             const float2 v2 = ptx::fadd2(c2, magic2);
             vb[j] = __float_as_uint(v2.x);
             vb[j + 1] = __float_as_uint(v2.y);
@@ -347,9 +355,11 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
             const __half2 bias2 = __halves2half2(__ushort_as_half(uint16_t(off)), __ushort_as_half(uint16_t(off)));
             // the low halves of two vb words, 0x6400 + Q each, are the fp16 values
             // 1024 + Q; one packed subtraction of 1024 + half leaves the codes s = Q - half
+            const __half2 lo2 = __float2half2_rn(float(-half)), hi2 = __float2half2_rn(float(half - 1));
             auto sub2 = [&](uint32_t v0, uint32_t v1) -> uint32_t {
                 uint32_t w = __byte_perm(v0, v1, 0x5410);
                 __half2 r = __hsub2(*reinterpret_cast<__half2*>(&w), bias2);
+                if constexpr (!SUMS) r = __hmax2(__hmin2(r, hi2), lo2);
                 return *reinterpret_cast<uint32_t*>(&r);
             };
             const uint32_t* h = vb;
