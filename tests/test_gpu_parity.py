@@ -386,7 +386,7 @@ def test_stage_from_device_int(ctx, oracle, code_fmt):
 @pytest.mark.parametrize("code_fmt", ROUTES)
 @pytest.mark.parametrize("M,N,K", [(4096, 3456, 1152), (4096, 1152, 4608), (4096, 1152, 1152), (1200, 2240, 2240),
                                    (77, 1280, 2048), (4096, 6720, 2240), (4096, 11200, 2240), (4096, 2240, 5600),
-                                   (256, 1280, 5120), (256, 10240, 1280), (1024, 640, 640)])
+                                   (256, 1280, 5120), (256, 10240, 1280), (1024, 640, 640), (16384, 4096, 4096)])
 def test_full_size_sampled_rows(ctx, oracle, code_fmt, M, N, K):
     """Full-size layer shapes of the backbones, checked on sampled token rows
     (the oracle computes those rows one by one)."""
