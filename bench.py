@@ -460,16 +460,18 @@ def run_zero_point(torch, tasq, workloads, shapes=((4096, 1152, 1152), (4096, 34
 
 
 # ------------------------------------------------------------ CPU oracle --
-def oracle_sample(workload: str, budget_s: float, rows: int = 32, seed: int = 0, max_layers=None):
+def oracle_sample(workload: str, budget_s: float, rows: int = 32, seed: int = 0, max_layers=None, threads=0):
     """Time the CPU oracle (act quant, int32 contraction, row sums, fp32
     epilogue) on `rows` token rows of successive layers of the workload until
-    the budget is spent.  Returns (ops, seconds, layers_done, rows, threads)."""
+    the budget is spent, on `threads` OpenMP threads (0: every core).
+    Returns (ops, seconds, layers_done, rows, threads)."""
     from oracle import oracle
     from paper_2608_03057_gb300 import workloads
 
     layers = workloads.inventory(workload)
     table = workloads.schedule_for(workload, len(layers))
     oracle.build()
+    oracle.set_threads(threads)
     ops = 0
     spent = 0.0
     done = 0
@@ -495,8 +497,7 @@ def oracle_sample(workload: str, budget_s: float, rows: int = 32, seed: int = 0,
             spent += time.perf_counter() - t0
             ops += 2 * rows * l.N * l.K
         done += 1
-    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    return ops, spent, done, rows, threads
+    return ops, spent, done, rows, oracle.threads()
 
 
 def run_reference(args):
@@ -712,6 +713,9 @@ def main():
         o, s, d, rows, threads = oracle_sample(args.workload, args.cpu_seconds, seed=args.seed)
         cpu = {"value": o / s / 1e12, "unit": UNIT, "cores": threads, "kind": "oracle",
                "sample": f"{rows} token rows of each of the first {d} layers of the step ({s:.1f} s)"}
+        o1, s1, d1, rows1, _ = oracle_sample(args.workload, min(8.0, args.cpu_seconds), seed=args.seed, threads=1)
+        cpu["single_thread"] = {"value": o1 / s1 / 1e12, "cores": 1,
+                                "sample": f"{rows1} token rows of each of the first {d1} layers ({s1:.1f} s)"}
 
     if rank == 0:
         bits = step.table.astype(np.float64)

@@ -70,6 +70,8 @@ def _lib():
             lib.oq_epilogue_zp_f32.argtypes = [P, i32, i32, i32, P, P, P, P, P, P, P, P, P]
             lib.oq_linear_zp_def_f64.argtypes = [P, P, P, i32, P, P, P, P, i32, i32, i32, P]
             lib.oq_conv3x3_code_sums.argtypes = [P, i32, i32, i32, i32, P, P]
+            lib.oq_set_threads.argtypes = [i32]
+            lib.oq_threads.restype = i32
             lib.oq_conv_epilogue_zp_f32.argtypes = [P, i64, i32, f32, f32, P, P, P, P, P, P, P, P]
             lib.oq_conv3x3_zp_def_f64.argtypes = [P, f32, f32, i32, i32, i32, i32, P, P, P, P, i32, i32, P]
             _LIB = lib
@@ -82,6 +84,15 @@ def _p(a):
 
 def _c(a, dtype):
     return np.ascontiguousarray(a, dtype=dtype)
+
+
+def set_threads(n: int) -> None:
+    """Threads of the oracle's OpenMP loops (n <= 0: every processor)."""
+    _lib().oq_set_threads(int(n))
+
+
+def threads() -> int:
+    return int(_lib().oq_threads())
 
 
 def f32_to_bf16_bits(y):

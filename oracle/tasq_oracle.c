@@ -37,6 +37,9 @@
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 #define OQ_SYMRANGE 0
 #define OQ_ASYM 1
@@ -503,4 +506,22 @@ void oq_conv3x3_zp_def_f64(const int8_t* s_x, float alpha, float zc, int B, int 
             y[p * Cout + n] = sum + (bias ? (double)bias[n] : 0.0);
         }
     }
+}
+
+/* Threads of the OpenMP loops above: n (n <= 0: every processor); and the
+ * number the next parallel loop will use.  Timing helpers, no arithmetic. */
+void oq_set_threads(int n) {
+#ifdef _OPENMP
+    omp_set_num_threads(n > 0 ? n : omp_get_num_procs());
+#else
+    (void)n;
+#endif
+}
+
+int oq_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
 }
