@@ -21,12 +21,16 @@
 //      into 128-byte-swizzled shared memory (a 2-D tile for a linear layer; a
 //      4-D NHWC box shifted by the 3x3 tap for a convolution, whose padding
 //      TMA fills with code 0).
-//   D: fp32 accumulators in tensor memory, double-buffered so the epilogue
-//      of one chunk overlaps the MMAs of the next.
+//   D: fp32 accumulators in tensor memory, double-buffered (192- and 64-token
+//      tiles) so the epilogue of one chunk overlaps the MMAs of the next, or
+//      single (256-token tiles, one tile per CTA).
 //
-// Warp roles (576 threads): warp 0 issues TMA; warp 1 allocates tensor
-// memory and issues the MMAs (one thread); warps 2..5 convert weights; warps
-// 6..17 drain accumulators and run the fused dequantization epilogue.  The
+// Warp roles (608 threads): warp 0 issues the activation TMA; warp 1
+// allocates tensor memory and issues the MMAs (one thread); warps 2..5 convert
+// weights (and, for a single-tile CTA, join the epilogue once the last K block
+// is converted); warps 6..17 drain accumulators and run the fused
+// dequantization epilogue (linear outputs leave through TMA stores of
+// swizzled [16 token][32 channel] boxes); warp 18 issues the weight TMA.  The
 // grid is persistent: one CTA per SM walks the output tiles.  Every wait is
 // bounded by the context's time limit; a wait that gives up records
 // TASQ_ERR_DEVICE_TIMEOUT, the CTA drains its copies in flight, frees its
