@@ -344,6 +344,38 @@ int tasq_masked_conv3x3_zp(tasq_ctx ctx, int layer, int stage, const void* d_cod
                            int Cin, const void* d_packed, int Cout, uint16_t* d_y, int32_t* d_acc,
                            tasq_stream stream);
 
+/* Launch plan of the tensor-core route for one contraction (see tasq_plan_tc). */
+typedef struct {
+    int tile_channels;      /* output channels per tile (MMA M): 128 */
+    int tile_tokens;        /* tokens per tile (MMA N): 64, 192 or 256 */
+    int acc_buffers;        /* fp32 accumulator buffers in tensor memory: 1 or 2 */
+    int tiles_ch;           /* channel tiles: ceil(N / 128) */
+    long long tiles_tok;    /* token tiles; a convolution tiles each image into boxes */
+    int box_rows, box_cols; /* convolution: token box of box_rows image rows x box_cols pixels
+                               (box_rows * box_cols == tile_tokens); 0 for a linear layer */
+    int splits;             /* K slices, each summed by its own CTAs (1: K is not split) */
+    int grid;               /* CTAs of the contraction kernel (persistent: at most num_sms) */
+    int reduce_grid;        /* CTAs of the split-K reduction kernel (0 when splits == 1) */
+    int kernels;            /* kernels the call enqueues: 1, 2 with split-K, 0 when M == 0 */
+} tasq_tc_plan;
+
+/*
+ * The launch plan that tasq_masked_gemm(_zp) or tasq_masked_conv3x3(_zp) on
+ * the tensor-core route (TASQ_ROUTE_TC) follows for this shape, on a device
+ * with `num_sms` SMs and a context's own split-K scratch.  The plan depends on
+ * the shape alone, not on the bits b or on the data.  Host-only: needs no
+ * context and no device, enqueues nothing.  Diagnostic (the paper has no
+ * counterpart): it lets a caller see how a layer is tiled without a GPU.
+ * kind TASQ_LINEAR: M tokens, N outputs, K inputs (B, H, W, Cin ignored).
+ * kind TASQ_CONV3X3: B, H, W, Cin and N = Cout (M = B*H*W and K = 9*Cin are
+ * implied; the M and K arguments are ignored).  *out is zeroed first.
+ * Returns TASQ_ERR_INVALID_ARG (bad kind, negative size, NULL out,
+ * num_sms < 1) or TASQ_ERR_UNSUPPORTED (a shape the contraction calls would
+ * reject on this route: K % 16, N % 8, Cin % 64 for a convolution), with the
+ * text in tasq_last_error(NULL) on the calling thread.
+ */
+int tasq_plan_tc(int kind, int M, int N, int K, int B, int H, int W, int Cin, int num_sms, tasq_tc_plan* out);
+
 /*
  * Per-tensor activation quantization without any allocation (no context).
  * The paper has no counterpart to this call: it exists for callers that

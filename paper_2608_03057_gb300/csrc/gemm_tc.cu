@@ -1006,8 +1006,82 @@ TokTiling token_tiling(const GemmArgs& a, int BT) {
     return t;
 }
 
+}  // namespace
+
+TcPlan plan_gemm_tc(int M, int N, int K, int B, int H, int W, int Cin, int num_sms, int64_t split_cap) {
+    TcPlan p{};
+    GemmArgs a{};
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.B = B;
+    a.H = H;
+    a.W = W;
+    a.Cin = Cin;
+    p.bch = BCH;
+    p.tiles_ch = (N + BCH - 1) / BCH;
+    p.splits = 1;
+    if (Cin && Cin % 64) {
+        p.why = "convolution needs Cin % 64 == 0";
+        return p;
+    }
+    if (M <= 0 || N <= 0) return p;
+    // The wide single-tile configuration when it covers the output in one wave
+    // of CTAs and the standard one would need more than one; the narrow one when
+    // the standard tiles would leave most SMs idle.
+    const int64_t std_tiles = p.tiles_ch * token_tiling(a, CfgStd::BT).tiles;
+    const int64_t wide_tiles = p.tiles_ch * token_tiling(a, CfgWide::BT).tiles;
+    if (std_tiles > num_sms && wide_tiles <= num_sms) {
+        p.bt = CfgWide::BT;
+        p.nacc = CfgWide::NACC;
+    } else if (std_tiles * 2 <= num_sms) {
+        p.bt = CfgNarrow::BT;
+        p.nacc = CfgNarrow::NACC;
+    } else {
+        p.bt = CfgStd::BT;
+        p.nacc = CfgStd::NACC;
+    }
+    const TokTiling tt = token_tiling(a, p.bt);  // conv: 2^bw_log2 divides BT (192 = 64 * 3, 256)
+    p.tiles_tok = tt.tiles;
+    p.bw_log2 = tt.bw_log2;
+    p.bhx = tt.bhx;
+    p.tiles_w = tt.tiles_w;
+    p.tiles_h = tt.tiles_h;
+    const int64_t tiles = int64_t(p.tiles_ch) * p.tiles_tok;
+    if (tiles > 0x7FFFFFFF) {
+        p.why = "too many tiles";
+        return p;
+    }
+    // Split K when the tiles alone would leave most SMs idle and each slice keeps
+    // at least 8 K blocks: a tile's fixed latency (pipeline fill, epilogue) is
+    // not reduced by splitting, only its K loop is.
+    if (p.nacc == 2 && split_cap > 0 && tiles * 2 <= num_sms) {
+        const int KT = (K + BK - 1) / BK;
+        int64_t S = num_sms / tiles;
+        S = S < KT / 8 ? S : KT / 8;
+        static const int max_splits = [] {
+            const char* v = getenv("TASQ_TC_MAX_SPLITS");  // tuning knob; default 16
+            return v ? atoi(v) : 16;
+        }();
+        S = S < max_splits ? S : max_splits;
+        const int64_t fit = split_cap / (int64_t(M) * N);
+        S = S < fit ? S : fit;
+        if (S >= 2) p.splits = int(S);
+    }
+    const int64_t works = tiles * p.splits;
+    p.grid = int(works < num_sms ? works : num_sms);
+    if (p.splits > 1) {
+        // the reduction reads 4 channels per thread, 256 threads per block
+        const int64_t blocks = (int64_t(M) * (N / 4) + 255) / 256;
+        p.reduce_grid = int(blocks < 8 * int64_t(num_sms) ? blocks : 8 * int64_t(num_sms));
+    }
+    return p;
+}
+
+namespace {
+
 template <class C>
-cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why, int* kernels) {
+cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, const char** why, int* kernels) {
     constexpr int BTOK = C::BT;
     auto encode = get_encode();
     if (!encode) {
@@ -1020,24 +1094,13 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
     p.tiles_ch = (a.N + BCH - 1) / BCH;
     CUtensorMap tm_x, tm_w, tm_y;
     CUresult r;
+    p.tiles_tok = int(plan.tiles_tok);
     if (p.conv) {
-        if (a.Cin % 64) {
-            *why = "convolution needs Cin % 64 == 0";
-            return cudaSuccess;
-        }
-        // box of bhx rows x 2^bwl pixels; 2^bwl divides BTOK (192 = 64 * 3, 256)
-        const TokTiling tt = token_tiling(a, BTOK);
-        p.bw_log2 = tt.bw_log2;
-        p.bhx = tt.bhx;
-        const int bw = 1 << tt.bw_log2;
-        p.tiles_w = tt.tiles_w;
-        p.tiles_h = tt.tiles_h;
-        const int64_t tok_tiles = tt.tiles;
-        if (tok_tiles * p.tiles_ch > 0x7FFFFFFF) {
-            *why = "too many tiles";
-            return cudaSuccess;
-        }
-        p.tiles_tok = int(tok_tiles);
+        p.bw_log2 = plan.bw_log2;
+        p.bhx = plan.bhx;
+        const int bw = 1 << plan.bw_log2;
+        p.tiles_w = plan.tiles_w;
+        p.tiles_h = plan.tiles_h;
         cuuint64_t dims[4] = {cuuint64_t(a.Cin), cuuint64_t(a.W), cuuint64_t(a.H), cuuint64_t(a.B)};
         cuuint64_t strides[3] = {cuuint64_t(a.Cin) * 2, cuuint64_t(a.W) * a.Cin * 2, cuuint64_t(a.H) * a.W * a.Cin * 2};
         cuuint32_t box[4] = {XK, cuuint32_t(bw), cuuint32_t(p.bhx), 1};
@@ -1046,7 +1109,6 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     } else {
-        p.tiles_tok = (a.M + BTOK - 1) / BTOK;
         cuuint64_t dims[2] = {cuuint64_t(a.K), cuuint64_t(a.M)};
         cuuint64_t strides[1] = {cuuint64_t(a.K) * 2};
         cuuint32_t box[2] = {XK, cuuint32_t(BTOK)};
@@ -1087,34 +1149,13 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
     } else {
         tm_y = tm_x;  // unused by the convolution instantiation
     }
-    const int64_t tiles = int64_t(p.tiles_ch) * p.tiles_tok;
-    // Split K when the tiles alone would leave most SMs idle and each slice keeps
-    // at least 8 K blocks: a tile's fixed latency (pipeline fill, epilogue) is
-    // not reduced by splitting, only its K loop is.
-    p.splits = 1;
-    p.split_out = nullptr;
-    if (C::NACC == 2 && a.split_buf && tiles * 2 <= num_sms) {
-        const int KT = (a.K + BK - 1) / BK;
-        int64_t S = num_sms / tiles;
-        S = S < KT / 8 ? S : KT / 8;
-        static const int max_splits = [] {
-            const char* v = getenv("TASQ_TC_MAX_SPLITS");  // tuning knob; default 16
-            return v ? atoi(v) : 16;
-        }();
-        S = S < max_splits ? S : max_splits;
-        const int64_t fit = a.split_cap / (int64_t(a.M) * a.N);
-        S = S < fit ? S : fit;
-        if (S >= 2) {
-            p.splits = int(S);
-            p.split_out = a.split_buf;
-        }
-    }
-    const int64_t works = tiles * p.splits;
-    const int units = int(works < num_sms ? works : num_sms);
+    p.splits = plan.splits;
+    p.split_out = plan.splits > 1 ? a.split_buf : nullptr;
+    const int units = plan.grid;
     static const bool verbose = getenv("TASQ_TC_VERBOSE") != nullptr;
     if (verbose)
-        fprintf(stderr, "tasq tc: M=%d N=%d K=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, (long long)tiles,
-                p.splits, units);
+        fprintf(stderr, "tasq tc: M=%d N=%d K=%d BT=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, BTOK,
+                (long long)p.tiles_ch * p.tiles_tok, p.splits, units);
     const int smem = smem_bytes<C>();
     auto kernel = p.conv ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
                          : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
@@ -1136,10 +1177,8 @@ cudaError_t launch_cfg(const GemmArgs& a, int num_sms, cudaStream_t st, const ch
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaSuccess) *kernels = 1;
     if (e == cudaSuccess && p.splits > 1) {
-        const int64_t total = int64_t(a.M) * (a.N / 4);
-        const int64_t blocks = (total + 255) / 256;
         cudaLaunchConfig_t rc{};
-        rc.gridDim = dim3(unsigned(blocks < 8 * num_sms ? blocks : 8 * num_sms));
+        rc.gridDim = dim3(unsigned(plan.reduce_grid));
         rc.blockDim = dim3(256);
         rc.stream = st;
         rc.attrs = attr;  // programmatic dependent launch
@@ -1173,15 +1212,15 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         return cudaSuccess;
     }
     if (a.M == 0 || a.N == 0) return cudaSuccess;
-    // The wide single-tile configuration when it covers the output in one wave
-    // of CTAs and the standard one would need more than one; the narrow one when
-    // the standard tiles would leave most SMs idle.
-    const int64_t tiles_ch = (a.N + BCH - 1) / BCH;
-    const int64_t std_tiles = tiles_ch * token_tiling(a, CfgStd::BT).tiles;
-    const int64_t wide_tiles = tiles_ch * token_tiling(a, CfgWide::BT).tiles;
-    if (std_tiles > num_sms && wide_tiles <= num_sms) return launch_cfg<CfgWide>(a, num_sms, st, why, kernels);
-    if (std_tiles * 2 <= num_sms) return launch_cfg<CfgNarrow>(a, num_sms, st, why, kernels);
-    return launch_cfg<CfgStd>(a, num_sms, st, why, kernels);
+    const TcPlan plan =
+        plan_gemm_tc(a.M, a.N, a.K, a.B, a.H, a.W, a.Cin, num_sms, a.split_buf ? a.split_cap : 0);
+    if (plan.why) {
+        *why = plan.why;
+        return cudaSuccess;
+    }
+    if (plan.bt == CfgWide::BT) return launch_cfg<CfgWide>(a, plan, st, why, kernels);
+    if (plan.bt == CfgNarrow::BT) return launch_cfg<CfgNarrow>(a, plan, st, why, kernels);
+    return launch_cfg<CfgStd>(a, plan, st, why, kernels);
 }
 
 #ifdef TASQ_TRACE

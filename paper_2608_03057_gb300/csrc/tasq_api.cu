@@ -441,3 +441,45 @@ TASQ_API int tasq_masked_conv3x3_zp(tasq_ctx ctx, int layer, int stage, const vo
     return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, d_code_sums,
                               B * H * W, d_packed, Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
 }
+
+TASQ_API int tasq_plan_tc(int kind, int M, int N, int K, int B, int H, int W, int Cin, int num_sms,
+                          tasq_tc_plan* out) {
+    const tasq_ctx ctx = nullptr;  // host-only call: errors go to tasq_last_error(NULL)
+    REQUIRE(out, TASQ_ERR_INVALID_ARG, "out is NULL");
+    *out = tasq_tc_plan{};
+    REQUIRE(kind == TASQ_LINEAR || kind == TASQ_CONV3X3, TASQ_ERR_INVALID_ARG, "kind %d", kind);
+    REQUIRE(num_sms > 0, TASQ_ERR_INVALID_ARG, "num_sms=%d", num_sms);
+    if (kind == TASQ_CONV3X3) {
+        // the checks of tasq_masked_conv3x3
+        REQUIRE(B >= 0 && H > 0 && W > 0 && Cin > 0, TASQ_ERR_INVALID_ARG, "B=%d H=%d W=%d Cin=%d", B, H, W, Cin);
+        REQUIRE(Cin % 16 == 0, TASQ_ERR_UNSUPPORTED, "conv: Cin=%d must be a multiple of 16", Cin);
+        REQUIRE((int64_t)B * H * W <= 0x7FFFFFFF && (int64_t)9 * Cin <= 0x7FFFFFFF, TASQ_ERR_UNSUPPORTED,
+                "too large");
+        M = B * H * W;
+        K = 9 * Cin;
+    } else {
+        B = 1;
+        H = W = Cin = 0;
+    }
+    // the checks every contraction call makes
+    REQUIRE(M >= 0 && N > 0 && K > 0, TASQ_ERR_INVALID_ARG, "M=%d N=%d K=%d", M, N, K);
+    REQUIRE(K % 16 == 0 && N % 8 == 0, TASQ_ERR_UNSUPPORTED, "need K %% 16 == 0 and N %% 8 == 0 (N=%d K=%d)", N, K);
+    const tasq::TcPlan p =
+        tasq::plan_gemm_tc(M, N, K, B, H, W, Cin, num_sms, tasq::kSplitBufBytes / int64_t(sizeof(int32_t)));
+    REQUIRE(!p.why, TASQ_ERR_UNSUPPORTED, "tensor-core route: %s", p.why);
+    out->tile_channels = p.bch;
+    out->tiles_ch = p.tiles_ch;
+    if (M == 0) return TASQ_OK;
+    out->tile_tokens = p.bt;
+    out->acc_buffers = p.nacc;
+    out->tiles_tok = p.tiles_tok;
+    if (Cin) {
+        out->box_rows = p.bhx;
+        out->box_cols = 1 << p.bw_log2;
+    }
+    out->splits = p.splits;
+    out->grid = p.grid;
+    out->reduce_grid = p.reduce_grid;
+    out->kernels = p.splits > 1 ? 2 : 1;
+    return TASQ_OK;
+}

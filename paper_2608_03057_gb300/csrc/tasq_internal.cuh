@@ -218,6 +218,25 @@ cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
 // *kernels: how many kernels the call enqueued (the contraction, plus the split-K
 // reduction when K is split).
 cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why, int* kernels);
+// Launch plan of the tensor-core route, decided on the host from the shape
+// alone: tile configuration, token tiling, K slices and grid.  launch_gemm_tc
+// launches exactly this plan.
+struct TcPlan {
+    int bch;              // output channels per tile (MMA M)
+    int bt;               // tokens per tile (MMA N): 64, 192 or 256
+    int nacc;             // accumulator buffers in tensor memory
+    int tiles_ch;         // 128-channel blocks
+    int64_t tiles_tok;    // token tiles
+    int bw_log2, bhx;     // conv: token box of bhx image rows x 2^bw_log2 pixels
+    int tiles_w, tiles_h; // conv: boxes across and down one image
+    int splits;           // K slices (1: K is not split)
+    int grid;             // CTAs of the contraction kernel
+    int reduce_grid;      // CTAs of the split-K reduction (0: K is not split)
+    const char* why;      // non-null: the route cannot take this shape
+};
+// Cin != 0 selects the convolution (M = B H W, K = 9 Cin); split_cap: elements
+// of split-K scratch (0: no split).
+TcPlan plan_gemm_tc(int M, int N, int K, int B, int H, int W, int Cin, int num_sms, int64_t split_cap);
 size_t gemm_tc_part_bytes(int num_sms);  // scratch the TC route needs for `num_sms` persistent CTAs
 constexpr int64_t kSplitBufBytes = int64_t(32) << 20;  // split-K partial sums (context scratch)
 cudaError_t launch_selftest_timeout(int* status, unsigned long long timeout_ns, cudaStream_t st);

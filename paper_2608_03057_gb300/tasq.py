@@ -32,6 +32,14 @@ _lock = threading.Lock()
 _lib = None
 
 
+class tasq_tc_plan(ctypes.Structure):
+    """The tasq_tc_plan struct of include/tasq.h."""
+    _fields_ = [("tile_channels", ctypes.c_int), ("tile_tokens", ctypes.c_int), ("acc_buffers", ctypes.c_int),
+                ("tiles_ch", ctypes.c_int), ("tiles_tok", ctypes.c_longlong), ("box_rows", ctypes.c_int),
+                ("box_cols", ctypes.c_int), ("splits", ctypes.c_int), ("grid", ctypes.c_int),
+                ("reduce_grid", ctypes.c_int), ("kernels", ctypes.c_int)]
+
+
 class TasqError(RuntimeError):
     def __init__(self, code: int, msg: str):
         super().__init__(f"tasq error {code}: {msg}")
@@ -73,6 +81,7 @@ def lib():
                 "tasq_masked_conv3x3": ([P, I, I, P, I, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_masked_conv3x3_zp": ([P, I, I, P, I, P, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_quant_act_tensor_noalloc": ([P, I, I, I, I, I, P, I, P, P, P], I),
+                "tasq_plan_tc": ([I, I, I, I, I, I, I, I, I, ctypes.POINTER(tasq_tc_plan)], I),
             }
             for name, (args, res) in sigs.items():
                 f = getattr(L, name)
@@ -234,3 +243,12 @@ def tasq_quant_act_tensor_noalloc(x, dtype, M, K, n_bits, mode, codes, code_fmt,
     _check(None, lib().tasq_quant_act_tensor_noalloc(_ptr(x), int(dtype), int(M), int(K), int(n_bits), int(mode),
                                                      _ptr(codes), int(code_fmt), _ptr(alpha), _ptr(zc),
                                                      _stream(stream)))
+
+
+def tasq_plan_tc(kind, M, N, K, B, H, W, Cin, num_sms) -> dict:
+    """Launch plan of the tensor-core route for one contraction shape (host only:
+    no context, no GPU).  Returns the tasq_tc_plan fields as a dict."""
+    out = tasq_tc_plan()
+    _check(None, lib().tasq_plan_tc(int(kind), int(M), int(N), int(K), int(B), int(H), int(W), int(Cin), int(num_sms),
+                                    ctypes.byref(out)))
+    return {name: getattr(out, name) for name, _ in tasq_tc_plan._fields_}

@@ -236,6 +236,46 @@ def test_split_k_repeated_launches(ctx, oracle, code_fmt, M, N, K):
     assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
 
 
+@pytest.mark.parametrize("kind,shape", [
+    (tasq.TASQ_LINEAR, (4096, 3456, 1152)),   # 192-token tiles, persistent
+    (tasq.TASQ_LINEAR, (4000, 1096, 384)),    # 256-token tiles
+    (tasq.TASQ_LINEAR, (300, 2304, 1152)),    # 64-token tiles
+    (tasq.TASQ_LINEAR, (64, 1152, 4608)),     # 64-token tiles, split K
+    (tasq.TASQ_CONV3X3, (1, 64, 64, 640, 640)),
+    (tasq.TASQ_CONV3X3, (2, 6, 6, 64, 128)),
+])
+def test_launches_follow_the_plan(ctx, kind, shape):
+    """The contraction enqueues the kernels tasq_plan_tc reports for its shape
+    on this GPU's SM count (two where K is split), and leaves no device error."""
+    torch = G.torch()
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    F16 = tasq.TASQ_CODES_F16
+    if kind == tasq.TASQ_LINEAR:
+        M, N, K = shape
+        plan = tasq.tasq_plan_tc(kind, M, N, K, 0, 0, 0, 0, sms)
+        Cin = 0
+    else:
+        B, H, W, Cin, N = shape
+        M, K = B * H * W, 9 * Cin
+        plan = tasq.tasq_plan_tc(kind, 0, N, 0, B, H, W, Cin, sms)
+    assert plan["kernels"] >= 1 and plan["grid"] <= sms
+    w = workloads.normal((N, K), 31, 0.02)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+    packed = G.pack(ctx, kind, sw, cw, G.dev(np.zeros(N, np.float32)), N, K, Cin)
+    tasq.tasq_set_schedule(ctx.h, np.array([[6]], np.uint8), 1, 1)
+    gran = tasq.TASQ_PER_TENSOR if kind == tasq.TASQ_CONV3X3 else tasq.TASQ_PER_TOKEN
+    k_in = Cin if Cin else K
+    codes, alpha, zc = G.quant_act(ctx, G.dev(workloads.normal((M, k_in), 32)), tasq.TASQ_F32, M, k_in, gran=gran,
+                                   code_fmt=F16)
+    before = tasq.tasq_kernel_count(ctx.h)
+    if kind == tasq.TASQ_LINEAR:
+        G.gemm(ctx, 0, 0, codes, F16, alpha, zc, M, packed, N, K, want_acc=False)
+    else:
+        G.conv(ctx, 0, 0, codes, F16, alpha, zc, B, H, W, Cin, packed, N, want_acc=False)
+    assert tasq.tasq_kernel_count(ctx.h) - before == plan["kernels"]
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
 @pytest.mark.parametrize("graph", [False, True])
 def test_two_layer_chain_reads_the_previous_output(ctx, oracle, graph):
     """Layer 2 quantizes layer 1's bf16 output, so every kernel depends on the one
