@@ -71,6 +71,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=list(WORKLOAD_NAMES), default="pixart")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-copy-streams", type=int, default=1,
+                    help="copy streams per direction in the end-to-end step (layers take them in turn)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU oracle sample budget")
     ap.add_argument("--seed", type=int, default=0)
@@ -640,30 +642,35 @@ def main():
     if not args.no_e2e:
         xh = [x.cpu().pin_memory() for x in step.x]
         yh = [torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for y in step.y]
-        s = torch.cuda.current_stream()
-        sh, sd = torch.cuda.Stream(), torch.cuda.Stream()
+        nc = max(1, args.e2e_copy_streams)
+        sh = [torch.cuda.Stream() for _ in range(nc)]
+        sd = [torch.cuda.Stream() for _ in range(nc)]
         evx = [torch.cuda.Event() for _ in range(L)]
         evy = [torch.cuda.Event() for _ in range(L)]
-        fork, join_h, join_d = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
+        fork = torch.cuda.Event()
+        joins = [torch.cuda.Event() for _ in range(2 * nc)]
 
         def e2e_step():
+            # the stream the kernels go to: under graph capture the capture stream, so
+            # that the copy streams fork from it and join it again and every copy is a
+            # node of the captured step
+            s = torch.cuda.current_stream()
             fork.record(s)
-            sh.wait_event(fork)
-            sd.wait_event(fork)
+            for c in sh + sd:
+                c.wait_event(fork)
             for i in range(L):
-                with torch.cuda.stream(sh):
+                with torch.cuda.stream(sh[i % nc]):
                     step.x[i].copy_(xh[i], non_blocking=True)
-                    evx[i].record(sh)
+                    evx[i].record(sh[i % nc])
                 s.wait_event(evx[i])
                 step.launch_layer(i)
                 evy[i].record(s)
-                with torch.cuda.stream(sd):
-                    sd.wait_event(evy[i])
+                with torch.cuda.stream(sd[i % nc]):
+                    sd[i % nc].wait_event(evy[i])
                     yh[i].copy_(step.y[i], non_blocking=True)
-            join_h.record(sh)
-            join_d.record(sd)
-            s.wait_event(join_h)
-            s.wait_event(join_d)
+            for c, j in zip(sh + sd, joins):
+                j.record(c)
+                s.wait_event(j)
         e2e_step()
         torch.cuda.synchronize()
         ge = torch.cuda.CUDAGraph()
@@ -675,6 +682,7 @@ def main():
         e2e = {"value": job_tops(step.ops, world, ms_e2e), "unit": UNIT,
                "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in xh)),
                "d2h_bytes_per_step": int(sum(y.numel() * y.element_size() for y in yh)),
+               "copy_streams_per_direction": nc,
                "ms_per_step": ms_e2e}
         del xh, yh, ge
 
