@@ -54,6 +54,15 @@ def kernel_sources_sha256() -> str:
         with open(os.path.join(here, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()
+
+
+def measured_traffic(workload: str):
+    """DRAM bytes per contraction launch from the recorded ncu capture of this
+    workload, or None when there is none or the kernel sources have changed since."""
+    tr = TRAFFIC.get(workload)
+    return tr["bytes_per_launch"] if tr and tr["sources_sha256"] == kernel_sources_sha256() else None
+
+
 UNIT = "TOPS"
 WORKLOAD_NAMES = {
     "pixart": "pixart_sigma_1024px_denoise_step",
@@ -689,8 +698,7 @@ def main():
     gemm_total_ms = sum(gemm_ms)
     achieved = step.ops / (gemm_total_ms * 1e-3) / 1e12
     peak = peaks["bf16_sus"]
-    tr = TRAFFIC.get(args.workload)
-    traffic = tr["bytes_per_launch"] if tr and tr["sources_sha256"] == kernel_sources_sha256() else None
+    traffic = measured_traffic(args.workload)
     alg_bytes = step.gemm_bytes() / len(step.layers)
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "traffic": traffic, "algorithmic_bytes_per_launch": alg_bytes,
