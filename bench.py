@@ -12,8 +12,11 @@ Default workload: the PixArt-Sigma-shaped DiT at 1024 px (224 layers, 4096
 image tokens, 300 text tokens, 20 stages, learned-style schedule).  The JSON
 line reports throughput in int8-equivalent TOPS (2*M*N*K per layer call,
 independent of b), ms per step, the same step under the all-8-bit schedule,
-the roofline of the dominant kernel, an end-to-end figure through the C ABI
-with host buffers, and the CPU oracle's throughput on a bounded sample.
+the roofline of the dominant kernel (from a replay of the step's launch
+sequence with only its contractions), an end-to-end figure through the C ABI
+with host buffers, and the CPU oracle's throughput on a bounded sample.  The
+other workloads (SANA-1.6B, SDXL-Turbo, the single 256x1152x1152 layer) are
+measured the same way in the same run, under "per_workload".
 
 --impl reference times the CPU oracle (the reference arm of this repository)
 on a bounded sample of the same workload, on the host cores.
@@ -36,11 +39,11 @@ import numpy as np
 
 METRIC = "masked W8A8 GEMM TOPS and % int8 tensor peak vs effective bits b; ms/denoise step"
 
-# DRAM bytes (read + write) per masked-contraction launch, averaged over the 224
-# launches of one PixArt-Sigma step, from one `ncu --metrics dram__bytes_read.sum,
-# dram__bytes_write.sum` capture (profiles/launch_list_pixart_sigma_step.md).  It
-# describes only the kernel sources it was measured on, identified by their SHA-256;
-# after any change to them the field reads null until the capture is repeated.
+# DRAM bytes (read + write) per masked-contraction launch of one workload, from one
+# `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` capture of the
+# contraction kernel.  It describes only the kernel sources it was measured on,
+# identified by their SHA-256; after any change to them the field reads null until
+# the capture is repeated.
 TRAFFIC = {"pixart": {"bytes_per_launch": 13552103,
                       "sources_sha256": "0f39c01cecb26ec53a3e3a85adeb6e5e983fff26bfd7a555d90c45588c25526a"}}
 KERNEL_SOURCES = ("gemm_tc.cu", "tc_ptx.cuh", "tasq_internal.cuh")
@@ -88,6 +91,8 @@ def parse_args():
     ap.add_argument("--blocks", type=int, default=0, help="keep only the first N transformer blocks (small cases)")
     ap.add_argument("--no-all8", action="store_true", help="skip the all-8-bit schedule comparison")
     ap.add_argument("--no-sweep", action="store_true", help="skip the GEMM sweep and the stage-switch test")
+    ap.add_argument("--no-per-workload", action="store_true",
+                    help="time only --workload, not the other workloads of the suite")
     return ap.parse_args()
 
 
@@ -196,35 +201,29 @@ class Step:
         self.gemm_ops = [l.ops for l in self.layers]
         self.conv = workloads.CONV3X3
 
-    def launch(self, events=None):
-        """Enqueue one step on the current stream (stage read from d_stage)."""
+    def launch(self, parts=("quant", "gemm")):
+        """Enqueue one step on the current stream (stage read from d_stage).
+        parts: which kernels of each layer to enqueue (the quantization, the
+        contraction, or both, in the step's order)."""
         for i in range(len(self.layers)):
-            self.launch_layer(i, events)
+            self.launch_layer(i, parts)
 
-    def launch_layer(self, i, events=None):
+    def launch_layer(self, i, parts=("quant", "gemm")):
         """Enqueue layer i (quantization + masked contraction) on the current stream."""
         t = self.tasq
         l = self.layers[i]
-        if l.kind == self.conv:
-            if events:
-                events[i][2].record()
-            t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.Cin, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TENSOR,
+        conv = l.kind == self.conv
+        if "quant" in parts:
+            gran = t.TASQ_PER_TENSOR if conv else t.TASQ_PER_TOKEN
+            t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.Cin if conv else l.K, 8, t.TASQ_SYMRANGE, gran,
                              self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
-            if events:
-                events[i][0].record()
-            t.tasq_masked_conv3x3(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B, l.H,
-                                  l.W, l.Cin, self.packed[i], l.N, self.y[i], None)
-        else:
-            if events:
-                events[i][2].record()
-            t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.K, 8, t.TASQ_SYMRANGE, t.TASQ_PER_TOKEN,
-                             self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
-            if events:
-                events[i][0].record()
-            t.tasq_masked_gemm(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
-                               self.packed[i], l.N, l.K, self.y[i], None)
-        if events:
-            events[i][1].record()
+        if "gemm" in parts:
+            if conv:
+                t.tasq_masked_conv3x3(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B, l.H,
+                                      l.W, l.Cin, self.packed[i], l.N, self.y[i], None)
+            else:
+                t.tasq_masked_gemm(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
+                                   self.packed[i], l.N, l.K, self.y[i], None)
 
     def launches_per_step(self):
         """Kernels the library enqueues for one step, counted by the library itself
@@ -237,33 +236,30 @@ class Step:
         return self._launches
 
     def act_bytes(self):
-        """HBM bytes of activation quantization per step (bf16 in, fp16 codes out, scales)."""
-        return sum(l.M * (l.Cin if l.Cin else l.K) * 4 + 8 * l.M for l in self.layers)
+        """Algorithmic HBM bytes of activation quantization per step: bf16 in,
+        one byte per code out (an int8 code; the tensor-core route holds it in
+        fp16, which doubles the bytes actually written), 8 bytes of scales per
+        token (per-tensor: per tensor)."""
+        return sum(l.M * (l.Cin if l.Cin else l.K) * 3 + 8 * l.M for l in self.layers)
 
     def gemm_bytes(self):
-        """Algorithmic HBM bytes of the contractions per step: fp16 codes in, int8 weights,
-        bf16 out, per-channel and per-token scalars."""
+        """Algorithmic HBM bytes of the contractions per step: int8 activation codes
+        (M K), int8 weights (N K), bf16 output (2 M N), per-token scales (8 M) and
+        per-channel scale, bias and the seven row sums (4 N (2 + 7))."""
         tot = 0
         for l in self.layers:
             k_in = l.Cin if l.Cin else l.K
-            tot += l.M * k_in * 2 + l.N * l.K + 2 * l.M * l.N + 12 * l.N + 8 * l.M
+            tot += l.M * k_in + l.N * l.K + 2 * l.M * l.N + 8 * l.M + 36 * l.N
         return tot
 
     def close(self):
         self.tasq.tasq_destroy(self.ctx)
 
 
-def make_events(torch, n, external):
-    kw = dict(enable_timing=True)
-    if external:
-        kw["external"] = True
-    return [(torch.cuda.Event(**kw), torch.cuda.Event(**kw), torch.cuda.Event(**kw)) for _ in range(n)]
-
-
-def capture(torch, step, events=None):
+def capture(torch, step, parts=("quant", "gemm")):
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, capture_error_mode="thread_local"):
-        step.launch(events)
+        step.launch(parts)
     return g
 
 
@@ -565,6 +561,156 @@ def job_tops(ops_per_rank: float, world: int, ms: float) -> float:
 
 
 # ------------------------------------------------------------------- main --
+# Denoising steps of the trajectory each workload's stages partition (stage of
+# step t = floor(t S / T), stage 0 the noisiest): 20 for the DiTs, 4 for the
+# distilled UNet; the single layer runs its 4 stages once each.
+TRAJECTORY_STEPS = {"pixart": 20, "sana": 20, "sdxl": 4, "single": 4}
+
+
+def stage_map(name: str, S: int):
+    from paper_2608_03057_gb300 import schedule
+    T = max(TRAJECTORY_STEPS[name], S)
+    return lambda k: schedule.stage_of_step(k % T, T, S)
+
+
+def e2e_measure(torch, tasq, step, n_steps, stage_of, copy_streams=1):
+    """The step end to end through the C ABI with host buffers: each layer's input
+    is copied in from pinned host memory on one stream and its output copied out on
+    another, the layers run in order on the compute stream, so the copies of other
+    layers overlap the kernels.  Everything is captured into one graph."""
+    L = len(step.layers)
+    xh = [x.cpu().pin_memory() for x in step.x]
+    yh = [torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for y in step.y]
+    nc = max(1, copy_streams)
+    sh = [torch.cuda.Stream() for _ in range(nc)]
+    sd = [torch.cuda.Stream() for _ in range(nc)]
+    evx = [torch.cuda.Event() for _ in range(L)]
+    evy = [torch.cuda.Event() for _ in range(L)]
+    fork = torch.cuda.Event()
+    joins = [torch.cuda.Event() for _ in range(2 * nc)]
+
+    def e2e_step():
+        # the stream the kernels go to: under graph capture the capture stream, so
+        # that the copy streams fork from it and join it again and every copy is a
+        # node of the captured step
+        s = torch.cuda.current_stream()
+        fork.record(s)
+        for c in sh + sd:
+            c.wait_event(fork)
+        for i in range(L):
+            with torch.cuda.stream(sh[i % nc]):
+                step.x[i].copy_(xh[i], non_blocking=True)
+                evx[i].record(sh[i % nc])
+            s.wait_event(evx[i])
+            step.launch_layer(i)
+            evy[i].record(s)
+            with torch.cuda.stream(sd[i % nc]):
+                sd[i % nc].wait_event(evy[i])
+                yh[i].copy_(step.y[i], non_blocking=True)
+        for c, j in zip(sh + sd, joins):
+            j.record(c)
+            s.wait_event(j)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    ge = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(ge, capture_error_mode="thread_local"):
+        e2e_step()
+    for k in range(3):  # the first replays of a new graph upload it and touch every pinned page
+        ge.replay()
+    torch.cuda.synchronize()
+    ms = timed_replays(torch, ge, step, n_steps, stage_of)
+    out = {"ms_per_step": ms, "copy_streams_per_direction": nc,
+           "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in xh)),
+           "d2h_bytes_per_step": int(sum(y.numel() * y.element_size() for y in yh))}
+    del xh, yh, ge
+    return out
+
+
+def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None, world=1, clocks=None,
+                     e2e=True, all8=True):
+    """Time one workload's denoising step (CUDA graph of the whole step, the stage
+    from a device int), then the same launch sequence with only its contractions
+    and with only its quantizations, the all-8-bit schedule on the same graph, and
+    the end-to-end step.  Returns the figures and the Step (closed by the caller)."""
+    from paper_2608_03057_gb300 import engine_model, schedule
+    step = Step(torch, tasq, workloads, name, args.seed, args.blocks if name in ("pixart", "sana") else 0)
+    S = step.S
+    stage_of = stage_map(name, S)
+    for k in range(2):  # eager launches first: they set kernel attributes outside any capture
+        step.d_stage.fill_(stage_of(k))
+        step.launch()
+    torch.cuda.synchronize()
+    assert tasq.tasq_device_status(step.ctx) == tasq.TASQ_OK
+    g = capture(torch, step)
+    g_gemm = capture(torch, step, parts=("gemm",))
+    g_quant = capture(torch, step, parts=("quant",))
+    for k in range(max(3, args.warmup)):
+        step.d_stage.fill_(stage_of(k))
+        g.replay()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+    if dist:
+        dist.barrier()
+    ms = timed_replays(torch, g, step, steps, stage_of)
+    clk = clocks.stop() if clocks else None
+    status = tasq.tasq_device_status(step.ctx)
+    if status != tasq.TASQ_OK:
+        raise SystemExit(f"device status {status} after the timed region ({name})")
+    ms = max_over_ranks(torch, dist, ms, "cuda")
+    # the same launch sequence with one kind of kernel left out: each launch still
+    # overlaps the previous one's tail (programmatic dependent launch), as in the step
+    ms_gemm = timed_replays(torch, g_gemm, step, steps, stage_of)
+    ms_quant = timed_replays(torch, g_quant, step, steps, stage_of)
+    L = len(step.layers)
+    ms8 = None
+    if all8:  # the all-8-bit schedule on the same captured graph (the table is re-read on the device)
+        tasq.tasq_set_schedule(step.ctx, workloads.schedule_constant(L, S, 8), L, S)
+        ms8 = timed_replays(torch, g, step, steps, stage_of)
+        tasq.tasq_set_schedule(step.ctx, step.table, L, S)
+    assert tasq.tasq_device_status(step.ctx) == tasq.TASQ_OK
+    e2e_out = None
+    if e2e:
+        e2e_out = e2e_measure(torch, tasq, step, max(5, steps // 10), stage_of, args.e2e_copy_streams)
+        e2e_out["ms_per_step"] = max_over_ranks(torch, dist, e2e_out["ms_per_step"], "cuda")
+        e2e_out = {"value": job_tops(step.ops, world, e2e_out["ms_per_step"]), "unit": UNIT, **e2e_out}
+    del g, g_gemm, g_quant
+
+    achieved = step.ops / (ms_gemm * 1e-3) / 1e12
+    peak = peaks["bf16"]
+    traffic = measured_traffic(name)
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": traffic, "algorithmic_bytes_per_launch": step.gemm_bytes() / L,
+                "kernel": "gemm_tc_kernel",
+                "peak_source": f"{peaks['src']} bf16 burst (cuBLAS); the fp16 tcgen05 MMA runs at the bf16 rate, "
+                               "and the contraction-only replay lasts well under a second",
+                "timing": "CUDA events around replays of the step's launch sequence with only its contractions "
+                          f"({steps} replays, {L} launches each, every launch overlapping the previous one's tail "
+                          "as in the step); achieved = int8-equivalent ops per step / that time"}
+    if traffic is not None:
+        roofline["traffic_note"] = ("mean DRAM bytes per contraction launch (ncu); inputs just written by the "
+                                    "quantization can stay in L2, so traffic may sit below the algorithmic bytes")
+    act_b = step.act_bytes()
+    bits = step.table.astype(np.float64)
+    ops_w = np.array(step.gemm_ops, np.float64)
+    eff_w = float((bits * ops_w[:, None]).sum() / (ops_w.sum() * S))
+    out = {
+        "workload": WORKLOAD_NAMES[name], "layers": L, "stages": S, "ms_per_step": ms,
+        "value": job_tops(step.ops, world, ms), "unit": UNIT, "ms_per_step_all8": ms8,
+        "effective_w_bits": eff_w, "rel_bitops": schedule.rel_bitops(eff_w, 8),
+        "engine_model_rel_cost": engine_model.schedule_cost(step.table, step.gemm_ops, 8),
+        "roofline": roofline,
+        "roofline_quant_act": {"bound": "hbm", "bytes_per_step": act_b, "achieved": act_b / (ms_quant * 1e-3) / 1e9,
+                               "peak": peaks["hbm"], "unit": "GB/s",
+                               "frac": act_b / (ms_quant * 1e-3) / 1e9 / peaks["hbm"], "ms_per_step": ms_quant,
+                               "bytes": "bf16 in, one byte per code out, 8 B of scales per group"},
+        "step_breakdown_ms": {"contractions_only": ms_gemm, "quantizations_only": ms_quant, "timed_step": ms},
+        "e2e": e2e_out, "clocks": clk,
+    }
+    return out, step
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -582,147 +728,36 @@ def main():
         dist.init_process_group("nccl")
     peaks = load_peaks()
 
-    step = Step(torch, tasq, workloads, args.workload, args.seed, args.blocks)
-    S = step.S
-    stage_of = lambda k: k % S
+    clocks = ClockSampler(local) if rank == 0 else None
+    head, step = measure_workload(torch, tasq, workloads, args.workload, args, peaks, args.steps, dist, world, clocks,
+                                  e2e=not args.no_e2e, all8=not args.no_all8)
+    launches = step.launches_per_step()
+    step.close()
+    del step
+    torch.cuda.empty_cache()
 
-    # eager warm-up (first launches set kernel attributes), then capture
-    for k in range(2):
-        step.d_stage.fill_(stage_of(k))
-        step.launch()
-    torch.cuda.synchronize()
-    assert tasq.tasq_device_status(step.ctx) == tasq.TASQ_OK
-    # the timed graph holds only the kernels (event nodes between kernels would
-    # block programmatic dependent launch); a second capture of the same launch
-    # sequence with an event around every kernel gives per-kernel durations
-    g = capture(torch, step, None)
-    external = True
-    try:
-        events = make_events(torch, len(step.layers), True)
-        g_ev = capture(torch, step, events)
-    except (TypeError, RuntimeError):
-        external = False
-        events = None
-    for k in range(args.warmup):
-        step.d_stage.fill_(stage_of(k))
-        g.replay()
-    torch.cuda.synchronize()
-
-    clocks = ClockSampler(local)
-    if rank == 0:
-        clocks.start()
-    if dist:
-        dist.barrier()
-    ms = timed_replays(torch, g, step, args.steps, stage_of)
-    clk = clocks.stop() if rank == 0 else None
-    status = tasq.tasq_device_status(step.ctx)
-    if status != tasq.TASQ_OK:
-        raise SystemExit(f"device status {status} after the timed region")
-
-    # per-kernel durations of the last timed replay
-    if external:  # instrumented replays right after the timed region
-        for k in range(3):
-            step.d_stage.fill_(stage_of(args.steps + k))
-            g_ev.replay()
-        torch.cuda.synchronize()
-    else:  # eager pass with events around each kernel
-        events = make_events(torch, len(step.layers), False)
-        step.d_stage.fill_(stage_of(args.steps - 1))
-        step.launch(events)
-        torch.cuda.synchronize()
-    gemm_ms = [events[i][0].elapsed_time(events[i][1]) for i in range(len(step.layers))]
-    quant_ms = [events[i][2].elapsed_time(events[i][0]) for i in range(len(step.layers))]
-
-    ms = max_over_ranks(torch, dist, ms, "cuda")
-    value = job_tops(step.ops, world, ms)
-
-    # the all-8-bit schedule on the same captured graph (same table buffer)
-    L = len(step.layers)
-    ms8 = None
-    if not args.no_all8:
-        tasq.tasq_set_schedule(step.ctx, workloads.schedule_constant(L, S, 8), L, S)
-        ms8 = timed_replays(torch, g, step, max(10, args.steps // 2), stage_of)
-        tasq.tasq_set_schedule(step.ctx, step.table, L, S)
-
-    # end to end through the C ABI with host buffers: each layer's input is copied in
-    # on one stream, its output copied out on another, the layers run in order on the
-    # compute stream, so the copies of other layers overlap the kernels
-    e2e = None
-    if not args.no_e2e:
-        xh = [x.cpu().pin_memory() for x in step.x]
-        yh = [torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for y in step.y]
-        nc = max(1, args.e2e_copy_streams)
-        sh = [torch.cuda.Stream() for _ in range(nc)]
-        sd = [torch.cuda.Stream() for _ in range(nc)]
-        evx = [torch.cuda.Event() for _ in range(L)]
-        evy = [torch.cuda.Event() for _ in range(L)]
-        fork = torch.cuda.Event()
-        joins = [torch.cuda.Event() for _ in range(2 * nc)]
-
-        def e2e_step():
-            # the stream the kernels go to: under graph capture the capture stream, so
-            # that the copy streams fork from it and join it again and every copy is a
-            # node of the captured step
-            s = torch.cuda.current_stream()
-            fork.record(s)
-            for c in sh + sd:
-                c.wait_event(fork)
-            for i in range(L):
-                with torch.cuda.stream(sh[i % nc]):
-                    step.x[i].copy_(xh[i], non_blocking=True)
-                    evx[i].record(sh[i % nc])
-                s.wait_event(evx[i])
-                step.launch_layer(i)
-                evy[i].record(s)
-                with torch.cuda.stream(sd[i % nc]):
-                    sd[i % nc].wait_event(evy[i])
-                    yh[i].copy_(step.y[i], non_blocking=True)
-            for c, j in zip(sh + sd, joins):
-                j.record(c)
-                s.wait_event(j)
-        e2e_step()
-        torch.cuda.synchronize()
-        ge = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(ge, capture_error_mode="thread_local"):
-            e2e_step()
-        n_e2e = max(5, args.steps // 10)
-        ms_e2e = timed_replays(torch, ge, step, n_e2e, stage_of)
-        ms_e2e = max_over_ranks(torch, dist, ms_e2e, "cuda")
-        e2e = {"value": job_tops(step.ops, world, ms_e2e), "unit": UNIT,
-               "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in xh)),
-               "d2h_bytes_per_step": int(sum(y.numel() * y.element_size() for y in yh)),
-               "copy_streams_per_direction": nc,
-               "ms_per_step": ms_e2e}
-        del xh, yh, ge
-
-    gemm_total_ms = sum(gemm_ms)
-    achieved = step.ops / (gemm_total_ms * 1e-3) / 1e12
-    peak = peaks["bf16_sus"]
-    traffic = measured_traffic(args.workload)
-    alg_bytes = step.gemm_bytes() / len(step.layers)
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                "traffic": traffic, "algorithmic_bytes_per_launch": alg_bytes,
-                "traffic_note": "mean DRAM bytes per contraction launch (ncu); inputs just written by the "
-                                "quantization stay in L2 and outputs leave L2 after the kernel, so traffic sits "
-                                "below the algorithmic bytes",
-                "kernel": "gemm_tc_kernel",
-                "peak_source": f"{peaks['src']} bf16 sustained (fp16 MMA runs at the bf16 rate)",
-                "timing": "CUDA events around each contraction in a replay of the step with event nodes "
-                          "between kernels, right after the timed region" if external
-                else "CUDA events around each contraction in an eager pass after the timed region"}
+    # the other workloads of the benchmark suite, each a full step of its own
+    per_workload = {}
+    if not args.no_per_workload:
+        for name in WORKLOAD_NAMES:
+            if name == args.workload:
+                continue
+            r, st = measure_workload(torch, tasq, workloads, name, args, peaks, max(10, min(args.steps, 50)), dist,
+                                     world, None, e2e=not args.no_e2e, all8=not args.no_all8)
+            st.close()
+            del st
+            torch.cuda.empty_cache()
+            per_workload[name] = r
 
     sweep = switch = zp = i8 = None
     if not args.no_sweep:
         sweep, switch = run_sweep(torch, tasq, workloads, seed=args.seed)
         zp = run_zero_point(torch, tasq, workloads, seed=args.seed)
-        # int8 tensor reference: the best int8 GEMM measured on this GPU (the library
-        # int8 GEMM, and this library's own mma.sync s8 route)
-        lt = int8_tensor_peak(torch)
-        s8 = s8_route_tops(torch, tasq, workloads)
-        best = max(x for x in (lt["tops"], s8["tops"]) if x)
-        i8 = {"tops": best, "source": "best measured int8 GEMM on this GPU",
-              "cublaslt_int8_gemm": lt, "mma_sync_s8_route": s8,
-              "step_pct": 100.0 * value / best}  # this step's int8-equivalent TOPS against it
+        # int8 GEMMs measured on this GPU, for context: the library int8 GEMM and this
+        # library's own mma.sync s8 route (sm_103a has no tcgen05 int8 kind)
+        i8 = {"cublaslt_int8_gemm": int8_tensor_peak(torch), "mma_sync_s8_route": s8_route_tops(torch, tasq, workloads),
+              "note": "context only; the contraction runs on the fp16 tcgen05 kind, whose peak is the "
+                      "measured bf16 cuBLAS rate"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -734,43 +769,38 @@ def main():
                                 "sample": f"{rows1} token rows of each of the first {d1} layers ({s1:.1f} s)"}
 
     if rank == 0:
-        bits = step.table.astype(np.float64)
-        ops_w = np.array(step.gemm_ops, np.float64)
-        eff_w = float((bits * ops_w[:, None]).sum() / (ops_w.sum() * S))
+        route_peak = {"tflops": peaks["bf16"], "source": f"{peaks['src']} bf16 cuBLAS burst",
+                      "step_frac": head["value"] / peaks["bf16"],
+                      "contractions_frac": head["roofline"]["frac"]}
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f16-exact-int8", "data": "synthetic",
-            "config": {"workload": WORKLOAD_NAMES[args.workload], "layers": L, "stages": S,
-                       "schedule": "seeded learned-style per-(layer, stage) bits", "effective_w_bits": eff_w,
-                       "rel_bitops": eff_w * 8 / 64, "route": "tcgen05 fp16 MMA, exact int32",
+            "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": head["ms_per_step"], "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f16-exact-int8", "data": "synthetic",
+            "config": {"workload": head["workload"], "layers": head["layers"], "stages": head["stages"],
+                       "schedule": "seeded learned-style per-(layer, stage) bits",
+                       "effective_w_bits": head["effective_w_bits"], "rel_bitops": head["rel_bitops"],
+                       "route": "tcgen05 fp16 MMA, exact int32",
                        "activations": "bf16 in HBM, per-token int8 codes held as fp16",
                        "l2": "inputs larger than L2 (per-step activations and weights exceed 129 MB)",
                        "graph": "whole step captured once; stage from a device int",
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
-            "ms_per_step_all8": ms8,
-            "roofline": roofline,
-            "roofline_quant_act": {"bound": "hbm", "bytes_per_step": step.act_bytes(),
-                                   "achieved": step.act_bytes() / (sum(quant_ms) * 1e-3) / 1e9,
-                                   "peak": peaks["hbm"], "unit": "GB/s",
-                                   "frac": step.act_bytes() / (sum(quant_ms) * 1e-3) / 1e9 / peaks["hbm"],
-                                   "ms_per_step": sum(quant_ms)},
-            "step_breakdown_ms": {"contractions": sum(gemm_ms), "act_quant": sum(quant_ms),
-                                  "timed_step": ms,
-                                  "note": "per-kernel sums come from the instrumented replay, where kernels "
-                                          "cannot overlap; the timed step lets each launch overlap the "
-                                          "previous kernel's tail"},
-            "e2e": e2e,
-            "gpu_launches": step.launches_per_step() * args.steps,
+            "ms_per_step_all8": head["ms_per_step_all8"],
+            "roofline": head["roofline"],
+            "roofline_quant_act": head["roofline_quant_act"],
+            "step_breakdown_ms": head["step_breakdown_ms"],
+            "engine_model_rel_cost": head["engine_model_rel_cost"],
+            "e2e": head["e2e"],
+            "gpu_launches": launches * args.steps,
             "cpu_baseline": cpu,
-            "clocks": clk,
+            "clocks": head["clocks"],
+            "route_peak": route_peak,
+            "per_workload": per_workload,
             "sweep_tops_by_b": sweep,
             "stage_switch": switch,
             "asym_weights": zp,
-            "int8_tensor_peak": i8,
+            "int8_gemm_context": i8,
         }
         print(json.dumps(line), flush=True)
-    step.close()
     if dist:
         dist.barrier()
         dist.destroy_process_group()

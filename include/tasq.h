@@ -101,8 +101,9 @@ typedef void* tasq_stream; /* cudaStream_t */
 int tasq_version(void);
 
 /* Create a context on CUDA device `device`.  Set-up call: allocates the
- * context's device status word, its reduction scratch and the tensor-core
- * route's accumulator scratch (96 KB per SM: about 14.6 MB on a GB300), and
+ * context's device status word, its reduction scratch, the bit table (room
+ * for 65,536 entries), the tensor-core route's accumulator scratch (96 KB per
+ * SM: about 14.6 MB on a GB300) and its split-K partial sums (32 MB), and
  * leaves the calling thread's current device unchanged.  *out is NULL on
  * failure. */
 int tasq_create(tasq_ctx* out, int device);
@@ -225,8 +226,16 @@ int tasq_pack_weights_zp(tasq_ctx ctx, int kind, const int8_t* d_sw, const float
 
 /*
  * Bit-allocation map (App. F.1): h_bits [L][S] uint8, each value in 2..8,
- * copied into device memory owned by the context.  Set-up call: allocates
- * (only when L*S grows), copies synchronously, validates every entry first.
+ * copied into device memory owned by the context.  Set-up call: validates
+ * every entry first, synchronizes the device, then copies synchronously.
+ * The context creates its table with room for 65,536 entries; the kernels
+ * read L and S from the device copy, not from their launch arguments, so a
+ * CUDA graph captured before this call runs the new schedule when replayed
+ * (a captured call whose layer or stage falls outside the new L x S records
+ * TASQ_ERR_DEVICE and writes nothing).  Only a schedule with more than
+ * 65,536 entries moves the table to a new buffer; graphs captured before
+ * that call keep reading the old buffer, which stays allocated, unchanged,
+ * until tasq_destroy, and must be captured again to see the new schedule.
  * Changing stage afterwards needs no host work: it is an argument of the
  * next call, or a device int (tasq_set_stage_device).
  */
@@ -393,7 +402,10 @@ int tasq_plan_tc(int kind, int M, int N, int K, int B, int H, int W, int Cin, in
  *    tensors return TASQ_ERR_UNSUPPORTED without launching anything.
  *  - The first call on a device looks up the array's device address once
  *    (cudaGetSymbolAddress, with that device current); make that first call
- *    before capturing a stream into a CUDA graph.
+ *    before capturing a stream into a CUDA graph.  The address is kept for
+ *    the life of the process: it does not survive cudaDeviceReset (or any
+ *    other reset of the device's primary context), after which this call
+ *    must not be used in that process.
  *  - Every call uses the same array, and each call rewrites the slots it
  *    reads, so nothing carries over between calls; but calls whose kernels
  *    overlap on the GPU (different streams, or one device used from several

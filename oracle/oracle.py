@@ -274,12 +274,6 @@ def linear_layer(x, w_s, c_w, bias, b, n_bits=8, mode=SYMRANGE):
     return dict(s_x=s_x, alpha=alpha, zc=zc, acc=acc, rs=rs, y=y, y_bf16=yb)
 
 
-def stage_of_step(step, n_steps, n_stages):
-    """Contiguous partition of the trajectory into stages (Sec. 3.2, stage-wise
-    sharing): stage = floor(step * S / T), stage 0 = the noisiest steps."""
-    return (step * n_stages) // n_steps
-
-
 def conv3x3_code_sums(s_x_nhwc):
     """Per output pixel: (sxw, Kv) = (sum of the in-bounds taps' input codes, Cin x in-bounds taps)."""
     s_x = _c(s_x_nhwc, np.int8)

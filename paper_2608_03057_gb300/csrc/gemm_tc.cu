@@ -46,45 +46,6 @@
 #include "tasq_internal.cuh"
 #include "tc_ptx.cuh"
 
-// Optional per-role timestamps of CTA 0 (build with -DTASQ_TRACE; compiled
-// out otherwise): role 0 producer, 1 MMA, 2 converter warp, 3 epilogue warp.
-// TE(ev) records, for every CTA, the global time (ns) and SM clock of one
-// event of its timeline: 0 entry, 1 set-up done, 2 inputs released (producer),
-// 3 first stage landed (converter), 4 first MMA issued, 5 last MMA committed,
-// 6 first accumulator ready, 7 last accumulator ready, 8 epilogue done,
-// 9 producer done, 10 exit.
-#ifdef TASQ_TRACE
-__device__ unsigned long long g_tasq_trace[4][256][8];
-__device__ unsigned long long g_tasq_ev[512][12][2];
-#define TQ(role, it, k)                                                          \
-    do {                                                                         \
-        if (blockIdx.x == 0 && (it) < 256) g_tasq_trace[role][it][k] = clock64(); \
-    } while (0)
-#define TE(ev)                                                    \
-    do {                                                          \
-        if (blockIdx.x < 512) {                                   \
-            g_tasq_ev[blockIdx.x][ev][0] = ptx::globaltimer();    \
-            g_tasq_ev[blockIdx.x][ev][1] = clock64();             \
-        }                                                         \
-    } while (0)
-// TF(call, k): steps of the epilogue's 16-column finishing of CTA 0, warp 6
-__device__ unsigned long long g_tasq_fin[64][8];
-#define TF(call, k)                                                                      \
-    do {                                                                                 \
-        if (blockIdx.x == 0 && warp == 6 && lane == 0 && (call) < 64) g_tasq_fin[call][k] = clock64(); \
-    } while (0)
-#else
-#define TQ(role, it, k) \
-    do {                \
-    } while (0)
-#define TE(ev) \
-    do {       \
-    } while (0)
-#define TF(call, k) \
-    do {            \
-    } while (0)
-#endif
-
 namespace tasq {
 namespace {
 
@@ -287,7 +248,6 @@ __global__ void __maxnreg__(96)
     constexpr int X_STAGES = C::X_STAGES, X_HALF = C::X_HALF, X_STAGE = C::X_STAGE, NACC = C::NACC;
     constexpr int Q = C::Q, DONE = C::DONE;
     constexpr int BT = C::BT, GPW = C::GPW;
-    if (threadIdx.x == 0) TE(0);
     extern __shared__ uint8_t smem_raw[];
     Smem<C>* s = reinterpret_cast<Smem<C>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const GemmArgs& a = p.a;
@@ -342,7 +302,6 @@ __global__ void __maxnreg__(96)
         if (warp == 1) ptx::tmem_dealloc(tmem, TMEM_COLS);
         return;
     }
-    if (threadIdx.x == 0) TE(1);
     if (warp == WPROD_WARP && lane == 0 && unit < works) {
         // pull the first weight tiles into L2 ahead of the weight ring
         const Work wk = work_item(p, unit, KT, chunk);
@@ -360,19 +319,16 @@ __global__ void __maxnreg__(96)
         // --------------------------------------------- activation producer
         if (lane == 0) {
             ptx::grid_dependency_wait();
-            TE(2);
             int u = 0;  // activation stages issued by this CTA
             bool ok = true;
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
                 const TileCoord tc = tile_coord<CONV, BT>(p, wk.t);
                 for (int kq = wk.kb_lo * Q; kq < wk.kb_hi * Q; ++kq, ++u) {
-                    TQ(0, u, 0);
                     if (u >= X_STAGES && !wt.wait(&s->done[(u - X_STAGES) % DONE], ((u - X_STAGES) / DONE) & 1)) {
                         ok = false;
                         break;
                     }
-                    TQ(0, u, 1);
                     const uint32_t fb = ptx::smem_u32(&s->xfull[u % X_STAGES]);
                     ptx::mbar_arrive_expect_tx(fb, X_STAGE);
                     const uint32_t dst = ptx::smem_u32(s->x[u % X_STAGES]);
@@ -390,7 +346,6 @@ __global__ void __maxnreg__(96)
                     }
                 }
             }
-            TE(9);
             // the next kernel may be launched while this grid drains
             ptx::grid_launch_dependents();
             // copies still in flight must land before the CTA may exit: the MMAs
@@ -437,7 +392,6 @@ __global__ void __maxnreg__(96)
                     const uint32_t d = tmem + C::ACC_COL + buf * BT;
                     const int kb0 = wk.kb_lo + c * chunk, kb_end = min(wk.kb_hi, kb0 + chunk);
                     for (int kb = kb0; kb < kb_end && ok; ++kb, ++it) {
-                        TQ(1, it, 0);
                         const uint32_t acol = tmem + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
                         for (int i = 0; i < Q; ++i) {
                             const int u = it * Q + i;
@@ -447,8 +401,6 @@ __global__ void __maxnreg__(96)
                                 break;
                             }
                             ptx::tc_fence_after();
-                            if (i == 0) TQ(1, it, 1);
-                            if (it == 0 && i == 0) TE(4);
                             for (int hh = 0; hh < 2 / Q; ++hh) {
                                 // one 64-wide swizzle atom; a K step of 16 codes is 32 bytes along its rows
                                 const uint64_t bdesc =
@@ -460,13 +412,10 @@ __global__ void __maxnreg__(96)
                             }
                             ptx::mma_commit(ptx::smem_u32(&s->done[u % DONE]));
                         }
-                        TQ(1, it, 2);
-                        TQ(1, it, 3);
                     }
                     if (ok) ptx::mma_commit(ptx::smem_u32(&s->accfull[buf]));
                 }
             }
-            TE(5);
             // every MMA issued must finish before tensor memory is released
             ptx::mma_commit(ptx::smem_u32(&s->drain));
             wt.wait(&s->drain, 0, true);
@@ -483,13 +432,10 @@ __global__ void __maxnreg__(96)
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
             for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rw.next()) {
-                if (warp == 2 && lane == 0) TQ(2, it, 0);
                 if (!wt.wait(&s->wfull[rw.slot], rw.phase)) {
                     ok = false;
                     break;
                 }
-                if (warp == 2 && lane == 0) TQ(2, it, 1);
-                if (warp == 2 && lane == 0 && it == 0) TE(3);
                 // 128 codes of row r; 16-byte chunk c sits at c ^ (r & 7) (128-byte swizzle).
                 // Mask and widen before waiting for the slot, so that only the
                 // tensor-memory store remains once the MMA releases it.
@@ -507,7 +453,6 @@ __global__ void __maxnreg__(96)
                 }
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->wempty[rw.slot]));
-                if (warp == 2 && lane == 0) TQ(2, it, 2);
                 // slot it % 2 last held K block it - 2: its MMAs must have finished
                 // (the last activation stage of block it - 2 completes after all its MMAs)
                 if (it >= ASLOTS && !wt.wait(&s->done[((it - ASLOTS) * Q + Q - 1) % DONE],
@@ -515,7 +460,6 @@ __global__ void __maxnreg__(96)
                     ok = false;
                     break;
                 }
-                if (warp == 2 && lane == 0) TQ(2, it, 3);
                 {
                     const uint32_t dst = lane_base + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
                     ptx::tmem_st32(dst, *reinterpret_cast<const uint32_t(*)[32]>(&f[0]));
@@ -525,7 +469,6 @@ __global__ void __maxnreg__(96)
                 ptx::tc_fence_before();
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->xfull[(it * Q) % X_STAGES]));
-                if (warp == 2 && lane == 0) TQ(2, it, 5);
             }
         }
     }
@@ -548,9 +491,6 @@ __global__ void __maxnreg__(96)
         const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
         constexpr bool zp = ZP;  // asymmetric weights: the four-term epilogue
         int cc = 0;
-#ifdef TASQ_TRACE
-        int fcall = 0;
-#endif
         bool ok = true;
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
@@ -640,7 +580,6 @@ __global__ void __maxnreg__(96)
             // FL: the accumulator values are float-held integers (single-chunk tiles), else int32
             auto finish16 = [&](int gi, int j0, const uint32_t (&v)[16], auto fl_tag, bool all_tok) {
                 constexpr bool fl = decltype(fl_tag)::value;
-                TF(fcall, 0);
                 [[maybe_unused]] const int g = part * gpw + gi;
                 const float* my_al = s->ep_al[e][gi];
                 const float* my_zc = s->ep_zc[e][gi];
@@ -683,19 +622,16 @@ __global__ void __maxnreg__(96)
                         yb2[2 * j4 + u / 2] = *reinterpret_cast<const uint32_t*>(&hb);
                     }
                 }
-                TF(fcall, 1);
                 // Transpose the warp's 32 channels x 16 tokens through shared memory:
                 // a [16 tokens][32 channels] bf16 box (64-byte rows).
                 // (convolutions only: linear layers finish in finish16f)
                 uint16_t* stg = s->ep_stage[e];
                 __syncwarp();
-                TF(fcall, 2);
 #pragma unroll
                 for (int j = 0; j < 16; ++j) stg[j * 32 + lane] = uint16_t(yb2[j >> 1] >> (16 * (j & 1)));
                 {
                     // the box's pixels need not be consecutive rows of y: 16-byte stores
                     __syncwarp();
-                    TF(fcall, 3);
                     const int qc = lane & 3;  // 8-channel chunk of the row
                     const int nq = tc.ch0 + (warp & 3) * 32 + qc * 8;
 #pragma unroll
@@ -707,10 +643,6 @@ __global__ void __maxnreg__(96)
                     }
                     __syncwarp();  // the box is read before the next one is written
                 }
-                TF(fcall, 4);
-#ifdef TASQ_TRACE
-                ++fcall;
-#endif
                 if (a.acc && n_ok) {  // int32 accumulators (a debugging output): plain stores
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
@@ -809,14 +741,10 @@ __global__ void __maxnreg__(96)
             int32_t* my_part = a.part + (int64_t(blockIdx.x) * EPI_WARPS + (e < EPI_WARPS ? e : 0)) * (MAX_GPW * 32 * 32) + lane;
             for (int c = 0; c < nchunks; ++c, ++cc) {
                 const int buf = cc % NACC;
-                if (warp == 6 && lane == 0) TQ(3, cc, 0);
                 if (!wt.wait(&s->accfull[buf], (cc / NACC) & 1)) {
                     ok = false;
                     break;
                 }
-                if (warp == 6 && lane == 0) TQ(3, cc, 1);
-                if (warp == 6 && lane == 0 && cc == 0) TE(6);
-                if (warp == 6 && lane == 0) TE(7);
                 ptx::tc_fence_after();
                 const uint32_t acc_base = lane_base + C::ACC_COL + buf * BT;
                 const bool last = c == nchunks - 1;
@@ -847,7 +775,6 @@ __global__ void __maxnreg__(96)
                                 else pp[j * 32] = x;
                             }
                         }
-                        if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 3 + 2 * h);
                         if (last && p.splits > 1) {
                             // exact int32 partial sums of this K slice, one coalesced
                             // 128-byte row per token
@@ -870,25 +797,21 @@ __global__ void __maxnreg__(96)
                                 else finish16(gi, h * 16, v, std::false_type{}, all_tok);
                             }
                         }
-                        if (warp == 6 && lane == 0 && gi == 0) TQ(3, cc, 4 + 2 * h);
                     }
                 }
                 ptx::tc_fence_before();
                 __syncwarp();
                 // (helper converter warps only join the tile's single chunk: nothing waits for them)
                 if (lane == 0 && e < EPI_WARPS) ptx::mbar_arrive(ptx::smem_u32(&s->accempty[buf]));
-                if (warp == 6 && lane == 0) TQ(3, cc, 2);
             }
         }
     }
 
-    if (warp == 6 && lane == 0) TE(8);
     // epilogue TMA stores complete before the CTA exits
     if (!CONV && lane == 0 &&
         ((warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS) || (helpers && warp >= 2 && warp < EPI_WARP0)))
         ptx::bulk_wait0();
     __syncthreads();
-    if (threadIdx.x == 0) TE(10);
     if (warp == 1) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, TMEM_COLS);
@@ -1222,17 +1145,5 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
     if (plan.bt == CfgNarrow::BT) return launch_cfg<CfgNarrow>(a, plan, st, why, kernels);
     return launch_cfg<CfgStd>(a, plan, st, why, kernels);
 }
-
-#ifdef TASQ_TRACE
-extern "C" __attribute__((visibility("default"))) int tasq_debug_trace(void* host, size_t bytes) {
-    return (int)cudaMemcpyFromSymbol(host, g_tasq_trace, bytes < sizeof(g_tasq_trace) ? bytes : sizeof(g_tasq_trace));
-}
-extern "C" __attribute__((visibility("default"))) int tasq_debug_fin(void* host, size_t bytes) {
-    return (int)cudaMemcpyFromSymbol(host, g_tasq_fin, bytes < sizeof(g_tasq_fin) ? bytes : sizeof(g_tasq_fin));
-}
-extern "C" __attribute__((visibility("default"))) int tasq_debug_events(void* host, size_t bytes) {
-    return (int)cudaMemcpyFromSymbol(host, g_tasq_ev, bytes < sizeof(g_tasq_ev) ? bytes : sizeof(g_tasq_ev));
-}
-#endif
 
 }  // namespace tasq

@@ -630,15 +630,19 @@ __global__ void selftest_timeout_kernel(int* status, unsigned long long timeout_
 }
 
 // Counts x / a pairs where the activation quantizer's quotient differs from
-// IEEE division (bit patterns compared).
-__global__ void selftest_quotients_kernel(const float* __restrict__ x, int nx, const float* __restrict__ a, int na,
-                                          unsigned long long* mismatches) {
+// IEEE division (bit patterns compared).  Each thread takes dividends and runs
+// them against every divisor (the divisors are read by all lanes at once).
+__global__ void __launch_bounds__(256) selftest_quotients_kernel(const float* __restrict__ x, int nx,
+                                                                 const float* __restrict__ a, int na,
+                                                                 unsigned long long* mismatches) {
     unsigned long long bad = 0;
-    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < int64_t(nx) * na;
-         i += int64_t(gridDim.x) * blockDim.x) {
-        const float xv = x[i % nx], av = a[i / nx];
-        const float ra = __frcp_rn(av);
-        bad += __float_as_uint(div_rn_by(xv, av, ra)) != __float_as_uint(__fdiv_rn(xv, av));
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < nx; i += int64_t(gridDim.x) * blockDim.x) {
+        const float xv = x[i];
+        for (int j = 0; j < na; ++j) {
+            const float av = a[j];
+            const float ra = __frcp_rn(av);
+            bad += __float_as_uint(div_rn_by(xv, av, ra)) != __float_as_uint(__fdiv_rn(xv, av));
+        }
     }
     for (int o = 16; o; o >>= 1) bad += __shfl_xor_sync(0xffffffffu, bad, o);
     if ((threadIdx.x & 31) == 0 && bad) atomicAdd(mismatches, bad);
@@ -648,7 +652,11 @@ __global__ void selftest_quotients_kernel(const float* __restrict__ x, int nx, c
 
 cudaError_t launch_selftest_quotients(const float* x, int nx, const float* a, int na, unsigned long long* mismatches,
                                       cudaStream_t st) {
-    selftest_quotients_kernel<<<1024, 256, 0, st>>>(x, nx, a, na, mismatches);
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int want = (nx + 255) / 256;
+    selftest_quotients_kernel<<<want < 8 * sms ? want : 8 * sms, 256, 0, st>>>(x, nx, a, na, mismatches);
     return cudaGetLastError();
 }
 

@@ -4,6 +4,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <vector>
 
 #include "tasq_internal.cuh"
 
@@ -15,8 +16,11 @@ struct tasq_ctx_s {
     int* d_words = nullptr;  // [0] status, [16..19] reduction scratch
     int32_t* d_part = nullptr;  // tensor-core route: int32 running sums of multi-chunk tiles
     int32_t* d_split = nullptr;  // tensor-core route: split-K partial sums
+    // bit table: a 16-byte header (int32 L, S) followed by the bits [L][S]; kernels
+    // read L and S from the header, so a captured graph follows later schedules
     uint8_t* d_table = nullptr;
-    size_t table_cap = 0;
+    size_t table_cap = 0;              // bits the current buffer holds
+    std::vector<uint8_t*> old_tables;  // replaced buffers, kept until tasq_destroy
     int L = 0, S = 0;
     const int32_t* d_stage = nullptr;
     int route = TASQ_ROUTE_AUTO;
@@ -96,11 +100,15 @@ TASQ_API int tasq_create(tasq_ctx* out, int device) {
     if (e == cudaSuccess) e = cudaMemset(ctx->d_words, 0, 256);
     if (e == cudaSuccess) e = cudaMalloc(&ctx->d_part, tasq::gemm_tc_part_bytes(ctx->num_sms));
     if (e == cudaSuccess) e = cudaMalloc(&ctx->d_split, tasq::kSplitBufBytes);
+    if (e == cudaSuccess) e = cudaMalloc(&ctx->d_table, tasq::kTableHeader + tasq::kTableCapacity);
+    if (e == cudaSuccess) e = cudaMemset(ctx->d_table, 0, tasq::kTableHeader);  // L = S = 0: no schedule yet
+    if (e == cudaSuccess) ctx->table_cap = tasq::kTableCapacity;
     cudaSetDevice(prev);
     if (e != cudaSuccess) {
         cudaFree(ctx->d_words);
         cudaFree(ctx->d_part);
         cudaFree(ctx->d_split);
+        cudaFree(ctx->d_table);
         delete ctx;
         return fail(nullptr, TASQ_ERR_CUDA, "allocating context buffers: %s", cudaGetErrorString(e));
     }
@@ -118,6 +126,7 @@ TASQ_API void tasq_destroy(tasq_ctx ctx) {
     cudaFree(ctx->d_part);
     cudaFree(ctx->d_split);
     cudaFree(ctx->d_table);
+    for (uint8_t* t : ctx->old_tables) cudaFree(t);
     cudaSetDevice(prev);
     delete ctx;
 }
@@ -258,13 +267,18 @@ TASQ_API int tasq_set_schedule(tasq_ctx ctx, const uint8_t* h_bits, int L, int S
     if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaDeviceSynchronize");
     size_t bytes = (size_t)L * S;
     if (bytes > ctx->table_cap) {
-        cudaFree(ctx->d_table);
-        ctx->d_table = nullptr;
-        ctx->table_cap = 0;
-        if ((e = cudaMalloc(&ctx->d_table, bytes)) != cudaSuccess) return cuda_fail(ctx, e, "allocating the table");
+        // a larger buffer; the old one stays allocated (graphs captured before this
+        // call still name it) until tasq_destroy
+        uint8_t* t = nullptr;
+        if ((e = cudaMalloc(&t, tasq::kTableHeader + bytes)) != cudaSuccess)
+            return cuda_fail(ctx, e, "allocating the table");
+        ctx->old_tables.push_back(ctx->d_table);
+        ctx->d_table = t;
         ctx->table_cap = bytes;
     }
-    if ((e = cudaMemcpy(ctx->d_table, h_bits, bytes, cudaMemcpyHostToDevice)) != cudaSuccess)
+    const int32_t dims[4] = {L, S, 0, 0};
+    if ((e = cudaMemcpy(ctx->d_table + tasq::kTableHeader, h_bits, bytes, cudaMemcpyHostToDevice)) != cudaSuccess ||
+        (e = cudaMemcpy(ctx->d_table, dims, sizeof dims, cudaMemcpyHostToDevice)) != cudaSuccess)
         return cuda_fail(ctx, e, "copying the table");
     ctx->L = L;
     ctx->S = S;
@@ -332,7 +346,7 @@ int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void*
                        const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int M,
                        const void* d_packed, int N, int K, int B, int H, int W, int Cin, uint16_t* d_y,
                        int32_t* d_acc, tasq_stream stream) {
-    REQUIRE(ctx->d_table, TASQ_ERR_INVALID_ARG, "no schedule: call tasq_set_schedule first");
+    REQUIRE(ctx->L > 0, TASQ_ERR_INVALID_ARG, "no schedule: call tasq_set_schedule first");
     REQUIRE(layer >= 0 && layer < ctx->L, TASQ_ERR_INVALID_ARG, "layer %d outside 0..%d", layer, ctx->L - 1);
     REQUIRE(stage >= -1 && stage < ctx->S, TASQ_ERR_INVALID_ARG, "stage %d outside -1..%d", stage, ctx->S - 1);
     REQUIRE(stage >= 0 || ctx->d_stage, TASQ_ERR_INVALID_ARG, "stage -1 needs tasq_set_stage_device");
@@ -365,7 +379,6 @@ int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void*
     a.d_stage = ctx->d_stage;
     a.layer = layer;
     a.stage = stage;
-    a.S = ctx->S;
     a.M = M;
     a.N = N;
     a.K = K;

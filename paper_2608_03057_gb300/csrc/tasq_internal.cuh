@@ -16,6 +16,10 @@ constexpr uint32_t kPackedMagic = 0x51534154u;  // "TASQ"
 constexpr int kBMin = 2, kBMax = 8, kNumB = kBMax - kBMin + 1;
 constexpr int kCertKBlock = 64;   // K block of the exactness certificate (TC route BK)
 constexpr int64_t kCertLimit = int64_t(1) << 17;  // 2^24 / 128: sum |w| bound per chunk
+// Bit table in device memory: a 16-byte header (int32 L, int32 S) then the bits
+// [L][S].  The context allocates room for kTableCapacity bits when it is created.
+constexpr int kTableHeader = 16;
+constexpr size_t kTableCapacity = 65536;
 
 struct PackedHeader {
     uint32_t magic;
@@ -72,9 +76,9 @@ struct GemmArgs {
     const int32_t* rs;        // [kNumB][N]
     const int32_t* ts;        // conv: [kNumB][N][9]
     const PackedHeader* hdr;  // device copy of the header
-    const uint8_t* table;     // [L][S]
+    const uint8_t* table;     // bit table: int32 L, S at offset 0, bits [L][S] at kTableHeader
     const int32_t* d_stage;   // used when stage < 0
-    int layer, stage, S;
+    int layer, stage;
     int M, N, K;
     int B, H, W, Cin;         // conv geometry (Cin == 0 for a linear layer)
     int per_tensor;
@@ -99,8 +103,11 @@ __device__ inline int resolve_bits(const GemmArgs& a) {
     const uint32_t magic = a.hdr->magic;
     const int hdr_n = a.hdr->N, hdr_k = a.hdr->K, hdr_zp = a.hdr->has_zp;
     const int stage = a.stage >= 0 ? a.stage : (a.d_stage ? *a.d_stage : -1);
-    const bool stage_ok = stage >= 0 && stage < a.S;
-    const int b = stage_ok ? a.table[a.layer * a.S + stage] : 0;
+    // the table's dimensions come from the device copy, so a graph captured before a
+    // later tasq_set_schedule reads that schedule's bits (or records the mismatch)
+    const int2 dims = *reinterpret_cast<const int2*>(a.table);
+    const bool stage_ok = stage >= 0 && stage < dims.y && a.layer < dims.x;
+    const int b = stage_ok ? a.table[kTableHeader + a.layer * dims.y + stage] : 0;
     // a buffer packed with zero offsets needs the code sums of the four-term epilogue
     if (!stage_ok || b < kBMin || b > kBMax || magic != kPackedMagic || hdr_n != a.N || hdr_k != a.K ||
         (hdr_zp && !a.code_sums)) {

@@ -807,3 +807,181 @@ def test_quotient_routine_matches_ieee_division(ctx):
     torch.cuda.synchronize()
     assert int(mism.item()) == 0
 
+
+
+def test_quotient_routine_matches_ieee_division_fp32(ctx):
+    """The same quotient routine on fp32 dividends (the per-token quantizer of an
+    fp32 input divides fp32 values): 10^8 seeded random bit patterns with
+    exponents that keep every quotient normal, against the same divisor set as
+    the bf16 test above.  Zero mismatches expected."""
+    torch = G.torch()
+    rng = workloads.rng(5)
+    a = np.concatenate([np.exp2(rng.uniform(-30, 30, 2000)), 2.0 ** np.arange(-30, 31),
+                        rng.uniform(1e-3, 5e-2, 1000)]).astype(np.float32)
+    ad = G.dev(a)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(12)
+    mism = torch.zeros((1,), dtype=torch.int64, device="cuda")
+    total = 0
+    while total < 100_000_000:
+        bits = torch.randint(-(2 ** 31), 2 ** 31 - 1, (30_000_000,), dtype=torch.int32, generator=gen, device="cuda")
+        e = (bits >> 23) & 0xFF
+        xs = bits[(e > 30) & (e < 225)].view(torch.float32).contiguous()
+        tasq.tasq_selftest_quotients(ctx.h, xs, xs.numel(), ad, a.size, mism)
+        total += xs.numel()
+        del bits, e, xs
+    torch.cuda.synchronize()
+    assert total >= 100_000_000
+    assert int(mism.item()) == 0
+
+
+# --------------------------------------- the sweep's shapes, uniform codes --
+
+SWEEP = [(M, KN) for M in (1024, 4096, 16384) for KN in (1152, 2240, 4096)]
+
+
+@pytest.mark.parametrize("M,KN", SWEEP)
+def test_sweep_shapes_uniform_codes(ctx, oracle, M, KN):
+    """The shape sweep at its own shapes: codes uniform in [-127, 127] for
+    activations and weights (sums of |w| far past one fp32-exact chunk), every
+    b = 2..8, on the tensor-core route.  The output is checked on sampled token
+    rows plus the last row, for the call without the int32 debug output (the
+    call the benchmark times) and, with it, the int32 accumulators as well.
+    M = 1024, K = N = 4096 runs the 256-token single-accumulator tiles over
+    several certified chunks."""
+    torch = G.torch()
+    N = K = KN
+    F16 = tasq.TASQ_CODES_F16
+    seed = 1000 + M + KN
+    s_x = workloads.uniform_codes((M, K), seed)
+    s_w = workloads.uniform_codes((N, K), seed + 1)
+    cw = workloads.uniform((N,), seed + 2, 1e-4, 2e-4)
+    bias = workloads.normal((N,), seed + 3, 0.02)
+    alpha = workloads.uniform((M,), seed + 4, 1e-3, 2e-3)
+    zc = workloads.uniform((M,), seed + 5, -0.5, 0.5)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, G.dev(s_w), G.dev(cw), G.dev(bias), N, K)
+    bits = list(range(2, 9))
+    tasq.tasq_set_schedule(ctx.h, np.array([bits], np.uint8), 1, len(bits))
+    codes = G.dev(s_x).to(torch.float16)
+    ad, zd = G.dev(alpha), G.dev(zc)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    plan = tasq.tasq_plan_tc(tasq.TASQ_LINEAR, M, N, K, 0, 0, 0, 0, sms)
+    chunk_kb, _ = G.packed_header(packed)
+    KT = (K + 127) // 128
+    nchunks = {b: -(-KT // max(1, min(KT, int(chunk_kb[b]) // 2))) for b in bits}
+    if (M, KN) == (1024, 4096) and sms >= 128:
+        assert plan["tile_tokens"] == 256 and plan["acc_buffers"] == 1, plan
+        assert nchunks[8] > 1, nchunks
+    rows = np.unique(np.concatenate([np.arange(0, M, max(1, M // 40)), [M - 1]]))
+    rows_d = torch.from_numpy(rows).cuda()
+    y_prod = G.empty((M, N), torch.int16)
+    for stage, b in enumerate(bits):
+        tasq.tasq_masked_gemm(ctx.h, 0, stage, codes, F16, ad, zd, M, packed, N, K, y_prod, None)
+        y_dbg, acc = G.gemm(ctx, 0, stage, codes, F16, ad, zd, M, packed, N, K)
+        ref_acc = oracle.gemm(s_x[rows], s_w, b)
+        got_acc = acc.index_select(0, rows_d).cpu().numpy()
+        assert np.array_equal(got_acc, ref_acc), f"b={b}: {(got_acc != ref_acc).sum()} int32 mismatches"
+        _, yb = oracle.epilogue_f32(ref_acc, alpha[rows], zc[rows], oracle.row_sums(s_w, b), cw, bias)
+        for y in (y_prod, y_dbg):
+            got = G.bf16_bits_host(y.index_select(0, rows_d))
+            assert G.assert_bf16_close(got, yb) == yb.size, f"b={b}: bf16 outputs differ in the last bit"
+        del y_dbg, acc
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+# ------------------------- the product call (no int32 output) vs the oracle --
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("M,N,K,full", [
+    (4096, 3456, 1152, False),  # 192-token tiles, two accumulators, persistent
+    (4000, 1096, 384, True),    # 256-token tiles, one accumulator, ragged tiles
+    (300, 1152, 1152, True),    # 64-token tiles, K split over slices
+    (77, 640, 2048, True),      # 64-token tiles, split K, ragged tokens
+    (1024, 4096, 4096, False),  # 256-token tiles over several certified chunks (N(0, 0.02) weights: one chunk)
+])
+def test_product_call_matches_oracle(ctx, oracle, code_fmt, M, N, K, full):
+    """tasq_masked_gemm with d_acc = NULL -- the call a network makes -- against
+    the oracle's bf16 output (not against the GPU's own debug call), one shape
+    per tile configuration of the tensor-core route."""
+    torch = G.torch()
+    bits = [8, 4, 2]
+    st = _setup_linear(ctx, oracle, M, N, K, bits, seed=M + K + 17, dtype=tasq.TASQ_BF16, code_fmt=code_fmt)
+    rows = np.arange(M) if full else np.unique(np.concatenate([np.arange(0, M, max(1, M // 48)), [M - 1]]))
+    rows_d = torch.from_numpy(rows).cuda()
+    for stage, b in enumerate(bits):
+        y, _ = G.gemm(ctx, 0, stage, st["codes"], code_fmt, st["alpha"], st["zc"], M, st["packed"], N, K,
+                      want_acc=False)
+        ref_acc = oracle.gemm(st["s_x"][rows], st["wq"]["s"], b)
+        _, yb = oracle.epilogue_f32(ref_acc, st["a"][rows], st["z"][rows], oracle.row_sums(st["wq"]["s"], b),
+                                    st["wq"]["c"], st["bias"])
+        got = G.bf16_bits_host(y.index_select(0, rows_d))
+        assert G.assert_bf16_close(got, yb) == yb.size, f"b={b}"
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+def test_conv_product_call_matches_oracle(ctx, oracle, code_fmt):
+    """tasq_masked_conv3x3 with d_acc = NULL against the oracle's bf16 output
+    (full check, border pixels included)."""
+    B, H, W, Cin, Cout = 1, 12, 20, 64, 136
+    x = workloads.normal((B, H, W, Cin), 301)
+    w = workloads.normal((Cout, 9 * Cin), 302, 0.03)
+    bias = workloads.normal((Cout,), 303, 0.02)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, Cout, 9 * Cin)
+    packed = G.pack(ctx, tasq.TASQ_CONV3X3, sw, cw, G.dev(bias), Cout, 9 * Cin, Cin)
+    tasq.tasq_set_schedule(ctx.h, np.array([[7, 3]], np.uint8), 1, 2)
+    M = B * H * W
+    codes, alpha, zc = G.quant_act(ctx, G.dev(x), tasq.TASQ_F32, M, Cin, 8, tasq.TASQ_SYMRANGE,
+                                   tasq.TASQ_PER_TENSOR, code_fmt)
+    wq = oracle.quant_weight(w)
+    s_x, a, z = oracle.quant_act(x.reshape(1, -1), 8, oracle.SYMRANGE, oracle.PER_TOKEN)
+    for stage, b in enumerate([7, 3]):
+        y, _ = G.conv(ctx, 0, stage, codes, code_fmt, alpha, zc, B, H, W, Cin, packed, Cout, want_acc=False)
+        acc, rs = oracle.conv3x3(s_x.reshape(B, H, W, Cin), wq["s"], b)
+        _, yb = oracle.epilogue_f32(acc, a, z, rs, wq["c"], bias, per_tensor=True, rs_per_row=True)
+        assert G.assert_bf16_close(G.bf16_bits_host(y), yb) == yb.size, f"b={b}"
+
+
+# -------------------------------- a captured graph follows the bit table --
+
+def test_graph_replay_follows_schedule_updates(ctx, oracle):
+    """A CUDA graph captured once keeps reading the context's bit table: after a
+    same-size tasq_set_schedule its replay runs the new bits; after a smaller
+    schedule that no longer holds the captured stage, the replay records
+    TASQ_ERR_DEVICE and writes nothing."""
+    torch = G.torch()
+    M, N, K = 256, 384, 640
+    st = _setup_linear(ctx, oracle, M, N, K, [8, 6], seed=77, code_fmt=tasq.TASQ_CODES_F16)
+    F16 = tasq.TASQ_CODES_F16
+    y = G.empty((M, N), torch.int16)
+
+    def call():
+        tasq.tasq_masked_gemm(ctx.h, 0, 1, st["codes"], F16, st["alpha"], st["zc"], M, st["packed"], N, K, y, None)
+
+    call()
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s), torch.cuda.graph(g, stream=s):
+        call()
+
+    def expect(b):
+        ref_acc = oracle.gemm(st["s_x"], st["wq"]["s"], b)
+        _, yb = oracle.epilogue_f32(ref_acc, st["a"], st["z"], oracle.row_sums(st["wq"]["s"], b), st["wq"]["c"],
+                                    st["bias"])
+        return yb
+
+    for table, b in (([[8, 6]], 6), ([[5, 3]], 3), ([[2, 7]], 7)):
+        tasq.tasq_set_schedule(ctx.h, np.array(table, np.uint8), 1, 2)
+        y.fill_(0)
+        g.replay()
+        torch.cuda.synchronize()
+        assert np.array_equal(G.bf16_bits_host(y), expect(b)), table
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+    # one stage only: the captured stage 1 is now out of range
+    tasq.tasq_set_schedule(ctx.h, np.array([[4]], np.uint8), 1, 1)
+    y.fill_(0)
+    g.replay()
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_ERR_DEVICE
+    assert not bool(y.any())
