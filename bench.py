@@ -161,15 +161,22 @@ class ClockSampler:
 
 # --------------------------------------------------------------- workload --
 class Step:
-    """Device-resident workload of one denoising step and its launch sequence."""
+    """Device-resident workload of one denoising step and its launch sequence.
 
-    def __init__(self, torch, tasq, workloads, name: str, seed: int, blocks: int = 0):
+    The step runs unit by unit: a unit is the layers that read one input (a
+    cross-attention's key and value projections; every other layer alone).  A
+    unit's input is quantized once and contracted by one call, at each member
+    layer's own precision from the bit table (tasq_masked_gemm_grouped for two
+    members).  Every layer keeps its own row of the table."""
+
+    def __init__(self, torch, tasq, workloads, name: str, seed: int, blocks: int = 0, group=True):
         self.torch, self.tasq = torch, tasq
         self.layers = workloads.inventory(name)
         self.table = workloads.schedule_for(name, len(self.layers))
         if blocks:
             keep = len(workloads.inventory_blocks(name, blocks))
             self.layers, self.table = self.layers[:keep], np.ascontiguousarray(self.table[:keep])
+        self.units = workloads.input_groups(self.layers) if group else [[i] for i in range(len(self.layers))]
         self.S = self.table.shape[1]
         self.ctx = tasq.tasq_create(torch.cuda.current_device())
         tasq.tasq_set_schedule(self.ctx, self.table, len(self.layers), self.S)
@@ -180,19 +187,24 @@ class Step:
         self.codes = torch.empty((max_mk,), dtype=torch.float16, device=dev)
         self.alpha = torch.empty((max_m,), dtype=torch.float32, device=dev)
         self.zc = torch.empty((max_m,), dtype=torch.float32, device=dev)
-        for i, l in enumerate(self.layers):
-            w = workloads.device_normal((l.N, l.K), seed * 100003 + 2 * i + 1, 0.02)
-            sw = torch.empty((l.N, l.K), dtype=torch.int8, device=dev)
-            cw = torch.empty((l.N,), dtype=torch.float32, device=dev)
-            tasq.tasq_quant_weights(self.ctx, w, tasq.TASQ_F32, l.N, l.K, sw, cw)
-            bias = workloads.device_normal((l.N,), seed * 100003 + 2 * i + 2, 0.02)
+        for unit in self.units:
+            l = self.layers[unit[0]]
+            N = sum(self.layers[i].N for i in unit)
+            # each member's weights and bias from its own seed, stacked along N
+            w = torch.cat([workloads.device_normal((self.layers[i].N, l.K), seed * 100003 + 2 * i + 1, 0.02)
+                           for i in unit])
+            bias = torch.cat([workloads.device_normal((self.layers[i].N,), seed * 100003 + 2 * i + 2, 0.02)
+                              for i in unit])
+            sw = torch.empty((N, l.K), dtype=torch.int8, device=dev)
+            cw = torch.empty((N,), dtype=torch.float32, device=dev)
+            tasq.tasq_quant_weights(self.ctx, w, tasq.TASQ_F32, N, l.K, sw, cw)
             kind = tasq.TASQ_CONV3X3 if l.kind == workloads.CONV3X3 else tasq.TASQ_LINEAR
-            pk = torch.empty((tasq.tasq_packed_bytes(kind, l.N, l.K),), dtype=torch.uint8, device=dev)
-            tasq.tasq_pack_weights(self.ctx, kind, sw, cw, bias, l.N, l.K, l.Cin, pk)
+            pk = torch.empty((tasq.tasq_packed_bytes(kind, N, l.K),), dtype=torch.uint8, device=dev)
+            tasq.tasq_pack_weights(self.ctx, kind, sw, cw, bias, N, l.K, l.Cin, pk)
             self.packed.append(pk)
             xs = (l.B, l.H, l.W, l.Cin) if l.kind == workloads.CONV3X3 else (l.M, l.K)
-            self.x.append(workloads.device_normal(xs, seed * 100003 + 1000003 + i, 1.0, torch.bfloat16))
-            self.y.append(torch.empty((l.M, l.N), dtype=torch.int16, device=dev))
+            self.x.append(workloads.device_normal(xs, seed * 100003 + 1000003 + unit[0], 1.0, torch.bfloat16))
+            self.y.append(torch.empty((l.M, N), dtype=torch.int16, device=dev))
             del w, sw, cw, bias
         self.d_stage = torch.zeros((4,), dtype=torch.int32, device=dev)
         tasq.tasq_set_stage_device(self.ctx, self.d_stage)
@@ -203,27 +215,32 @@ class Step:
 
     def launch(self, parts=("quant", "gemm")):
         """Enqueue one step on the current stream (stage read from d_stage).
-        parts: which kernels of each layer to enqueue (the quantization, the
+        parts: which kernels of each unit to enqueue (the quantization, the
         contraction, or both, in the step's order)."""
-        for i in range(len(self.layers)):
-            self.launch_layer(i, parts)
+        for u in range(len(self.units)):
+            self.launch_unit(u, parts)
 
-    def launch_layer(self, i, parts=("quant", "gemm")):
-        """Enqueue layer i (quantization + masked contraction) on the current stream."""
+    def launch_unit(self, u, parts=("quant", "gemm")):
+        """Enqueue unit u (one quantization + one masked contraction) on the current stream."""
         t = self.tasq
-        l = self.layers[i]
+        unit = self.units[u]
+        l = self.layers[unit[0]]
+        N = self.y[u].shape[1]
         conv = l.kind == self.conv
         if "quant" in parts:
             gran = t.TASQ_PER_TENSOR if conv else t.TASQ_PER_TOKEN
-            t.tasq_quant_act(self.ctx, self.x[i], t.TASQ_BF16, l.M, l.Cin if conv else l.K, 8, t.TASQ_SYMRANGE, gran,
+            t.tasq_quant_act(self.ctx, self.x[u], t.TASQ_BF16, l.M, l.Cin if conv else l.K, 8, t.TASQ_SYMRANGE, gran,
                              self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
         if "gemm" in parts:
             if conv:
-                t.tasq_masked_conv3x3(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B, l.H,
-                                      l.W, l.Cin, self.packed[i], l.N, self.y[i], None)
+                t.tasq_masked_conv3x3(self.ctx, unit[0], -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B,
+                                      l.H, l.W, l.Cin, self.packed[u], N, self.y[u], None)
+            elif len(unit) == 1:
+                t.tasq_masked_gemm(self.ctx, unit[0], -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
+                                   self.packed[u], N, l.K, self.y[u], None)
             else:
-                t.tasq_masked_gemm(self.ctx, i, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
-                                   self.packed[i], l.N, l.K, self.y[i], None)
+                t.tasq_masked_gemm_grouped(self.ctx, unit, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc,
+                                           l.M, self.packed[u], N, l.K, self.y[u], None)
 
     def launches_per_step(self):
         """Kernels the library enqueues for one step, counted by the library itself
@@ -235,22 +252,23 @@ class Step:
             self._launches = self.tasq.tasq_kernel_count(self.ctx) - before
         return self._launches
 
+    def _unit_shapes(self):
+        for u, unit in enumerate(self.units):
+            l = self.layers[unit[0]]
+            yield l, (l.Cin if l.Cin else l.K), self.y[u].shape[1]
+
     def act_bytes(self):
         """Algorithmic HBM bytes of activation quantization per step: bf16 in,
         one byte per code out (an int8 code; the tensor-core route holds it in
         fp16, which doubles the bytes actually written), 8 bytes of scales per
         token (per-tensor: per tensor)."""
-        return sum(l.M * (l.Cin if l.Cin else l.K) * 3 + 8 * l.M for l in self.layers)
+        return sum(l.M * k_in * 3 + 8 * l.M for l, k_in, _ in self._unit_shapes())
 
     def gemm_bytes(self):
         """Algorithmic HBM bytes of the contractions per step: int8 activation codes
         (M K), int8 weights (N K), bf16 output (2 M N), per-token scales (8 M) and
         per-channel scale, bias and the seven row sums (4 N (2 + 7))."""
-        tot = 0
-        for l in self.layers:
-            k_in = l.Cin if l.Cin else l.K
-            tot += l.M * k_in + l.N * l.K + 2 * l.M * l.N + 8 * l.M + 36 * l.N
-        return tot
+        return sum(l.M * k_in + N * l.K + 2 * l.M * N + 8 * l.M + 36 * N for l, k_in, N in self._unit_shapes())
 
     def close(self):
         self.tasq.tasq_destroy(self.ctx)
@@ -574,11 +592,11 @@ def stage_map(name: str, S: int):
 
 
 def e2e_measure(torch, tasq, step, n_steps, stage_of, copy_streams=1):
-    """The step end to end through the C ABI with host buffers: each layer's input
+    """The step end to end through the C ABI with host buffers: each unit's input
     is copied in from pinned host memory on one stream and its output copied out on
-    another, the layers run in order on the compute stream, so the copies of other
-    layers overlap the kernels.  Everything is captured into one graph."""
-    L = len(step.layers)
+    another, the units run in order on the compute stream, so the copies of other
+    units overlap the kernels.  Everything is captured into one graph."""
+    L = len(step.units)
     xh = [x.cpu().pin_memory() for x in step.x]
     yh = [torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for y in step.y]
     nc = max(1, copy_streams)
@@ -602,7 +620,7 @@ def e2e_measure(torch, tasq, step, n_steps, stage_of, copy_streams=1):
                 step.x[i].copy_(xh[i], non_blocking=True)
                 evx[i].record(sh[i % nc])
             s.wait_event(evx[i])
-            step.launch_layer(i)
+            step.launch_unit(i)
             evy[i].record(s)
             with torch.cuda.stream(sd[i % nc]):
                 sd[i % nc].wait_event(evy[i])
@@ -680,13 +698,14 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     achieved = step.ops / (ms_gemm * 1e-3) / 1e12
     peak = peaks["bf16"]
     traffic = measured_traffic(name)
+    U = len(step.units)
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                "traffic": traffic, "algorithmic_bytes_per_launch": step.gemm_bytes() / L,
+                "traffic": traffic, "algorithmic_bytes_per_launch": step.gemm_bytes() / U,
                 "kernel": "gemm_tc_kernel",
                 "peak_source": f"{peaks['src']} bf16 burst (cuBLAS); the fp16 tcgen05 MMA runs at the bf16 rate, "
                                "and the contraction-only replay lasts well under a second",
                 "timing": "CUDA events around replays of the step's launch sequence with only its contractions "
-                          f"({steps} replays, {L} launches each, every launch overlapping the previous one's tail "
+                          f"({steps} replays, {U} calls each, every launch overlapping the previous one's tail "
                           "as in the step); achieved = int8-equivalent ops per step / that time"}
     if traffic is not None:
         roofline["traffic_note"] = ("mean DRAM bytes per contraction launch (ncu); inputs just written by the "
@@ -696,7 +715,7 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     ops_w = np.array(step.gemm_ops, np.float64)
     eff_w = float((bits * ops_w[:, None]).sum() / (ops_w.sum() * S))
     out = {
-        "workload": WORKLOAD_NAMES[name], "layers": L, "stages": S, "ms_per_step": ms,
+        "workload": WORKLOAD_NAMES[name], "layers": L, "contraction_calls": U, "stages": S, "ms_per_step": ms,
         "value": job_tops(step.ops, world, ms), "unit": UNIT, "ms_per_step_all8": ms8,
         "effective_w_bits": eff_w, "rel_bitops": schedule.rel_bitops(eff_w, 8),
         "engine_model_rel_cost": engine_model.schedule_cost(step.table, step.gemm_ops, 8),
@@ -776,7 +795,10 @@ def main():
             "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": max(3, args.warmup), "ms_per_step": head["ms_per_step"], "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f16-exact-int8", "data": "synthetic",
-            "config": {"workload": head["workload"], "layers": head["layers"], "stages": head["stages"],
+            "config": {"workload": head["workload"], "layers": head["layers"],
+                       "contraction_calls": head["contraction_calls"], "stages": head["stages"],
+                       "shared_inputs": "a cross-attention's key and value projections read one input: one "
+                                        "quantization and one grouped contraction, each layer at its own b",
                        "schedule": "seeded learned-style per-(layer, stage) bits",
                        "effective_w_bits": head["effective_w_bits"], "rel_bitops": head["rel_bitops"],
                        "route": "tcgen05 fp16 MMA, exact int32",

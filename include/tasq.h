@@ -67,7 +67,7 @@
 extern "C" {
 #endif
 
-#define TASQ_ABI_VERSION 2
+#define TASQ_ABI_VERSION 3
 
 /* Return codes. */
 enum {
@@ -301,6 +301,28 @@ int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, 
 int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt, const float* d_alpha,
                      const float* d_zc, int M, const void* d_packed, int N, int K, uint16_t* d_y, int32_t* d_acc,
                      tasq_stream stream);
+
+/*
+ * Grouped masked linear layers: `groups` (1..4) layers that read the same
+ * activations -- e.g. the key and value projections of a cross-attention,
+ * which both take the text tokens -- contracted in one launch, each at its own
+ * operating precision b_g = table[h_layers[g]][stage] (App. F.1: the bit map
+ * is per layer).  The layers' stored weights are packed together, once, as one
+ * TASQ_LINEAR buffer of N = groups * Ng rows ([layer 0's Ng rows][layer 1's]
+ * ...; tasq_pack_weights on the concatenated [N][K] codes, scales and biases),
+ * and member g owns output channels [g Ng, (g + 1) Ng).  Output channel n of
+ * member g is exactly what tasq_masked_gemm computes for layer h_layers[g]
+ * alone (same contraction, mask and epilogue at b_g), so d_y [M][N] holds the
+ * members' outputs side by side (and d_acc their int32 accumulators).
+ * h_layers: host array of `groups` layer indices, read during the call.
+ * Needs N % groups == 0 and Ng % 8 == 0; other arguments and rules as
+ * tasq_masked_gemm (groups == 1 is tasq_masked_gemm).  The activations are
+ * quantized once for the group, and the launch overhead is paid once.
+ * Enqueue call.
+ */
+int tasq_masked_gemm_grouped(tasq_ctx ctx, const int32_t* h_layers, int groups, int stage, const void* d_codes,
+                             int code_fmt, const float* d_alpha, const float* d_zc, int M, const void* d_packed,
+                             int N, int K, uint16_t* d_y, int32_t* d_acc, tasq_stream stream);
 
 /*
  * Masked linear layer with asymmetric weights (Eq. weight_dequant with the

@@ -44,13 +44,17 @@ __device__ inline void mma_s8(int (&d)[4], const uint32_t (&a)[4], uint32_t b0, 
 template <bool CONV, bool ZP>
 __global__ void __launch_bounds__(THREADS) gemm_s8_kernel(const GemmArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
-    const int b = resolve_bits(a);
-    if (b == 0) return;
-    const uint32_t wmask = mask_word(b);
+    const uint32_t gbits = resolve_group_bits(a);
+    if (gbits == 0) return;
+    const int b = int(gbits & 15u);  // the layer's b (member 0 of a grouped call)
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int wm = warp >> 2, wn = warp & 3;  // 2 x 4 warps, 64 x 32 each
     const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM;
+    // weight fragment ni of this thread holds channel n0 + wn * 32 + ni * 8 + lane / 4
+    uint32_t wmask[4];
+#pragma unroll
+    for (int ni = 0; ni < 4; ++ni) wmask[ni] = mask_word(channel_bits(a, gbits, n0 + wn * 32 + ni * 8 + (lane >> 2)));
     const int M = a.M, N = a.N, K = a.K;
     const int8_t* __restrict__ X = reinterpret_cast<const int8_t*>(a.x);
     const int8_t* __restrict__ Wt = a.w;
@@ -136,10 +140,10 @@ __global__ void __launch_bounds__(THREADS) gemm_s8_kernel(const GemmArgs a) {
                 int r = wn * 32 + j * 16 + (lane & 7) + ((lane >> 4) << 3);
                 uint32_t t0, t1, t2, t3;
                 ldmatrix_x4(sB + swz(r, ks * 2 + ((lane >> 3) & 1)), t0, t1, t2, t3);
-                bf[2 * j][0] = t0 & wmask;
-                bf[2 * j][1] = t1 & wmask;
-                bf[2 * j + 1][0] = t2 & wmask;
-                bf[2 * j + 1][1] = t3 & wmask;
+                bf[2 * j][0] = t0 & wmask[2 * j];
+                bf[2 * j][1] = t1 & wmask[2 * j];
+                bf[2 * j + 1][0] = t2 & wmask[2 * j + 1];
+                bf[2 * j + 1][1] = t3 & wmask[2 * j + 1];
             }
 #pragma unroll
             for (int mi = 0; mi < 4; ++mi)
@@ -151,7 +155,6 @@ __global__ void __launch_bounds__(THREADS) gemm_s8_kernel(const GemmArgs a) {
 
     // ------------------------------------------------------------ epilogue
     const int g = lane >> 2, t4 = lane & 3;
-    const int32_t* rs_b = a.rs + int64_t(b - kBMin) * N;
     const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * N * 9 : nullptr;
 #pragma unroll
     for (int ni = 0; ni < 4; ++ni) {
@@ -159,6 +162,8 @@ __global__ void __launch_bounds__(THREADS) gemm_s8_kernel(const GemmArgs a) {
         if (n >= N) continue;
         const float cw0 = a.cw[n], cw1 = a.cw[n + 1];
         const float bi0 = a.bias[n], bi1 = a.bias[n + 1];
+        // row sums at the channel's b (n and n + 1 belong to one member: group_n % 8 == 0)
+        const int32_t* rs_b = a.rs + int64_t(channel_bits(a, gbits, n) - kBMin) * N;
         const int rsl0 = CONV ? 0 : rs_b[n], rsl1 = CONV ? 0 : rs_b[n + 1];
         // asymmetric weights: zero offsets per channel, activation sums per token
         constexpr bool zp = ZP;

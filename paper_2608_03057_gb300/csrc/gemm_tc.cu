@@ -284,11 +284,18 @@ __global__ void __maxnreg__(96)
     int cert[kNumB];
 #pragma unroll
     for (int i = 0; i < kNumB; ++i) cert[i] = a.hdr->chunk_kb[kBMin + i];
-    const int b = resolve_bits(a);
-    int chunk_kb = 1;
+    // b of every member layer (one member unless the call is grouped); b = member 0's
+    const uint32_t gbits = resolve_group_bits(a);
+    const int b = int(gbits & 15u);
+    // the shortest certified chunk over the members' precisions is valid for all of them
+    int chunk_kb = 0x7FFFFFFF;
 #pragma unroll
-    for (int i = 0; i < kNumB; ++i)
-        if (b == kBMin + i) chunk_kb = cert[i];
+    for (int g = 0; g < kMaxGroups; ++g) {
+        const int bg = int((gbits >> (4 * g)) & 15u);
+#pragma unroll
+        for (int i = 0; i < kNumB; ++i)
+            if (g < a.groups && bg == kBMin + i) chunk_kb = min(chunk_kb, cert[i]);
+    }
     const int KT = (a.K + BK - 1) / BK;
     // certificate is in 64-wide K blocks; a run of c64 of them covers c64/2 of ours
     int chunk = chunk_kb / (BK / kCertKBlock);
@@ -424,13 +431,14 @@ __global__ void __maxnreg__(96)
         // ------------------------------------------- weight mask + convert
         const int q = warp & 3;             // tensor-memory lane quadrant
         const int r = q * 32 + lane;        // channel row within the tile
-        const uint32_t m = mask_word(b);
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         Ring<W_STAGES> rw;
         int it = 0;
         bool ok = true;
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
+            // this row's channel runs at its layer's b (a grouped call holds several layers)
+            const uint32_t m = mask_word(channel_bits(a, gbits, tile_coord<CONV, BT>(p, wk.t).ch0 + r));
             for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rw.next()) {
                 if (!wt.wait(&s->wfull[rw.slot], rw.phase)) {
                     ok = false;
@@ -487,8 +495,9 @@ __global__ void __maxnreg__(96)
         const int gpw = helpers ? (C::GROUPS + EPI_PARTS) / (EPI_PARTS + 1) : GPW;  // groups per share
         const int r = q * 32 + lane;
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
-        const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
+        // row sums at each channel's b (convolutions are never grouped)
         const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
+        auto rs_of = [&](int n) { return a.rs[int64_t(channel_bits(a, gbits, n) - kBMin) * a.N + n]; };
         constexpr bool zp = ZP;  // asymmetric weights: the four-term epilogue
         int cc = 0;
         bool ok = true;
@@ -513,7 +522,7 @@ __global__ void __maxnreg__(96)
 #pragma unroll
                     for (int i = 0; i < 9; ++i) ts[i] = __int2float_rn(ts_b[int64_t(n) * 9 + i]);
                 } else {
-                    rs = __int2float_rn(rs_b[n]);
+                    rs = __int2float_rn(rs_of(n));
                 }
             }
 
@@ -527,7 +536,7 @@ __global__ void __maxnreg__(96)
                     const bool ok_k = nk < a.N;
                     cwf[k] = ok_k ? a.cw[nk] : 0.f;
                     biasf[k] = ok_k ? a.bias[nk] : 0.f;
-                    rsf[k] = ok_k ? __int2float_rn(rs_b[nk]) : 0.f;
+                    rsf[k] = ok_k ? __int2float_rn(rs_of(nk)) : 0.f;
                     zcwf[k] = ok_k && zp ? a.zcw[nk] : 0.f;
                 }
             }
@@ -824,11 +833,11 @@ __global__ void __maxnreg__(96)
 __global__ void __launch_bounds__(256) splitk_epilogue_kernel(const GemmArgs a, const int32_t* __restrict__ parts,
                                                               int S) {
     ptx::grid_dependency_wait();
-    const int b = resolve_bits(a);
-    if (b == 0) return;
+    const uint32_t gbits = resolve_group_bits(a);
+    if (gbits == 0) return;
+    const int b = int(gbits & 15u);
     const int N4 = a.N / 4;
     const int64_t total = int64_t(a.M) * N4;
-    const int32_t* rs_b = a.rs + int64_t(b - kBMin) * a.N;
     const int32_t* ts_b = a.Cin ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
     for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < total; i += int64_t(gridDim.x) * blockDim.x) {
         const int m = int(i / N4);
@@ -870,7 +879,8 @@ __global__ void __launch_bounds__(256) splitk_epilogue_kernel(const GemmArgs a, 
                 for (int k9 = 0; k9 < 9; ++k9)
                     rsum = __fadd_rn(rsum, (tap >> k9) & 1 ? __int2float_rn(ts_b[int64_t(n + q) * 9 + k9]) : 0.f);
             } else {
-                rsum = __int2float_rn(rs_b[n + q]);
+                // the four channels n..n+3 belong to one member (group_n % 8 == 0)
+                rsum = __int2float_rn(a.rs[int64_t(channel_bits(a, gbits, n) - kBMin) * a.N + n + q]);
             }
             float u = __fmaf_rn(zc, rsum, __int2float_rn(accs[q]));
             if (zp) u = __fmaf_rn(a.zcw[n + q], t, u);

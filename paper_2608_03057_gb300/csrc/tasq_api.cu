@@ -342,17 +342,24 @@ TASQ_API int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M
 
 namespace {
 
-int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void* d_codes, int code_fmt,
-                       const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int M,
+// layers[0..groups): the member layers of a grouped call (one for a single layer)
+int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, int stage, const void* d_codes,
+                       int code_fmt, const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int M,
                        const void* d_packed, int N, int K, int B, int H, int W, int Cin, uint16_t* d_y,
                        int32_t* d_acc, tasq_stream stream) {
     REQUIRE(ctx->L > 0, TASQ_ERR_INVALID_ARG, "no schedule: call tasq_set_schedule first");
-    REQUIRE(layer >= 0 && layer < ctx->L, TASQ_ERR_INVALID_ARG, "layer %d outside 0..%d", layer, ctx->L - 1);
+    REQUIRE(layers && groups >= 1 && groups <= tasq::kMaxGroups, TASQ_ERR_INVALID_ARG, "groups %d outside 1..%d",
+            groups, tasq::kMaxGroups);
+    for (int g = 0; g < groups; ++g)
+        REQUIRE(layers[g] >= 0 && layers[g] < ctx->L, TASQ_ERR_INVALID_ARG, "layer %d outside 0..%d", layers[g],
+                ctx->L - 1);
     REQUIRE(stage >= -1 && stage < ctx->S, TASQ_ERR_INVALID_ARG, "stage %d outside -1..%d", stage, ctx->S - 1);
     REQUIRE(stage >= 0 || ctx->d_stage, TASQ_ERR_INVALID_ARG, "stage -1 needs tasq_set_stage_device");
     REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16, TASQ_ERR_INVALID_ARG, "code_fmt %d", code_fmt);
     REQUIRE(M >= 0 && N > 0 && K > 0, TASQ_ERR_INVALID_ARG, "M=%d N=%d K=%d", M, N, K);
     REQUIRE(K % 16 == 0 && N % 8 == 0, TASQ_ERR_UNSUPPORTED, "need K %% 16 == 0 and N %% 8 == 0 (N=%d K=%d)", N, K);
+    REQUIRE(groups == 1 || (N % groups == 0 && (N / groups) % 8 == 0), TASQ_ERR_UNSUPPORTED,
+            "grouped call: N=%d must split into %d members of a multiple of 8 channels", N, groups);
     int route = ctx->route;
     if (route == TASQ_ROUTE_AUTO) route = code_fmt == TASQ_CODES_F16 ? TASQ_ROUTE_TC : TASQ_ROUTE_MMA_S8;
     REQUIRE((route == TASQ_ROUTE_TC) == (code_fmt == TASQ_CODES_F16), TASQ_ERR_UNSUPPORTED,
@@ -377,8 +384,11 @@ int masked_contraction(tasq_ctx ctx, int kind, int layer, int stage, const void*
     a.hdr = reinterpret_cast<const tasq::PackedHeader*>(p);
     a.table = ctx->d_table;
     a.d_stage = ctx->d_stage;
-    a.layer = layer;
+    a.layer = layers[0];
     a.stage = stage;
+    a.groups = groups;
+    a.group_n = N / groups;
+    for (int g = 0; g < groups; ++g) a.layers[g] = layers[g];
     a.M = M;
     a.N = N;
     a.K = K;
@@ -417,8 +427,8 @@ TASQ_API int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_
                               const float* d_alpha, const float* d_zc, int M, const void* d_packed, int N, int K,
                               uint16_t* d_y, int32_t* d_acc, tasq_stream stream) {
     CHECK_CTX(ctx);
-    return masked_contraction(ctx, TASQ_LINEAR, layer, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, M, d_packed,
-                              N, K, 1, 0, 0, 0, d_y, d_acc, stream);
+    return masked_contraction(ctx, TASQ_LINEAR, &layer, 1, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, M,
+                              d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream);
 }
 
 TASQ_API int tasq_masked_gemm_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
@@ -427,7 +437,19 @@ TASQ_API int tasq_masked_gemm_zp(tasq_ctx ctx, int layer, int stage, const void*
                                  tasq_stream stream) {
     CHECK_CTX(ctx);
     REQUIRE(M == 0 || d_code_sums, TASQ_ERR_INVALID_ARG, "NULL pointer");
-    return masked_contraction(ctx, TASQ_LINEAR, layer, stage, d_codes, code_fmt, d_alpha, d_zc, d_code_sums, M,
+    return masked_contraction(ctx, TASQ_LINEAR, &layer, 1, stage, d_codes, code_fmt, d_alpha, d_zc, d_code_sums, M,
+                              d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream);
+}
+
+TASQ_API int tasq_masked_gemm_grouped(tasq_ctx ctx, const int32_t* h_layers, int groups, int stage,
+                                      const void* d_codes, int code_fmt, const float* d_alpha, const float* d_zc,
+                                      int M, const void* d_packed, int N, int K, uint16_t* d_y, int32_t* d_acc,
+                                      tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(h_layers, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    int layers[tasq::kMaxGroups] = {};
+    for (int g = 0; g < groups && g < tasq::kMaxGroups; ++g) layers[g] = h_layers[g];
+    return masked_contraction(ctx, TASQ_LINEAR, layers, groups, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, M,
                               d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream);
 }
 
@@ -438,8 +460,8 @@ TASQ_API int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void*
     REQUIRE(B >= 0 && H > 0 && W > 0 && Cin > 0, TASQ_ERR_INVALID_ARG, "B=%d H=%d W=%d Cin=%d", B, H, W, Cin);
     REQUIRE(Cin % 16 == 0, TASQ_ERR_UNSUPPORTED, "conv: Cin=%d must be a multiple of 16", Cin);
     REQUIRE((int64_t)B * H * W <= 0x7FFFFFFF && (int64_t)9 * Cin <= 0x7FFFFFFF, TASQ_ERR_UNSUPPORTED, "too large");
-    return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, B * H * W,
-                              d_packed, Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
+    return masked_contraction(ctx, TASQ_CONV3X3, &layer, 1, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr,
+                              B * H * W, d_packed, Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
 }
 
 TASQ_API int tasq_masked_conv3x3_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
@@ -451,7 +473,7 @@ TASQ_API int tasq_masked_conv3x3_zp(tasq_ctx ctx, int layer, int stage, const vo
     REQUIRE(Cin % 16 == 0, TASQ_ERR_UNSUPPORTED, "conv: Cin=%d must be a multiple of 16", Cin);
     REQUIRE((int64_t)B * H * W <= 0x7FFFFFFF && (int64_t)9 * Cin <= 0x7FFFFFFF, TASQ_ERR_UNSUPPORTED, "too large");
     REQUIRE(B == 0 || d_code_sums, TASQ_ERR_INVALID_ARG, "NULL pointer");
-    return masked_contraction(ctx, TASQ_CONV3X3, layer, stage, d_codes, code_fmt, d_alpha, d_zc, d_code_sums,
+    return masked_contraction(ctx, TASQ_CONV3X3, &layer, 1, stage, d_codes, code_fmt, d_alpha, d_zc, d_code_sums,
                               B * H * W, d_packed, Cout, 9 * Cin, B, H, W, Cin, d_y, d_acc, stream);
 }
 

@@ -20,6 +20,8 @@ constexpr int64_t kCertLimit = int64_t(1) << 17;  // 2^24 / 128: sum |w| bound p
 // [L][S].  The context allocates room for kTableCapacity bits when it is created.
 constexpr int kTableHeader = 16;
 constexpr size_t kTableCapacity = 65536;
+// Most layers one grouped contraction call may hold.
+constexpr int kMaxGroups = 4;
 
 struct PackedHeader {
     uint32_t magic;
@@ -79,6 +81,12 @@ struct GemmArgs {
     const uint8_t* table;     // bit table: int32 L, S at offset 0, bits [L][S] at kTableHeader
     const int32_t* d_stage;   // used when stage < 0
     int layer, stage;
+    // Grouped call: `groups` layers that read the same activations, stored as one
+    // packed buffer of their weights concatenated along N; member g owns output
+    // channels [g * group_n, (g + 1) * group_n) and runs at its own b.
+    int groups;               // 1 for a single layer
+    int group_n;              // N / groups
+    int layers[kMaxGroups];   // member layers (layers[0] == layer)
     int M, N, K;
     int B, H, W, Cin;         // conv geometry (Cin == 0 for a linear layer)
     int per_tensor;
@@ -96,9 +104,11 @@ struct GemmArgs {
     const int32_t* code_sums;  // [M] sum_k s_x[m][k] (conv: per input pixel), or NULL (two-term epilogue)
 };
 
-// Resolves b for this launch on the device; returns 0 (and records an error)
-// when the stage or the table entry is out of range or the header mismatches.
-__device__ inline int resolve_bits(const GemmArgs& a) {
+// Resolves the operating precision of every member layer of this launch on
+// the device, packed four bits per member (member g in bits 4g..4g+3); returns
+// 0 (and records an error) when the stage or a table entry is out of range or
+// the header mismatches.  A single layer is the group of one.
+__device__ inline uint32_t resolve_group_bits(const GemmArgs& a) {
     // the header fields and the stage do not depend on one another: load them together
     const uint32_t magic = a.hdr->magic;
     const int hdr_n = a.hdr->N, hdr_k = a.hdr->K, hdr_zp = a.hdr->has_zp;
@@ -106,15 +116,30 @@ __device__ inline int resolve_bits(const GemmArgs& a) {
     // the table's dimensions come from the device copy, so a graph captured before a
     // later tasq_set_schedule reads that schedule's bits (or records the mismatch)
     const int2 dims = *reinterpret_cast<const int2*>(a.table);
-    const bool stage_ok = stage >= 0 && stage < dims.y && a.layer < dims.x;
-    const int b = stage_ok ? a.table[kTableHeader + a.layer * dims.y + stage] : 0;
-    // a buffer packed with zero offsets needs the code sums of the four-term epilogue
-    if (!stage_ok || b < kBMin || b > kBMax || magic != kPackedMagic || hdr_n != a.N || hdr_k != a.K ||
-        (hdr_zp && !a.code_sums)) {
+    bool ok = stage >= 0 && stage < dims.y && magic == kPackedMagic && hdr_n == a.N && hdr_k == a.K &&
+              !(hdr_zp && !a.code_sums);  // a buffer packed with zero offsets needs the code sums
+    uint32_t packed = 0;
+#pragma unroll
+    for (int g = 0; g < kMaxGroups; ++g) {
+        if (g < a.groups) {
+            const int layer = a.layers[g];
+            const bool in = ok && layer < dims.x;
+            const int b = in ? a.table[kTableHeader + layer * dims.y + stage] : 0;
+            ok = in && b >= kBMin && b <= kBMax;
+            packed |= uint32_t(b & 15) << (4 * g);
+        }
+    }
+    if (!ok) {
         set_status(a.status, TASQ_ERR_DEVICE);
         return 0;
     }
-    return b;
+    return packed;
+}
+
+// b of output channel n from the packed member bits.
+__device__ __forceinline__ int channel_bits(const GemmArgs& a, uint32_t packed_bits, int n) {
+    const int g = a.groups > 1 ? min(n / a.group_n, a.groups - 1) : 0;
+    return int((packed_bits >> (4 * g)) & 15u);
 }
 
 // x / a rounded to nearest even, from ra = RN(1/a): the quotient estimate

@@ -78,6 +78,7 @@ def lib():
                 "tasq_quant_act_sums": ([P, P, I, I, I, I, I, I, P, I, P, P, P, P], I),
                 "tasq_masked_gemm": ([P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_gemm_zp": ([P, I, I, P, I, P, P, P, I, P, I, I, P, P, P], I),
+                "tasq_masked_gemm_grouped": ([P, P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_conv3x3": ([P, I, I, P, I, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_masked_conv3x3_zp": ([P, I, I, P, I, P, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_quant_act_tensor_noalloc": ([P, I, I, I, I, I, P, I, P, P, P], I),
@@ -222,6 +223,15 @@ def tasq_masked_gemm_zp(ctx, layer, stage, codes, code_fmt, alpha, zc, code_sums
 def tasq_masked_gemm(ctx, layer, stage, codes, code_fmt, alpha, zc, M, packed, N, K, y, acc=None, stream=None) -> None:
     _check(ctx, lib().tasq_masked_gemm(ctx, int(layer), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha), _ptr(zc),
                                        int(M), _ptr(packed), int(N), int(K), _ptr(y), _ptr(acc), _stream(stream)))
+
+
+def tasq_masked_gemm_grouped(ctx, layers, stage, codes, code_fmt, alpha, zc, M, packed, N, K, y, acc=None,
+                             stream=None) -> None:
+    """layers: the member layer indices (a sequence of 1..4 ints)."""
+    h = (ctypes.c_int32 * len(layers))(*[int(v) for v in layers])
+    _check(ctx, lib().tasq_masked_gemm_grouped(ctx, h, len(layers), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
+                                               _ptr(zc), int(M), _ptr(packed), int(N), int(K), _ptr(y), _ptr(acc),
+                                               _stream(stream)))
 
 
 def tasq_masked_conv3x3(ctx, layer, stage, codes, code_fmt, alpha, zc, B, H, W, Cin, packed, Cout, y, acc=None,

@@ -167,6 +167,36 @@ def sdxl_turbo() -> List[Layer]:
     return out
 
 
+# Layers that read the same input tensor: the key and value projections of a
+# cross-attention both take the text tokens.
+SHARED_INPUT_PAIRS = ((".cross.k", ".cross.v"), (".attn2.k", ".attn2.v"))
+
+
+def input_groups(layers: List[Layer]) -> List[List[int]]:
+    """The inventory as units of layers that read one input: a cross-attention's
+    key and value projections form a unit of two (consecutive, same M and K),
+    every other layer a unit of its own.  Indices follow the inventory."""
+    out: List[List[int]] = []
+    i = 0
+    while i < len(layers):
+        l = layers[i]
+        if i + 1 < len(layers):
+            m = layers[i + 1]
+            for a, b in SHARED_INPUT_PAIRS:
+                if (l.name.endswith(a) and m.name.endswith(b) and l.name[:-len(a)] == m.name[:-len(b)]
+                        and (l.M, l.K, l.kind) == (m.M, m.K, m.kind)):
+                    out.append([i, i + 1])
+                    i += 2
+                    break
+            else:
+                out.append([i])
+                i += 1
+            continue
+        out.append([i])
+        i += 1
+    return out
+
+
 def sweep_shapes():
     """GEMM sweep: M x (K = N) x b."""
     for M in (1024, 4096, 16384):

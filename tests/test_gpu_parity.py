@@ -11,6 +11,7 @@ import pytest
 
 from paper_2608_03057_gb300 import tasq, workloads
 from tests import gpu_layer as G
+from tests import gpu_layer as GL
 
 pytestmark = pytest.mark.gpu
 
@@ -985,3 +986,59 @@ def test_graph_replay_follows_schedule_updates(ctx, oracle):
     g.replay()
     assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_ERR_DEVICE
     assert not bool(y.any())
+
+
+# --------------------------------------------- grouped contraction call --
+
+@pytest.mark.parametrize("code_fmt", ROUTES)
+@pytest.mark.parametrize("M,Ng,K,G", [(300, 1152, 1152, 2), (77, 1280, 2048, 2), (513, 136, 1168, 3),
+                                      (129, 264, 2240, 4)])
+def test_grouped_members_match_single_layers(ctx, oracle, code_fmt, M, Ng, K, G):
+    """One grouped launch over G layers that share their activations (weights
+    packed once, concatenated along N) equals, member by member, the oracle's
+    single layer at that member's own b.  Members straddle 128-channel tiles
+    (Ng = 136, 264) and two shapes split K on the tensor-core route."""
+    N = G * Ng
+    w = workloads.normal((N, K), 400 + M, 0.02)
+    bias = workloads.normal((N,), 401 + M, 0.02)
+    x = workloads.normal((M, K), 402 + M)
+    sw, cw, _ = GL.quant_weights(ctx, GL.dev(w), tasq.TASQ_F32, N, K)
+    packed = GL.pack(ctx, tasq.TASQ_LINEAR, sw, cw, GL.dev(bias), N, K)
+    table = np.array([[8, 3], [2, 7], [5, 5], [6, 4]], np.uint8)
+    tasq.tasq_set_schedule(ctx.h, table, 4, 2)
+    layers = [2, 0, 3, 1][:G]
+    codes, alpha, zc = GL.quant_act(ctx, GL.dev(x), tasq.TASQ_F32, M, K, 8, tasq.TASQ_SYMRANGE,
+                                    tasq.TASQ_PER_TOKEN, code_fmt)
+    wq = oracle.quant_weight(w)
+    s_x, a, z = oracle.quant_act(x)
+    for stage in range(2):
+        for want_acc in (True, False):
+            y = GL.empty((M, N), GL.torch().int16)
+            acc = GL.empty((M, N), GL.torch().int32) if want_acc else None
+            tasq.tasq_masked_gemm_grouped(ctx.h, layers, stage, codes, code_fmt, alpha, zc, M, packed, N, K, y, acc)
+            yh = GL.bf16_bits_host(y)
+            acch = acc.cpu().numpy() if want_acc else None
+            for g, layer in enumerate(layers):
+                b = int(table[layer, stage])
+                sl = slice(g * Ng, (g + 1) * Ng)
+                ref = oracle.gemm(s_x, wq["s"][sl], b)
+                if want_acc:
+                    assert np.array_equal(acch[:, sl], ref), (g, b)
+                _, yb = oracle.epilogue_f32(ref, a, z, oracle.row_sums(wq["s"][sl], b), wq["c"][sl], bias[sl])
+                assert GL.assert_bf16_close(yh[:, sl], yb) == yb.size, (g, b)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+def test_grouped_call_rejects_bad_groups(ctx):
+    torch = GL.torch()
+    buf = torch.zeros((1 << 16,), dtype=torch.uint8, device="cuda")
+    tasq.tasq_set_schedule(ctx.h, np.array([[8], [4]], np.uint8), 2, 1)
+    F16 = tasq.TASQ_CODES_F16
+    for layers, N, code in (([0, 1, 0, 1, 0], 80, tasq.TASQ_ERR_INVALID_ARG),  # more than 4 members
+                            ([0, 2], 64, tasq.TASQ_ERR_INVALID_ARG),           # no layer 2
+                            ([0, 1, 1], 64, tasq.TASQ_ERR_UNSUPPORTED),        # 64 channels do not split in 3
+                            ([0, 1], 40, tasq.TASQ_ERR_UNSUPPORTED)):          # 20-channel members
+        with pytest.raises(tasq.TasqError) as e:
+            tasq.tasq_masked_gemm_grouped(ctx.h, layers, 0, buf, F16, buf, buf, 16, buf, N, 64, buf, None)
+        assert e.value.code == code, layers
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK

@@ -225,3 +225,20 @@ def test_rejected_shapes(args, code):
     with pytest.raises(tasq.TasqError) as e:
         tasq.tasq_plan_tc(tasq.TASQ_LINEAR, 64, 128, 1024, 0, 0, 0, 0, 0)
     assert e.value.code == tasq.TASQ_ERR_INVALID_ARG
+
+
+def test_input_groups_pair_cross_attention_keys_and_values():
+    """The benchmark's units: each cross-attention's key and value projections
+    (same block, same input shape) share one input; nothing else is grouped."""
+    from paper_2608_03057_gb300 import workloads
+    for name, pairs in (("pixart", 28), ("sana", 20), ("sdxl", 70), ("single", 0)):
+        layers = workloads.inventory(name)
+        units = workloads.input_groups(layers)
+        assert sorted(i for u in units for i in u) == list(range(len(layers)))
+        two = [u for u in units if len(u) == 2]
+        assert len(two) == pairs
+        for a, b in two:
+            la, lb = layers[a], layers[b]
+            assert b == a + 1 and (la.M, la.K) == (lb.M, lb.K)
+            assert la.name.rsplit(".", 1)[1] == "k" and lb.name.rsplit(".", 1)[1] == "v"
+            assert la.name.rsplit(".", 1)[0] == lb.name.rsplit(".", 1)[0]
