@@ -419,6 +419,67 @@ def s8_route_tops(torch, tasq, workloads, n=4096, reps=10):
     return {"shape": [n, n, n], "b": 8, "tops": 2.0 * n ** 3 / (ms * 1e-3) / 1e12}
 
 
+def run_small_m_weight_bytes(torch, tasq, shapes=((300, 1152, 1152), (300, 2304, 1152), (77, 1280, 2048),
+                                                  (256, 1280, 1280)), layers=128, seed=0):
+    """How much of a small-M contraction's time is reading its weights from HBM:
+    each shape (b = 3, 64-token tiles) as a CUDA graph of `layers` back-to-back
+    calls, either all on one packed layer (its weights stay in L2) or each on a
+    different packed layer of the same shape (`layers` x N x K bytes, more than
+    L2 holds, so every call reads its weights from HBM); the activation codes are
+    the same buffer in both.  A layout that streams only the selected weight
+    planes (e.g. hi/lo-nibble planes, half the bytes at b <= 4) could save at
+    most half of the difference per call."""
+    ctx = tasq.tasq_create(torch.cuda.current_device())
+    tasq.tasq_set_schedule(ctx, np.array([[3]] * layers, np.uint8), layers, 1)
+    out = []
+    for si, (M, N, K) in enumerate(shapes):
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed * 1000 + 700 + si)
+        nbytes = tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, N, K)
+        pks = []
+        for _ in range(layers):
+            sw = torch.randint(-127, 128, (N, K), generator=g, device="cuda", dtype=torch.int8)
+            cw = torch.rand((N,), generator=g, device="cuda") * 1e-3 + 1e-4
+            pk = torch.empty((nbytes,), dtype=torch.uint8, device="cuda")
+            tasq.tasq_pack_weights(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K, 0, pk)
+            pks.append(pk)
+            del sw, cw
+        codes = torch.randint(-127, 128, (M, K), generator=g, device="cuda", dtype=torch.int8).to(torch.float16)
+        al = torch.rand((M,), generator=g, device="cuda") * 1e-2 + 1e-3
+        zc = torch.full((M,), 0.5, device="cuda")
+        y = torch.empty((M, N), dtype=torch.int16, device="cuda")
+
+        def graph_us(which):
+            def seq():
+                for i in range(layers):
+                    j = which(i)
+                    tasq.tasq_masked_gemm(ctx, j, 0, codes, tasq.TASQ_CODES_F16, al, zc, M, pks[j], N, K, y)
+            seq()
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+                seq()
+            best = None
+            for _ in range(4):
+                gr.replay()
+                torch.cuda.synchronize()
+                t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                t0.record()
+                gr.replay()
+                t1.record()
+                torch.cuda.synchronize()
+                us = t0.elapsed_time(t1) * 1e3 / layers
+                best = us if best is None else min(best, us)
+            return best
+
+        warm = graph_us(lambda i: 0)
+        cold = graph_us(lambda i: i)
+        out.append({"M": M, "N": N, "K": K, "b": 3, "weight_bytes": N * K, "us_weights_in_l2": warm,
+                    "us_weights_from_hbm": cold, "max_saving_us_half_weight_bytes": max(0.0, cold - warm) / 2})
+        del pks, codes, al, zc, y
+    tasq.tasq_destroy(ctx)
+    return out
+
+
 def run_zero_point(torch, tasq, workloads, shapes=((4096, 1152, 1152), (4096, 3456, 1152), (300, 1152, 1152)),
                    reps=20, seed=0):
     """Asymmetric weights (App. A.1.1 on each channel's [min, max], a real zero
@@ -730,6 +791,13 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     return out, step
 
 
+def clk_mhz(clk):
+    """The median SM clock sampled during the timed region, else the maximum SM clock."""
+    if clk and clk.get("sm_mhz"):
+        return float(clk["sm_mhz"])
+    return 2070.0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -768,10 +836,13 @@ def main():
             torch.cuda.empty_cache()
             per_workload[name] = r
 
-    sweep = switch = zp = i8 = None
+    sweep = switch = zp = i8 = small_m = mma_kinds = None
     if not args.no_sweep:
         sweep, switch = run_sweep(torch, tasq, workloads, seed=args.seed)
         zp = run_zero_point(torch, tasq, workloads, seed=args.seed)
+        small_m = run_small_m_weight_bytes(torch, tasq, seed=args.seed)
+        from paper_2608_03057_gb300 import mma_probe
+        mma_kinds = mma_probe.run(clk_mhz(head["clocks"]))
         # int8 GEMMs measured on this GPU, for context: the library int8 GEMM and this
         # library's own mma.sync s8 route (sm_103a has no tcgen05 int8 kind)
         i8 = {"cublaslt_int8_gemm": int8_tensor_peak(torch), "mma_sync_s8_route": s8_route_tops(torch, tasq, workloads),
@@ -820,6 +891,8 @@ def main():
             "sweep_tops_by_b": sweep,
             "stage_switch": switch,
             "asym_weights": zp,
+            "small_m_weight_bytes": small_m,
+            "mma_kinds": mma_kinds,
             "int8_gemm_context": i8,
         }
         print(json.dumps(line), flush=True)

@@ -408,6 +408,23 @@ typedef struct {
 int tasq_plan_tc(int kind, int M, int N, int K, int B, int H, int W, int Cin, int num_sms, tasq_tc_plan* out);
 
 /*
+ * Probe of the tensor-core MMA kinds (diagnostic; the paper has no
+ * counterpart).  Launches `ctas` CTAs (one per SM); each loads A (128 rows)
+ * and B (n rows) of 128 bytes per row from d_a / d_b (row-major bytes: fp16
+ * values for kind 0, e4m3 values for kind 1), and one thread issues 4 * reps
+ * tcgen05.mma of that kind (kind 0: kind::f16, 16 elements of K per
+ * instruction; kind 1: kind::f8f6f4 with e4m3 A and B, 32 elements), M = 128,
+ * N = n, accumulating D = reps * A . B^T (over the 64 or 128 elements of a row)
+ * in fp32 in tensor memory.  d_cycles[i] receives CTA i's clock cycles from the
+ * first MMA to the completion of the last (0 if that wait gave up after 2 s);
+ * CTA 0 writes D to d_d [128][n] fp32.  16 <= n <= 256, n % 16 == 0,
+ * 1 <= reps <= 2^20, 1 <= ctas <= 1024.  Enqueue call; no context.  Errors are
+ * described by tasq_last_error(NULL) on the calling thread.
+ */
+int tasq_probe_mma(int kind, int n, int reps, const uint8_t* d_a, const uint8_t* d_b, float* d_d,
+                   unsigned long long* d_cycles, int ctas, tasq_stream stream);
+
+/*
  * Per-tensor activation quantization without any allocation (no context).
  * The paper has no counterpart to this call: it exists for callers that
  * cannot allocate device memory at run time -- for example an inference

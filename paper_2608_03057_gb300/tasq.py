@@ -83,6 +83,7 @@ def lib():
                 "tasq_masked_conv3x3_zp": ([P, I, I, P, I, P, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_quant_act_tensor_noalloc": ([P, I, I, I, I, I, P, I, P, P, P], I),
                 "tasq_plan_tc": ([I, I, I, I, I, I, I, I, I, ctypes.POINTER(tasq_tc_plan)], I),
+                "tasq_probe_mma": ([I, I, I, P, P, P, P, I, P], I),
             }
             for name, (args, res) in sigs.items():
                 f = getattr(L, name)
@@ -262,3 +263,9 @@ def tasq_plan_tc(kind, M, N, K, B, H, W, Cin, num_sms) -> dict:
     _check(None, lib().tasq_plan_tc(int(kind), int(M), int(N), int(K), int(B), int(H), int(W), int(Cin), int(num_sms),
                                     ctypes.byref(out)))
     return {name: getattr(out, name) for name, _ in tasq_tc_plan._fields_}
+
+
+def tasq_probe_mma(kind, n, reps, a, b, d, cycles, ctas, stream=None) -> None:
+    """Tensor-core MMA kind probe (diagnostic; see include/tasq.h)."""
+    _check(None, lib().tasq_probe_mma(int(kind), int(n), int(reps), _ptr(a), _ptr(b), _ptr(d), _ptr(cycles), int(ctas),
+                                      _stream(stream)))
