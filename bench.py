@@ -69,6 +69,7 @@ def measured_traffic(workload: str):
 UNIT = "TOPS"
 WORKLOAD_NAMES = {
     "pixart": "pixart_sigma_1024px_denoise_step",
+    "pixart_a4": "pixart_sigma_1024px_denoise_step_a4_w4a4_budget",
     "sana": "sana_1600m_1024px_denoise_step",
     "sdxl": "sdxl_turbo_512px_denoise_step",
     "single": "single_linear_256x1152x1152",
@@ -173,6 +174,10 @@ class Step:
         self.torch, self.tasq = torch, tasq
         self.layers = workloads.inventory(name)
         self.table = workloads.schedule_for(name, len(self.layers))
+        # activation precision; at n <= 4 the codes also come as e5m2 bytes, so that
+        # linear contractions at b <= 4 run on the 8-bit-float tensor-core kind
+        self.act_bits = workloads.ACT_BITS.get(name, 8)
+        self.code_fmt = tasq.TASQ_CODES_F16_E5M2 if self.act_bits <= 4 else tasq.TASQ_CODES_F16
         if blocks:
             keep = len(workloads.inventory_blocks(name, blocks))
             self.layers, self.table = self.layers[:keep], np.ascontiguousarray(self.table[:keep])
@@ -184,7 +189,7 @@ class Step:
         self.packed, self.x, self.y = [], [], []
         max_mk = max(l.M * (l.Cin if l.Cin else l.K) for l in self.layers)
         max_m = max(l.M for l in self.layers)
-        self.codes = torch.empty((max_mk,), dtype=torch.float16, device=dev)
+        self.codes = torch.empty((max_mk * (3 if self.act_bits <= 4 else 2) // 2,), dtype=torch.float16, device=dev)
         self.alpha = torch.empty((max_m,), dtype=torch.float32, device=dev)
         self.zc = torch.empty((max_m,), dtype=torch.float32, device=dev)
         for unit in self.units:
@@ -229,17 +234,17 @@ class Step:
         conv = l.kind == self.conv
         if "quant" in parts:
             gran = t.TASQ_PER_TENSOR if conv else t.TASQ_PER_TOKEN
-            t.tasq_quant_act(self.ctx, self.x[u], t.TASQ_BF16, l.M, l.Cin if conv else l.K, 8, t.TASQ_SYMRANGE, gran,
-                             self.codes, t.TASQ_CODES_F16, self.alpha, self.zc)
+            t.tasq_quant_act(self.ctx, self.x[u], t.TASQ_BF16, l.M, l.Cin if conv else l.K, self.act_bits,
+                             t.TASQ_SYMRANGE, gran, self.codes, self.code_fmt, self.alpha, self.zc)
         if "gemm" in parts:
             if conv:
-                t.tasq_masked_conv3x3(self.ctx, unit[0], -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.B,
+                t.tasq_masked_conv3x3(self.ctx, unit[0], -1, self.codes, self.code_fmt, self.alpha, self.zc, l.B,
                                       l.H, l.W, l.Cin, self.packed[u], N, self.y[u], None)
             elif len(unit) == 1:
-                t.tasq_masked_gemm(self.ctx, unit[0], -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc, l.M,
+                t.tasq_masked_gemm(self.ctx, unit[0], -1, self.codes, self.code_fmt, self.alpha, self.zc, l.M,
                                    self.packed[u], N, l.K, self.y[u], None)
             else:
-                t.tasq_masked_gemm_grouped(self.ctx, unit, -1, self.codes, t.TASQ_CODES_F16, self.alpha, self.zc,
+                t.tasq_masked_gemm_grouped(self.ctx, unit, -1, self.codes, self.code_fmt, self.alpha, self.zc,
                                            l.M, self.packed[u], N, l.K, self.y[u], None)
 
     def launches_per_step(self):
@@ -364,6 +369,55 @@ def run_sweep(torch, tasq, workloads, shapes=None, reps=10, seed=0):
         del sw, cw, pk, codes, al, zc, y
     tasq.tasq_destroy(ctx)
     return out, switch
+
+
+def run_sweep_a4(torch, tasq, workloads, shapes=((4096, 4096), (16384, 4096), (4096, 1152)), reps=10, seed=0):
+    """The shape sweep with 4-bit activation codes (uniform in [-8, 7]) in the dual
+    fp16 + e5m2 storage: b <= 4 runs the K loop on the e5m2 tensor-core kind, b >= 5
+    on the fp16 codes.  TOPS (2 M N K per call) per b."""
+    ctx = tasq.tasq_create(torch.cuda.current_device())
+    table = workloads.schedule_for("sweep", 1)  # stages 0..6 <-> b = 2..8
+    tasq.tasq_set_schedule(ctx, table, 1, table.shape[1])
+    F8 = tasq.TASQ_CODES_F16_E5M2
+    out = []
+    for si, (M, KN) in enumerate(shapes):
+        N = K = KN
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed * 1000 + 300 + si)
+        sw = torch.randint(-127, 128, (N, K), generator=g, device="cuda", dtype=torch.int8)
+        cw = torch.rand((N,), generator=g, device="cuda") * 1e-3 + 1e-4
+        pk = torch.empty((tasq.tasq_packed_bytes(tasq.TASQ_LINEAR, N, K),), dtype=torch.uint8, device="cuda")
+        tasq.tasq_pack_weights(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K, 0, pk)
+        s = torch.randint(-8, 8, (M, K), generator=g, device="cuda", dtype=torch.int8)
+        codes = torch.empty((3 * M * K,), dtype=torch.uint8, device="cuda")
+        codes[:2 * M * K].view(torch.float16).copy_(s.view(-1).to(torch.float16))
+        codes[2 * M * K:].view(torch.float8_e5m2).copy_(s.view(-1).to(torch.float8_e5m2))
+        al = torch.rand((M,), generator=g, device="cuda") * 1e-2 + 1e-3
+        zc = torch.full((M,), 0.5, device="cuda")
+        y = torch.empty((M, N), dtype=torch.int16, device="cuda")
+        row = {"M": M, "K": K, "N": N, "act_bits": 4, "tops_by_b": {}}
+        for b in range(2, 9):
+            stage = b - 2
+            call = lambda: tasq.tasq_masked_gemm(ctx, 0, stage, codes, F8, al, zc, M, pk, N, K, y)
+            call()
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, capture_error_mode="thread_local"):
+                for _ in range(reps):
+                    call()
+            gr.replay()
+            torch.cuda.synchronize()
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record()
+            gr.replay()
+            t1.record()
+            torch.cuda.synchronize()
+            us = t0.elapsed_time(t1) * 1e3 / reps
+            row["tops_by_b"][b] = 2.0 * M * N * K / (us * 1e-6) / 1e12
+        out.append(row)
+        del sw, cw, pk, s, codes, al, zc, y
+    assert tasq.tasq_device_status(ctx) == tasq.TASQ_OK
+    tasq.tasq_destroy(ctx)
+    return out
 
 
 def int8_tensor_peak(torch, n=8192, reps=20):
@@ -643,7 +697,7 @@ def job_tops(ops_per_rank: float, world: int, ms: float) -> float:
 # Denoising steps of the trajectory each workload's stages partition (stage of
 # step t = floor(t S / T), stage 0 the noisiest): 20 for the DiTs, 4 for the
 # distilled UNet; the single layer runs its 4 stages once each.
-TRAJECTORY_STEPS = {"pixart": 20, "sana": 20, "sdxl": 4, "single": 4}
+TRAJECTORY_STEPS = {"pixart": 20, "pixart_a4": 20, "sana": 20, "sdxl": 4, "single": 4}
 
 
 def stage_map(name: str, S: int):
@@ -713,7 +767,7 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     and with only its quantizations, the all-8-bit schedule on the same graph, and
     the end-to-end step.  Returns the figures and the Step (closed by the caller)."""
     from paper_2608_03057_gb300 import engine_model, schedule
-    step = Step(torch, tasq, workloads, name, args.seed, args.blocks if name in ("pixart", "sana") else 0)
+    step = Step(torch, tasq, workloads, name, args.seed, args.blocks if name in ("pixart", "pixart_a4", "sana") else 0)
     S = step.S
     stage_of = stage_map(name, S)
     for k in range(2):  # eager launches first: they set kernel attributes outside any capture
@@ -748,6 +802,15 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
         tasq.tasq_set_schedule(step.ctx, workloads.schedule_constant(L, S, 8), L, S)
         ms8 = timed_replays(torch, g, step, steps, stage_of)
         tasq.tasq_set_schedule(step.ctx, step.table, L, S)
+    # at 4-bit activations linear layers run the K loop on the e5m2 kind for b <= 4: the
+    # same graph replayed with every (layer, stage) at one b shows the step time against b
+    ms_by_b = None
+    if step.act_bits <= 4:
+        ms_by_b = {}
+        for bb in (2, 4, 5, 6, 8):
+            tasq.tasq_set_schedule(step.ctx, workloads.schedule_constant(L, S, bb), L, S)
+            ms_by_b[bb] = timed_replays(torch, g, step, steps, stage_of)
+        tasq.tasq_set_schedule(step.ctx, step.table, L, S)
     assert tasq.tasq_device_status(step.ctx) == tasq.TASQ_OK
     e2e_out = None
     if e2e:
@@ -778,8 +841,9 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     out = {
         "workload": WORKLOAD_NAMES[name], "layers": L, "contraction_calls": U, "stages": S, "ms_per_step": ms,
         "value": job_tops(step.ops, world, ms), "unit": UNIT, "ms_per_step_all8": ms8,
-        "effective_w_bits": eff_w, "rel_bitops": schedule.rel_bitops(eff_w, 8),
-        "engine_model_rel_cost": engine_model.schedule_cost(step.table, step.gemm_ops, 8),
+        "act_bits": step.act_bits, "ms_per_step_constant_b": ms_by_b,
+        "effective_w_bits": eff_w, "rel_bitops": schedule.rel_bitops(eff_w, step.act_bits),
+        "engine_model_rel_cost": engine_model.schedule_cost(step.table, step.gemm_ops, step.act_bits),
         "roofline": roofline,
         "roofline_quant_act": {"bound": "hbm", "bytes_per_step": act_b, "achieved": act_b / (ms_quant * 1e-3) / 1e9,
                                "peak": peaks["hbm"], "unit": "GB/s",
@@ -836,9 +900,10 @@ def main():
             torch.cuda.empty_cache()
             per_workload[name] = r
 
-    sweep = switch = zp = i8 = small_m = mma_kinds = None
+    sweep = switch = zp = i8 = small_m = mma_kinds = sweep_a4 = None
     if not args.no_sweep:
         sweep, switch = run_sweep(torch, tasq, workloads, seed=args.seed)
+        sweep_a4 = run_sweep_a4(torch, tasq, workloads, seed=args.seed)
         zp = run_zero_point(torch, tasq, workloads, seed=args.seed)
         small_m = run_small_m_weight_bytes(torch, tasq, seed=args.seed)
         from paper_2608_03057_gb300 import mma_probe
@@ -889,6 +954,7 @@ def main():
             "route_peak": route_peak,
             "per_workload": per_workload,
             "sweep_tops_by_b": sweep,
+            "sweep_a4_tops_by_b": sweep_a4,
             "stage_switch": switch,
             "asym_weights": zp,
             "small_m_weight_bytes": small_m,

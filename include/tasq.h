@@ -85,8 +85,18 @@ enum { TASQ_SYMRANGE = 0, TASQ_ASYM = 1 };                /* quantization range 
 enum { TASQ_PER_TOKEN = 0, TASQ_PER_TENSOR = 1 };         /* activation granularity */
 /* Storage of activation codes s = Q - 2^(n-1): one signed byte, or the same
  * integer held exactly in an IEEE fp16 (the operand type of the tensor-core
- * route; every integer in [-128, 127] is exact in fp16). */
-enum { TASQ_CODES_S8 = 0, TASQ_CODES_F16 = 1 };
+ * route; every integer in [-128, 127] is exact in fp16).  TASQ_CODES_F16_E5M2
+ * (activation precision n <= 4, |s| <= 8) stores the fp16 codes [M][K] and,
+ * right after them, the same codes as OCP e5m2 bytes [M][K] (every integer of
+ * magnitude <= 8 has at most three significant bits and is exact in e5m2):
+ * 3 * M * K bytes.  With it a linear tensor-core contraction runs its K loop on
+ * the 8-bit-float MMA kind (twice the K per instruction) whenever the operating
+ * precision is b <= 4, because the masked weight code mask_b(s_w) then has at
+ * most three significant bits and is exact in e5m2 too (unsplit launches); for
+ * b > 4, split-K launches and convolutions it reads the fp16 codes.  Either way
+ * the bound |s| <= 8 lets an exact fp32 chunk run 16 times as long as the one
+ * certified for 8-bit codes; codes outside it are outside the format. */
+enum { TASQ_CODES_S8 = 0, TASQ_CODES_F16 = 1, TASQ_CODES_F16_E5M2 = 2 };
 /* Contraction routes.  TC: tcgen05 MMA on fp16-held integer codes with fp32
  * accumulation in tensor memory, drained to int32 in chunks whose exactness
  * is certified at pack time (needs TASQ_CODES_F16).  MMA_S8: warp-level
@@ -411,9 +421,10 @@ int tasq_plan_tc(int kind, int M, int N, int K, int B, int H, int W, int Cin, in
  * Probe of the tensor-core MMA kinds (diagnostic; the paper has no
  * counterpart).  Launches `ctas` CTAs (one per SM); each loads A (128 rows)
  * and B (n rows) of 128 bytes per row from d_a / d_b (row-major bytes: fp16
- * values for kind 0, e4m3 values for kind 1), and one thread issues 4 * reps
- * tcgen05.mma of that kind (kind 0: kind::f16, 16 elements of K per
- * instruction; kind 1: kind::f8f6f4 with e4m3 A and B, 32 elements), M = 128,
+ * values for kind 0, e4m3 values for kind 1, e5m2 values for kind 2), and one
+ * thread issues 4 * reps tcgen05.mma of that kind (kind 0: kind::f16, 16
+ * elements of K per instruction; kind 1: kind::f8f6f4 with e4m3 A and B, kind 2:
+ * kind::f8f6f4 with e5m2 A and B, 32 elements), M = 128,
  * N = n, accumulating D = reps * A . B^T (over the 64 or 128 elements of a row)
  * in fp32 in tensor memory.  d_cycles[i] receives CTA i's clock cycles from the
  * first MMA to the completion of the last (0 if that wait gave up after 2 s);

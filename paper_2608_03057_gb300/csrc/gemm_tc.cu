@@ -54,10 +54,11 @@ constexpr int BK = 128;           // K per weight stage and per tensor-memory sl
 constexpr int XK = 64;            // K per activation TMA box (one 128-byte swizzle atom of fp16 codes)
 constexpr int W_STAGES = 3;
 constexpr int ASLOTS = 2;         // converted-weight slots in tensor memory
-constexpr int EPI_WARP0 = 6;      // first epilogue warp
-constexpr int EPI_WARPS = 12;     // three per tensor-memory lane quadrant
-constexpr int EPI_PARTS = EPI_WARPS / 4;           // epilogue warps per lane quadrant
-constexpr int WPROD_WARP = EPI_WARP0 + EPI_WARPS;  // weight-tile producer
+// Warps 2 .. 17 are converters (4, one per tensor-memory lane quadrant, or 8, two per
+// quadrant each widening half of a K block) followed by epilogue warps (12 or 8).
+constexpr int MID_WARPS = 16;
+constexpr int MAX_EPI_WARPS = 12;
+constexpr int WPROD_WARP = 2 + MID_WARPS;  // weight-tile producer
 constexpr int THREADS = (WPROD_WARP + 1) * 32;
 constexpr int W_STAGE = BCH * BK;       // 16 KB int8 codes, 128-byte rows
 constexpr uint32_t A_SLOT_COLS = BK / 2;
@@ -72,10 +73,15 @@ static_assert(BK == 2 * XK, "a stage is two 64-wide swizzle atoms");
 // accumulator then only has to wait for the drain between certified chunks.
 // <64, 2>: for launches with few tokens, three times as many CTAs as <192, 2>
 // and a third of its per-tile epilogue.
-template <int BT_, int NACC_>
+template <int BT_, int NACC_, int CONV_WARPS_ = 4>
 struct Cfg {
     static constexpr int BT = BT_;
     static constexpr int NACC = NACC_;
+    static constexpr int CONV_WARPS = CONV_WARPS_;           // converter warps (4 or 8)
+    static constexpr int CONV_SPLIT = CONV_WARPS / 4;        // converters per lane quadrant (K split)
+    static constexpr int EPI_WARP0 = 2 + CONV_WARPS;         // first epilogue warp
+    static constexpr int EPI_WARPS = MID_WARPS - CONV_WARPS; // epilogue warps
+    static constexpr int EPI_PARTS = EPI_WARPS / 4;          // epilogue warps per lane quadrant
     // Q activation stages per K block: 1 (a 128-K stage, one wait per K block on
     // the MMA thread) or 2 (64-K stages released half a block earlier, for the
     // N = 256 tile, whose MMAs leave the issuing thread time for a second wait)
@@ -86,20 +92,28 @@ struct Cfg {
     static constexpr int DONE = 2 * X_STAGES;            // stage-completion barriers (ring of MMA commits)
     static constexpr int GROUPS = BT / 32;               // 32-token column groups of the accumulator
     static constexpr int GPW = (GROUPS + EPI_PARTS - 1) / EPI_PARTS;  // groups per epilogue warp
-    // the single-tile configuration lets the 4 converter warps, idle once the last K
-    // block is converted, drain a fourth share of the tile's groups
-    static constexpr int EPI_SLOTS = EPI_WARPS + (NACC == 1 ? 4 : 0);
+    // the single-tile configuration lets 4 converter warps, idle once the last K block
+    // is converted, drain a fourth share of the tile's groups
+    static constexpr bool HELPERS = NACC == 1 && CONV_WARPS == 4;
+    static constexpr int EPI_SLOTS = EPI_WARPS + (HELPERS ? 4 : 0);
     static constexpr uint32_t ACC_COL = 0;               // NACC x BT fp32 accumulators
     static constexpr uint32_t A_COL = NACC * BT;         // ASLOTS x BK/2 columns (fp16 pairs)
     static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BT);
+    static constexpr uint32_t IDESC8 = ptx::idesc_e5m2_f32(BCH, BT);  // the 8-bit route
     static_assert(DONE % X_STAGES == 0 && DONE >= (ASLOTS + 1) * Q, "completion ring covers both reuse distances");
     static_assert(Q == 1 || X_STAGES % 2 == 0, "first-half stages must keep their parity");
     static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
     static_assert(GPW <= MAX_GPW && BT <= 256 && BT % 32 == 0, "tile shape");
+    static_assert((CONV_WARPS == 4 || CONV_WARPS == 8) && EPI_WARPS <= MAX_EPI_WARPS, "warp roles");
 };
 using CfgStd = Cfg<192, 2>;
 using CfgWide = Cfg<256, 1>;
 using CfgNarrow = Cfg<64, 2>;  // few tokens (cross-attention keys and values): more CTAs, shorter epilogue
+// The two-accumulator tiles for linear layers whose codes also come as e5m2: the 8-bit
+// route's block of two weight tiles is shared out between two converter warps per lane
+// quadrant (one tile each), with eight epilogue warps.
+using CfgStdF8 = Cfg<192, 2, 8>;
+using CfgNarrowF8 = Cfg<64, 2, 8>;
 
 // Synchronisation is arranged so that the single MMA-issuing thread, whose
 // per-instruction cost bounds the K loop, does one wait and one commit per
@@ -135,7 +149,8 @@ struct Smem {
 template <class C>
 constexpr int smem_bytes() { return int(sizeof(Smem<C>)) + 1024; }
 static_assert(smem_bytes<CfgStd>() <= 227 * 1024 && smem_bytes<CfgWide>() <= 227 * 1024 &&
-                  smem_bytes<CfgNarrow>() <= 227 * 1024,
+                  smem_bytes<CfgNarrow>() <= 227 * 1024 && smem_bytes<CfgStdF8>() <= 227 * 1024 &&
+                  smem_bytes<CfgNarrowF8>() <= 227 * 1024,
               "shared memory per CTA");
 
 struct TcParams {
@@ -216,6 +231,14 @@ __device__ __forceinline__ void widen4(uint32_t w, uint32_t m, uint32_t& lo, uin
     hi = *reinterpret_cast<uint32_t*>(&h);
 }
 
+// e5m2 bytes of four masked codes whose values have at most three significant bits
+// (b <= 4): the upper bytes of their fp16 values (see ptx::e5m2x4).
+__device__ __forceinline__ uint32_t masked_e5m2x4(uint32_t w, uint32_t m) {
+    uint32_t lo, hi;
+    widen4(w, m, lo, hi);
+    return ptx::e5m2x4(lo, hi);
+}
+
 struct TileCoord {
     int ch0;  // first channel of the tile's 128 rows
     int tok0, img, h0, w0;
@@ -238,43 +261,41 @@ __device__ __forceinline__ TileCoord tile_coord(const TcParams& p, int t) {
     return c;
 }
 
-// CONV selects the implicit-GEMM 3x3 convolution (one instantiation per
-// operand layout, so neither pays for the other's index arithmetic); ZP the
-// four-term epilogue of asymmetric weights.
-template <bool CONV, bool ZP, class C>
+// Whether a launch whose codes also come as e5m2 takes the 8-bit route: every member
+// layer's b is known (the table lookup succeeded) and at most 4, so that its masked
+// weight codes have at most three significant bits.
+__device__ __forceinline__ bool f8_route(const GemmArgs& a, uint32_t gbits) {
+    bool f8 = gbits != 0;
+#pragma unroll
+    for (int g = 0; g < kMaxGroups; ++g)
+        if (g < a.groups && int((gbits >> (4 * g)) & 15u) > kBMaxF8) f8 = false;
+    return f8;
+}
+
+// CONV selects the implicit-GEMM 3x3 convolution (one instantiation per operand
+// layout, so neither pays for the other's index arithmetic); ZP the four-term
+// epilogue of asymmetric weights; F8 a linear layer whose codes also come as e5m2
+// bytes (tm_x8): when every member's b is <= 4 the K loop runs on the 8-bit route
+// (kind::f8f6f4 MMAs with e5m2 operands, 32 codes of K per instruction), else on
+// the fp16 codes as usual.
+template <bool CONV, bool ZP, class C, bool F8 = false>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
-                   const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_y) {
+                   const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_y,
+                   const __grid_constant__ CUtensorMap tm_x8) {
     constexpr int X_STAGES = C::X_STAGES, X_HALF = C::X_HALF, X_STAGE = C::X_STAGE, NACC = C::NACC;
     constexpr int Q = C::Q, DONE = C::DONE;
     constexpr int BT = C::BT, GPW = C::GPW;
+    constexpr int EPI_WARP0 = C::EPI_WARP0, EPI_WARPS = C::EPI_WARPS, EPI_PARTS = C::EPI_PARTS;
+    constexpr int CONV_WARPS = C::CONV_WARPS;
     extern __shared__ uint8_t smem_raw[];
     Smem<C>* s = reinterpret_cast<Smem<C>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const GemmArgs& a = p.a;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const Waiter<C> wt{s, &a};
 
-    // Set-up that does not depend on b (barriers, tensor memory, descriptor prefetch)
-    // overlaps the loads that resolve it.
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < X_STAGES; ++i)  // producer's expect_tx (+ the 4 converter warps on first stages)
-            ptx::mbar_init(ptx::smem_u32(&s->xfull[i]), i % Q == 0 ? 1 + 4 : 1);
-        for (int i = 0; i < DONE; ++i) ptx::mbar_init(ptx::smem_u32(&s->done[i]), 1);  // the MMA commit
-        for (int i = 0; i < W_STAGES; ++i) {
-            ptx::mbar_init(ptx::smem_u32(&s->wfull[i]), 1);
-            ptx::mbar_init(ptx::smem_u32(&s->wempty[i]), 4);  // the 4 converter warps
-        }
-        for (int i = 0; i < NACC; ++i) {
-            ptx::mbar_init(ptx::smem_u32(&s->accfull[i]), 1);
-            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS);
-        }
-        ptx::mbar_init(ptx::smem_u32(&s->drain), 1);
-        s->abort = 0;
-        ptx::fence_mbar_init();
-        ptx::prefetch_tmap(&tm_x);
-        ptx::prefetch_tmap(&tm_w);
-        if constexpr (!CONV) ptx::prefetch_tmap(&tm_y);
-    }
+    // Set-up that does not depend on b (tensor memory, descriptor prefetch) overlaps the
+    // loads that resolve it.
     if (warp == 1) {
         ptx::tmem_alloc(ptx::smem_u32(&s->tmem_base), TMEM_COLS);
         ptx::tmem_relinquish();
@@ -296,10 +317,38 @@ __global__ void __maxnreg__(96)
         for (int i = 0; i < kNumB; ++i)
             if (g < a.groups && bg == kBMin + i) chunk_kb = min(chunk_kb, cert[i]);
     }
-    const int KT = (a.K + BK - 1) / BK;
-    // certificate is in 64-wide K blocks; a run of c64 of them covers c64/2 of ours
-    int chunk = chunk_kb / (BK / kCertKBlock);
-    chunk = chunk < 1 ? 1 : (chunk > KT ? KT : chunk);
+    // The 8-bit route (uniform over the grid).  Its K block is 256 codes: their e5m2 bytes
+    // fill exactly the activation stage, the tensor-memory weight slot and the MMA
+    // descriptors of a 128-code fp16 block (a 128-byte row segment per 32-byte K step
+    // either way), so both routes share every ring; only the MMA kind, the activation
+    // tensor map, the weight tiles per block (two) and the converters' arithmetic differ.
+    // It needs an unsplit launch and an exact chunk of at least one such block.
+    const int64_t chunk_k64 = int64_t(chunk_kb) * a.chunk_scale;  // exact chunk in 64-code blocks
+    const bool f8 = F8 && p.splits == 1 && chunk_k64 >= 2 * BK / kCertKBlock && f8_route(a, gbits);
+    const int KBLK = f8 ? 2 * BK : BK;  // codes of K per block
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < X_STAGES; ++i)  // producer's expect_tx (+ the converter warps on first stages)
+            ptx::mbar_init(ptx::smem_u32(&s->xfull[i]), i % Q == 0 ? 1 + CONV_WARPS : 1);
+        for (int i = 0; i < DONE; ++i) ptx::mbar_init(ptx::smem_u32(&s->done[i]), 1);  // the MMA commit
+        for (int i = 0; i < W_STAGES; ++i) {
+            ptx::mbar_init(ptx::smem_u32(&s->wfull[i]), 1);
+            ptx::mbar_init(ptx::smem_u32(&s->wempty[i]), CONV_WARPS);  // every converter warp, every tile
+        }
+        for (int i = 0; i < NACC; ++i) {
+            ptx::mbar_init(ptx::smem_u32(&s->accfull[i]), 1);
+            ptx::mbar_init(ptx::smem_u32(&s->accempty[i]), EPI_WARPS);
+        }
+        ptx::mbar_init(ptx::smem_u32(&s->drain), 1);
+        s->abort = 0;
+        ptx::fence_mbar_init();
+        ptx::prefetch_tmap(f8 ? &tm_x8 : &tm_x);
+        ptx::prefetch_tmap(&tm_w);
+        if constexpr (!CONV) ptx::prefetch_tmap(&tm_y);
+    }
+    const int KT = (a.K + KBLK - 1) / KBLK;
+    // the exact chunk is in 64-wide K blocks; a run of c64 of them covers c64 / (KBLK / 64) of ours
+    const int64_t chunk64 = chunk_k64 / (KBLK / kCertKBlock);
+    const int chunk = chunk64 < 1 ? 1 : (chunk64 > KT ? KT : int(chunk64));
     const int works = p.tiles_ch * p.tiles_tok * p.splits;
     const int unit = int(blockIdx.x), units = int(gridDim.x);
     __syncthreads();
@@ -313,7 +362,7 @@ __global__ void __maxnreg__(96)
         // pull the first weight tiles into L2 ahead of the weight ring
         const Work wk = work_item(p, unit, KT, chunk);
         const int ch0 = tile_coord<CONV, BT>(p, wk.t).ch0;
-        for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * BK, ch0);
+        for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * KBLK, ch0);
     }
     // Programmatic dependent launch: this grid may start while the previous kernel
     // (normally the quantization of this layer's activations) still runs.  Only the
@@ -337,16 +386,20 @@ __global__ void __maxnreg__(96)
                         break;
                     }
                     const uint32_t fb = ptx::smem_u32(&s->xfull[u % X_STAGES]);
-                    ptx::mbar_arrive_expect_tx(fb, X_STAGE);
                     const uint32_t dst = ptx::smem_u32(s->x[u % X_STAGES]);
+                    ptx::mbar_arrive_expect_tx(fb, X_STAGE);
 #pragma unroll
                     for (int hh = 0; hh < 2 / Q; ++hh) {
+                        // box hh of the stage: 128 bytes of each token's row, 64 fp16 codes
+                        // or 128 e5m2 codes
                         const int kh = kq * (BK / Q) + hh * XK;
                         if constexpr (CONV) {
                             // a 128-wide K block may straddle two taps when Cin % 128 == 64
                             const int tap = kh / a.Cin, c0 = kh - tap * a.Cin;
                             ptx::tma_load_4d(dst + hh * X_HALF, &tm_x, fb, c0, tc.w0 + tap % 3 - 1, tc.h0 + tap / 3 - 1,
                                              tc.img);
+                        } else if (F8 && f8) {
+                            ptx::tma_load_2d(dst + hh * X_HALF, &tm_x8, fb, 2 * kh, tc.tok0);
                         } else {
                             ptx::tma_load_2d(dst + hh * X_HALF, &tm_x, fb, kh, tc.tok0);
                         }
@@ -366,17 +419,18 @@ __global__ void __maxnreg__(96)
             Ring<W_STAGES> rw;
             int nw = 0;
             bool ok = true;
+            const int wpb = f8 ? 2 : 1;  // 128-code weight tiles per K block
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
                 const int ch0 = tile_coord<CONV, BT>(p, wk.t).ch0;
-                for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++nw, rw.next()) {
+                for (int kw = wk.kb_lo * wpb; kw < wk.kb_hi * wpb; ++kw, ++nw, rw.next()) {
                     if (!wt.wait(&s->wempty[rw.slot], rw.phase ^ 1)) {
                         ok = false;
                         break;
                     }
                     const uint32_t fb = ptx::smem_u32(&s->wfull[rw.slot]);
                     ptx::mbar_arrive_expect_tx(fb, W_STAGE);
-                    ptx::tma_load_2d(ptx::smem_u32(s->w[rw.slot]), &tm_w, fb, kb * BK, ch0);
+                    ptx::tma_load_2d(ptx::smem_u32(s->w[rw.slot]), &tm_w, fb, kw * BK, ch0);
                 }
             }
             for (int j = nw - W_STAGES < 0 ? 0 : nw - W_STAGES; j < nw; ++j)
@@ -409,13 +463,20 @@ __global__ void __maxnreg__(96)
                             }
                             ptx::tc_fence_after();
                             for (int hh = 0; hh < 2 / Q; ++hh) {
-                                // one 64-wide swizzle atom; a K step of 16 codes is 32 bytes along its rows
+                                // one 128-byte swizzle atom per row (64 fp16 or 128 e5m2 codes); a K
+                                // step (16 fp16 or 32 e5m2 codes) is 32 bytes along its rows
                                 const uint64_t bdesc =
                                     ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[u % X_STAGES] + hh * X_HALF));
-                                const int k0 = (i * (2 / Q) + hh) * (XK / 16);  // K step of 16 within the block
-                                for (int kk = 0; kk < XK / 16; ++kk)
-                                    ptx::mma_f16_ts(d, acol + (k0 + kk) * 8, bdesc + uint64_t((kk * 32) >> 4), C::IDESC,
-                                                    (kb > kb0 || k0 + kk > 0) ? 1u : 0u);
+                                const int k0 = (i * (2 / Q) + hh) * (XK / 16);  // K step within the block
+                                if (F8 && f8) {
+                                    for (int kk = 0; kk < XK / 16; ++kk)
+                                        ptx::mma_f8_ts(d, acol + (k0 + kk) * 8, bdesc + uint64_t((kk * 32) >> 4),
+                                                       C::IDESC8, (kb > kb0 || k0 + kk > 0) ? 1u : 0u);
+                                } else {
+                                    for (int kk = 0; kk < XK / 16; ++kk)
+                                        ptx::mma_f16_ts(d, acol + (k0 + kk) * 8, bdesc + uint64_t((kk * 32) >> 4),
+                                                        C::IDESC, (kb > kb0 || k0 + kk > 0) ? 1u : 0u);
+                                }
                             }
                             ptx::mma_commit(ptx::smem_u32(&s->done[u % DONE]));
                         }
@@ -429,8 +490,17 @@ __global__ void __maxnreg__(96)
         }
     } else if (warp < EPI_WARP0) {
         // ------------------------------------------- weight mask + convert
-        const int q = warp & 3;             // tensor-memory lane quadrant
-        const int r = q * 32 + lane;        // channel row within the tile
+        // Converter warp c serves the 32 channel rows of lane quadrant c % 4 and part
+        // kp = (c - 2) / 4 of each K block: the fp16 route's block (one 128-code weight
+        // tile) is cut into CONV_SPLIT runs of codes, the 8-bit route's block (two tiles)
+        // into CONV_SPLIT runs of tiles.  Either way a part fills 64 / CONV_SPLIT
+        // tensor-memory columns of the block's slot.
+        constexpr int SPLIT = C::CONV_SPLIT;
+        constexpr int CH = 8 / SPLIT;        // fp16 route: 16-byte chunks of a row per part
+        constexpr int NF = 64 / SPLIT;       // 32-bit words (columns) per part and block
+        const int q = warp & 3;              // tensor-memory lane quadrant
+        const int kp = (warp - 2) >> 2;      // K part
+        const int r = q * 32 + lane;         // channel row within the tile
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         Ring<W_STAGES> rw;
         int it = 0;
@@ -439,28 +509,59 @@ __global__ void __maxnreg__(96)
             const Work wk = work_item(p, w, KT, chunk);
             // this row's channel runs at its layer's b (a grouped call holds several layers)
             const uint32_t m = mask_word(channel_bits(a, gbits, tile_coord<CONV, BT>(p, wk.t).ch0 + r));
-            for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it, rw.next()) {
-                if (!wt.wait(&s->wfull[rw.slot], rw.phase)) {
-                    ok = false;
-                    break;
-                }
-                // 128 codes of row r; 16-byte chunk c sits at c ^ (r & 7) (128-byte swizzle).
-                // Mask and widen before waiting for the slot, so that only the
+            for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it) {
+                // Row r of a tile holds 128 codes; 16-byte chunk c sits at c ^ (r & 7) (128-byte
+                // swizzle).  Mask and widen before waiting for the slot, so that only the
                 // tensor-memory store remains once the MMA releases it.
-                uint32_t f[64];
-                {
+                uint32_t f[NF];
+                if (F8 && f8) {
+                    // e5m2 (b <= 4): one word per 4 codes, 32 words per tile.  Every
+                    // converter warp passes both tiles of the block through the ring in
+                    // order (a part that skipped the other part's tiles could wait on a
+                    // slot two phases ahead, which one parity bit cannot tell apart) and
+                    // converts its own: both tiles, or tile kp of two parts.
+#pragma unroll
+                    for (int t = 0; t < 2; ++t) {
+                        if (!wt.wait(&s->wfull[rw.slot], rw.phase)) {
+                            ok = false;
+                            break;
+                        }
+                        if (SPLIT == 1 || t == kp) {
+                            const int o = SPLIT == 1 ? 32 * t : 0;
+                            const uint8_t* row = s->w[rw.slot] + r * BK;
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) {
+                                const uint4 u = *reinterpret_cast<const uint4*>(row + ((c ^ (r & 7)) << 4));
+                                f[o + 4 * c + 0] = masked_e5m2x4(u.x, m);
+                                f[o + 4 * c + 1] = masked_e5m2x4(u.y, m);
+                                f[o + 4 * c + 2] = masked_e5m2x4(u.z, m);
+                                f[o + 4 * c + 3] = masked_e5m2x4(u.w, m);
+                            }
+                        }
+                        __syncwarp();
+                        if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->wempty[rw.slot]));
+                        rw.next();
+                    }
+                    if (!ok) break;
+                } else {
+                    // fp16: two words per 4 codes
+                    if (!wt.wait(&s->wfull[rw.slot], rw.phase)) {
+                        ok = false;
+                        break;
+                    }
                     const uint8_t* row = s->w[rw.slot] + r * BK;
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        const uint4 u = *reinterpret_cast<const uint4*>(row + ((c ^ (r & 7)) << 4));
+                    for (int c = 0; c < CH; ++c) {
+                        const uint4 u = *reinterpret_cast<const uint4*>(row + (((kp * CH + c) ^ (r & 7)) << 4));
                         widen4(u.x, m, f[8 * c + 0], f[8 * c + 1]);
                         widen4(u.y, m, f[8 * c + 2], f[8 * c + 3]);
                         widen4(u.z, m, f[8 * c + 4], f[8 * c + 5]);
                         widen4(u.w, m, f[8 * c + 6], f[8 * c + 7]);
                     }
+                    __syncwarp();
+                    if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->wempty[rw.slot]));
+                    rw.next();
                 }
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->wempty[rw.slot]));
                 // slot it % 2 last held K block it - 2: its MMAs must have finished
                 // (the last activation stage of block it - 2 completes after all its MMAs)
                 if (it >= ASLOTS && !wt.wait(&s->done[((it - ASLOTS) * Q + Q - 1) % DONE],
@@ -469,9 +570,10 @@ __global__ void __maxnreg__(96)
                     break;
                 }
                 {
-                    const uint32_t dst = lane_base + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
-                    ptx::tmem_st32(dst, *reinterpret_cast<const uint32_t(*)[32]>(&f[0]));
-                    ptx::tmem_st32(dst + 32, *reinterpret_cast<const uint32_t(*)[32]>(&f[32]));
+                    const uint32_t dst = lane_base + C::A_COL + (it % ASLOTS) * A_SLOT_COLS + kp * NF;
+#pragma unroll
+                    for (int h = 0; h < NF / 32; ++h)
+                        ptx::tmem_st32(dst + 32 * h, *reinterpret_cast<const uint32_t(*)[32]>(&f[32 * h]));
                 }
                 ptx::tmem_wait_st();
                 ptx::tc_fence_before();
@@ -483,7 +585,7 @@ __global__ void __maxnreg__(96)
     // Helper mode (uniform over the CTA): a single-tile CTA whose tile is one
     // certified chunk (linear layers) drains it with the converter warps too,
     // four warps per lane quadrant instead of three.
-    const bool helpers = !CONV && C::NACC == 1 && unit < works && works <= units &&
+    const bool helpers = !CONV && C::HELPERS && unit < works && works <= units &&
                          work_item(p, unit, KT, chunk).nch == 1;
     if ((warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS) || (helpers && warp >= 2 && warp < EPI_WARP0)) {
         // ------------------------------------- accumulator drain + epilogue
@@ -912,7 +1014,7 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 
 }  // namespace
 
-size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * EPI_WARPS * MAX_GPW * 32 * 32 * sizeof(int32_t); }
+size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * MAX_EPI_WARPS * MAX_GPW * 32 * 32 * sizeof(int32_t); }
 
 namespace {
 
@@ -1025,7 +1127,7 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
     p.a = a;
     p.conv = a.Cin != 0;
     p.tiles_ch = (a.N + BCH - 1) / BCH;
-    CUtensorMap tm_x, tm_w, tm_y;
+    CUtensorMap tm_x, tm_w, tm_y, tm_x8;
     CUresult r;
     p.tiles_tok = int(plan.tiles_tok);
     if (p.conv) {
@@ -1053,6 +1155,24 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
     if (r != CUDA_SUCCESS) {
         *why = "activation tensor map rejected";
         return cudaSuccess;
+    }
+    const bool f8 = !p.conv && a.x8 != nullptr;
+    if (f8) {
+        // the same codes as e5m2 bytes [M][K]: 128 codes of a token are one
+        // 128-byte swizzle atom
+        cuuint64_t dims[2] = {cuuint64_t(a.K), cuuint64_t(a.M)};
+        cuuint64_t strides[1] = {cuuint64_t(a.K)};
+        cuuint32_t box[2] = {BK, cuuint32_t(BTOK)};
+        cuuint32_t es[2] = {1, 1};
+        r = encode(&tm_x8, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(a.x8), dims, strides, box, es,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) {
+            *why = "e5m2 activation tensor map rejected";
+            return cudaSuccess;
+        }
+    } else {
+        tm_x8 = tm_x;  // unused
     }
     {
         cuuint64_t dims[2] = {cuuint64_t(a.K), cuuint64_t(a.N)};
@@ -1090,8 +1210,15 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
         fprintf(stderr, "tasq tc: M=%d N=%d K=%d BT=%d tiles=%lld splits=%d grid=%d\n", a.M, a.N, a.K, BTOK,
                 (long long)p.tiles_ch * p.tiles_tok, p.splits, units);
     const int smem = smem_bytes<C>();
-    auto kernel = p.conv ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
-                         : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
+    auto kernel = [&] {
+        // the eight-converter tiles only serve linear layers with e5m2 codes
+        if constexpr (C::CONV_WARPS == 8)
+            return a.code_sums ? gemm_tc_kernel<false, true, C, true> : gemm_tc_kernel<false, false, C, true>;
+        else
+            return p.conv ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
+                   : f8   ? (a.code_sums ? gemm_tc_kernel<false, true, C, true> : gemm_tc_kernel<false, false, C, true>)
+                          : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
+    }();
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     // programmatic dependent launch: the grid may start while the previous
@@ -1106,7 +1233,7 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w, tm_y);
+    e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w, tm_y, tm_x8);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaSuccess) *kernels = 1;
     if (e == cudaSuccess && p.splits > 1) {
@@ -1151,9 +1278,11 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         *why = plan.why;
         return cudaSuccess;
     }
+    const bool x8 = a.Cin == 0 && a.x8 != nullptr;  // a linear layer with e5m2 codes
     if (plan.bt == CfgWide::BT) return launch_cfg<CfgWide>(a, plan, st, why, kernels);
-    if (plan.bt == CfgNarrow::BT) return launch_cfg<CfgNarrow>(a, plan, st, why, kernels);
-    return launch_cfg<CfgStd>(a, plan, st, why, kernels);
+    if (plan.bt == CfgNarrow::BT)
+        return x8 ? launch_cfg<CfgNarrowF8>(a, plan, st, why, kernels) : launch_cfg<CfgNarrow>(a, plan, st, why, kernels);
+    return x8 ? launch_cfg<CfgStdF8>(a, plan, st, why, kernels) : launch_cfg<CfgStd>(a, plan, st, why, kernels);
 }
 
 }  // namespace tasq

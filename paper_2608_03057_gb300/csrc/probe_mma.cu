@@ -1,9 +1,10 @@
 // Diagnostic probe of the 5th-generation tensor-core MMA kinds on this GPU
 // (no counterpart in the paper): cycles per tcgen05.mma and the exactness of
 // integer-valued operands, for kind::f16 (the exact route's operand type) and
-// kind::f8f6f4 with e4m3 operands (every integer of magnitude <= 16 is exact
-// in e4m3, so a weight truncated to b <= 5 planes times a 4-bit activation code
-// could run on it).  Both operands come from shared memory in the 128-byte
+// kind::f8f6f4 with e4m3 operands (every integer of magnitude <= 16 is exact)
+// or e5m2 operands (integers with at most three significant bits, such as a
+// weight truncated to b <= 4 planes and a 4-bit activation code: the operand
+// type of the 8-bit route).  Both operands come from shared memory in the 128-byte
 // swizzled K-major layout the contraction kernels use; one swizzle atom (128
 // bytes of every row) is contracted `reps` times into an fp32 accumulator in
 // tensor memory, so D = reps * (A . B^T over the atom) -- a long accumulation
@@ -43,8 +44,9 @@ __device__ __forceinline__ void mma_ss(uint32_t d, uint64_t adesc, uint64_t bdes
     }
 }
 
-// KIND 0: f16 x f16 (16 elements = 32 bytes per K step); KIND 1: e4m3 x e4m3
-// (32 elements = 32 bytes per K step).  Either way an atom row is four K steps.
+// KIND 0: f16 x f16 (16 elements = 32 bytes per K step); KIND 1: e4m3 x e4m3,
+// KIND 2: e5m2 x e5m2 (32 elements = 32 bytes per K step).  Either way an atom
+// row is four K steps.
 template <int KIND>
 __global__ void __launch_bounds__(128) probe_mma_kernel(const uint8_t* __restrict__ ga, const uint8_t* __restrict__ gb,
                                                         int n, int reps, float* __restrict__ gd,
@@ -77,8 +79,9 @@ __global__ void __launch_bounds__(128) probe_mma_kernel(const uint8_t* __restric
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem;
-    // instruction descriptor: fp32 D; A and B format 0 (f16 for kind::f16, e4m3 for kind::f8f6f4)
-    const uint32_t idesc = ptx::idesc_f16_f32(PM, n);
+    // instruction descriptor: fp32 D; A and B format 0 (f16 for kind::f16, e4m3 for
+    // kind::f8f6f4) or 1 (e5m2 for kind::f8f6f4)
+    const uint32_t idesc = KIND == 2 ? ptx::idesc_e5m2_f32(PM, n) : ptx::idesc_f16_f32(PM, n);
     bool ok = true;
     if (threadIdx.x == 0) {
         const uint64_t adesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->a));
@@ -128,8 +131,8 @@ extern "C" __attribute__((visibility("default"))) int tasq_probe_mma(int kind, i
                                                                     unsigned long long* d_cycles, int ctas,
                                                                     tasq_stream stream) {
     using namespace tasq;
-    if (kind != 0 && kind != 1) {
-        set_noctx_error("kind must be 0 (f16) or 1 (e4m3)");
+    if (kind < 0 || kind > 2) {
+        set_noctx_error("kind must be 0 (f16), 1 (e4m3) or 2 (e5m2)");
         return TASQ_ERR_INVALID_ARG;
     }
     if (n < 16 || n > MAX_N || n % 16 || reps < 1 || reps > (1 << 20) || ctas < 1 || ctas > 1024 || !d_a || !d_b ||
@@ -144,7 +147,7 @@ extern "C" __attribute__((visibility("default"))) int tasq_probe_mma(int kind, i
     // at least 120 KB of shared memory: one CTA per SM, so that no CTA waits for
     // another's tensor memory (each allocates all 512 columns)
     const int smem = int(sizeof(ProbeSmem)) + 1024 > 120 * 1024 ? int(sizeof(ProbeSmem)) + 1024 : 120 * 1024;
-    auto kernel = kind == 0 ? probe_mma_kernel<0> : probe_mma_kernel<1>;
+    auto kernel = kind == 0 ? probe_mma_kernel<0> : kind == 1 ? probe_mma_kernel<1> : probe_mma_kernel<2>;
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e == cudaSuccess) {
         kernel<<<ctas, 128, smem, (cudaStream_t)stream>>>(d_a, d_b, n, reps, d_d, d_cycles, 2000000000ull);

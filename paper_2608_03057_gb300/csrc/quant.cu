@@ -82,7 +82,9 @@ __device__ inline int act_code(float x, float alpha, float ralpha, float z, int 
     return min(max(q, 0), qmax) - half;
 }
 
-__device__ inline void store8_codes(void* out, int code_fmt, int64_t i, const int s[8]) {
+// Codes s[0..7] of 8-element group i: int8, or fp16 (and, for TASQ_CODES_F16_E5M2,
+// the same codes as e5m2 bytes at out8).
+__device__ inline void store8_codes(void* out, int code_fmt, int64_t i, const int s[8], void* out8 = nullptr) {
     if (code_fmt == TASQ_CODES_S8) {
         uint2 pk;
         pk.x = (s[0] & 0xFF) | ((s[1] & 0xFF) << 8) | ((s[2] & 0xFF) << 16) | ((uint32_t)(s[3] & 0xFF) << 24);
@@ -98,6 +100,8 @@ __device__ inline void store8_codes(void* out, int code_fmt, int64_t i, const in
         pk.z = h[4] | (h[5] << 16);
         pk.w = h[6] | (h[7] << 16);
         reinterpret_cast<uint4*>(out)[i] = pk;
+        if (code_fmt == TASQ_CODES_F16_E5M2)
+            reinterpret_cast<uint2*>(out8)[i] = make_uint2(ptx::e5m2x4(pk.x, pk.y), ptx::e5m2x4(pk.z, pk.w));
     }
 }
 
@@ -187,6 +191,8 @@ __global__ void __launch_bounds__(256) quant_act_token_kernel(const void* __rest
     scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
     const float ralpha = __frcp_rn(alpha);
     char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (code_fmt == TASQ_CODES_S8 ? 1 : 2);
+    // TASQ_CODES_F16_E5M2: the e5m2 copy follows the M x K fp16 codes
+    char* out8 = reinterpret_cast<char*>(codes) + int64_t(M) * K * 2 + int64_t(m) * K;
     int csum = 0;
     for (int i = lane; i < groups; i += 32) {
         float v[8];
@@ -197,7 +203,7 @@ __global__ void __launch_bounds__(256) quant_act_token_kernel(const void* __rest
             s[j] = act_code(v[j], alpha, ralpha, z, qmax, half);
             csum += s[j];
         }
-        store8_codes(out, code_fmt, i, s);
+        store8_codes(out, code_fmt, i, s, out8);
     }
     if (code_sums) csum = warp_sum(csum);
     if (lane == 0) {
@@ -300,6 +306,8 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
     // end in the 16 bits 0x6400 + rint(u) (for 0 <= rint(u) <= 255)
     const float2 magic2 = make_float2(12608512.0f, 12608512.0f);
     char* out = reinterpret_cast<char*>(codes) + int64_t(m) * K * (CODES == TASQ_CODES_S8 ? 1 : 2);
+    // TASQ_CODES_F16_E5M2: the e5m2 copy follows the M x K fp16 codes
+    char* out8 = reinterpret_cast<char*>(codes) + int64_t(M) * K * 2 + int64_t(m) * K;
     int csum = 0;  // sum of this lane's codes Q - half (kept only when code_sums is set)
 #pragma unroll
     for (int k = 0; k < NPL; ++k) {
@@ -370,8 +378,12 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
                 pk.z = sub2(h[4 % EPC], h[5 % EPC]);
                 pk.w = sub2(h[6 % EPC], h[7 % EPC]);
                 reinterpret_cast<uint4*>(out)[c] = pk;
+                if constexpr (CODES == TASQ_CODES_F16_E5M2)
+                    reinterpret_cast<uint2*>(out8)[c] = make_uint2(ptx::e5m2x4(pk.x, pk.y), ptx::e5m2x4(pk.z, pk.w));
             } else {
-                reinterpret_cast<uint2*>(out)[c] = make_uint2(sub2(h[0], h[1]), sub2(h[2 % EPC], h[3 % EPC]));
+                const uint2 pk = make_uint2(sub2(h[0], h[1]), sub2(h[2 % EPC], h[3 % EPC]));
+                reinterpret_cast<uint2*>(out)[c] = pk;
+                if constexpr (CODES == TASQ_CODES_F16_E5M2) reinterpret_cast<uint32_t*>(out8)[c] = ptx::e5m2x4(pk.x, pk.y);
             }
         }
     }
@@ -398,8 +410,11 @@ cudaError_t launch_rowreg(const void* x, int M, int K, int n_bits, int mode, voi
     auto kernel = code_fmt == TASQ_CODES_S8
                       ? (sums ? quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_S8, true>
                               : quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_S8, false>)
-                      : (sums ? quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16, true>
-                              : quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16, false>);
+                  : code_fmt == TASQ_CODES_F16
+                      ? (sums ? quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16, true>
+                              : quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16, false>)
+                      : (sums ? quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16_E5M2, true>
+                              : quant_act_rowreg_kernel<NPL, DTYPE, TASQ_CODES_F16_E5M2, false>);
     cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, x, M, K, n_bits, mode, codes, alpha, zc, sums);
     return e == cudaSuccess ? cudaGetLastError() : e;
 }
@@ -483,7 +498,7 @@ __global__ void __launch_bounds__(256) quant_act_tensor_kernel(const void* __res
         int s[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j) s[j] = act_code(v[j], alpha, ralpha, z, qmax, half);
-        store8_codes(codes, code_fmt, i, s);
+        store8_codes(codes, code_fmt, i, s, reinterpret_cast<char*>(codes) + groups * 16);
     }
     if (blockIdx.x == 0 && threadIdx.x == 0) {
         alpha_out[0] = alpha;

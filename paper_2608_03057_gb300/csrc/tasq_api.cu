@@ -299,8 +299,11 @@ int quant_act(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, int n_bits
     REQUIRE(dtype == TASQ_F32 || dtype == TASQ_BF16, TASQ_ERR_INVALID_ARG, "dtype %d", dtype);
     REQUIRE(mode == TASQ_SYMRANGE || mode == TASQ_ASYM, TASQ_ERR_INVALID_ARG, "mode %d", mode);
     REQUIRE(gran == TASQ_PER_TOKEN || gran == TASQ_PER_TENSOR, TASQ_ERR_INVALID_ARG, "gran %d", gran);
-    REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16, TASQ_ERR_INVALID_ARG, "code_fmt %d", code_fmt);
+    REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16 || code_fmt == TASQ_CODES_F16_E5M2,
+            TASQ_ERR_INVALID_ARG, "code_fmt %d", code_fmt);
     REQUIRE(n_bits >= 2 && n_bits <= 8, TASQ_ERR_INVALID_ARG, "n_bits %d outside 2..8", n_bits);
+    REQUIRE(code_fmt != TASQ_CODES_F16_E5M2 || n_bits <= 4, TASQ_ERR_UNSUPPORTED,
+            "e5m2 codes need n_bits <= 4 (codes of magnitude <= 8), got %d", n_bits);
     REQUIRE(M >= 0 && K > 0, TASQ_ERR_INVALID_ARG, "M=%d K=%d", M, K);
     REQUIRE(K % 16 == 0, TASQ_ERR_UNSUPPORTED, "K=%d must be a multiple of 16", K);
     if (M == 0) return TASQ_OK;
@@ -355,14 +358,15 @@ int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, in
                 ctx->L - 1);
     REQUIRE(stage >= -1 && stage < ctx->S, TASQ_ERR_INVALID_ARG, "stage %d outside -1..%d", stage, ctx->S - 1);
     REQUIRE(stage >= 0 || ctx->d_stage, TASQ_ERR_INVALID_ARG, "stage -1 needs tasq_set_stage_device");
-    REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16, TASQ_ERR_INVALID_ARG, "code_fmt %d", code_fmt);
+    REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16 || code_fmt == TASQ_CODES_F16_E5M2,
+            TASQ_ERR_INVALID_ARG, "code_fmt %d", code_fmt);
     REQUIRE(M >= 0 && N > 0 && K > 0, TASQ_ERR_INVALID_ARG, "M=%d N=%d K=%d", M, N, K);
     REQUIRE(K % 16 == 0 && N % 8 == 0, TASQ_ERR_UNSUPPORTED, "need K %% 16 == 0 and N %% 8 == 0 (N=%d K=%d)", N, K);
     REQUIRE(groups == 1 || (N % groups == 0 && (N / groups) % 8 == 0), TASQ_ERR_UNSUPPORTED,
             "grouped call: N=%d must split into %d members of a multiple of 8 channels", N, groups);
     int route = ctx->route;
-    if (route == TASQ_ROUTE_AUTO) route = code_fmt == TASQ_CODES_F16 ? TASQ_ROUTE_TC : TASQ_ROUTE_MMA_S8;
-    REQUIRE((route == TASQ_ROUTE_TC) == (code_fmt == TASQ_CODES_F16), TASQ_ERR_UNSUPPORTED,
+    if (route == TASQ_ROUTE_AUTO) route = code_fmt == TASQ_CODES_S8 ? TASQ_ROUTE_MMA_S8 : TASQ_ROUTE_TC;
+    REQUIRE((route == TASQ_ROUTE_TC) == (code_fmt != TASQ_CODES_S8), TASQ_ERR_UNSUPPORTED,
             "route %d cannot read code format %d", route, code_fmt);
     if (M == 0) return TASQ_OK;
     REQUIRE(d_codes && d_alpha && d_zc && d_packed && d_y, TASQ_ERR_INVALID_ARG, "NULL pointer");
@@ -374,6 +378,13 @@ int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, in
     const char* p = reinterpret_cast<const char*>(d_packed);
     tasq::GemmArgs a{};
     a.x = d_codes;
+    // the e5m2 copy of the codes follows the M x K fp16 codes (linear layers use it)
+    a.x8 = code_fmt == TASQ_CODES_F16_E5M2 && kind == TASQ_LINEAR
+               ? static_cast<const char*>(d_codes) + int64_t(M) * K * 2
+               : nullptr;
+    // the certificate bounds sum |mask_b(s_w)| for codes of magnitude <= 128; codes of
+    // magnitude <= 8 keep 16 times as long a run below 2^24
+    a.chunk_scale = code_fmt == TASQ_CODES_F16_E5M2 ? 128 / tasq::kF8CodeMax : 1;
     a.alpha = d_alpha;
     a.zc = d_zc;
     a.w = reinterpret_cast<const int8_t*>(p + lay.off_w);

@@ -22,6 +22,13 @@ constexpr int kTableHeader = 16;
 constexpr size_t kTableCapacity = 65536;
 // Most layers one grouped contraction call may hold.
 constexpr int kMaxGroups = 4;
+// Largest operating precision whose masked weight codes are exact in e5m2: mask_b(v)
+// is t * 2^(8-b) with |t| <= 2^(b-1), at most three significant bits for b <= 4.
+constexpr int kBMaxF8 = 4;
+// Largest activation code magnitude of TASQ_CODES_F16_E5M2 (n <= 4): the exact
+// chunk of the tensor-core route is 128 / kF8CodeMax times the one certified for
+// 8-bit codes.
+constexpr int kF8CodeMax = 8;
 
 struct PackedHeader {
     uint32_t magic;
@@ -70,6 +77,8 @@ __device__ inline void set_status(int* status, int code) {
 // ---------------------------------------------------------------------------
 struct GemmArgs {
     const void* x;            // codes: [M][K] (linear) or NHWC (conv)
+    const void* x8;           // the same codes as e5m2 bytes [M][K] (linear layers), or NULL
+    int chunk_scale;          // exact-chunk multiplier: 128 / the largest code magnitude (1 for 8-bit codes)
     const float* alpha;       // [M] or [1]
     const float* zc;
     const int8_t* w;          // stored codes [N][K]

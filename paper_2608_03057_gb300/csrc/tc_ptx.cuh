@@ -117,6 +117,22 @@ __device__ __forceinline__ void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uin
         "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
         "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate));
 }
+// D[tmem] (+)= A[tmem] * B[smem]^T, kind::f8f6f4 (8-bit float A and B, of the
+// types the instruction descriptor names), fp32 accumulator, 32 elements of K.
+__device__ __forceinline__ void mma_f8_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{\n.reg .pred p;\n"
+        "setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+// Four e5m2 bytes (element j in byte j) from two fp16 pairs holding values with
+// at most three significant bits.  e5m2 is the upper byte of fp16 (sign, the same
+// 5-bit exponent with the same bias, the 2 leading mantissa bits), so for such
+// values, whose lower 8 mantissa bits are zero, the upper bytes are the e5m2
+// encodings exactly.
+__device__ __forceinline__ uint32_t e5m2x4(uint32_t h01, uint32_t h23) { return __byte_perm(h01, h23, 0x7531); }
 // Arrive on an mbarrier once every tcgen05 op issued so far by this thread completes.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
@@ -144,6 +160,13 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
         "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]),
         "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]),
         "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+        "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
         : "memory");
 }
 // 32 lanes x 16 consecutive 32-bit columns.
@@ -217,6 +240,10 @@ __host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
     return (1u << 4)                 // D format: fp32
            | (0u << 7) | (0u << 10)  // A, B format: fp16
            | (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
+}
+// The same for kind::f8f6f4 with e5m2 A and B (format code 1 in both fields).
+__host__ __device__ constexpr uint32_t idesc_e5m2_f32(int M, int N) {
+    return idesc_f16_f32(M, N) | (1u << 7) | (1u << 10);
 }
 
 }  // namespace ptx

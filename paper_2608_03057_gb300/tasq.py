@@ -25,7 +25,7 @@ TASQ_LINEAR, TASQ_CONV3X3 = 0, 1
 TASQ_F32, TASQ_BF16 = 0, 1
 TASQ_SYMRANGE, TASQ_ASYM = 0, 1
 TASQ_PER_TOKEN, TASQ_PER_TENSOR = 0, 1
-TASQ_CODES_S8, TASQ_CODES_F16 = 0, 1
+TASQ_CODES_S8, TASQ_CODES_F16, TASQ_CODES_F16_E5M2 = 0, 1, 2
 TASQ_ROUTE_AUTO, TASQ_ROUTE_TC, TASQ_ROUTE_MMA_S8 = 0, 1, 2
 
 _lock = threading.Lock()

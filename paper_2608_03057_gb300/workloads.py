@@ -233,6 +233,10 @@ def schedule_for(config: str, L: int, seed: int = 7) -> np.ndarray:
         return schedule_uniform(L, 20, (2, 3, 4, 6, 8), seed)
     if config == "sdxl":
         return schedule_uniform(L, 4, (4, 5, 6, 8), seed)
+    if config == "pixart_a4":
+        # 4-bit activations at the W4A4 computational budget: operating precisions
+        # averaging 4 bits (the quality table's W4A4-budget row has Eff. W 3.98)
+        return schedule_uniform(L, 20, (2, 3, 4, 5, 6), seed)
     if config == "single":
         return np.array([[8, 6, 4, 3]], np.uint8)
     if config == "sweep":
@@ -242,7 +246,7 @@ def schedule_for(config: str, L: int, seed: int = 7) -> np.ndarray:
 
 def inventory_blocks(config: str, blocks: int) -> List[Layer]:
     """The first `blocks` transformer blocks of a DiT inventory (small cases)."""
-    if config == "pixart":
+    if config in ("pixart", "pixart_a4"):
         return pixart_sigma(blocks=blocks)
     if config == "sana":
         return sana_1600m(blocks=blocks)
@@ -250,7 +254,12 @@ def inventory_blocks(config: str, blocks: int) -> List[Layer]:
 
 
 def inventory(config: str) -> List[Layer]:
-    return {"single": single_linear, "pixart": pixart_sigma, "sana": sana_1600m, "sdxl": sdxl_turbo}[config]()
+    return {"single": single_linear, "pixart": pixart_sigma, "pixart_a4": pixart_sigma, "sana": sana_1600m,
+            "sdxl": sdxl_turbo}[config]()
+
+
+# Activation precision n of each workload (8 unless listed).
+ACT_BITS = {"pixart_a4": 4}
 
 
 # ----------------------------------------------------------------------------

@@ -1042,3 +1042,216 @@ def test_grouped_call_rejects_bad_groups(ctx):
             tasq.tasq_masked_gemm_grouped(ctx.h, layers, 0, buf, F16, buf, buf, 16, buf, N, 64, buf, None)
         assert e.value.code == code, layers
     assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+# ------------------------------- e5m2 codes: the K loop on the 8-bit-float MMA kind --
+
+F8 = tasq.TASQ_CODES_F16_E5M2
+
+
+def _e5m2_part(codes, M, K):
+    """The e5m2 copy that follows the M x K fp16 codes, decoded on the host."""
+    torch = G.torch()
+    raw = codes.view(torch.uint8)[2 * M * K:3 * M * K].cpu()
+    return raw.view(torch.float8_e5m2).float().numpy().reshape(M, K)
+
+
+@pytest.mark.parametrize("n_bits", [2, 3, 4])
+@pytest.mark.parametrize("gran", [tasq.TASQ_PER_TOKEN, tasq.TASQ_PER_TENSOR])
+@pytest.mark.parametrize("dtype", [tasq.TASQ_F32, tasq.TASQ_BF16])
+def test_quant_act_e5m2_copy_bitexact(ctx, oracle, n_bits, gran, dtype):
+    """TASQ_CODES_F16_E5M2: the fp16 codes equal the oracle's codes, and the e5m2
+    copy after them holds the same integers, element for element."""
+    torch = G.torch()
+    M, K = 333, 1152 if gran == tasq.TASQ_PER_TOKEN else 640
+    x = workloads.normal((M, K), 71 + n_bits)
+    x[5, 7] = 9.0
+    if dtype == tasq.TASQ_BF16:
+        xd, x = G.to_bf16(x)
+    else:
+        xd = G.dev(x)
+    codes = G.empty((3 * M * K // 2,), torch.float16)  # 3 M K bytes
+    g = 1 if gran == tasq.TASQ_PER_TENSOR else M
+    alpha, zc = G.empty((g,), torch.float32), G.empty((g,), torch.float32)
+    tasq.tasq_quant_act(ctx.h, xd, dtype, M, K, n_bits, tasq.TASQ_SYMRANGE, gran, codes, F8, alpha, zc)
+    torch.cuda.synchronize()
+    if gran == tasq.TASQ_PER_TOKEN:
+        s, a, z = oracle.quant_act(x, n_bits, oracle.SYMRANGE, oracle.PER_TOKEN)
+    else:
+        s, a, z = oracle.quant_act(x.reshape(1, -1), n_bits, oracle.SYMRANGE, oracle.PER_TOKEN)
+        s = s.reshape(M, K)
+    f16 = codes[:M * K].float().cpu().numpy().reshape(M, K)
+    assert np.array_equal(f16, s.astype(np.float32))
+    assert np.array_equal(_e5m2_part(codes, M, K), s.astype(np.float32))
+    assert np.array_equal(alpha.cpu().numpy(), a) and np.array_equal(zc.cpu().numpy(), z)
+
+
+def test_e5m2_codes_need_four_bits_or_fewer(ctx):
+    torch = G.torch()
+    buf = torch.zeros((1 << 16,), dtype=torch.uint8, device="cuda")
+    with pytest.raises(tasq.TasqError) as e:
+        tasq.tasq_quant_act(ctx.h, buf, tasq.TASQ_F32, 16, 64, 5, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, buf, F8,
+                            buf, buf)
+    assert e.value.code == tasq.TASQ_ERR_UNSUPPORTED
+
+
+def _setup_f8(ctx, oracle, M, N, K, bits, seed, n_bits=4, uniform_w=False):
+    w = workloads.normal((N, K), seed + 1, 0.02)
+    bias = workloads.normal((N,), seed + 2, 0.02)
+    x = workloads.normal((M, K), seed)
+    if uniform_w:
+        s_w = workloads.uniform_codes((N, K), seed + 3)
+        cw = workloads.uniform((N,), seed + 4, 1e-4, 2e-4)
+        packed = G.pack(ctx, tasq.TASQ_LINEAR, G.dev(s_w), G.dev(cw), G.dev(bias), N, K)
+        wq = dict(s=s_w, c=cw)
+    else:
+        sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+        packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, G.dev(bias), N, K)
+        wq = oracle.quant_weight(w)
+    tasq.tasq_set_schedule(ctx.h, np.array([bits], np.uint8), 1, len(bits))
+    torch = G.torch()
+    codes = G.empty((3 * M * K // 2,), torch.float16)
+    alpha, zc = G.empty((M,), torch.float32), G.empty((M,), torch.float32)
+    tasq.tasq_quant_act(ctx.h, G.dev(x), tasq.TASQ_F32, M, K, n_bits, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, codes,
+                        F8, alpha, zc)
+    s_x, a, z = oracle.quant_act(x, n_bits, oracle.SYMRANGE, oracle.PER_TOKEN)
+    return dict(packed=packed, codes=codes, alpha=alpha, zc=zc, wq=wq, s_x=s_x, a=a, z=z, bias=bias)
+
+
+@pytest.mark.parametrize("M,N,K,full", [
+    (256, 1152, 1152, True),    # 64-token tiles
+    (4000, 1096, 384, True),    # 256-token tiles, one accumulator: two activation stages per 256-code block
+    (4096, 3456, 1152, False),  # 192-token tiles, two accumulators
+    (77, 640, 2048, True),      # 64-token tiles, split K
+    (513, 72, 64, True),        # K shorter than one block
+    (300, 136, 1168, True),     # ragged last K block
+])
+@pytest.mark.parametrize("n_bits", [3, 4])
+def test_f8_route_every_b(ctx, oracle, M, N, K, full, n_bits):
+    """Codes in the dual format: at b <= 4 the K loop runs on the e5m2 MMA kind
+    (unsplit launches), at b = 5..8 on the fp16 codes; every b gives the oracle's
+    exact int32 accumulators and bf16 outputs, with and without the int32 output."""
+    torch = G.torch()
+    bits = list(range(2, 9))
+    st = _setup_f8(ctx, oracle, M, N, K, bits, seed=M + N + n_bits, n_bits=n_bits)
+    rows = np.arange(M) if full else np.unique(np.concatenate([np.arange(0, M, max(1, M // 48)), [M - 1]]))
+    rows_d = torch.from_numpy(rows).cuda()
+    y_prod = G.empty((M, N), torch.int16)
+    for stage, b in enumerate(bits):
+        tasq.tasq_masked_gemm(ctx.h, 0, stage, st["codes"], F8, st["alpha"], st["zc"], M, st["packed"], N, K, y_prod,
+                              None)
+        y, acc = G.gemm(ctx, 0, stage, st["codes"], F8, st["alpha"], st["zc"], M, st["packed"], N, K)
+        ref = oracle.gemm(st["s_x"][rows], st["wq"]["s"], b)
+        got = acc.index_select(0, rows_d).cpu().numpy()
+        assert np.array_equal(got, ref), f"b={b}: {(got != ref).sum()} int32 mismatches"
+        _, yb = oracle.epilogue_f32(ref, st["a"][rows], st["z"][rows], oracle.row_sums(st["wq"]["s"], b),
+                                    st["wq"]["c"], st["bias"])
+        for yy in (y, y_prod):
+            assert G.assert_bf16_close(G.bf16_bits_host(yy.index_select(0, rows_d)), yb) == yb.size, b
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+def test_f8_route_uniform_codes(ctx, oracle):
+    """Uniform weight codes in [-127, 127] and K = 4096 at M = 1024 (single-
+    accumulator tiles), on either path."""
+    torch = G.torch()
+    M, N, K = 1024, 4096, 4096
+    bits = [2, 4, 5, 8]
+    st = _setup_f8(ctx, oracle, M, N, K, bits, seed=91, uniform_w=True)
+    rows = np.unique(np.concatenate([np.arange(0, M, 37), [M - 1]]))
+    rows_d = torch.from_numpy(rows).cuda()
+    for stage, b in enumerate(bits):
+        y, acc = G.gemm(ctx, 0, stage, st["codes"], F8, st["alpha"], st["zc"], M, st["packed"], N, K)
+        ref = oracle.gemm(st["s_x"][rows], st["wq"]["s"], b)
+        assert np.array_equal(acc.index_select(0, rows_d).cpu().numpy(), ref), b
+
+
+def test_f8_codes_lengthen_the_exact_chunk(ctx, oracle):
+    """Codes of magnitude <= 8 (the e5m2 format) let an exact fp32 chunk run 16
+    times as far as the run certified for 8-bit codes.  Odd extreme operands
+    (weight codes +127 / -125, activation code 7 on the positive rows; -8 on
+    the others) over K = 40960 make the positive rows' products odd and the row
+    totals ~2^25, so a chunk one doubling too long would round its fp32 partial
+    sum; at b = 8 (fp16 codes) and b = 4 (e5m2 kind, a multiple of 16 per
+    product) the int32 accumulators must equal the oracle's."""
+    torch = G.torch()
+    M, N, K = 640, 1152, 40960  # 90 tiles of 64 tokens: one unsplit wave
+    col = torch.where(torch.arange(N, device="cuda") % 2 == 0, 127, -125).to(torch.int8)
+    s_w = col[:, None].expand(N, K).contiguous()
+    cw = torch.full((N,), 1e-4, device="cuda")
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, s_w, cw, None, N, K)
+    sign = torch.where(torch.arange(M, device="cuda") % 3 == 0, -1.0, 1.0)
+    x = sign[:, None].expand(M, K).contiguous()
+    bits = [8, 4]
+    tasq.tasq_set_schedule(ctx.h, np.array([bits], np.uint8), 1, len(bits))
+    codes = G.empty((3 * M * K // 2,), torch.float16)
+    alpha, zc = G.empty((M,), torch.float32), G.empty((M,), torch.float32)
+    tasq.tasq_quant_act(ctx.h, x, tasq.TASQ_F32, M, K, 4, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, codes, F8,
+                        alpha, zc)
+    rows = np.array([0, 1, 2, 300, M - 1])
+    s_x, _, _ = oracle.quant_act(np.where(rows % 3 == 0, -1.0, 1.0)[:, None] * np.ones((1, K)), 4, oracle.SYMRANGE,
+                                 oracle.PER_TOKEN)
+    assert np.array_equal(codes[:M * K].view(M, K)[torch.from_numpy(rows).cuda()].cpu().numpy(), s_x)
+    assert (s_x[rows % 3 != 0] == 7).all()  # odd codes on the positive rows
+    s_w_host = np.where(np.arange(N) % 2 == 0, 127, -125).astype(np.int8)[:, None] * np.ones((1, K), np.int8)
+    for stage, b in enumerate(bits):
+        _, acc = G.gemm(ctx, 0, stage, codes, F8, alpha, zc, M, packed, N, K)
+        ref = oracle.gemm(s_x, s_w_host, b)
+        assert np.abs(ref).max() > 2 ** 24
+        got = acc.index_select(0, torch.from_numpy(rows).cuda()).cpu().numpy()
+        assert np.array_equal(got, ref), f"b={b}: {(got != ref).sum()} mismatches"
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+def test_f8_route_grouped_members_choose_the_path_together(ctx, oracle):
+    """A grouped call runs on the e5m2 kind only when every member's b is <= 4;
+    either way each member equals the oracle's single layer at its b."""
+    torch = G.torch()
+    M, Ng, K = 300, 1152, 1152
+    N = 2 * Ng
+    w = workloads.normal((N, K), 501, 0.02)
+    bias = workloads.normal((N,), 502, 0.02)
+    x = workloads.normal((M, K), 503)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, G.dev(bias), N, K)
+    table = np.array([[3, 4], [2, 7]], np.uint8)  # stage 0: (3, 2) e5m2; stage 1: (4, 7) fp16
+    tasq.tasq_set_schedule(ctx.h, table, 2, 2)
+    codes = G.empty((3 * M * K // 2,), torch.float16)
+    alpha, zc = G.empty((M,), torch.float32), G.empty((M,), torch.float32)
+    tasq.tasq_quant_act(ctx.h, G.dev(x), tasq.TASQ_F32, M, K, 4, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, codes, F8,
+                        alpha, zc)
+    wq = oracle.quant_weight(w)
+    s_x, a, z = oracle.quant_act(x, 4, oracle.SYMRANGE, oracle.PER_TOKEN)
+    for stage in range(2):
+        y = G.empty((M, N), torch.int16)
+        acc = G.empty((M, N), torch.int32)
+        tasq.tasq_masked_gemm_grouped(ctx.h, [0, 1], stage, codes, F8, alpha, zc, M, packed, N, K, y, acc)
+        yh, acch = G.bf16_bits_host(y), acc.cpu().numpy()
+        for g in range(2):
+            b = int(table[g, stage])
+            sl = slice(g * Ng, (g + 1) * Ng)
+            ref = oracle.gemm(s_x, wq["s"][sl], b)
+            assert np.array_equal(acch[:, sl], ref), (stage, g)
+            _, yb = oracle.epilogue_f32(ref, a, z, oracle.row_sums(wq["s"][sl], b), wq["c"][sl], bias[sl])
+            assert G.assert_bf16_close(yh[:, sl], yb) == yb.size
+
+
+def test_e5m2_codes_in_a_convolution_use_the_fp16_codes(ctx, oracle):
+    """A 3x3 convolution given dual-format codes reads their fp16 part."""
+    torch = G.torch()
+    B, H, W, Cin, Cout = 1, 8, 8, 64, 16
+    x = workloads.normal((B, H, W, Cin), 511)
+    w = workloads.normal((Cout, 9 * Cin), 512, 0.03)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, Cout, 9 * Cin)
+    packed = G.pack(ctx, tasq.TASQ_CONV3X3, sw, cw, None, Cout, 9 * Cin, Cin)
+    tasq.tasq_set_schedule(ctx.h, np.array([[4]], np.uint8), 1, 1)
+    M = B * H * W
+    codes = G.empty((3 * M * Cin // 2,), torch.float16)
+    alpha, zc = G.empty((1,), torch.float32), G.empty((1,), torch.float32)
+    tasq.tasq_quant_act(ctx.h, G.dev(x), tasq.TASQ_F32, M, Cin, 4, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TENSOR, codes,
+                        F8, alpha, zc)
+    y, acc = G.conv(ctx, 0, 0, codes, F8, alpha, zc, B, H, W, Cin, packed, Cout)
+    wq = oracle.quant_weight(w)
+    s_x, a, z = oracle.quant_act(x.reshape(1, -1), 4, oracle.SYMRANGE, oracle.PER_TOKEN)
+    ref, rs = oracle.conv3x3(s_x.reshape(B, H, W, Cin), wq["s"], 4)
+    assert np.array_equal(acc.cpu().numpy(), ref)
