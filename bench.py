@@ -286,6 +286,27 @@ def capture(torch, step, parts=("quant", "gemm")):
     return g
 
 
+def f8_op_share(tasq, step, steps, stage_of, num_sms):
+    """Share of a step's int8-equivalent ops that run on the 8-bit-float route,
+    over the stages of `steps` timed replays: linear units with e5m2 codes whose
+    members are all at b <= 4, in unsplit launches (the route's conditions)."""
+    if step.code_fmt != tasq.TASQ_CODES_F16_E5M2:
+        return 0.0
+    f8 = tot = 0.0
+    for k in range(steps):
+        s = stage_of(k)
+        for u, unit in enumerate(step.units):
+            l = step.layers[unit[0]]
+            ops = sum(step.layers[i].ops for i in unit)
+            tot += ops
+            if l.kind == step.conv or any(int(step.table[i, s]) > 4 for i in unit):
+                continue
+            plan = tasq.tasq_plan_tc(tasq.TASQ_LINEAR, l.M, step.y[u].shape[1], l.K, 0, 0, 0, 0, num_sms)
+            if plan["splits"] == 1:
+                f8 += ops
+    return f8 / tot if tot else 0.0
+
+
 def timed_replays(torch, g, step, steps, stage_of):
     s = torch.cuda.current_stream()
     t0 = torch.cuda.Event(enable_timing=True)
@@ -820,14 +841,21 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     del g, g_gemm, g_quant
 
     achieved = step.ops / (ms_gemm * 1e-3) / 1e12
-    peak = peaks["bf16"]
+    # ops on the 8-bit-float route (4-bit codes, b <= 4) run at twice the bf16 rate (the
+    # nominal fp8 : bf16 ratio, and the probe's equal cycles per MMA for twice the K): the
+    # peak is the ops-weighted harmonic mean of the two rates
+    phi = f8_op_share(tasq, step, steps, stage_of, torch.cuda.get_device_properties(0).multi_processor_count)
+    peak = peaks["bf16"] / ((1.0 - phi) + phi / 2.0)
     traffic = measured_traffic(name)
     U = len(step.units)
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "traffic": traffic, "algorithmic_bytes_per_launch": step.gemm_bytes() / U,
                 "kernel": "gemm_tc_kernel",
                 "peak_source": f"{peaks['src']} bf16 burst (cuBLAS); the fp16 tcgen05 MMA runs at the bf16 rate, "
-                               "and the contraction-only replay lasts well under a second",
+                               "and the contraction-only replay lasts well under a second"
+                               + (f"; {phi:.3f} of the ops on the 8-bit-float route at twice that rate "
+                                  "(ops-weighted harmonic mean)" if phi else ""),
+                "f8_op_share": phi,
                 "timing": "CUDA events around replays of the step's launch sequence with only its contractions "
                           f"({steps} replays, {U} calls each, every launch overlapping the previous one's tail "
                           "as in the step); achieved = int8-equivalent ops per step / that time"}
