@@ -70,6 +70,7 @@ UNIT = "TOPS"
 WORKLOAD_NAMES = {
     "pixart": "pixart_sigma_1024px_denoise_step",
     "pixart_a4": "pixart_sigma_1024px_denoise_step_a4_w4a4_budget",
+    "pixart_lr": "pixart_sigma_1024px_denoise_step_with_rank32_lowrank_branch",
     "sana": "sana_1600m_1024px_denoise_step",
     "sdxl": "sdxl_turbo_512px_denoise_step",
     "single": "single_linear_256x1152x1152",
@@ -178,6 +179,9 @@ class Step:
         # linear contractions at b <= 4 run on the 8-bit-float tensor-core kind
         self.act_bits = workloads.ACT_BITS.get(name, 8)
         self.code_fmt = tasq.TASQ_CODES_F16_E5M2 if self.act_bits <= 4 else tasq.TASQ_CODES_F16
+        # 16-bit low-rank branch beside every linear layer: one call per layer
+        self.rank = workloads.LOWRANK.get(name, 0)
+        group = group and not self.rank
         if blocks:
             keep = len(workloads.inventory_blocks(name, blocks))
             self.layers, self.table = self.layers[:keep], np.ascontiguousarray(self.table[:keep])
@@ -192,6 +196,9 @@ class Step:
         self.codes = torch.empty((max_mk * (3 if self.act_bits <= 4 else 2) // 2,), dtype=torch.float16, device=dev)
         self.alpha = torch.empty((max_m,), dtype=torch.float32, device=dev)
         self.zc = torch.empty((max_m,), dtype=torch.float32, device=dev)
+        self.l1, self.l2 = [], []
+        if self.rank:
+            self.u = torch.empty((max_m, 64), dtype=torch.int16, device=dev)  # u' rows of 64 fp16
         for unit in self.units:
             l = self.layers[unit[0]]
             N = sum(self.layers[i].N for i in unit)
@@ -210,6 +217,16 @@ class Step:
             xs = (l.B, l.H, l.W, l.Cin) if l.kind == workloads.CONV3X3 else (l.M, l.K)
             self.x.append(workloads.device_normal(xs, seed * 100003 + 1000003 + unit[0], 1.0, torch.bfloat16))
             self.y.append(torch.empty((l.M, N), dtype=torch.int16, device=dev))
+            if self.rank and l.kind != workloads.CONV3X3:
+                # the branch's factors (bf16 bits): l2 [rank][K] and l1 [N][rank]
+                i = unit[0]
+                self.l2.append(workloads.device_normal((self.rank, l.K), seed * 100003 + 3000003 + i, 0.05,
+                                                       torch.bfloat16).view(torch.int16))
+                self.l1.append(workloads.device_normal((N, self.rank), seed * 100003 + 4000003 + i, 0.05,
+                                                       torch.bfloat16).view(torch.int16))
+            else:
+                self.l1.append(None)
+                self.l2.append(None)
             del w, sw, cw, bias
         self.d_stage = torch.zeros((4,), dtype=torch.int32, device=dev)
         tasq.tasq_set_stage_device(self.ctx, self.d_stage)
@@ -240,6 +257,12 @@ class Step:
             if conv:
                 t.tasq_masked_conv3x3(self.ctx, unit[0], -1, self.codes, self.code_fmt, self.alpha, self.zc, l.B,
                                       l.H, l.W, l.Cin, self.packed[u], N, self.y[u], None)
+            elif self.l1[u] is not None:
+                # the low-rank branch: its down-projection of this input, then the layer
+                t.tasq_lowrank_down(self.ctx, self.x[u], t.TASQ_BF16, l.M, l.K, self.l2[u], self.rank, self.alpha,
+                                    self.u)
+                t.tasq_masked_gemm_lr(self.ctx, unit[0], -1, self.codes, self.code_fmt, self.alpha, self.zc, l.M,
+                                      self.packed[u], N, l.K, self.u, self.l1[u], self.rank, self.y[u], None)
             elif len(unit) == 1:
                 t.tasq_masked_gemm(self.ctx, unit[0], -1, self.codes, self.code_fmt, self.alpha, self.zc, l.M,
                                    self.packed[u], N, l.K, self.y[u], None)
@@ -718,7 +741,7 @@ def job_tops(ops_per_rank: float, world: int, ms: float) -> float:
 # Denoising steps of the trajectory each workload's stages partition (stage of
 # step t = floor(t S / T), stage 0 the noisiest): 20 for the DiTs, 4 for the
 # distilled UNet; the single layer runs its 4 stages once each.
-TRAJECTORY_STEPS = {"pixart": 20, "pixart_a4": 20, "sana": 20, "sdxl": 4, "single": 4}
+TRAJECTORY_STEPS = {"pixart": 20, "pixart_a4": 20, "pixart_lr": 20, "sana": 20, "sdxl": 4, "single": 4}
 
 
 def stage_map(name: str, S: int):
@@ -788,7 +811,8 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     and with only its quantizations, the all-8-bit schedule on the same graph, and
     the end-to-end step.  Returns the figures and the Step (closed by the caller)."""
     from paper_2608_03057_gb300 import engine_model, schedule
-    step = Step(torch, tasq, workloads, name, args.seed, args.blocks if name in ("pixart", "pixart_a4", "sana") else 0)
+    step = Step(torch, tasq, workloads, name, args.seed,
+                args.blocks if name in ("pixart", "pixart_a4", "pixart_lr", "sana") else 0)
     S = step.S
     stage_of = stage_map(name, S)
     for k in range(2):  # eager launches first: they set kernel attributes outside any capture

@@ -67,7 +67,7 @@
 extern "C" {
 #endif
 
-#define TASQ_ABI_VERSION 3
+#define TASQ_ABI_VERSION 4
 
 /* Return codes. */
 enum {
@@ -333,6 +333,41 @@ int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_codes, in
 int tasq_masked_gemm_grouped(tasq_ctx ctx, const int32_t* h_layers, int groups, int stage, const void* d_codes,
                              int code_fmt, const float* d_alpha, const float* d_zc, int M, const void* d_packed,
                              int N, int K, uint16_t* d_y, int32_t* d_acc, tasq_stream stream);
+
+/*
+ * 16-bit low-rank branch of an SVD-split linear layer (the frozen SVD branch
+ * that the paper's SVDQuant+TASQ pipelines carry beside the masked weights:
+ * rank 32 for the 4-bit setting, 16 for the 6-bit one, Sec. 4 setup and the
+ * training-setting table): y = Q(x) Q_b(R)^T + (x l2^T) l1^T.  The masked
+ * contraction adds the up-projection inside its accumulator, in the
+ * accumulator's units, as one more K block of fp16 tensor-core MMAs after the
+ * last one of each output tile:
+ *   acc'[m][n] = acc[m][n] + sum_j u'[m][j] * fp16(l1[n][j] * RN(1 / c_w[n])),
+ *   u'[m][j] = fp16((sum_k bf16(x[m][k]) * l2[j][k]) / alpha[m]),
+ * so that the epilogue's alpha[m] * c_w[n] scales it back to u . l1; the
+ * epilogue then runs as for tasq_masked_gemm on acc' (held in fp32).
+ *
+ * tasq_lowrank_down: u' above (the sum over k accumulated in fp32 on the tensor
+ * cores, order unspecified; one IEEE division by alpha[m]; fp16 rounding to
+ * nearest even) into d_u [M][64] fp16 bits, columns >= rank zero.  d_x: the
+ * layer's input [M][K], fp32 or bf16 (dtype; fp32 rounded to bf16 first);
+ * d_l2: [rank][K] bf16 bits; d_alpha: [M] per-token scales of the layer's
+ * activation codes (tasq_quant_act, per token).  rank 16 or 32, K % 16 == 0;
+ * d_x 8-byte (fp32) or 4-byte (bf16) aligned, d_l2 4-byte and d_u 16-byte
+ * aligned.  Enqueue call (one kernel), after the quantization.
+ *
+ * tasq_masked_gemm_lr: tasq_masked_gemm with the branch.  d_u: from
+ * tasq_lowrank_down on this layer's input; d_l1: [N][rank] bf16 bits, 16-byte
+ * aligned.  d_acc must be NULL (the accumulator carries the branch's fraction).
+ * Tensor-core route only (fp16 or fp16 + e5m2 codes; the branch's block is fp16
+ * either way); the launch is never split along K.  Other arguments as
+ * tasq_masked_gemm.  Enqueue call.
+ */
+int tasq_lowrank_down(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, const uint16_t* d_l2, int rank,
+                      const float* d_alpha, uint16_t* d_u, tasq_stream stream);
+int tasq_masked_gemm_lr(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt, const float* d_alpha,
+                        const float* d_zc, int M, const void* d_packed, int N, int K, const uint16_t* d_u,
+                        const uint16_t* d_l1, int rank, uint16_t* d_y, int32_t* d_acc, tasq_stream stream);
 
 /*
  * Masked linear layer with asymmetric weights (Eq. weight_dequant with the

@@ -309,3 +309,32 @@ def conv3x3_zp_def_f64(s_x_nhwc, alpha, zc, s_w, c_w, z, bias, b):
     _lib().oq_conv3x3_zp_def_f64(_p(s_x), float(alpha), float(zc), B, H, W, Cin, _p(s_w), _p(_c(c_w, np.float32)),
                                  _p(_c(z, np.float32)), _p(bias), Cout, int(b), _p(y))
     return y
+
+
+# ------------------------------------------------ 16-bit low-rank branch --
+# The frozen SVD low-rank branch that the paper's SVDQuant+TASQ pipelines keep
+# beside the masked int8 weights (rank 32 for the 4-bit setting, 16 for the
+# 6-bit one; the training-setting passage of the appendix): the layer computes
+# y = Q(x) Q_b(R)^T + (x l2^T) l1^T, the branch on 16-bit (bf16) numbers.
+# Readings: x enters the branch rounded to bf16; the branch's value is the exact
+# sum, added to the dequantized main branch before the output's bf16 rounding.
+# Plain numpy: fp64 matrix products of bf16 values.
+
+def bf16_round(x):
+    """fp32 values rounded to the nearest bf16 (ties to even), as fp32."""
+    return bf16_bits_to_f32(f32_to_bf16_bits(np.asarray(x, np.float32)))
+
+
+def lowrank_down(x, l2_bits):
+    """u = sum_k bf16(x[m][k]) * l2[j][k] (fp64): x [M][K] fp32, l2 [r][K] bf16 bits."""
+    return bf16_round(x).astype(np.float64) @ bf16_bits_to_f32(l2_bits).astype(np.float64).T
+
+
+def lowrank_up(u, l1_bits):
+    """lr[m][n] = sum_j u[m][j] * l1[n][j] (fp64), l1 [N][r] bf16 bits."""
+    return np.asarray(u, np.float64) @ bf16_bits_to_f32(l1_bits).astype(np.float64).T
+
+
+def linear_lowrank_def_f64(s_x, alpha, zc, s_w, c_w, bias, b, lr):
+    """The dequantized masked linear layer plus its low-rank branch, fp64."""
+    return linear_def_f64(s_x, alpha, zc, s_w, c_w, bias, b) + np.asarray(lr, np.float64)

@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 OBJ = os.path.join(HERE, "_build")
 LIB_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(LIB_DIR, "libtasq.so")
-SOURCES = ["tasq_api.cu", "quant.cu", "gemm_s8.cu", "gemm_tc.cu", "probe_mma.cu"]
+SOURCES = ["tasq_api.cu", "quant.cu", "gemm_s8.cu", "gemm_tc.cu", "probe_mma.cu", "lowrank.cu"]
 HEADERS = ["tasq_internal.cuh", "tc_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

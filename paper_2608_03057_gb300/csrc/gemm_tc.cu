@@ -277,12 +277,16 @@ __device__ __forceinline__ bool f8_route(const GemmArgs& a, uint32_t gbits) {
 // epilogue of asymmetric weights; F8 a linear layer whose codes also come as e5m2
 // bytes (tm_x8): when every member's b is <= 4 the K loop runs on the 8-bit route
 // (kind::f8f6f4 MMAs with e5m2 operands, 32 codes of K per instruction), else on
-// the fp16 codes as usual.
-template <bool CONV, bool ZP, class C, bool F8 = false>
+// the fp16 codes as usual; LR a linear layer with a 16-bit low-rank branch: after
+// the last K block of each tile one more block of fp16 MMAs adds
+// u'[m] . (l1[n] / c_w[n]) to the accumulator (u' in tm_u, the weights' block
+// converted from l1 by the converters), so that the epilogue's dequantization
+// scales it back to u . l1 (unsplit launches only).
+template <bool CONV, bool ZP, class C, bool F8 = false, bool LR = false>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_y,
-                   const __grid_constant__ CUtensorMap tm_x8) {
+                   const __grid_constant__ CUtensorMap tm_x8, const __grid_constant__ CUtensorMap tm_u) {
     constexpr int X_STAGES = C::X_STAGES, X_HALF = C::X_HALF, X_STAGE = C::X_STAGE, NACC = C::NACC;
     constexpr int Q = C::Q, DONE = C::DONE;
     constexpr int BT = C::BT, GPW = C::GPW;
@@ -380,7 +384,8 @@ __global__ void __maxnreg__(96)
             for (int w = unit; w < works && ok; w += units) {
                 const Work wk = work_item(p, w, KT, chunk);
                 const TileCoord tc = tile_coord<CONV, BT>(p, wk.t);
-                for (int kq = wk.kb_lo * Q; kq < wk.kb_hi * Q; ++kq, ++u) {
+                // (LR: the tile's last block is the low-rank block, stages of u' rows)
+                for (int kq = wk.kb_lo * Q; kq < (wk.kb_hi + (LR ? 1 : 0)) * Q; ++kq, ++u) {
                     if (u >= X_STAGES && !wt.wait(&s->done[(u - X_STAGES) % DONE], ((u - X_STAGES) / DONE) & 1)) {
                         ok = false;
                         break;
@@ -393,7 +398,11 @@ __global__ void __maxnreg__(96)
                         // box hh of the stage: 128 bytes of each token's row, 64 fp16 codes
                         // or 128 e5m2 codes
                         const int kh = kq * (BK / Q) + hh * XK;
-                        if constexpr (CONV) {
+                        if (LR && kq >= wk.kb_hi * Q) {
+                            // u' columns 0..63; the block's other boxes lie past the 64
+                            // columns and are filled with zeros
+                            ptx::tma_load_2d(dst + hh * X_HALF, &tm_u, fb, kh - wk.kb_hi * BK, tc.tok0);
+                        } else if constexpr (CONV) {
                             // a 128-wide K block may straddle two taps when Cin % 128 == 64
                             const int tap = kh / a.Cin, c0 = kh - tap * a.Cin;
                             ptx::tma_load_4d(dst + hh * X_HALF, &tm_x, fb, c0, tc.w0 + tap % 3 - 1, tc.h0 + tap / 3 - 1,
@@ -451,9 +460,12 @@ __global__ void __maxnreg__(96)
                     }
                     ptx::tc_fence_after();
                     const uint32_t d = tmem + C::ACC_COL + buf * BT;
-                    const int kb0 = wk.kb_lo + c * chunk, kb_end = min(wk.kb_hi, kb0 + chunk);
+                    const int kb0 = wk.kb_lo + c * chunk;
+                    // (LR: the last chunk also takes the low-rank block, kb == kb_hi)
+                    const int kb_end = min(wk.kb_hi, kb0 + chunk) + (LR && c == wk.nch - 1 ? 1 : 0);
                     for (int kb = kb0; kb < kb_end && ok; ++kb, ++it) {
                         const uint32_t acol = tmem + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
+                        const bool lrb = LR && kb == wk.kb_hi;  // the low-rank block: fp16, 64 columns of K
                         for (int i = 0; i < Q; ++i) {
                             const int u = it * Q + i;
                             // activations landed (and, for i == 0, the converters wrote slot it % 2)
@@ -468,7 +480,12 @@ __global__ void __maxnreg__(96)
                                 const uint64_t bdesc =
                                     ptx::sw128_kmajor_desc(ptx::smem_u32(s->x[u % X_STAGES] + hh * X_HALF));
                                 const int k0 = (i * (2 / Q) + hh) * (XK / 16);  // K step within the block
-                                if (F8 && f8) {
+                                if (lrb) {
+                                    if (k0 == 0)
+                                        for (int kk = 0; kk < XK / 16; ++kk)
+                                            ptx::mma_f16_ts(d, acol + kk * 8, bdesc + uint64_t((kk * 32) >> 4),
+                                                            C::IDESC, 1u);
+                                } else if (F8 && f8) {
                                     for (int kk = 0; kk < XK / 16; ++kk)
                                         ptx::mma_f8_ts(d, acol + (k0 + kk) * 8, bdesc + uint64_t((kk * 32) >> 4),
                                                        C::IDESC8, (kb > kb0 || k0 + kk > 0) ? 1u : 0u);
@@ -509,12 +526,41 @@ __global__ void __maxnreg__(96)
             const Work wk = work_item(p, w, KT, chunk);
             // this row's channel runs at its layer's b (a grouped call holds several layers)
             const uint32_t m = mask_word(channel_bits(a, gbits, tile_coord<CONV, BT>(p, wk.t).ch0 + r));
-            for (int kb = wk.kb_lo; kb < wk.kb_hi; ++kb, ++it) {
+            if constexpr (LR) {  // the low-rank block's l1 row, read after the tile's K blocks
+                const int n = tile_coord<CONV, BT>(p, wk.t).ch0 + r;
+                if (kp == 0 && n < a.N) asm volatile("prefetch.global.L1 [%0];" ::"l"(a.lr_l1 + int64_t(n) * a.lr_rank));
+            }
+            // (LR: the tile's last block is the low-rank block, kb == kb_hi)
+            for (int kb = wk.kb_lo; kb < wk.kb_hi + (LR ? 1 : 0); ++kb, ++it) {
                 // Row r of a tile holds 128 codes; 16-byte chunk c sits at c ^ (r & 7) (128-byte
                 // swizzle).  Mask and widen before waiting for the slot, so that only the
                 // tensor-memory store remains once the MMA releases it.
                 uint32_t f[NF];
-                if (F8 && f8) {
+                if (LR && kb == wk.kb_hi) {
+                    // the low-rank block's weights: fp16(l1[n][j] * RN(1 / c_w[n])) for the
+                    // rank columns j (the first part's first words), zeros elsewhere; no
+                    // tile of the weight ring
+#pragma unroll
+                    for (int i = 0; i < NF; ++i) f[i] = 0u;
+                    const int n = tile_coord<CONV, BT>(p, wk.t).ch0 + r;
+                    if (kp == 0 && n < a.N) {
+                        const float rcw = __frcp_rn(a.cw[n]);
+                        const uint4* lp = reinterpret_cast<const uint4*>(a.lr_l1 + int64_t(n) * a.lr_rank);
+#pragma unroll
+                        for (int q4 = 0; q4 < 4; ++q4) {  // rank 32: four 16-byte loads; rank 16: two
+                            if (q4 >= a.lr_rank / 8) break;
+                            const uint4 v = __ldg(lp + q4);
+                            const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float lo = __fmul_rn(__uint_as_float(wv[i] << 16), rcw);
+                                const float hi = __fmul_rn(__uint_as_float(wv[i] & 0xFFFF0000u), rcw);
+                                const __half2 h = __floats2half2_rn(lo, hi);
+                                f[4 * q4 + i] = *reinterpret_cast<const uint32_t*>(&h);
+                            }
+                        }
+                    }
+                } else if (F8 && f8) {
                     // e5m2 (b <= 4): one word per 4 codes, 32 words per tile.  Every
                     // converter warp passes both tiles of the block through the ring in
                     // order (a part that skipped the other part's tiles could wait on a
@@ -880,6 +926,11 @@ __global__ void __maxnreg__(96)
                             int32_t* pp = my_part + (gi * 32 + h * 16) * 32;
 #pragma unroll
                             for (int j = 0; j < 16; ++j) {
+                                if (LR && last) {
+                                    // the last chunk holds the low-rank block's fraction: keep it
+                                    v[j] = __float_as_uint(__fadd_rn(__int2float_rn(pp[j * 32]), __uint_as_float(v[j])));
+                                    continue;
+                                }
                                 int x = __float2int_rn(__uint_as_float(v[j]));
                                 if (c > 0) x += pp[j * 32];
                                 if (last) v[j] = uint32_t(x);
@@ -901,7 +952,7 @@ __global__ void __maxnreg__(96)
                             }
                         } else if (last) {
                             if constexpr (!CONV) {
-                                if (nchunks == 1) finish16f(gi, h * 16, v, std::true_type{});
+                                if (nchunks == 1 || LR) finish16f(gi, h * 16, v, std::true_type{});
                                 else finish16f(gi, h * 16, v, std::false_type{});
                             } else {
                                 if (nchunks == 1) finish16(gi, h * 16, v, std::true_type{}, all_tok);
@@ -1127,7 +1178,7 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
     p.a = a;
     p.conv = a.Cin != 0;
     p.tiles_ch = (a.N + BCH - 1) / BCH;
-    CUtensorMap tm_x, tm_w, tm_y, tm_x8;
+    CUtensorMap tm_x, tm_w, tm_y, tm_x8, tm_u;
     CUresult r;
     p.tiles_tok = int(plan.tiles_tok);
     if (p.conv) {
@@ -1174,6 +1225,22 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
     } else {
         tm_x8 = tm_x;  // unused
     }
+    if (a.lr_rank) {
+        // the low-rank block's activations: u' [M][64] fp16, one 64-wide box per stage half
+        cuuint64_t dims[2] = {cuuint64_t(kLowRankCols), cuuint64_t(a.M)};
+        cuuint64_t strides[1] = {cuuint64_t(kLowRankCols) * 2};
+        cuuint32_t box[2] = {XK, cuuint32_t(BTOK)};
+        cuuint32_t es[2] = {1, 1};
+        r = encode(&tm_u, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<uint16_t*>(a.lr_u), dims, strides, box, es,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) {
+            *why = "low-rank tensor map rejected";
+            return cudaSuccess;
+        }
+    } else {
+        tm_u = tm_x;  // unused
+    }
     {
         cuuint64_t dims[2] = {cuuint64_t(a.K), cuuint64_t(a.N)};
         cuuint64_t strides[1] = {cuuint64_t(a.K)};
@@ -1211,13 +1278,17 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
                 (long long)p.tiles_ch * p.tiles_tok, p.splits, units);
     const int smem = smem_bytes<C>();
     auto kernel = [&] {
-        // the eight-converter tiles only serve linear layers with e5m2 codes
+        // the eight-converter tiles only serve linear layers with e5m2 codes; the
+        // low-rank branch only symmetric linear layers
         if constexpr (C::CONV_WARPS == 8)
-            return a.code_sums ? gemm_tc_kernel<false, true, C, true> : gemm_tc_kernel<false, false, C, true>;
+            return a.lr_rank     ? gemm_tc_kernel<false, false, C, true, true>
+                   : a.code_sums ? gemm_tc_kernel<false, true, C, true>
+                                 : gemm_tc_kernel<false, false, C, true>;
         else
-            return p.conv ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
-                   : f8   ? (a.code_sums ? gemm_tc_kernel<false, true, C, true> : gemm_tc_kernel<false, false, C, true>)
-                          : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
+            return p.conv      ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
+                   : a.lr_rank ? (f8 ? gemm_tc_kernel<false, false, C, true, true> : gemm_tc_kernel<false, false, C, false, true>)
+                   : f8        ? (a.code_sums ? gemm_tc_kernel<false, true, C, true> : gemm_tc_kernel<false, false, C, true>)
+                               : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
     }();
     cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
@@ -1233,7 +1304,7 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w, tm_y, tm_x8);
+    e = cudaLaunchKernelEx(&cfg, kernel, p, tm_x, tm_w, tm_y, tm_x8, tm_u);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e == cudaSuccess) *kernels = 1;
     if (e == cudaSuccess && p.splits > 1) {
@@ -1272,8 +1343,9 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         return cudaSuccess;
     }
     if (a.M == 0 || a.N == 0) return cudaSuccess;
+    // (the split-K reduction has no low-rank term: such launches stay unsplit)
     const TcPlan plan =
-        plan_gemm_tc(a.M, a.N, a.K, a.B, a.H, a.W, a.Cin, num_sms, a.split_buf ? a.split_cap : 0);
+        plan_gemm_tc(a.M, a.N, a.K, a.B, a.H, a.W, a.Cin, num_sms, a.split_buf && !a.lr_rank ? a.split_cap : 0);
     if (plan.why) {
         *why = plan.why;
         return cudaSuccess;

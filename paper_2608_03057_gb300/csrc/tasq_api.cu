@@ -349,7 +349,8 @@ namespace {
 int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, int stage, const void* d_codes,
                        int code_fmt, const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int M,
                        const void* d_packed, int N, int K, int B, int H, int W, int Cin, uint16_t* d_y,
-                       int32_t* d_acc, tasq_stream stream) {
+                       int32_t* d_acc, tasq_stream stream, const uint16_t* d_lr_u = nullptr,
+                       const uint16_t* d_lr_l1 = nullptr, int lr_rank = 0) {
     REQUIRE(ctx->L > 0, TASQ_ERR_INVALID_ARG, "no schedule: call tasq_set_schedule first");
     REQUIRE(layers && groups >= 1 && groups <= tasq::kMaxGroups, TASQ_ERR_INVALID_ARG, "groups %d outside 1..%d",
             groups, tasq::kMaxGroups);
@@ -373,6 +374,12 @@ int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, in
     REQUIRE(aligned16(d_codes) && aligned16(d_y) && aligned16(d_acc), TASQ_ERR_UNSUPPORTED,
             "pointers must be 16-byte aligned");
     REQUIRE((reinterpret_cast<uintptr_t>(d_packed) & 255u) == 0, TASQ_ERR_UNSUPPORTED, "d_packed must be 256-byte aligned");
+    if (lr_rank) {
+        REQUIRE(route == TASQ_ROUTE_TC, TASQ_ERR_UNSUPPORTED, "the low-rank branch runs on the tensor-core route");
+        REQUIRE(d_lr_u && d_lr_l1, TASQ_ERR_INVALID_ARG, "NULL pointer");
+        REQUIRE(!d_acc, TASQ_ERR_INVALID_ARG, "no int32 accumulators with the low-rank branch (d_acc must be NULL)");
+        REQUIRE(aligned16(d_lr_u) && aligned16(d_lr_l1), TASQ_ERR_UNSUPPORTED, "d_u and d_l1 must be 16-byte aligned");
+    }
 
     const tasq::PackedHeader lay = tasq::packed_layout(kind, N, K);
     const char* p = reinterpret_cast<const char*>(d_packed);
@@ -417,6 +424,9 @@ int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, in
     a.timeout_ns = ctx->timeout_ns;
     a.zcw = reinterpret_cast<const float*>(p + lay.off_zcw);
     a.code_sums = d_code_sums;
+    a.lr_u = d_lr_u;
+    a.lr_l1 = d_lr_l1;
+    a.lr_rank = lr_rank;
     cudaError_t e;
     int kernels = 0;
     if (route == TASQ_ROUTE_TC) {
@@ -440,6 +450,36 @@ TASQ_API int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_
     CHECK_CTX(ctx);
     return masked_contraction(ctx, TASQ_LINEAR, &layer, 1, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, M,
                               d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream);
+}
+
+TASQ_API int tasq_masked_gemm_lr(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,
+                                 const float* d_alpha, const float* d_zc, int M, const void* d_packed, int N, int K,
+                                 const uint16_t* d_u, const uint16_t* d_l1, int rank, uint16_t* d_y, int32_t* d_acc,
+                                 tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(rank == 16 || rank == 32, TASQ_ERR_INVALID_ARG, "rank %d: 16 or 32", rank);
+    return masked_contraction(ctx, TASQ_LINEAR, &layer, 1, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, M,
+                              d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream, d_u, d_l1, rank);
+}
+
+TASQ_API int tasq_lowrank_down(tasq_ctx ctx, const void* d_x, int dtype, int M, int K, const uint16_t* d_l2, int rank,
+                               const float* d_alpha, uint16_t* d_u, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(dtype == TASQ_F32 || dtype == TASQ_BF16, TASQ_ERR_INVALID_ARG, "dtype %d", dtype);
+    REQUIRE(rank == 16 || rank == 32, TASQ_ERR_INVALID_ARG, "rank %d: 16 or 32", rank);
+    REQUIRE(M >= 0 && K > 0, TASQ_ERR_INVALID_ARG, "M=%d K=%d", M, K);
+    REQUIRE(K % 16 == 0, TASQ_ERR_UNSUPPORTED, "K=%d must be a multiple of 16", K);
+    if (M == 0) return TASQ_OK;
+    REQUIRE(d_x && d_l2 && d_alpha && d_u, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    REQUIRE((reinterpret_cast<uintptr_t>(d_x) & (dtype == TASQ_F32 ? 7u : 3u)) == 0 &&
+                (reinterpret_cast<uintptr_t>(d_l2) & 3u) == 0 && aligned16(d_u),
+            TASQ_ERR_UNSUPPORTED,
+            "d_x must be 8-byte (fp32) or 4-byte (bf16) aligned, d_l2 4-byte and d_u 16-byte aligned");
+    const cudaError_t e =
+        tasq::launch_lowrank_down(d_x, dtype, M, K, d_l2, rank, d_alpha, 0, d_u, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "low-rank launch");
+    ctx->kernels += 1;
+    return TASQ_OK;
 }
 
 TASQ_API int tasq_masked_gemm_zp(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,

@@ -111,6 +111,12 @@ struct GemmArgs {
     // With code_sums set the epilogue adds zcw[n] * t[m], t = sum_k (s_x + zc).
     const float* zcw;          // [N] from the packed buffer (zeros for a symmetric pack)
     const int32_t* code_sums;  // [M] sum_k s_x[m][k] (conv: per input pixel), or NULL (two-term epilogue)
+    // 16-bit low-rank branch of an SVD-split layer (linear layers): one more K block
+    // after the last one of each tile adds sum_j u'[m][j] * fp16(l1[n][j] / c_w[n]) to
+    // the accumulator, u' = fp16((x . l2^T)[m][j] / alpha[m]) from tasq_lowrank_down.
+    const uint16_t* lr_u;      // fp16 [M][kLowRankCols] u' (columns >= lr_rank zero), or NULL
+    const uint16_t* lr_l1;     // bf16 [N][lr_rank]
+    int lr_rank;               // 0, 16 or 32
 };
 
 // Resolves the operating precision of every member layer of this launch on
@@ -256,6 +262,11 @@ cudaError_t launch_code_row_sums(const void* codes, int code_fmt, int M, int K, 
 cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float* zcw, const float* bias, int N, int K,
                         int Cin, void* packed, cudaStream_t st);
 cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
+// u' = fp16((bf16(x) . l2^T) / alpha[m]) into [M][64] fp16 (columns >= rank zero;
+// rank 16 or 32; K % 16 == 0; alpha per token, or one value when per_tensor)
+cudaError_t launch_lowrank_down(const void* x, int dtype, int M, int K, const uint16_t* l2, int rank,
+                                const float* alpha, int per_tensor, uint16_t* u, cudaStream_t st);
+constexpr int kLowRankCols = 64;  // fp16 columns of a u' row (one 128-byte swizzle atom)
 // *kernels: how many kernels the call enqueued (the contraction, plus the split-K
 // reduction when K is split).
 cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, const char** why, int* kernels);

@@ -133,6 +133,17 @@ __device__ __forceinline__ void mma_f8_ts(uint32_t d_tmem, uint32_t a_tmem, uint
 // values, whose lower 8 mantissa bits are zero, the upper bytes are the e5m2
 // encodings exactly.
 __device__ __forceinline__ uint32_t e5m2x4(uint32_t h01, uint32_t h23) { return __byte_perm(h01, h23, 0x7531); }
+// Warp-level D (+)= A . B, m16n8k16, bf16 operands, fp32 accumulators (the
+// register fragments of the PTX ISA's mma.m16n8k16 layout: a = 4 x bf16x2 of
+// rows g / g + 8 and columns 2t / 2t + 8, b = 2 x bf16x2 of rows 2t / 2t + 8 and
+// column g, d = rows g / g + 8 x columns 2t, 2t + 1; g = lane / 4, t = lane % 4).
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
 // Arrive on an mbarrier once every tcgen05 op issued so far by this thread completes.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");

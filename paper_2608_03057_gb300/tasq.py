@@ -78,6 +78,8 @@ def lib():
                 "tasq_quant_act_sums": ([P, P, I, I, I, I, I, I, P, I, P, P, P, P], I),
                 "tasq_masked_gemm": ([P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_gemm_zp": ([P, I, I, P, I, P, P, P, I, P, I, I, P, P, P], I),
+                "tasq_masked_gemm_lr": ([P, I, I, P, I, P, P, I, P, I, I, P, P, I, P, P, P], I),
+                "tasq_lowrank_down": ([P, P, I, I, I, P, I, P, P, P], I),
                 "tasq_masked_gemm_grouped": ([P, P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_conv3x3": ([P, I, I, P, I, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_masked_conv3x3_zp": ([P, I, I, P, I, P, P, P, I, I, I, I, P, I, P, P, P], I),
@@ -219,6 +221,18 @@ def tasq_masked_gemm_zp(ctx, layer, stage, codes, code_fmt, alpha, zc, code_sums
     _check(ctx, lib().tasq_masked_gemm_zp(ctx, int(layer), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
                                           _ptr(zc), _ptr(code_sums), int(M), _ptr(packed), int(N), int(K), _ptr(y),
                                           _ptr(acc), _stream(stream)))
+
+
+def tasq_lowrank_down(ctx, x, dtype, M, K, l2, rank, alpha, u, stream=None) -> None:
+    _check(ctx, lib().tasq_lowrank_down(ctx, _ptr(x), int(dtype), int(M), int(K), _ptr(l2), int(rank), _ptr(alpha),
+                                        _ptr(u), _stream(stream)))
+
+
+def tasq_masked_gemm_lr(ctx, layer, stage, codes, code_fmt, alpha, zc, M, packed, N, K, u, l1, rank, y, acc=None,
+                        stream=None) -> None:
+    _check(ctx, lib().tasq_masked_gemm_lr(ctx, int(layer), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
+                                          _ptr(zc), int(M), _ptr(packed), int(N), int(K), _ptr(u), _ptr(l1), int(rank),
+                                          _ptr(y), _ptr(acc), _stream(stream)))
 
 
 def tasq_masked_gemm(ctx, layer, stage, codes, code_fmt, alpha, zc, M, packed, N, K, y, acc=None, stream=None) -> None:

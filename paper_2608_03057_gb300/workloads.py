@@ -227,7 +227,7 @@ def schedule_constant(L: int, S: int, b: int) -> np.ndarray:
 
 
 def schedule_for(config: str, L: int, seed: int = 7) -> np.ndarray:
-    if config == "pixart":
+    if config in ("pixart", "pixart_lr"):
         return schedule_uniform(L, 20, (3, 4, 5, 6, 8), seed, edge_stages=2)
     if config == "sana":
         return schedule_uniform(L, 20, (2, 3, 4, 6, 8), seed)
@@ -246,7 +246,7 @@ def schedule_for(config: str, L: int, seed: int = 7) -> np.ndarray:
 
 def inventory_blocks(config: str, blocks: int) -> List[Layer]:
     """The first `blocks` transformer blocks of a DiT inventory (small cases)."""
-    if config in ("pixart", "pixart_a4"):
+    if config in ("pixart", "pixart_a4", "pixart_lr"):
         return pixart_sigma(blocks=blocks)
     if config == "sana":
         return sana_1600m(blocks=blocks)
@@ -254,12 +254,15 @@ def inventory_blocks(config: str, blocks: int) -> List[Layer]:
 
 
 def inventory(config: str) -> List[Layer]:
-    return {"single": single_linear, "pixart": pixart_sigma, "pixart_a4": pixart_sigma, "sana": sana_1600m,
-            "sdxl": sdxl_turbo}[config]()
+    return {"single": single_linear, "pixart": pixart_sigma, "pixart_a4": pixart_sigma, "pixart_lr": pixart_sigma,
+            "sana": sana_1600m, "sdxl": sdxl_turbo}[config]()
 
 
 # Activation precision n of each workload (8 unless listed).
 ACT_BITS = {"pixart_a4": 4}
+# Rank of the 16-bit low-rank branch beside every linear layer (SVDQuant+TASQ: a
+# frozen SVD branch of rank 32 in the 4-bit setting, 16 in the 6-bit one), or 0.
+LOWRANK = {"pixart_lr": 32}
 
 
 # ----------------------------------------------------------------------------

@@ -1255,3 +1255,143 @@ def test_e5m2_codes_in_a_convolution_use_the_fp16_codes(ctx, oracle):
     s_x, a, z = oracle.quant_act(x.reshape(1, -1), 4, oracle.SYMRANGE, oracle.PER_TOKEN)
     ref, rs = oracle.conv3x3(s_x.reshape(B, H, W, Cin), wq["s"], 4)
     assert np.array_equal(acc.cpu().numpy(), ref)
+
+
+# ------------------------------------------------ 16-bit low-rank branch --
+
+def _bf16_bits(a):
+    torch = G.torch()
+    return torch.from_numpy(np.asarray(a, np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def _dev_bits(bits):
+    torch = G.torch()
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).cuda()
+
+
+def _ulp(v, mant):
+    """Spacing of a float format with `mant` stored mantissa bits at |v|."""
+    e = np.floor(np.log2(np.maximum(np.abs(v), 2.0 ** -60)))
+    return 2.0 ** (e - mant)
+
+
+def _down_sums(oracle, x, l2_bits):
+    """sum_k |bf16(x) l2| per (row, rank): the fp32 accumulation's error scale."""
+    return np.abs(oracle.bf16_round(x).astype(np.float64)) @ np.abs(
+        oracle.bf16_bits_to_f32(l2_bits).astype(np.float64)).T
+
+
+@pytest.mark.parametrize("M,K,r,dtype", [(300, 1152, 32, tasq.TASQ_BF16), (4096, 1152, 16, tasq.TASQ_F32),
+                                         (77, 2048, 32, tasq.TASQ_F32), (17, 16, 16, tasq.TASQ_BF16),
+                                         (33, 48, 32, tasq.TASQ_F32)])
+def test_lowrank_down_parity(ctx, oracle, M, K, r, dtype):
+    """u' = fp16((bf16(x) . l2^T) / alpha) in rows of 64 fp16 against the oracle's
+    u / alpha, within the fp32 accumulation (K 2^-23 sum |x_b l2|) and one fp16
+    rounding; columns past the rank are zero (16 rows per CTA in eight K slices,
+    ragged M, K shorter than eight steps)."""
+    torch = G.torch()
+    x = workloads.normal((M, K), 801 + M)
+    l2 = _bf16_bits(workloads.normal((r, K), 802 + K, 0.05))
+    alpha = workloads.uniform((M,), 805 + M, 0.005, 0.02).astype(np.float32)
+    if dtype == tasq.TASQ_BF16:
+        xd, x = G.to_bf16(x)
+    else:
+        xd = G.dev(x)
+    u = G.empty((M, 64), torch.int16)
+    tasq.tasq_lowrank_down(ctx.h, xd, dtype, M, K, _dev_bits(l2), r, G.dev(alpha), u)
+    got = u.cpu().numpy().view(np.float16).astype(np.float64)
+    ref = oracle.lowrank_down(x, l2) / alpha[:, None].astype(np.float64)
+    tol = K * 2.0 ** -23 * _down_sums(oracle, x, l2) / alpha[:, None] + _ulp(np.abs(ref) + 1e-30, 10) * 1.01
+    assert np.all(np.abs(got[:, :r] - ref) <= tol)
+    assert not got[:, r:].any()
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+@pytest.mark.parametrize("M,N,K,r,full,act_bits", [
+    (256, 1152, 1152, 32, True, 8),    # 64-token tiles
+    (4000, 1096, 384, 16, True, 8),    # 256-token tiles (two stages per block), ragged channel tile
+    (4096, 3456, 1152, 32, False, 8),  # 192-token tiles, two accumulators
+    (77, 640, 2048, 32, True, 8),      # a shape the plan would split along K: kept whole
+    (4096, 1152, 4608, 32, False, 4),  # e5m2 codes, 8-bit-float route at b <= 4
+    (300, 512, 1168, 16, True, 4),     # e5m2 codes, ragged last K block
+])
+def test_masked_gemm_lr_parity(ctx, oracle, M, N, K, r, full, act_bits):
+    """The layer with its low-rank branch against the fp64 definition (masked
+    layer plus (x_b l2^T) l1^T), at every b: within one bf16 ulp, the fp32
+    epilogue chain, and the branch's 16-bit roundings (u' and l1 / c_w in fp16:
+    2^-10 of each product) and fp32 accumulations."""
+    torch = G.torch()
+    bits = [8, 5, 4, 2]
+    if act_bits <= 4:
+        st = _setup_f8(ctx, oracle, M, N, K, bits, seed=M + N + r, n_bits=act_bits)
+        x = workloads.normal((M, K), M + N + r)  # the input _setup_f8 quantized
+        fmt = F8
+    else:
+        w = workloads.normal((N, K), M + 11, 0.02)
+        bias = workloads.normal((N,), M + 12, 0.02)
+        x = workloads.normal((M, K), M + 13)
+        sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+        packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, G.dev(bias), N, K)
+        tasq.tasq_set_schedule(ctx.h, np.array([bits], np.uint8), 1, len(bits))
+        codes = G.empty((M, K), torch.float16)
+        alpha, zc = G.empty((M,), torch.float32), G.empty((M,), torch.float32)
+        tasq.tasq_quant_act(ctx.h, G.dev(x), tasq.TASQ_F32, M, K, 8, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, codes,
+                            tasq.TASQ_CODES_F16, alpha, zc)
+        s_x, a, z = oracle.quant_act(x, 8, oracle.SYMRANGE, oracle.PER_TOKEN)
+        st = dict(packed=packed, codes=codes, alpha=alpha, zc=zc, wq=oracle.quant_weight(w), s_x=s_x, a=a, z=z,
+                  bias=bias)
+        fmt = tasq.TASQ_CODES_F16
+    l2 = _bf16_bits(workloads.normal((r, K), 803 + K, 0.05))
+    l1 = _bf16_bits(workloads.normal((N, r), 804 + N, 0.05))
+    u = G.empty((M, 64), torch.int16)
+    tasq.tasq_lowrank_down(ctx.h, G.dev(x), tasq.TASQ_F32, M, K, _dev_bits(l2), r, st["alpha"], u)
+    rows = np.arange(M) if full else np.unique(np.concatenate([np.arange(0, M, max(1, M // 40)), [M - 1]]))
+    rows_d = torch.from_numpy(rows).cuda()
+    u_ref = oracle.lowrank_down(x[rows], l2)
+    lr = oracle.lowrank_up(u_ref, l1)
+    l1a = np.abs(oracle.bf16_bits_to_f32(l1).astype(np.float64))
+    branch_err = (2.0 ** -9 * np.abs(u_ref) + K * 2.0 ** -22 * _down_sums(oracle, x[rows], l2)) @ l1a.T
+    scale = np.abs(st["a"][rows].astype(np.float64)[:, None] * st["wq"]["c"].astype(np.float64)[None, :])
+    for stage, b in enumerate(bits):
+        y = G.empty((M, N), torch.int16)
+        tasq.tasq_masked_gemm_lr(ctx.h, 0, stage, st["codes"], fmt, st["alpha"], st["zc"], M, st["packed"], N, K, u,
+                                 _dev_bits(l1), r, y, None)
+        s_w = st["wq"]["s"]
+        ydef = oracle.linear_lowrank_def_f64(st["s_x"][rows], st["a"][rows], st["z"][rows], s_w, st["wq"]["c"],
+                                            st["bias"], b, lr)
+        acc = oracle.gemm(st["s_x"][rows], s_w, b).astype(np.float64)
+        rs = oracle.row_sums(s_w, b).astype(np.float64)
+        chain = 2.0 ** -18 * (scale * (np.abs(acc) + np.abs(st["z"][rows, None] * rs[None, :])) + np.abs(lr)
+                              + np.abs(st["bias"])[None, :])
+        got = oracle.bf16_bits_to_f32(G.bf16_bits_host(y.index_select(0, rows_d))).astype(np.float64)
+        tol = _ulp(np.maximum(np.abs(ydef), np.abs(got)), 7) + chain + branch_err
+        bad = np.abs(got - ydef) > tol
+        assert not bad.any(), (b, bad.sum(), np.abs(got - ydef)[bad][:5], tol[bad][:5])
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+def test_lowrank_bad_arguments(ctx):
+    torch = G.torch()
+    buf = torch.zeros((1 << 16,), dtype=torch.uint8, device="cuda")
+    tasq.tasq_set_schedule(ctx.h, np.array([[8]], np.uint8), 1, 1)
+    for rank in (8, 64):
+        with pytest.raises(tasq.TasqError) as e:
+            tasq.tasq_lowrank_down(ctx.h, buf, tasq.TASQ_F32, 16, 64, buf, rank, buf, buf)
+        assert e.value.code == tasq.TASQ_ERR_INVALID_ARG
+    with pytest.raises(tasq.TasqError) as e:  # K not a multiple of 16
+        tasq.tasq_lowrank_down(ctx.h, buf, tasq.TASQ_BF16, 16, 40, buf, 16, buf, buf)
+    assert e.value.code == tasq.TASQ_ERR_UNSUPPORTED
+    with pytest.raises(tasq.TasqError) as e:  # u must be 16-byte aligned
+        tasq.tasq_lowrank_down(ctx.h, buf, tasq.TASQ_BF16, 16, 64, buf, 16, buf, buf.data_ptr() + 8)
+    assert e.value.code == tasq.TASQ_ERR_UNSUPPORTED
+    with pytest.raises(tasq.TasqError) as e:  # int8 codes: the mma.sync s8 route has no low-rank block
+        tasq.tasq_masked_gemm_lr(ctx.h, 0, 0, buf, tasq.TASQ_CODES_S8, buf, buf, 16, buf, 64, 64, buf, buf, 16, buf)
+    assert e.value.code == tasq.TASQ_ERR_UNSUPPORTED
+    with pytest.raises(tasq.TasqError) as e:  # rank outside 16 / 32
+        tasq.tasq_masked_gemm_lr(ctx.h, 0, 0, buf, tasq.TASQ_CODES_F16, buf, buf, 16, buf, 64, 64, buf, buf, 24, buf)
+    assert e.value.code == tasq.TASQ_ERR_INVALID_ARG
+    with pytest.raises(tasq.TasqError) as e:  # no int32 accumulators with the branch
+        tasq.tasq_masked_gemm_lr(ctx.h, 0, 0, buf, tasq.TASQ_CODES_F16, buf, buf, 16, buf, 64, 64, buf, buf, 16, buf,
+                                 buf)
+    assert e.value.code == tasq.TASQ_ERR_INVALID_ARG
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK

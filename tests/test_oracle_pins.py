@@ -530,3 +530,48 @@ def test_effective_bits_weights_by_ops():
     tab = np.array([[8, 4], [2, 4]], np.uint8)
     eb = schedule.effective_bits(tab, [3, 1])
     assert eb[0] == pytest.approx((8 * 3 + 2) / 4) and eb[1] == 4.0
+
+
+# ------------------------------------------------ 16-bit low-rank branch --
+
+def test_lowrank_down_identity_rows_select_columns(oracle):
+    # l2 = the first 16 rows of the identity: u = bf16(x[:, :16]) exactly (one product per sum)
+    rng = np.random.default_rng(5)
+    x = rng.standard_normal((7, 48)).astype(np.float32)
+    l2 = np.zeros((16, 48), np.float32)
+    l2[np.arange(16), np.arange(16)] = 1.0
+    u = oracle.lowrank_down(x, oracle.f32_to_bf16_bits(l2))
+    assert np.array_equal(u, oracle.bf16_round(x[:, :16]).astype(np.float64))
+    # a permutation of the rank rows permutes the columns of u
+    perm = rng.permutation(16)
+    u2 = oracle.lowrank_down(x, oracle.f32_to_bf16_bits(l2[perm]))
+    assert np.array_equal(u2, u[:, perm])
+
+
+def test_lowrank_branch_equals_the_product_of_its_factors(oracle):
+    # small integers: every bf16 value and every sum is exact, so
+    # (x l2^T) l1^T must equal x (l1 l2)^T computed in int64
+    rng = np.random.default_rng(6)
+    M, K, N, r = 9, 64, 24, 32
+    x = rng.integers(-2, 3, (M, K))
+    l2 = rng.integers(-1, 2, (r, K))
+    l1 = rng.integers(-3, 4, (N, r))
+    u = oracle.lowrank_down(x.astype(np.float32), oracle.f32_to_bf16_bits(l2.astype(np.float32)))
+    lr = oracle.lowrank_up(u, oracle.f32_to_bf16_bits(l1.astype(np.float32)))
+    assert np.array_equal(lr, (x @ (l1 @ l2).T).astype(np.float64))
+    assert np.array_equal(u, (x @ l2.T).astype(np.float64))
+
+
+def test_lowrank_layer_adds_the_branch_to_the_dequantized_layer(oracle):
+    # with a zero branch the layer is the plain masked layer; a constant branch shifts every output
+    rng = np.random.default_rng(7)
+    s_x = rng.integers(-128, 128, (5, 32)).astype(np.int8)
+    s_w = rng.integers(-128, 128, (6, 32)).astype(np.int8)
+    alpha = rng.uniform(0.01, 0.02, 5).astype(np.float32)
+    zc = rng.uniform(-1, 1, 5).astype(np.float32)
+    c_w = rng.uniform(1e-3, 2e-3, 6).astype(np.float32)
+    bias = rng.uniform(-0.1, 0.1, 6).astype(np.float32)
+    y0 = oracle.linear_def_f64(s_x, alpha, zc, s_w, c_w, bias, 5)
+    assert np.array_equal(oracle.linear_lowrank_def_f64(s_x, alpha, zc, s_w, c_w, bias, 5, np.zeros((5, 6))), y0)
+    y1 = oracle.linear_lowrank_def_f64(s_x, alpha, zc, s_w, c_w, bias, 5, np.full((5, 6), 0.25))
+    assert np.allclose(y1 - y0, 0.25, rtol=0, atol=1e-12)
