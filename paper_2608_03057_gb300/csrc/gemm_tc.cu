@@ -1050,6 +1050,8 @@ __global__ void __launch_bounds__(256) splitk_epilogue_kernel(const GemmArgs a, 
     ptx::grid_launch_dependents();
 }
 
+}  // namespace
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
@@ -1062,8 +1064,6 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     }
     return fn;
 }
-
-}  // namespace
 
 size_t gemm_tc_part_bytes(int num_sms) { return size_t(num_sms) * MAX_EPI_WARPS * MAX_GPW * 32 * 32 * sizeof(int32_t); }
 

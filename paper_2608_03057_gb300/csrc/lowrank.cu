@@ -18,11 +18,15 @@
 // layer's quantization: only the final division by alpha waits for it.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
+#include <cudaTypedefs.h>
 
 #include "tasq_internal.cuh"
 #include "tc_ptx.cuh"
 
 namespace tasq {
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode();  // gemm_tc.cu
+
 namespace {
 
 // Eight bf16 of x[row][k..k+7] (16 bytes); zeros past M
@@ -160,10 +164,217 @@ __global__ void __launch_bounds__(kDownWarps * 32, 2)
     }
 }
 
+// ---------------------------------------------------------------------------
+// The same down-projection on the 5th-generation tensor cores, for bf16 x: a CTA
+// of four warps per 128 rows computes D[128 rows][R] = x_tile . l2^T in tensor
+// memory, tcgen05.mma kind::f16 with bf16 A (x, [128][64] per stage) and B (l2,
+// [R][64] per stage), both K-major in the 128-byte swizzle, brought in by TMA
+// through a ring of kTcStages stages (one thread loads, one thread issues the
+// four K = 16 MMAs per stage).  Each warp then reads its 32 rows of D and writes
+// u' = fp16(D / alpha).  Every wait is bounded: on a timeout the kernel records
+// TASQ_ERR_DEVICE_TIMEOUT and skips its output.
+constexpr int kTcStages = 4;
+constexpr int kTcRows = 128;
+
+template <int R>
+struct DownTcSmem {
+    alignas(1024) uint8_t xs[kTcStages][kTcRows * 128];
+    alignas(1024) uint8_t ls[kTcStages][R * 128];
+    uint64_t full[kTcStages], empty[kTcStages], done;
+    uint32_t tmem;
+    int abort;
+};
+
+__device__ __forceinline__ bool bounded_wait(uint32_t bar, uint32_t parity, unsigned long long timeout_ns,
+                                             int* abort, bool ignore_abort = false) {
+    if (ptx::mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = ptx::globaltimer();
+    for (uint32_t it = 1;; ++it) {
+        if (ptx::mbar_try_wait(bar, parity)) return true;
+        if ((it & 63) == 0) {
+            if (!ignore_abort && *(volatile int*)abort) return false;
+            if (ptx::globaltimer() - t0 > timeout_ns) {
+                *(volatile int*)abort = 1;
+                return false;
+            }
+        }
+    }
+}
+
+template <int R>
+__global__ void __launch_bounds__(128)
+    lowrank_down_tc_kernel(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_l2, int M,
+                           int K, const float* __restrict__ alpha, int per_tensor, uint16_t* __restrict__ u,
+                           int* status, unsigned long long timeout_ns) {
+    extern __shared__ uint8_t smem_raw[];
+    DownTcSmem<R>* s =
+        reinterpret_cast<DownTcSmem<R>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * kTcRows;
+    const int KB = (K + 63) / 64;
+    constexpr uint32_t kStageBytes = kTcRows * 128 + R * 128;
+    // D: fp32, bf16 A and B (format code 1 in both fields), M = 128, N = R
+    constexpr uint32_t idesc = ptx::idesc_f16_f32(kTcRows, R) | (1u << 7) | (1u << 10);
+    if (warp == 0) {
+        ptx::tmem_alloc(ptx::smem_u32(&s->tmem), 32);
+        ptx::tmem_relinquish();
+        ptx::tc_fence_before();
+    }
+    if (threadIdx.x == 32) {
+        for (int i = 0; i < kTcStages; ++i) {
+            ptx::mbar_init(ptx::smem_u32(&s->full[i]), 1);
+            ptx::mbar_init(ptx::smem_u32(&s->empty[i]), 1);
+        }
+        ptx::mbar_init(ptx::smem_u32(&s->done), 1);
+        s->abort = 0;
+        ptx::fence_mbar_init();
+        ptx::prefetch_tmap(&tm_x);
+        ptx::prefetch_tmap(&tm_l2);
+    }
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = s->tmem;
+    bool ok = true;
+    int issued = 0;  // producer: stages loaded
+    if (threadIdx.x == 0) {
+        // producer: x is the layer's input and l2 a weight, both written before the
+        // quantization this launch overlaps
+        for (int kb = 0; kb < KB && ok; ++kb, ++issued) {
+            const int st = kb % kTcStages;
+            if (kb >= kTcStages &&
+                !bounded_wait(ptx::smem_u32(&s->empty[st]), ((kb / kTcStages) - 1) & 1, timeout_ns, &s->abort)) {
+                ok = false;
+                break;
+            }
+            const uint32_t fb = ptx::smem_u32(&s->full[st]);
+            ptx::mbar_arrive_expect_tx(fb, kStageBytes);
+            ptx::tma_load_2d(ptx::smem_u32(s->xs[st]), &tm_x, fb, kb * 64, m0);
+            ptx::tma_load_2d(ptx::smem_u32(s->ls[st]), &tm_l2, fb, kb * 64, 0);
+        }
+    } else if (threadIdx.x == 32) {
+        // MMA issuer
+        for (int kb = 0; kb < KB && ok; ++kb) {
+            const int st = kb % kTcStages;
+            if (!bounded_wait(ptx::smem_u32(&s->full[st]), (kb / kTcStages) & 1, timeout_ns, &s->abort)) {
+                ok = false;
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint64_t adesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->xs[st]));
+            const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_u32(s->ls[st]));
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)  // K steps of 16 bf16 = 32 bytes along the rows
+                asm volatile(
+                    "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+                    "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
+                    "l"(adesc + uint64_t(2 * kk)), "l"(bdesc + uint64_t(2 * kk)), "r"(idesc),
+                    "r"((kb | kk) ? 1u : 0u));
+            ptx::mma_commit(ptx::smem_u32(&s->empty[st]));
+        }
+        ptx::mma_commit(ptx::smem_u32(&s->done));
+    }
+    __syncwarp();
+    // the contraction that reads u' may start its set-up; alpha comes from the
+    // previous kernel (the layer's quantization)
+    ptx::grid_launch_dependents();
+    ptx::grid_dependency_wait();
+    const bool got = bounded_wait(ptx::smem_u32(&s->done), 0, timeout_ns, &s->abort);
+    ptx::tc_fence_after();
+    if (got && !*(volatile int*)&s->abort) {
+        uint32_t v[32];
+        if constexpr (R == 32) {
+            ptx::tmem_ld32(tmem + (uint32_t(warp * 32) << 16), v);
+        } else {
+            ptx::tmem_ld16(tmem + (uint32_t(warp * 32) << 16), *reinterpret_cast<uint32_t(*)[16]>(&v[0]));
+        }
+        ptx::tmem_wait_ld();
+        const int m = m0 + warp * 32 + lane;
+        if (m < M) {
+            const float al = alpha[per_tensor ? 0 : m];
+            uint32_t h[32];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const float a0 = 2 * j < R ? __fdiv_rn(__uint_as_float(v[2 * j]), al) : 0.f;
+                const float a1 = 2 * j + 1 < R ? __fdiv_rn(__uint_as_float(v[2 * j + 1]), al) : 0.f;
+                const __half2 hh = __floats2half2_rn(a0, a1);
+                h[j] = *reinterpret_cast<const uint32_t*>(&hh);
+            }
+#pragma unroll
+            for (int j = 16; j < 32; ++j) h[j] = 0u;
+            uint4* dst = reinterpret_cast<uint4*>(u + int64_t(m) * 64);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) dst[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+        }
+    }
+    if (threadIdx.x == 0) {
+        // copies still in flight land before the CTA may exit (only after an abort can
+        // the MMA issuer have left a loaded stage unread)
+        for (int kb = issued - kTcStages < 0 ? 0 : issued - kTcStages; kb < issued; ++kb)
+            bounded_wait(ptx::smem_u32(&s->full[kb % kTcStages]), (kb / kTcStages) & 1, timeout_ns, &s->abort, true);
+        if (*(volatile int*)&s->abort) set_status(status, TASQ_ERR_DEVICE_TIMEOUT);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, 32);
+    }
+}
+
+}  // namespace
+
+namespace {
+
+// The tensor-core kernel for bf16 x (16-byte aligned x and l2); false when its
+// tensor maps cannot be encoded.
+template <int R>
+bool launch_down_tc(const void* x, int M, int K, const uint16_t* l2, const float* alpha, int per_tensor, uint16_t* u,
+                    int* status, unsigned long long timeout_ns, cudaStream_t st, cudaError_t* err) {
+    auto encode = get_encode();
+    if (!encode) return false;
+    CUtensorMap tm_x, tm_l2;
+    cuuint64_t dx[2] = {cuuint64_t(K), cuuint64_t(M)}, dl[2] = {cuuint64_t(K), cuuint64_t(R)};
+    cuuint64_t sx[1] = {cuuint64_t(K) * 2}, sl[1] = {cuuint64_t(K) * 2};
+    cuuint32_t bx[2] = {64, kTcRows}, bl[2] = {64, R}, es[2] = {1, 1};
+    if (encode(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dx, sx, bx, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
+        encode(&tm_l2, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(l2), dl, sl, bl, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return false;
+    const int smem = int(sizeof(DownTcSmem<R>)) + 1024;
+    cudaError_t e = cudaFuncSetAttribute(lowrank_down_tc_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess) {
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3(unsigned((M + kTcRows - 1) / kTcRows));
+        cfg.blockDim = dim3(128);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, lowrank_down_tc_kernel<R>, tm_x, tm_l2, M, K, alpha, per_tensor, u, status,
+                               timeout_ns);
+        if (e == cudaSuccess) e = cudaGetLastError();
+    }
+    *err = e;
+    return true;
+}
+
 }  // namespace
 
 cudaError_t launch_lowrank_down(const void* x, int dtype, int M, int K, const uint16_t* l2, int rank,
-                                const float* alpha, int per_tensor, uint16_t* u, cudaStream_t st) {
+                                const float* alpha, int per_tensor, uint16_t* u, int* status,
+                                unsigned long long timeout_ns, cudaStream_t st) {
+    if (dtype == TASQ_BF16 && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(l2)) & 15u) == 0) {
+        cudaError_t e = cudaSuccess;
+        if (rank == 16 ? launch_down_tc<16>(x, M, K, l2, alpha, per_tensor, u, status, timeout_ns, st, &e)
+                       : launch_down_tc<32>(x, M, K, l2, alpha, per_tensor, u, status, timeout_ns, st, &e))
+            return e;
+    }
     const unsigned grid = unsigned((M + 15) / 16), block = kDownWarps * 32;
     auto launch = [&](auto kernel, size_t smem) {
         cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));

@@ -475,8 +475,8 @@ TASQ_API int tasq_lowrank_down(tasq_ctx ctx, const void* d_x, int dtype, int M, 
                 (reinterpret_cast<uintptr_t>(d_l2) & 3u) == 0 && aligned16(d_u),
             TASQ_ERR_UNSUPPORTED,
             "d_x must be 8-byte (fp32) or 4-byte (bf16) aligned, d_l2 4-byte and d_u 16-byte aligned");
-    const cudaError_t e =
-        tasq::launch_lowrank_down(d_x, dtype, M, K, d_l2, rank, d_alpha, 0, d_u, (cudaStream_t)stream);
+    const cudaError_t e = tasq::launch_lowrank_down(d_x, dtype, M, K, d_l2, rank, d_alpha, 0, d_u, ctx->d_words,
+                                                    ctx->timeout_ns, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(ctx, e, "low-rank launch");
     ctx->kernels += 1;
     return TASQ_OK;

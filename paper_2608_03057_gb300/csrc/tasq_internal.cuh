@@ -263,9 +263,11 @@ cudaError_t launch_pack(int kind, const int8_t* sw, const float* cw, const float
                         int Cin, void* packed, cudaStream_t st);
 cudaError_t launch_gemm_s8(const GemmArgs& a, int num_sms, cudaStream_t st);
 // u' = fp16((bf16(x) . l2^T) / alpha[m]) into [M][64] fp16 (columns >= rank zero;
-// rank 16 or 32; K % 16 == 0; alpha per token, or one value when per_tensor)
+// rank 16 or 32; K % 16 == 0; alpha per token, or one value when per_tensor).
+// status / timeout_ns: the device status word and the bound of the kernel's waits.
 cudaError_t launch_lowrank_down(const void* x, int dtype, int M, int K, const uint16_t* l2, int rank,
-                                const float* alpha, int per_tensor, uint16_t* u, cudaStream_t st);
+                                const float* alpha, int per_tensor, uint16_t* u, int* status,
+                                unsigned long long timeout_ns, cudaStream_t st);
 constexpr int kLowRankCols = 64;  // fp16 columns of a u' row (one 128-byte swizzle atom)
 // *kernels: how many kernels the call enqueued (the contraction, plus the split-K
 // reduction when K is split).

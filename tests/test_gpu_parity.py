@@ -1283,12 +1283,15 @@ def _down_sums(oracle, x, l2_bits):
 
 @pytest.mark.parametrize("M,K,r,dtype", [(300, 1152, 32, tasq.TASQ_BF16), (4096, 1152, 16, tasq.TASQ_F32),
                                          (77, 2048, 32, tasq.TASQ_F32), (17, 16, 16, tasq.TASQ_BF16),
-                                         (33, 48, 32, tasq.TASQ_F32)])
+                                         (33, 48, 32, tasq.TASQ_F32), (4096, 1152, 32, tasq.TASQ_BF16),
+                                         (200, 4608, 16, tasq.TASQ_BF16)])
 def test_lowrank_down_parity(ctx, oracle, M, K, r, dtype):
     """u' = fp16((bf16(x) . l2^T) / alpha) in rows of 64 fp16 against the oracle's
     u / alpha, within the fp32 accumulation (K 2^-23 sum |x_b l2|) and one fp16
-    rounding; columns past the rank are zero (16 rows per CTA in eight K slices,
-    ragged M, K shorter than eight steps)."""
+    rounding; columns past the rank are zero.  bf16 x takes the tensor-core kernel
+    (128 rows per CTA, ragged M, K shorter than one 64-wide stage, several trips
+    round the stage ring), fp32 x the warp-MMA kernel (ragged M, K shorter than
+    its sixteen slices)."""
     torch = G.torch()
     x = workloads.normal((M, K), 801 + M)
     l2 = _bf16_bits(workloads.normal((r, K), 802 + K, 0.05))
