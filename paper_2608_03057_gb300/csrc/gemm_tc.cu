@@ -53,7 +53,7 @@ constexpr int BCH = 128;          // output channels per tile (MMA M)
 constexpr int BK = 128;           // K per weight stage and per tensor-memory slot of converted weights
 constexpr int XK = 64;            // K per activation TMA box (one 128-byte swizzle atom of fp16 codes)
 constexpr int W_STAGES = 3;
-constexpr int ASLOTS = 2;         // converted-weight slots in tensor memory
+constexpr int ASLOTS = 2;         // converted-weight slots in tensor memory (the configurations' default)
 // Warps 2 .. 17 are converters (4, one per tensor-memory lane quadrant, or 8, two per
 // quadrant each widening half of a K block) followed by epilogue warps (12 or 8).
 constexpr int MID_WARPS = 16;
@@ -73,10 +73,11 @@ static_assert(BK == 2 * XK, "a stage is two 64-wide swizzle atoms");
 // accumulator then only has to wait for the drain between certified chunks.
 // <64, 2>: for launches with few tokens, three times as many CTAs as <192, 2>
 // and a third of its per-tile epilogue.
-template <int BT_, int NACC_, int CONV_WARPS_ = 4>
+template <int BT_, int NACC_, int CONV_WARPS_ = 4, int AS_ = ASLOTS>
 struct Cfg {
     static constexpr int BT = BT_;
     static constexpr int NACC = NACC_;
+    static constexpr int AS = AS_;  // converted-weight slots in tensor memory
     static constexpr int CONV_WARPS = CONV_WARPS_;           // converter warps (4 or 8)
     static constexpr int CONV_SPLIT = CONV_WARPS / 4;        // converters per lane quadrant (K split)
     static constexpr int EPI_WARP0 = 2 + CONV_WARPS;         // first epilogue warp
@@ -100,9 +101,9 @@ struct Cfg {
     static constexpr uint32_t A_COL = NACC * BT;         // ASLOTS x BK/2 columns (fp16 pairs)
     static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BT);
     static constexpr uint32_t IDESC8 = ptx::idesc_e5m2_f32(BCH, BT);  // the 8-bit route
-    static_assert(DONE % X_STAGES == 0 && DONE >= (ASLOTS + 1) * Q, "completion ring covers both reuse distances");
+    static_assert(DONE % X_STAGES == 0 && DONE >= (AS + 1) * Q, "completion ring covers both reuse distances");
     static_assert(Q == 1 || X_STAGES % 2 == 0, "first-half stages must keep their parity");
-    static_assert(A_COL + ASLOTS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
+    static_assert(A_COL + AS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
     static_assert(GPW <= MAX_GPW && BT <= 256 && BT % 32 == 0, "tile shape");
     static_assert((CONV_WARPS == 4 || CONV_WARPS == 8) && EPI_WARPS <= MAX_EPI_WARPS, "warp roles");
 };
@@ -464,11 +465,11 @@ __global__ void __maxnreg__(96)
                     // (LR: the last chunk also takes the low-rank block, kb == kb_hi)
                     const int kb_end = min(wk.kb_hi, kb0 + chunk) + (LR && c == wk.nch - 1 ? 1 : 0);
                     for (int kb = kb0; kb < kb_end && ok; ++kb, ++it) {
-                        const uint32_t acol = tmem + C::A_COL + (it % ASLOTS) * A_SLOT_COLS;
+                        const uint32_t acol = tmem + C::A_COL + (it % C::AS) * A_SLOT_COLS;
                         const bool lrb = LR && kb == wk.kb_hi;  // the low-rank block: fp16, 64 columns of K
                         for (int i = 0; i < Q; ++i) {
                             const int u = it * Q + i;
-                            // activations landed (and, for i == 0, the converters wrote slot it % 2)
+                            // activations landed (and, for i == 0, the converters wrote slot it % AS)
                             if (!wt.wait(&s->xfull[u % X_STAGES], (u / X_STAGES) & 1)) {
                                 ok = false;
                                 break;
@@ -608,15 +609,15 @@ __global__ void __maxnreg__(96)
                     if (lane == 0) ptx::mbar_arrive(ptx::smem_u32(&s->wempty[rw.slot]));
                     rw.next();
                 }
-                // slot it % 2 last held K block it - 2: its MMAs must have finished
-                // (the last activation stage of block it - 2 completes after all its MMAs)
-                if (it >= ASLOTS && !wt.wait(&s->done[((it - ASLOTS) * Q + Q - 1) % DONE],
-                                             (((it - ASLOTS) * Q + Q - 1) / DONE) & 1)) {
+                // slot it % AS last held K block it - AS: its MMAs must have finished
+                // (the last activation stage of that block completes after all its MMAs)
+                if (it >= C::AS && !wt.wait(&s->done[((it - C::AS) * Q + Q - 1) % DONE],
+                                            (((it - C::AS) * Q + Q - 1) / DONE) & 1)) {
                     ok = false;
                     break;
                 }
                 {
-                    const uint32_t dst = lane_base + C::A_COL + (it % ASLOTS) * A_SLOT_COLS + kp * NF;
+                    const uint32_t dst = lane_base + C::A_COL + (it % C::AS) * A_SLOT_COLS + kp * NF;
 #pragma unroll
                     for (int h = 0; h < NF / 32; ++h)
                         ptx::tmem_st32(dst + 32 * h, *reinterpret_cast<const uint32_t(*)[32]>(&f[32 * h]));
