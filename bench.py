@@ -788,18 +788,51 @@ def e2e_measure(torch, tasq, step, n_steps, stage_of, copy_streams=1):
             j.record(c)
             s.wait_event(j)
 
-    e2e_step()
-    torch.cuda.synchronize()
-    ge = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(ge, capture_error_mode="thread_local"):
-        e2e_step()
-    for k in range(3):  # the first replays of a new graph upload it and touch every pinned page
-        ge.replay()
-    torch.cuda.synchronize()
+    def copies_only(h2d, d2h):
+        # the step's own copies on the same streams, without its kernels: the time the
+        # host link alone needs for them, measured beside the end-to-end figure
+        s = torch.cuda.current_stream()
+        fork.record(s)
+        for c in sh + sd:
+            c.wait_event(fork)
+        for i in range(L):
+            if h2d:
+                with torch.cuda.stream(sh[i % nc]):
+                    step.x[i].copy_(xh[i], non_blocking=True)
+            if d2h:
+                with torch.cuda.stream(sd[i % nc]):
+                    yh[i].copy_(step.y[i], non_blocking=True)
+        for c, j in zip(sh + sd, joins):
+            j.record(c)
+            s.wait_event(j)
+
+    def graph_of(fn):
+        fn()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            fn()
+        for k in range(3):  # the first replays of a new graph upload it and touch every pinned page
+            g.replay()
+        torch.cuda.synchronize()
+        return g
+
+    bi = int(sum(x.numel() * x.element_size() for x in xh))
+    bo = int(sum(y.numel() * y.element_size() for y in yh))
+    ge = graph_of(e2e_step)
     ms = timed_replays(torch, ge, step, n_steps, stage_of)
+    link = {}
+    for key, h2d, d2h in (("h2d_only", True, False), ("d2h_only", False, True), ("both", True, True)):
+        gc = graph_of(lambda: copies_only(h2d, d2h))
+        link[key + "_ms"] = timed_replays(torch, gc, step, 3, stage_of)
+        del gc
+    link["h2d_gbs"] = bi / link["h2d_only_ms"] / 1e6
+    link["d2h_gbs"] = bo / link["d2h_only_ms"] / 1e6
+    link["both_gbs"] = (bi + bo) / link["both_ms"] / 1e6
     out = {"ms_per_step": ms, "copy_streams_per_direction": nc,
-           "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in xh)),
-           "d2h_bytes_per_step": int(sum(y.numel() * y.element_size() for y in yh))}
+           "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo,
+           # the same copies with no kernels, timed right after the end-to-end replays
+           "copies_only": link}
     del xh, yh, ge
     return out
 
