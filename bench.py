@@ -67,6 +67,15 @@ def measured_traffic(workload: str):
 
 
 UNIT = "TOPS"
+# Units of the step (layers that read one input: one quantization, one contraction call).
+GROUPINGS = {
+    "text": "every layer that reads the text tokens (the key and value projections of all cross-attention "
+            "blocks) in one unit per shape, first in the step: one quantization and one contraction launch "
+            "with the member list in device memory, each layer at its own b",
+    "pairs": "a cross-attention's key and value projections read one input: one quantization and one grouped "
+             "contraction, each layer at its own b",
+    "none": "every layer its own quantization and contraction",
+}
 WORKLOAD_NAMES = {
     "pixart": "pixart_sigma_1024px_denoise_step",
     "pixart_a4": "pixart_sigma_1024px_denoise_step_a4_w4a4_budget",
@@ -95,6 +104,8 @@ def parse_args():
     ap.add_argument("--no-sweep", action="store_true", help="skip the GEMM sweep and the stage-switch test")
     ap.add_argument("--no-per-workload", action="store_true",
                     help="time only --workload, not the other workloads of the suite")
+    ap.add_argument("--grouping", choices=list(GROUPINGS), default="text",
+                    help="which layers share one quantization and one contraction launch")
     return ap.parse_args()
 
 
@@ -165,13 +176,16 @@ class ClockSampler:
 class Step:
     """Device-resident workload of one denoising step and its launch sequence.
 
-    The step runs unit by unit: a unit is the layers that read one input (a
-    cross-attention's key and value projections; every other layer alone).  A
-    unit's input is quantized once and contracted by one call, at each member
-    layer's own precision from the bit table (tasq_masked_gemm_grouped for two
-    members).  Every layer keeps its own row of the table."""
+    The step runs unit by unit: a unit is the layers that read one input.  With
+    grouping "text" (the default) every layer that reads the text tokens -- the key
+    and value projections of all cross-attention blocks -- is in one unit per shape,
+    first in the step, contracted by tasq_masked_gemm_shared_input; with "pairs" each
+    cross-attention's key and value projections form a unit (tasq_masked_gemm_grouped);
+    every other layer is a unit alone.  A unit's input is quantized once and
+    contracted by one call, at each member layer's own precision from the bit table.
+    Every layer keeps its own row of the table."""
 
-    def __init__(self, torch, tasq, workloads, name: str, seed: int, blocks: int = 0, group=True):
+    def __init__(self, torch, tasq, workloads, name: str, seed: int, blocks: int = 0, grouping="text"):
         self.torch, self.tasq = torch, tasq
         self.layers = workloads.inventory(name)
         self.table = workloads.schedule_for(name, len(self.layers))
@@ -181,11 +195,21 @@ class Step:
         self.code_fmt = tasq.TASQ_CODES_F16_E5M2 if self.act_bits <= 4 else tasq.TASQ_CODES_F16
         # 16-bit low-rank branch beside every linear layer: one call per layer
         self.rank = workloads.LOWRANK.get(name, 0)
-        group = group and not self.rank
+        if self.rank:
+            grouping = "none"
+        self.grouping = grouping
         if blocks:
             keep = len(workloads.inventory_blocks(name, blocks))
             self.layers, self.table = self.layers[:keep], np.ascontiguousarray(self.table[:keep])
-        self.units = workloads.input_groups(self.layers) if group else [[i] for i in range(len(self.layers))]
+        if grouping == "text":
+            self.units = workloads.shared_input_units(self.layers)
+        elif grouping == "pairs":
+            self.units = workloads.input_groups(self.layers)
+        else:
+            self.units = [[i] for i in range(len(self.layers))]
+        # units contracted with the member list in device memory
+        self.d_layers = [torch.tensor(unit, dtype=torch.int32, device="cuda") if grouping == "text" and len(unit) > 1
+                         else None for unit in self.units]
         self.S = self.table.shape[1]
         self.ctx = tasq.tasq_create(torch.cuda.current_device())
         tasq.tasq_set_schedule(self.ctx, self.table, len(self.layers), self.S)
@@ -263,6 +287,9 @@ class Step:
                                     self.u)
                 t.tasq_masked_gemm_lr(self.ctx, unit[0], -1, self.codes, self.code_fmt, self.alpha, self.zc, l.M,
                                       self.packed[u], N, l.K, self.u, self.l1[u], self.rank, self.y[u], None)
+            elif self.d_layers[u] is not None:
+                t.tasq_masked_gemm_shared_input(self.ctx, self.d_layers[u], len(unit), -1, self.codes, self.code_fmt,
+                                                self.alpha, self.zc, l.M, self.packed[u], N, l.K, self.y[u], None)
             elif len(unit) == 1:
                 t.tasq_masked_gemm(self.ctx, unit[0], -1, self.codes, self.code_fmt, self.alpha, self.zc, l.M,
                                    self.packed[u], N, l.K, self.y[u], None)
@@ -325,7 +352,7 @@ def f8_op_share(tasq, step, steps, stage_of, num_sms):
             if l.kind == step.conv or any(int(step.table[i, s]) > 4 for i in unit):
                 continue
             plan = tasq.tasq_plan_tc(tasq.TASQ_LINEAR, l.M, step.y[u].shape[1], l.K, 0, 0, 0, 0, num_sms)
-            if plan["splits"] == 1:
+            if plan["splits"] == 1 or step.d_layers[u] is not None:  # (member lists in device memory: unsplit)
                 f8 += ops
     return f8 / tot if tot else 0.0
 
@@ -845,7 +872,7 @@ def measure_workload(torch, tasq, workloads, name, args, peaks, steps, dist=None
     the end-to-end step.  Returns the figures and the Step (closed by the caller)."""
     from paper_2608_03057_gb300 import engine_model, schedule
     step = Step(torch, tasq, workloads, name, args.seed,
-                args.blocks if name in ("pixart", "pixart_a4", "pixart_lr", "sana") else 0)
+                args.blocks if name in ("pixart", "pixart_a4", "pixart_lr", "sana") else 0, args.grouping)
     S = step.S
     stage_of = stage_map(name, S)
     for k in range(2):  # eager launches first: they set kernel attributes outside any capture
@@ -1018,8 +1045,7 @@ def main():
             "scaling": "weak", "vs_baseline": None, "dtype": "f16-exact-int8", "data": "synthetic",
             "config": {"workload": head["workload"], "layers": head["layers"],
                        "contraction_calls": head["contraction_calls"], "stages": head["stages"],
-                       "shared_inputs": "a cross-attention's key and value projections read one input: one "
-                                        "quantization and one grouped contraction, each layer at its own b",
+                       "shared_inputs": GROUPINGS[args.grouping],
                        "schedule": "seeded learned-style per-(layer, stage) bits",
                        "effective_w_bits": head["effective_w_bits"], "rel_bitops": head["rel_bitops"],
                        "route": "tcgen05 fp16 MMA, exact int32",

@@ -67,7 +67,7 @@
 extern "C" {
 #endif
 
-#define TASQ_ABI_VERSION 4
+#define TASQ_ABI_VERSION 5
 
 /* Return codes. */
 enum {
@@ -333,6 +333,32 @@ int tasq_masked_gemm(tasq_ctx ctx, int layer, int stage, const void* d_codes, in
 int tasq_masked_gemm_grouped(tasq_ctx ctx, const int32_t* h_layers, int groups, int stage, const void* d_codes,
                              int code_fmt, const float* d_alpha, const float* d_zc, int M, const void* d_packed,
                              int N, int K, uint16_t* d_y, int32_t* d_acc, tasq_stream stream);
+
+/*
+ * Many masked linear layers that read one input, in one launch: the grouped
+ * call with its member list in device memory, for up to 256 members -- e.g. the
+ * key and value projections of every cross-attention block of a denoising
+ * step, which all take the same text tokens (the caption embedding is computed
+ * once per forward pass), so that their activations are quantized once and
+ * their weights streamed by one launch.  Member g is layer d_layers[g] and
+ * runs at b_g = table[d_layers[g]][stage] (App. F.1: the bit map is per
+ * layer); it owns output channels [g Ng, (g + 1) Ng), Ng = N / n_layers, of
+ * one TASQ_LINEAR buffer packed from the members' [Ng][K] codes, scales and
+ * biases concatenated along N, and its outputs are exactly what
+ * tasq_masked_gemm computes for that layer alone.  d_layers: device int32
+ * array of n_layers (1..256) layer indices, 4-byte aligned, owned by the
+ * caller and read by every launch (a graph that captured the call reads it at
+ * each replay); an index outside 0..L-1 is found on the device and recorded
+ * as TASQ_ERR_DEVICE in the status word (tasq_device_status), with no output
+ * written.  Needs N % n_layers == 0, Ng % 8 == 0, fp16 codes
+ * (TASQ_CODES_F16 or TASQ_CODES_F16_E5M2) and the tensor-core route; the
+ * launch is never split along K.  Other arguments and rules as
+ * tasq_masked_gemm.  Enqueue call.
+ */
+int tasq_masked_gemm_shared_input(tasq_ctx ctx, const int32_t* d_layers, int n_layers, int stage,
+                                  const void* d_codes, int code_fmt, const float* d_alpha, const float* d_zc, int M,
+                                  const void* d_packed, int N, int K, uint16_t* d_y, int32_t* d_acc,
+                                  tasq_stream stream);
 
 /*
  * 16-bit low-rank branch of an SVD-split linear layer (the frozen SVD branch

@@ -146,6 +146,10 @@ struct Smem {
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
+    // a member list in device memory: each member's b, and per warp the set of the
+    // precisions its members run at (bit b; bit 0 for a member that did not resolve)
+    uint8_t mbits[kMaxMembers];
+    uint32_t wpresent[THREADS / 32];
 };
 template <class C>
 constexpr int smem_bytes() { return int(sizeof(Smem<C>)) + 1024; }
@@ -282,8 +286,10 @@ __device__ __forceinline__ bool f8_route(const GemmArgs& a, uint32_t gbits) {
 // the last K block of each tile one more block of fp16 MMAs adds
 // u'[m] . (l1[n] / c_w[n]) to the accumulator (u' in tm_u, the weights' block
 // converted from l1 by the converters), so that the epilogue's dequantization
-// scales it back to u . l1 (unsplit launches only).
-template <bool CONV, bool ZP, class C, bool F8 = false, bool LR = false>
+// scales it back to u . l1 (unsplit launches only); MANY a grouped linear layer whose
+// member list is in device memory (a.d_layers, up to kMaxMembers members; unsplit
+// launches only): every CTA resolves each member's b into shared memory.
+template <bool CONV, bool ZP, class C, bool F8 = false, bool LR = false, bool MANY = false>
 __global__ void __maxnreg__(96)
     gemm_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tm_x,
                    const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_y,
@@ -310,17 +316,46 @@ __global__ void __maxnreg__(96)
     int cert[kNumB];
 #pragma unroll
     for (int i = 0; i < kNumB; ++i) cert[i] = a.hdr->chunk_kb[kBMin + i];
-    // b of every member layer (one member unless the call is grouped); b = member 0's
-    const uint32_t gbits = resolve_group_bits(a);
+    // b of every member layer (one member unless the call is grouped); b = member 0's.
+    // A member list in device memory (MANY): one thread per member resolves its b into
+    // shared memory and each warp gathers the set of precisions present; gbits then
+    // stands for that set (bit b for each b present, 0 when a member did not resolve)
+    // once the barrier below has passed.
+    uint32_t gbits = 0;
+    if constexpr (MANY) {
+        uint32_t present = 0;
+        if (int(threadIdx.x) < a.groups) {
+            const int bg = resolve_member_bits(a, int(threadIdx.x));
+            s->mbits[threadIdx.x] = uint8_t(bg);
+            present = 1u << bg;
+        }
+        present = __reduce_or_sync(0xFFFFFFFFu, present);
+        if (lane == 0) s->wpresent[warp] = present;
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < THREADS / 32; ++i) gbits |= s->wpresent[i];
+        if (gbits & 1u) {
+            if (threadIdx.x == 0) set_status(a.status, TASQ_ERR_DEVICE);
+            gbits = 0;
+        }
+    } else {
+        gbits = resolve_group_bits(a);
+    }
     const int b = int(gbits & 15u);
     // the shortest certified chunk over the members' precisions is valid for all of them
     int chunk_kb = 0x7FFFFFFF;
-#pragma unroll
-    for (int g = 0; g < kMaxGroups; ++g) {
-        const int bg = int((gbits >> (4 * g)) & 15u);
+    if constexpr (MANY) {
 #pragma unroll
         for (int i = 0; i < kNumB; ++i)
-            if (g < a.groups && bg == kBMin + i) chunk_kb = min(chunk_kb, cert[i]);
+            if ((gbits >> (kBMin + i)) & 1u) chunk_kb = min(chunk_kb, cert[i]);
+    } else {
+#pragma unroll
+        for (int g = 0; g < kMaxGroups; ++g) {
+            const int bg = int((gbits >> (4 * g)) & 15u);
+#pragma unroll
+            for (int i = 0; i < kNumB; ++i)
+                if (g < a.groups && bg == kBMin + i) chunk_kb = min(chunk_kb, cert[i]);
+        }
     }
     // The 8-bit route (uniform over the grid).  Its K block is 256 codes: their e5m2 bytes
     // fill exactly the activation stage, the tensor-memory weight slot and the MMA
@@ -329,7 +364,8 @@ __global__ void __maxnreg__(96)
     // tensor map, the weight tiles per block (two) and the converters' arithmetic differ.
     // It needs an unsplit launch and an exact chunk of at least one such block.
     const int64_t chunk_k64 = int64_t(chunk_kb) * a.chunk_scale;  // exact chunk in 64-code blocks
-    const bool f8 = F8 && p.splits == 1 && chunk_k64 >= 2 * BK / kCertKBlock && f8_route(a, gbits);
+    const bool f8 = F8 && p.splits == 1 && chunk_k64 >= 2 * BK / kCertKBlock &&
+                    (MANY ? gbits != 0 && (gbits >> (kBMaxF8 + 1)) == 0 : f8_route(a, gbits));
     const int KBLK = f8 ? 2 * BK : BK;  // codes of K per block
     if (threadIdx.x == 0) {
         for (int i = 0; i < X_STAGES; ++i)  // producer's expect_tx (+ the converter warps on first stages)
@@ -359,7 +395,7 @@ __global__ void __maxnreg__(96)
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem_base;
-    if (b == 0) {  // uniform across the grid (a launch-wide check, recorded in the status word)
+    if (MANY ? gbits == 0 : b == 0) {  // uniform across the grid (a launch-wide check, recorded in the status word)
         if (warp == 1) ptx::tmem_dealloc(tmem, TMEM_COLS);
         return;
     }
@@ -369,6 +405,11 @@ __global__ void __maxnreg__(96)
         const int ch0 = tile_coord<CONV, BT>(p, wk.t).ch0;
         for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * KBLK, ch0);
     }
+    // b of output channel n: its member layer's
+    auto bits_of = [&](int n) {
+        if constexpr (MANY) return int(s->mbits[min(n / a.group_n, a.groups - 1)]);
+        else return channel_bits(a, gbits, n);
+    };
     // Programmatic dependent launch: this grid may start while the previous kernel
     // (normally the quantization of this layer's activations) still runs.  Only the
     // activation codes and the per-token scales come from it, so only the warps that
@@ -526,7 +567,7 @@ __global__ void __maxnreg__(96)
         for (int w = unit; w < works && ok; w += units) {
             const Work wk = work_item(p, w, KT, chunk);
             // this row's channel runs at its layer's b (a grouped call holds several layers)
-            const uint32_t m = mask_word(channel_bits(a, gbits, tile_coord<CONV, BT>(p, wk.t).ch0 + r));
+            const uint32_t m = mask_word(bits_of(tile_coord<CONV, BT>(p, wk.t).ch0 + r));
             if constexpr (LR) {  // the low-rank block's l1 row, read after the tile's K blocks
                 const int n = tile_coord<CONV, BT>(p, wk.t).ch0 + r;
                 if (kp == 0 && n < a.N) asm volatile("prefetch.global.L1 [%0];" ::"l"(a.lr_l1 + int64_t(n) * a.lr_rank));
@@ -646,7 +687,7 @@ __global__ void __maxnreg__(96)
         const uint32_t lane_base = tmem + (uint32_t(q * 32) << 16);
         // row sums at each channel's b (convolutions are never grouped)
         const int32_t* ts_b = CONV ? a.ts + int64_t(b - kBMin) * a.N * 9 : nullptr;
-        auto rs_of = [&](int n) { return a.rs[int64_t(channel_bits(a, gbits, n) - kBMin) * a.N + n]; };
+        auto rs_of = [&](int n) { return a.rs[int64_t(bits_of(n) - kBMin) * a.N + n]; };
         constexpr bool zp = ZP;  // asymmetric weights: the four-term epilogue
         int cc = 0;
         bool ok = true;
@@ -1282,11 +1323,14 @@ cudaError_t launch_cfg(const GemmArgs& a, const TcPlan& plan, cudaStream_t st, c
         // the eight-converter tiles only serve linear layers with e5m2 codes; the
         // low-rank branch only symmetric linear layers
         if constexpr (C::CONV_WARPS == 8)
-            return a.lr_rank     ? gemm_tc_kernel<false, false, C, true, true>
+            return a.d_layers    ? gemm_tc_kernel<false, false, C, true, false, true>
+                   : a.lr_rank   ? gemm_tc_kernel<false, false, C, true, true>
                    : a.code_sums ? gemm_tc_kernel<false, true, C, true>
                                  : gemm_tc_kernel<false, false, C, true>;
         else
-            return p.conv      ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
+            return p.conv        ? (a.code_sums ? gemm_tc_kernel<true, true, C> : gemm_tc_kernel<true, false, C>)
+                   : a.d_layers ? (f8 ? gemm_tc_kernel<false, false, C, true, false, true>
+                                      : gemm_tc_kernel<false, false, C, false, false, true>)
                    : a.lr_rank ? (f8 ? gemm_tc_kernel<false, false, C, true, true> : gemm_tc_kernel<false, false, C, false, true>)
                    : f8        ? (a.code_sums ? gemm_tc_kernel<false, true, C, true> : gemm_tc_kernel<false, false, C, true>)
                                : (a.code_sums ? gemm_tc_kernel<false, true, C> : gemm_tc_kernel<false, false, C>);
@@ -1344,9 +1388,10 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int num_sms, cudaStream_t st, cons
         return cudaSuccess;
     }
     if (a.M == 0 || a.N == 0) return cudaSuccess;
-    // (the split-K reduction has no low-rank term: such launches stay unsplit)
-    const TcPlan plan =
-        plan_gemm_tc(a.M, a.N, a.K, a.B, a.H, a.W, a.Cin, num_sms, a.split_buf && !a.lr_rank ? a.split_cap : 0);
+    // (the split-K reduction has no low-rank term and reads at most kMaxGroups members'
+    // precisions from the arguments: such launches stay unsplit)
+    const TcPlan plan = plan_gemm_tc(a.M, a.N, a.K, a.B, a.H, a.W, a.Cin, num_sms,
+                                     a.split_buf && !a.lr_rank && !a.d_layers ? a.split_cap : 0);
     if (plan.why) {
         *why = plan.why;
         return cudaSuccess;

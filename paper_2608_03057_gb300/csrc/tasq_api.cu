@@ -345,18 +345,26 @@ TASQ_API int tasq_quant_act_sums(tasq_ctx ctx, const void* d_x, int dtype, int M
 
 namespace {
 
-// layers[0..groups): the member layers of a grouped call (one for a single layer)
+// layers[0..groups): the member layers of a grouped call (one for a single layer), or
+// d_layers[0..groups): the same list in device memory (then layers is unused)
 int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, int stage, const void* d_codes,
                        int code_fmt, const float* d_alpha, const float* d_zc, const int32_t* d_code_sums, int M,
                        const void* d_packed, int N, int K, int B, int H, int W, int Cin, uint16_t* d_y,
                        int32_t* d_acc, tasq_stream stream, const uint16_t* d_lr_u = nullptr,
-                       const uint16_t* d_lr_l1 = nullptr, int lr_rank = 0) {
+                       const uint16_t* d_lr_l1 = nullptr, int lr_rank = 0, const int32_t* d_layers = nullptr) {
     REQUIRE(ctx->L > 0, TASQ_ERR_INVALID_ARG, "no schedule: call tasq_set_schedule first");
-    REQUIRE(layers && groups >= 1 && groups <= tasq::kMaxGroups, TASQ_ERR_INVALID_ARG, "groups %d outside 1..%d",
-            groups, tasq::kMaxGroups);
-    for (int g = 0; g < groups; ++g)
-        REQUIRE(layers[g] >= 0 && layers[g] < ctx->L, TASQ_ERR_INVALID_ARG, "layer %d outside 0..%d", layers[g],
-                ctx->L - 1);
+    if (d_layers) {
+        REQUIRE(groups >= 1 && groups <= tasq::kMaxMembers, TASQ_ERR_INVALID_ARG, "layers %d outside 1..%d", groups,
+                tasq::kMaxMembers);
+        REQUIRE((reinterpret_cast<uintptr_t>(d_layers) & 3u) == 0, TASQ_ERR_UNSUPPORTED,
+                "d_layers must be 4-byte aligned");
+    } else {
+        REQUIRE(layers && groups >= 1 && groups <= tasq::kMaxGroups, TASQ_ERR_INVALID_ARG,
+                "groups %d outside 1..%d", groups, tasq::kMaxGroups);
+        for (int g = 0; g < groups; ++g)
+            REQUIRE(layers[g] >= 0 && layers[g] < ctx->L, TASQ_ERR_INVALID_ARG, "layer %d outside 0..%d", layers[g],
+                    ctx->L - 1);
+    }
     REQUIRE(stage >= -1 && stage < ctx->S, TASQ_ERR_INVALID_ARG, "stage %d outside -1..%d", stage, ctx->S - 1);
     REQUIRE(stage >= 0 || ctx->d_stage, TASQ_ERR_INVALID_ARG, "stage -1 needs tasq_set_stage_device");
     REQUIRE(code_fmt == TASQ_CODES_S8 || code_fmt == TASQ_CODES_F16 || code_fmt == TASQ_CODES_F16_E5M2,
@@ -369,6 +377,8 @@ int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, in
     if (route == TASQ_ROUTE_AUTO) route = code_fmt == TASQ_CODES_S8 ? TASQ_ROUTE_MMA_S8 : TASQ_ROUTE_TC;
     REQUIRE((route == TASQ_ROUTE_TC) == (code_fmt != TASQ_CODES_S8), TASQ_ERR_UNSUPPORTED,
             "route %d cannot read code format %d", route, code_fmt);
+    REQUIRE(!d_layers || route == TASQ_ROUTE_TC, TASQ_ERR_UNSUPPORTED,
+            "a member list in device memory needs the tensor-core route");
     if (M == 0) return TASQ_OK;
     REQUIRE(d_codes && d_alpha && d_zc && d_packed && d_y, TASQ_ERR_INVALID_ARG, "NULL pointer");
     REQUIRE(aligned16(d_codes) && aligned16(d_y) && aligned16(d_acc), TASQ_ERR_UNSUPPORTED,
@@ -402,11 +412,16 @@ int masked_contraction(tasq_ctx ctx, int kind, const int* layers, int groups, in
     a.hdr = reinterpret_cast<const tasq::PackedHeader*>(p);
     a.table = ctx->d_table;
     a.d_stage = ctx->d_stage;
-    a.layer = layers[0];
     a.stage = stage;
     a.groups = groups;
     a.group_n = N / groups;
-    for (int g = 0; g < groups; ++g) a.layers[g] = layers[g];
+    if (d_layers) {
+        a.layer = -1;
+        a.d_layers = d_layers;
+    } else {
+        a.layer = layers[0];
+        for (int g = 0; g < groups; ++g) a.layers[g] = layers[g];
+    }
     a.M = M;
     a.N = N;
     a.K = K;
@@ -502,6 +517,17 @@ TASQ_API int tasq_masked_gemm_grouped(tasq_ctx ctx, const int32_t* h_layers, int
     for (int g = 0; g < groups && g < tasq::kMaxGroups; ++g) layers[g] = h_layers[g];
     return masked_contraction(ctx, TASQ_LINEAR, layers, groups, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr, M,
                               d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream);
+}
+
+TASQ_API int tasq_masked_gemm_shared_input(tasq_ctx ctx, const int32_t* d_layers, int n_layers, int stage,
+                                           const void* d_codes, int code_fmt, const float* d_alpha,
+                                           const float* d_zc, int M, const void* d_packed, int N, int K,
+                                           uint16_t* d_y, int32_t* d_acc, tasq_stream stream) {
+    CHECK_CTX(ctx);
+    REQUIRE(d_layers, TASQ_ERR_INVALID_ARG, "NULL pointer");
+    REQUIRE(code_fmt != TASQ_CODES_S8, TASQ_ERR_UNSUPPORTED, "a member list in device memory needs fp16 codes");
+    return masked_contraction(ctx, TASQ_LINEAR, nullptr, n_layers, stage, d_codes, code_fmt, d_alpha, d_zc, nullptr,
+                              M, d_packed, N, K, 1, 0, 0, 0, d_y, d_acc, stream, nullptr, nullptr, 0, d_layers);
 }
 
 TASQ_API int tasq_masked_conv3x3(tasq_ctx ctx, int layer, int stage, const void* d_codes, int code_fmt,

@@ -20,8 +20,11 @@ constexpr int64_t kCertLimit = int64_t(1) << 17;  // 2^24 / 128: sum |w| bound p
 // [L][S].  The context allocates room for kTableCapacity bits when it is created.
 constexpr int kTableHeader = 16;
 constexpr size_t kTableCapacity = 65536;
-// Most layers one grouped contraction call may hold.
+// Most layers one grouped contraction call may hold: with the member list in
+// the call's arguments (kMaxGroups), or in device memory (kMaxMembers; the
+// tensor-core route resolves every member's b into shared memory).
 constexpr int kMaxGroups = 4;
+constexpr int kMaxMembers = 256;
 // Largest operating precision whose masked weight codes are exact in e5m2: mask_b(v)
 // is t * 2^(8-b) with |t| <= 2^(b-1), at most three significant bits for b <= 4.
 constexpr int kBMaxF8 = 4;
@@ -95,7 +98,8 @@ struct GemmArgs {
     // channels [g * group_n, (g + 1) * group_n) and runs at its own b.
     int groups;               // 1 for a single layer
     int group_n;              // N / groups
-    int layers[kMaxGroups];   // member layers (layers[0] == layer)
+    int layers[kMaxGroups];   // member layers (layers[0] == layer) when d_layers is NULL
+    const int32_t* d_layers;  // member layers in device memory (up to kMaxMembers), or NULL
     int M, N, K;
     int B, H, W, Cin;         // conv geometry (Cin == 0 for a linear layer)
     int per_tensor;
@@ -155,6 +159,21 @@ __device__ inline uint32_t resolve_group_bits(const GemmArgs& a) {
 __device__ __forceinline__ int channel_bits(const GemmArgs& a, uint32_t packed_bits, int n) {
     const int g = a.groups > 1 ? min(n / a.group_n, a.groups - 1) : 0;
     return int((packed_bits >> (4 * g)) & 15u);
+}
+
+// b of member g of a call whose member list is in device memory (a.d_layers), or 0
+// when the stage, the layer index or its table entry is out of range or the header
+// mismatches (the caller records the error).
+__device__ inline int resolve_member_bits(const GemmArgs& a, int g) {
+    const uint32_t magic = a.hdr->magic;
+    const int hdr_n = a.hdr->N, hdr_k = a.hdr->K, hdr_zp = a.hdr->has_zp;
+    const int stage = a.stage >= 0 ? a.stage : (a.d_stage ? *a.d_stage : -1);
+    const int layer = a.d_layers[g];
+    const int2 dims = *reinterpret_cast<const int2*>(a.table);
+    const bool ok = stage >= 0 && stage < dims.y && magic == kPackedMagic && hdr_n == a.N && hdr_k == a.K &&
+                    !(hdr_zp && !a.code_sums) && layer >= 0 && layer < dims.x;
+    const int b = ok ? a.table[kTableHeader + layer * dims.y + stage] : 0;
+    return b >= kBMin && b <= kBMax ? b : 0;
 }
 
 // x / a rounded to nearest even, from ra = RN(1/a): the quotient estimate

@@ -81,6 +81,7 @@ def lib():
                 "tasq_masked_gemm_lr": ([P, I, I, P, I, P, P, I, P, I, I, P, P, I, P, P, P], I),
                 "tasq_lowrank_down": ([P, P, I, I, I, P, I, P, P, P], I),
                 "tasq_masked_gemm_grouped": ([P, P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
+                "tasq_masked_gemm_shared_input": ([P, P, I, I, P, I, P, P, I, P, I, I, P, P, P], I),
                 "tasq_masked_conv3x3": ([P, I, I, P, I, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_masked_conv3x3_zp": ([P, I, I, P, I, P, P, P, I, I, I, I, P, I, P, P, P], I),
                 "tasq_quant_act_tensor_noalloc": ([P, I, I, I, I, I, P, I, P, P, P], I),
@@ -247,6 +248,14 @@ def tasq_masked_gemm_grouped(ctx, layers, stage, codes, code_fmt, alpha, zc, M, 
     _check(ctx, lib().tasq_masked_gemm_grouped(ctx, h, len(layers), int(stage), _ptr(codes), int(code_fmt), _ptr(alpha),
                                                _ptr(zc), int(M), _ptr(packed), int(N), int(K), _ptr(y), _ptr(acc),
                                                _stream(stream)))
+
+
+def tasq_masked_gemm_shared_input(ctx, d_layers, n_layers, stage, codes, code_fmt, alpha, zc, M, packed, N, K, y,
+                                  acc=None, stream=None) -> None:
+    """d_layers: device int32 array of the n_layers member layer indices."""
+    _check(ctx, lib().tasq_masked_gemm_shared_input(ctx, _ptr(d_layers), int(n_layers), int(stage), _ptr(codes),
+                                                    int(code_fmt), _ptr(alpha), _ptr(zc), int(M), _ptr(packed), int(N),
+                                                    int(K), _ptr(y), _ptr(acc), _stream(stream)))
 
 
 def tasq_masked_conv3x3(ctx, layer, stage, codes, code_fmt, alpha, zc, B, H, W, Cin, packed, Cout, y, acc=None,

@@ -197,6 +197,33 @@ def input_groups(layers: List[Layer]) -> List[List[int]]:
     return out
 
 
+# Layers that read the text tokens: the key and value projections of every
+# cross-attention block.  In all three networks the text embedding is computed once
+# per forward pass and is the same tensor for every block.
+TEXT_INPUT_SUFFIXES = (".cross.k", ".cross.v", ".attn2.k", ".attn2.v")
+MAX_SHARED_MEMBERS = 256
+
+
+def shared_input_units(layers: List[Layer], max_members: int = MAX_SHARED_MEMBERS) -> List[List[int]]:
+    """The inventory as units of layers that read one input, with every layer that
+    reads the text tokens gathered into units of one shape (kind, M, N, K) each, at
+    most max_members layers per unit, in inventory order within a unit.  These units
+    come first (their input does not depend on the image tokens, so they can run
+    before any block); every other layer is a unit of its own, in inventory order."""
+    shared = {}
+    rest: List[List[int]] = []
+    for i, l in enumerate(layers):
+        if l.name.endswith(TEXT_INPUT_SUFFIXES):
+            shared.setdefault((l.kind, l.M, l.N, l.K), []).append(i)
+        else:
+            rest.append([i])
+    units: List[List[int]] = []
+    for members in shared.values():  # shapes in order of first appearance
+        for j in range(0, len(members), max_members):
+            units.append(members[j:j + max_members])
+    return units + rest
+
+
 def sweep_shapes():
     """GEMM sweep: M x (K = N) x b."""
     for M in (1024, 4096, 16384):

@@ -1236,6 +1236,129 @@ def test_f8_route_grouped_members_choose_the_path_together(ctx, oracle):
             assert G.assert_bf16_close(yh[:, sl], yb) == yb.size
 
 
+# ------------------------- members listed in device memory (one shared input) --
+
+@pytest.mark.parametrize("code_fmt,n_bits", [(tasq.TASQ_CODES_F16, 8), (F8, 4)], ids=["f16", "e5m2"])
+@pytest.mark.parametrize("M,Ng,K,L", [(300, 128, 256, 56), (77, 136, 256, 9), (33, 8, 128, 256),
+                                      (200, 64, 1152, 40), (129, 1152, 384, 3)])
+def test_shared_input_members_match_single_layers(ctx, oracle, code_fmt, n_bits, M, Ng, K, L):
+    """tasq_masked_gemm_shared_input: L layers (up to 256) that read one input, listed
+    in device memory in a shuffled order, contracted by one launch; each member equals
+    the oracle's single layer at its own b.  Stage 0 draws every b from 2..8 (fp16
+    route), stage 1 from 2..4 (the e5m2 kind when the codes come as e5m2), and the
+    stage is also read from the device int.  Members straddle 128-channel tiles
+    (Ng = 8, 64, 136) or span several (Ng = 1152)."""
+    torch = G.torch()
+    N = L * Ng
+    w = workloads.normal((N, K), 700 + L, 0.02)
+    bias = workloads.normal((N,), 701 + L, 0.02)
+    x = workloads.normal((M, K), 702 + L)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, G.dev(bias), N, K)
+    r = workloads.rng(703 + L)
+    n_table = L + 5  # the table holds layers that are not members too
+    table = np.stack([r.integers(2, 9, n_table), r.integers(2, 5, n_table)], 1).astype(np.uint8)
+    tasq.tasq_set_schedule(ctx.h, table, n_table, 2)
+    layers = r.permutation(n_table)[:L].astype(np.int32)
+    d_layers = G.dev(layers)
+    f8 = code_fmt == F8
+    codes = G.empty(((3 if f8 else 2) * M * K // 2,), torch.float16)
+    alpha, zc = G.empty((M,), torch.float32), G.empty((M,), torch.float32)
+    tasq.tasq_quant_act(ctx.h, G.dev(x), tasq.TASQ_F32, M, K, n_bits, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN, codes,
+                        code_fmt, alpha, zc)
+    wq = oracle.quant_weight(w)
+    s_x, a, z = oracle.quant_act(x, n_bits, oracle.SYMRANGE, oracle.PER_TOKEN)
+    d_stage = torch.zeros((4,), dtype=torch.int32, device="cuda")
+    tasq.tasq_set_stage_device(ctx.h, d_stage)
+    try:
+        for stage, call_stage in ((0, 0), (1, 1), (1, -1)):
+            d_stage.fill_(stage)
+            y = G.empty((M, N), torch.int16)
+            acc = G.empty((M, N), torch.int32)
+            tasq.tasq_masked_gemm_shared_input(ctx.h, d_layers, L, call_stage, codes, code_fmt, alpha, zc, M, packed,
+                                               N, K, y, acc)
+            yh, acch = G.bf16_bits_host(y), acc.cpu().numpy()
+            for g, layer in enumerate(layers):
+                b = int(table[layer, stage])
+                sl = slice(g * Ng, (g + 1) * Ng)
+                ref = oracle.gemm(s_x, wq["s"][sl], b)
+                assert np.array_equal(acch[:, sl], ref), (stage, g, b)
+                _, yb = oracle.epilogue_f32(ref, a, z, oracle.row_sums(wq["s"][sl], b), wq["c"][sl], bias[sl])
+                assert G.assert_bf16_close(yh[:, sl], yb) == yb.size, (stage, g, b)
+    finally:
+        tasq.tasq_set_stage_device(ctx.h, None)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
+def test_shared_input_in_a_graph_and_bad_members(ctx, oracle):
+    """The member list is read at every replay of a captured call (a later change
+    of the list or of the bit table shows in the next replay); a layer index outside
+    the table is found on the device, recorded as TASQ_ERR_DEVICE, and no output is
+    written.  Host-side checks: the member count, the channel split, the code format
+    and a NULL list."""
+    torch = G.torch()
+    M, Ng, K, L = 64, 128, 256, 6
+    N = L * Ng
+    w = workloads.normal((N, K), 711, 0.02)
+    x = workloads.normal((M, K), 712)
+    sw, cw, _ = G.quant_weights(ctx, G.dev(w), tasq.TASQ_F32, N, K)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, None, N, K)
+    table = np.array([[2 + i % 7] for i in range(8)], np.uint8)
+    tasq.tasq_set_schedule(ctx.h, table, 8, 1)
+    codes, alpha, zc = G.quant_act(ctx, G.dev(x), tasq.TASQ_F32, M, K, 8, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN,
+                                   tasq.TASQ_CODES_F16)
+    wq = oracle.quant_weight(w)
+    s_x, a, z = oracle.quant_act(x)
+    d_layers = G.dev(np.arange(L, dtype=np.int32))
+    y = G.empty((M, N), torch.int16)
+
+    def call():
+        tasq.tasq_masked_gemm_shared_input(ctx.h, d_layers, L, 0, codes, tasq.TASQ_CODES_F16, alpha, zc, M, packed, N,
+                                           K, y, None)
+
+    call()
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s), torch.cuda.graph(g, stream=s):
+        call()
+
+    def check(layers):
+        yh = G.bf16_bits_host(y)
+        for m, layer in enumerate(layers):
+            b = int(table[layer, 0])
+            sl = slice(m * Ng, (m + 1) * Ng)
+            ref = oracle.gemm(s_x, wq["s"][sl], b)
+            _, yb = oracle.epilogue_f32(ref, a, z, oracle.row_sums(wq["s"][sl], b), wq["c"][sl])
+            assert np.array_equal(yh[:, sl], yb), (m, layer, b)
+
+    for layers in ([0, 1, 2, 3, 4, 5], [7, 6, 5, 4, 3, 2]):
+        d_layers.copy_(torch.tensor(layers, dtype=torch.int32))
+        y.fill_(0)
+        g.replay()
+        torch.cuda.synchronize()
+        check(layers)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+    d_layers.copy_(torch.tensor([0, 1, 2, 8, 4, 5], dtype=torch.int32))  # layer 8: not in the table
+    y.fill_(0)
+    g.replay()
+    torch.cuda.synchronize()
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_ERR_DEVICE
+    assert not bool(y.any())
+    buf = torch.zeros((1 << 16,), dtype=torch.uint8, device="cuda")
+    big = G.dev(np.zeros(300, np.int32))
+    for dl, n, NN, fmt, code in ((big, 257, 257 * 8, tasq.TASQ_CODES_F16, tasq.TASQ_ERR_INVALID_ARG),  # > 256
+                                 (big, 0, 64, tasq.TASQ_CODES_F16, tasq.TASQ_ERR_INVALID_ARG),          # none
+                                 (big, 3, 64, tasq.TASQ_CODES_F16, tasq.TASQ_ERR_UNSUPPORTED),          # 64 / 3
+                                 (big, 2, 64, tasq.TASQ_CODES_S8, tasq.TASQ_ERR_UNSUPPORTED),           # int8 codes
+                                 (None, 2, 64, tasq.TASQ_CODES_F16, tasq.TASQ_ERR_INVALID_ARG)):        # no list
+        with pytest.raises(tasq.TasqError) as e:
+            tasq.tasq_masked_gemm_shared_input(ctx.h, dl, n, 0, buf, fmt, buf, buf, 16, buf, NN, 64, buf, None)
+        assert e.value.code == code, (n, NN, fmt)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
 def test_e5m2_codes_in_a_convolution_use_the_fp16_codes(ctx, oracle):
     """A 3x3 convolution given dual-format codes reads their fp16 part."""
     torch = G.torch()

@@ -242,3 +242,26 @@ def test_input_groups_pair_cross_attention_keys_and_values():
             assert b == a + 1 and (la.M, la.K) == (lb.M, lb.K)
             assert la.name.rsplit(".", 1)[1] == "k" and lb.name.rsplit(".", 1)[1] == "v"
             assert la.name.rsplit(".", 1)[0] == lb.name.rsplit(".", 1)[0]
+
+
+def test_shared_input_units_gather_every_text_projection():
+    """The benchmark's default units: every layer that reads the text tokens (the key
+    and value projections of all cross-attention blocks) in one unit per shape, at
+    most 256 layers, placed first; every other layer alone, in inventory order."""
+    from paper_2608_03057_gb300 import workloads
+    for name, sizes in (("pixart", [56]), ("sana", [40]), ("sdxl", [20, 120]), ("single", [])):
+        layers = workloads.inventory(name)
+        units = workloads.shared_input_units(layers)
+        assert sorted(i for u in units for i in u) == list(range(len(layers)))
+        shared = [u for u in units if len(u) > 1]
+        assert [len(u) for u in shared] == sizes
+        assert units[:len(shared)] == shared
+        for u in shared:
+            assert all(layers[i].name.rsplit(".", 1)[1] in ("k", "v") for i in u)
+            assert len({(layers[i].kind, layers[i].M, layers[i].N, layers[i].K) for i in u}) == 1
+            assert u == sorted(u)
+        rest = [u[0] for u in units[len(shared):]]
+        assert rest == sorted(rest) and all(len(u) == 1 for u in units[len(shared):])
+        assert not any(layers[i].name.endswith(workloads.TEXT_INPUT_SUFFIXES) for i in rest)
+    layers = workloads.inventory("sdxl")
+    assert [len(u) for u in workloads.shared_input_units(layers, 50) if len(u) > 1] == [20, 50, 50, 20]
