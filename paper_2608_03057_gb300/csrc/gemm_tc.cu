@@ -97,6 +97,9 @@ struct Cfg {
     // is converted, drain a fourth share of the tile's groups
     static constexpr bool HELPERS = NACC == 1 && CONV_WARPS == 4;
     static constexpr int EPI_SLOTS = EPI_WARPS + (HELPERS ? 4 : 0);
+    // output boxes ([16 tokens][32 channels] bf16, 1 KB) one epilogue warp stores per tile:
+    // two per 32-token group it drains (the converter helpers drain at most as many)
+    static constexpr int PIECES = 2 * GPW;
     static constexpr uint32_t ACC_COL = 0;               // NACC x BT fp32 accumulators
     static constexpr uint32_t A_COL = NACC * BT;         // ASLOTS x BK/2 columns (fp16 pairs)
     static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BT);
@@ -105,6 +108,8 @@ struct Cfg {
     static_assert(Q == 1 || X_STAGES % 2 == 0, "first-half stages must keep their parity");
     static_assert(A_COL + AS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
     static_assert(GPW <= MAX_GPW && BT <= 256 && BT % 32 == 0, "tile shape");
+    static_assert(!HELPERS || (GROUPS + EPI_PARTS) / (EPI_PARTS + 1) <= GPW, "helpers drain at most GPW groups");
+    static_assert(EPI_SLOTS * PIECES * 1024 <= X_STAGES * X_STAGE, "a CTA's last tile stages its boxes in the ring");
     static_assert((CONV_WARPS == 4 || CONV_WARPS == 8) && EPI_WARPS <= MAX_EPI_WARPS, "warp roles");
 };
 using CfgStd = Cfg<192, 2>;
@@ -331,7 +336,7 @@ __global__ void __maxnreg__(96)
         }
         present = __reduce_or_sync(0xFFFFFFFFu, present);
         if (lane == 0) s->wpresent[warp] = present;
-        __syncthreads();
+        ptx::cta_sync();
 #pragma unroll
         for (int i = 0; i < THREADS / 32; ++i) gbits |= s->wpresent[i];
         if (gbits & 1u) {
@@ -392,7 +397,7 @@ __global__ void __maxnreg__(96)
     const int chunk = chunk64 < 1 ? 1 : (chunk64 > KT ? KT : int(chunk64));
     const int works = p.tiles_ch * p.tiles_tok * p.splits;
     const int unit = int(blockIdx.x), units = int(gridDim.x);
-    __syncthreads();
+    ptx::cta_sync();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem_base;
     if (MANY ? gbits == 0 : b == 0) {  // uniform across the grid (a launch-wide check, recorded in the status word)
@@ -735,6 +740,9 @@ __global__ void __maxnreg__(96)
             // each of this warp's two groups, written to this warp's shared scratch before
             // the accumulator wait, so the global loads' latency hides under the MMAs.
             bool all_tok_g[GPW];
+            // where this tile's output boxes are staged: this warp's box (step 0), or (the
+            // CTA's last tile) a 1 KB box per piece in the activation ring
+            uint32_t stg_base = ptx::smem_u32(s->ep_stage[e]), stg_step = 0;
             __syncwarp();  // the previous tile's reads of the scratch are done
 #pragma unroll
             for (int gi = 0; gi < GPW; ++gi) {
@@ -894,8 +902,11 @@ __global__ void __maxnreg__(96)
                         pk[k][tp] = *reinterpret_cast<const uint32_t*>(&hb);
                     }
                 }
-                uint16_t* stg = s->ep_stage[e];
-                if (lane == 0) ptx::bulk_wait_read0();  // the previous box has left the buffer
+                // The CTA's last tile stages every box in its own 1 KB of the activation ring,
+                // idle once the tile's last MMA has completed, so no box waits for the store
+                // of the one before; other tiles share this warp's box.
+                const uint32_t stg = stg_base + uint32_t(gi * 2 + (j0 >> 4)) * stg_step;
+                if (stg_step == 0 && lane == 0) ptx::bulk_wait_read0();  // the previous box has left the buffer
                 __syncwarp();
                 {
                     // stored matrix i = lane / 8: (channel block, token block) = (i & 1, i >> 1), plus
@@ -904,7 +915,7 @@ __global__ void __maxnreg__(96)
                     // so the eight rows of each stored matrix fall in eight different bank groups
                     const int i = lane >> 3, kr = lane & 7;
                     const int t = (i >> 1) * 8 + kr, sw = (t >> 1) & 3;
-                    const uint32_t row = ptx::smem_u32(stg) + uint32_t(t * 64);
+                    const uint32_t row = stg + uint32_t(t * 64);
                     ptx::stmatrix_x4_trans(row + uint32_t((((i & 1)) ^ sw) << 4), pk[0][0], pk[1][0], pk[0][1], pk[1][1]);
                     ptx::stmatrix_x4_trans(row + uint32_t(((2 + (i & 1)) ^ sw) << 4), pk[2][0], pk[3][0], pk[2][1],
                                            pk[3][1]);
@@ -913,7 +924,7 @@ __global__ void __maxnreg__(96)
                 __syncwarp();
                 const int xc = tc.ch0 + q * 32, yt = tc.tok0 + g * 32 + j0;
                 if (lane == 0 && xc < a.N && yt < a.M) {
-                    ptx::tma_store_2d(&tm_y, ptx::smem_u32(stg), xc, yt);
+                    ptx::tma_store_2d(&tm_y, stg, xc, yt);
                     ptx::bulk_commit();
                 }
                 if (a.acc) {  // int32 accumulators (a debugging output): plain stores
@@ -947,6 +958,13 @@ __global__ void __maxnreg__(96)
                 ptx::tc_fence_after();
                 const uint32_t acc_base = lane_base + C::ACC_COL + buf * BT;
                 const bool last = c == nchunks - 1;
+                // the last chunk of the CTA's last tile: no activation stage is loaded or read
+                // again (its last MMA has completed), so the ring can hold the output boxes
+                if (!CONV && last && w + units >= works) {
+                    stg_base = ptx::smem_u32(&s->x[0][0]) + uint32_t(e * C::PIECES) * 1024u;
+                    stg_step = 1024;
+                    ptx::fence_proxy_async_smem();  // after the ring's TMA writes and MMA reads
+                }
 #pragma unroll 1
                 for (int gi = 0; gi < gpw; ++gi) {
                     const int g = part * gpw + gi;
@@ -1011,15 +1029,18 @@ __global__ void __maxnreg__(96)
         }
     }
 
-    // epilogue TMA stores complete before the CTA exits
-    if (!CONV && lane == 0 &&
-        ((warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS) || (helpers && warp >= 2 && warp < EPI_WARP0)))
-        ptx::bulk_wait0();
-    __syncthreads();
+    // every thread of the CTA, the epilogue's last tensor-memory reads included, is past
+    // its role before tensor memory is released (a barrier that counts threads: see
+    // ptx::cta_sync)
+    ptx::cta_sync();
     if (warp == 1) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, TMEM_COLS);
     }
+    // epilogue TMA stores complete before the CTA exits
+    if (!CONV && lane == 0 &&
+        ((warp >= EPI_WARP0 && warp < EPI_WARP0 + EPI_WARPS) || (helpers && warp >= 2 && warp < EPI_WARP0)))
+        ptx::bulk_wait0();
 }
 
 // Split-K second half: adds the slices' exact int32 partial sums in slice

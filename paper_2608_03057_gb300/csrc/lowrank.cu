@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(kDownWarps * 32, 2)
         red(warp)[g + 8][nt * 8 + 2 * t] = d[nt][2];
         red(warp)[g + 8][nt * 8 + 2 * t + 1] = d[nt][3];
     }
-    __syncthreads();
+    ptx::cta_sync();
     // u' rows of 64 fp16: the rank columns, then zeros
     for (int i = threadIdx.x; i < 16 * 64; i += blockDim.x) {
         const int row = i >> 6, col = i & 63, m = m0 + row;
@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(128)
         ptx::prefetch_tmap(&tm_x);
         ptx::prefetch_tmap(&tm_l2);
     }
-    __syncthreads();
+    ptx::cta_sync();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem;
     bool ok = true;
@@ -314,7 +314,7 @@ __global__ void __launch_bounds__(128)
         if (*(volatile int*)&s->abort) set_status(status, TASQ_ERR_DEVICE_TIMEOUT);
     }
     ptx::tc_fence_before();
-    __syncthreads();
+    ptx::cta_sync();
     if (warp == 0) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, 32);

@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(128) probe_mma_kernel(const uint8_t* __restric
         ptx::tmem_relinquish();
         ptx::tc_fence_before();
     }
-    __syncthreads();
+    ptx::cta_sync();
     ptx::tc_fence_after();
     const uint32_t tmem = s->tmem;
     // instruction descriptor: fp32 D; A and B format 0 (f16 for kind::f16, e4m3 for
@@ -103,7 +103,7 @@ __global__ void __launch_bounds__(128) probe_mma_kernel(const uint8_t* __restric
         const long long c1 = clock64();
         cycles[blockIdx.x] = ok ? (unsigned long long)(c1 - c0) : 0ull;
     }
-    __syncthreads();
+    ptx::cta_sync();
     ptx::tc_fence_after();
     if (blockIdx.x == 0 && cycles[0] != 0) {
         // D rows = TMEM lanes: warp w reads lanes 32 w .. 32 w + 31, 16 columns at a time
@@ -116,7 +116,7 @@ __global__ void __launch_bounds__(128) probe_mma_kernel(const uint8_t* __restric
         }
     }
     ptx::tc_fence_before();
-    __syncthreads();
+    ptx::cta_sync();
     if (warp == 0) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, 512);

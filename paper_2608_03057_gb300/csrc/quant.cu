@@ -464,7 +464,7 @@ __global__ void __launch_bounds__(256) tensor_range_kernel(const void* __restric
         slo[warp] = lo;
         shi[warp] = hi;
     }
-    __syncthreads();
+    ptx::cta_sync();
     if (threadIdx.x == 0) {
         for (int i = 1; i < int(blockDim.x >> 5); ++i) {
             lo = fminf(lo, slo[i]);
@@ -554,7 +554,7 @@ __global__ void __launch_bounds__(256) pack_sums_kernel(const int8_t* __restrict
     __shared__ int red[kNumB][9];
     if (threadIdx.x < kNumB * 9) red[threadIdx.x / 9][threadIdx.x % 9] = 0;
     for (int i = threadIdx.x; i < kNumB * KB; i += blockDim.x) smem_sums[i] = 0;
-    __syncthreads();
+    ptx::cta_sync();
     // per-thread partials: [b][tap] signed sums; block abs sums via shared atomics
     int part[kNumB][9];
 #pragma unroll
@@ -583,7 +583,7 @@ __global__ void __launch_bounds__(256) pack_sums_kernel(const int8_t* __restrict
             for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
             if ((threadIdx.x & 31) == 0 && s) atomicAdd(&red[bi][t], s);
         }
-    __syncthreads();
+    ptx::cta_sync();
     if (threadIdx.x < kNumB) {
         int bi = threadIdx.x;
         int tot = 0;
@@ -597,7 +597,7 @@ __global__ void __launch_bounds__(256) pack_sums_kernel(const int8_t* __restrict
     // chunks) make the property monotone in C, so the minimum over channels is
     // valid for every channel.  C = (shortest window whose sum exceeds the
     // bound) - 1, found by two pointers over the non-negative block sums.
-    __syncthreads();
+    ptx::cta_sync();
     if (threadIdx.x < kNumB) {
         const int bi = threadIdx.x;
         const int* S = smem_sums + bi * KB;
@@ -794,7 +794,7 @@ __global__ void __launch_bounds__(256) noalloc_range_kernel(const void* __restri
         slo[warp] = lo;
         shi[warp] = hi;
     }
-    __syncthreads();
+    ptx::cta_sync();
     if (threadIdx.x == 0) {
         for (int i = 1; i < int(blockDim.x >> 5); ++i) {
             lo = fminf(lo, slo[i]);
@@ -824,7 +824,7 @@ __global__ void __launch_bounds__(256) noalloc_quant_kernel(const void* __restri
             s_hi = hi;
         }
     }
-    __syncthreads();
+    ptx::cta_sync();
     float lo = s_lo, hi = s_hi;
     if (mode == TASQ_SYMRANGE) {
         hi = fmaxf(fabsf(lo), fabsf(hi));

@@ -20,6 +20,12 @@ __device__ __forceinline__ uint64_t globaltimer() {
 // Block until the preceding kernel in the stream has completed and its memory
 // is visible (a no-op when this grid was launched without the PDL attribute).
 __device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// CTA-wide barrier 0 in its non-aligned form, which counts the threads that arrive:
+// correct when the lanes of a warp reach it at different times (after role code that
+// only lane 0 runs).  __syncthreads compiles to the aligned form, which expects each
+// warp to arrive converged; after such role code a traced build saw it let a CTA pass
+// 1-2 us before its epilogue warps arrived, even with __syncwarp in front of it.
+__device__ __forceinline__ void cta_sync() { asm volatile("barrier.sync 0;" ::: "memory"); }
 // Allow the next kernel in the stream to be launched ahead of this grid's exit.
 __device__ __forceinline__ void grid_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
