@@ -404,12 +404,6 @@ __global__ void __maxnreg__(96)
         if (warp == 1) ptx::tmem_dealloc(tmem, TMEM_COLS);
         return;
     }
-    if (warp == WPROD_WARP && lane == 0 && unit < works) {
-        // pull the first weight tiles into L2 ahead of the weight ring
-        const Work wk = work_item(p, unit, KT, chunk);
-        const int ch0 = tile_coord<CONV, BT>(p, wk.t).ch0;
-        for (int kb = wk.kb_lo; kb < wk.kb_hi && kb < wk.kb_lo + 8; ++kb) ptx::tma_prefetch_2d(&tm_w, kb * KBLK, ch0);
-    }
     // b of output channel n: its member layer's
     auto bits_of = [&](int n) {
         if constexpr (MANY) return int(s->mbits[min(n / a.group_n, a.groups - 1)]);
@@ -487,6 +481,12 @@ __global__ void __maxnreg__(96)
                     const uint32_t fb = ptx::smem_u32(&s->wfull[rw.slot]);
                     ptx::mbar_arrive_expect_tx(fb, W_STAGE);
                     ptx::tma_load_2d(ptx::smem_u32(s->w[rw.slot]), &tm_w, fb, kw * BK, ch0);
+                    if (nw == W_STAGES - 1) {
+                        // the ring is full: pull the first tile's next weight tiles into L2
+                        // ahead of it (after its first loads, which the converters wait for)
+                        for (int k2 = kw + 1; k2 < wk.kb_hi * wpb && k2 < (wk.kb_lo + 8) * wpb; ++k2)
+                            ptx::tma_prefetch_2d(&tm_w, k2 * BK, ch0);
+                    }
                 }
             }
             for (int j = nw - W_STAGES < 0 ? 0 : nw - W_STAGES; j < nw; ++j)
