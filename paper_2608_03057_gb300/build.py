@@ -17,7 +17,7 @@ OBJ = os.path.join(HERE, "_build")
 LIB_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(LIB_DIR, "libtasq.so")
 SOURCES = ["tasq_api.cu", "quant.cu", "gemm_s8.cu", "gemm_tc.cu", "probe_mma.cu", "lowrank.cu"]
-HEADERS = ["tasq_internal.cuh", "tc_ptx.cuh"]
+HEADERS = ["tasq_internal.cuh", "tc_ptx.cuh", "act_quant.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -7,6 +7,7 @@
 #include <cstdio>
 #include <mutex>
 
+#include "act_quant.cuh"
 #include "tasq_internal.cuh"
 #include "tc_ptx.cuh"
 
@@ -55,21 +56,6 @@ __device__ inline int warp_sum(int v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
-}
-
-// Quantization range of a group: [lo, hi] -> (alpha, z) in the fp32 order
-// alpha = (hi - lo) / denom, z = -lo / alpha; a constant group gets alpha = 1
-// and z = half (symmetric range) or -lo.
-__device__ inline void scale_of_range(float lo, float hi, float denom, float half, int mode, float* alpha,
-                                      float* z) {
-    float range = __fsub_rn(hi, lo);
-    if (range == 0.0f) {
-        *alpha = 1.0f;
-        *z = (mode == TASQ_SYMRANGE) ? half : -lo;
-    } else {
-        *alpha = __fdiv_rn(range, denom);
-        *z = __fdiv_rn(-lo, *alpha);
-    }
 }
 
 // Activation code: Q = clamp(rint(x / alpha + z), 0, qmax), s = Q - half.
@@ -292,14 +278,9 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
     }
     lo = warp_min(lo);
     hi = warp_max(hi);
-    if (mode == TASQ_SYMRANGE) {
-        hi = fmaxf(fabsf(lo), fabsf(hi));
-        lo = -hi;
-    }
+    const RowScale rs = row_scale(lo, hi, n_bits, mode);
+    const float alpha = rs.alpha, z = rs.z, ralpha = rs.ralpha;
     const int half = 1 << (n_bits - 1), qmax = (1 << n_bits) - 1;
-    float alpha, z;
-    scale_of_range(lo, hi, float(qmax), float(half), mode, &alpha, &z);
-    const float ralpha = __frcp_rn(alpha);
     const float qmaxf = float(qmax);
     const float2 ra2 = make_float2(ralpha, ralpha), na2 = make_float2(-alpha, -alpha), z2 = make_float2(z, z);
     // 1.5 * 2^23 + 0x6400: RN(u + this) is the integer rint(u) + this, whose fp32 bits
@@ -313,6 +294,13 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
     for (int k = 0; k < NPL; ++k) {
         const int c = lane + 32 * k;
         if (c >= chunks) continue;
+        if constexpr (DTYPE == TASQ_BF16 && CODES != TASQ_CODES_S8 && !SUMS) {
+            const uint4 pk = codes8_f16_of_bf16(d[k], rs, half);
+            reinterpret_cast<uint4*>(out)[c] = pk;
+            if constexpr (CODES == TASQ_CODES_F16_E5M2)
+                reinterpret_cast<uint2*>(out8)[c] = make_uint2(ptx::e5m2x4(pk.x, pk.y), ptx::e5m2x4(pk.z, pk.w));
+            continue;
+        }
         // vb[j]: fp32 bits of Q + 1.5 * 2^23 + 0x6400 with Q = clamp(rint(x / alpha + z),
         // 0, qmax), so the low 16 bits are 0x6400 + Q (clamping u to the integer bounds
         // before rounding gives the same Q as rounding first); x / alpha as div_rn_by.  Element pairs: every packed
