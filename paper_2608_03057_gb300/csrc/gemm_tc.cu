@@ -20,7 +20,9 @@
 //   B: the activation codes, held as fp16 integers in HBM, brought by TMA
 //      into 128-byte-swizzled shared memory (a 2-D tile for a linear layer; a
 //      4-D NHWC box shifted by the 3x3 tap for a convolution, whose padding
-//      TMA fills with code 0).
+//      TMA fills with code 0).  4-bit codes also come as e5m2 bytes; with every
+//      member at b <= 4 a linear layer's K loop runs on the 8-bit-float MMA kind
+//      (256-code K blocks of two weight tiles).
 //   D: fp32 accumulators in tensor memory, double-buffered (192- and 64-token
 //      tiles) so the epilogue of one chunk overlaps the MMAs of the next, or
 //      single (256-token tiles, one tile per CTA).
@@ -30,11 +32,15 @@
 // weights (and, for a single-tile CTA, join the epilogue once the last K block
 // is converted); warps 6..17 drain accumulators and run the fused
 // dequantization epilogue (linear outputs leave through TMA stores of
-// swizzled [16 token][32 channel] boxes); warp 18 issues the weight TMA.  The
-// grid is persistent: one CTA per SM walks the output tiles.  Every wait is
-// bounded by the context's time limit; a wait that gives up records
-// TASQ_ERR_DEVICE_TIMEOUT, the CTA drains its copies in flight, frees its
-// tensor memory and returns.
+// swizzled [16 token][32 channel] boxes, staged in the idle activation ring on
+// the CTA's last tile); warp 18 issues the weight TMA.  The grid is persistent:
+// one CTA per SM walks the output tiles.  A call may hold several layers that
+// read one input, each at its own b (channels [g Ng, (g+1) Ng) are member g's),
+// listed in the arguments or, up to kMaxMembers, in device memory.  The roles
+// diverge within warps, so the CTA's barriers count threads (ptx::cta_sync).
+// Every wait is bounded by the context's time limit; a wait that gives up
+// records TASQ_ERR_DEVICE_TIMEOUT, the CTA drains its copies in flight, frees
+// its tensor memory and returns.
 #include <cstdio>
 #include <cstdlib>
 #include <type_traits>
