@@ -111,6 +111,10 @@ struct Cfg {
     static constexpr uint32_t IDESC = ptx::idesc_f16_f32(BCH, BT);
     static constexpr uint32_t IDESC8 = ptx::idesc_e5m2_f32(BCH, BT);  // the 8-bit route
     static_assert(DONE % X_STAGES == 0 && DONE >= (AS + 1) * Q, "completion ring covers both reuse distances");
+    // A converter arrives on K block j's first-stage barrier after the MMAs of block j - AS
+    // completed; that barrier last served block j - X_STAGES / Q, whose phase must be closed
+    // by then, or the arrival would count toward the wrong phase.
+    static_assert(AS * Q <= X_STAGES, "converter arrivals stay within the stage ring");
     static_assert(Q == 1 || X_STAGES % 2 == 0, "first-half stages must keep their parity");
     static_assert(A_COL + AS * A_SLOT_COLS <= TMEM_COLS, "tensor memory budget");
     static_assert(GPW <= MAX_GPW && BT <= 256 && BT % 32 == 0, "tile shape");
@@ -120,12 +124,15 @@ struct Cfg {
 };
 using CfgStd = Cfg<192, 2>;
 using CfgWide = Cfg<256, 1>;
-using CfgNarrow = Cfg<64, 2>;  // few tokens (cross-attention keys and values): more CTAs, shorter epilogue
+// few tokens (cross-attention keys and values): more CTAs, shorter epilogue; its tensor memory
+// has room for a third converted-weight slot (2 x 64 + 3 x 64 columns), which gives the
+// converters a block more of slack (measured ~1-2 % per layer)
+using CfgNarrow = Cfg<64, 2, 4, 3>;
 // The two-accumulator tiles for linear layers whose codes also come as e5m2: the 8-bit
 // route's block of two weight tiles is shared out between two converter warps per lane
 // quadrant (one tile each), with eight epilogue warps.
 using CfgStdF8 = Cfg<192, 2, 8>;
-using CfgNarrowF8 = Cfg<64, 2, 8>;
+using CfgNarrowF8 = Cfg<64, 2, 8, 3>;
 
 // Synchronisation is arranged so that the single MMA-issuing thread, whose
 // per-instruction cost bounds the K loop, does one wait and one commit per
@@ -133,11 +140,11 @@ using CfgNarrowF8 = Cfg<64, 2, 8>;
 //   xfull[u % X_STAGES]  completes when its activation bytes have landed (TMA
 //                 transaction bytes) and, for the first stage of a K block,
 //                 when the four converter warps have written the block's
-//                 weights into tensor-memory slot j % 2;
+//                 weights into tensor-memory slot j % AS;
 //   done[u % DONE]  completes when the MMAs reading stage u have finished; the
 //                 activation producer waits on it before refilling the stage
 //                 with u + X_STAGES, the converters (on the last stage of block
-//                 j) before overwriting slot j % 2 with block j + 2.
+//                 j) before overwriting slot j % AS with block j + AS.
 // The weight ring is separate: a weight stage is released as soon as the
 // converters have read it, so weight tiles run several K blocks ahead.
 template <class C>
