@@ -1290,6 +1290,42 @@ def test_shared_input_members_match_single_layers(ctx, oracle, code_fmt, n_bits,
     assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
 
 
+@pytest.mark.parametrize("M,Ng,K,L", [(300, 1152, 1152, 56), (77, 1280, 2048, 120)], ids=["pixart_text", "sdxl_text"])
+def test_shared_input_full_size_sampled_rows(ctx, oracle, M, Ng, K, L):
+    """The text units at the sizes the bench runs them (every cross-attention key and value
+    projection of PixArt-Sigma's 28 blocks, of SDXL-Turbo's 60 width-1280 blocks) in the
+    same launch: sampled token rows (the first, the last and six in between) of every
+    member's output against the oracle's single layer at that member's b."""
+    torch = G.torch()
+    N = L * Ng
+    wd = workloads.device_normal((N, K), 730 + L, 0.02)
+    sw, cw, _ = G.quant_weights(ctx, wd, tasq.TASQ_F32, N, K)
+    del wd
+    bias = workloads.normal((N,), 731 + L, 0.02)
+    packed = G.pack(ctx, tasq.TASQ_LINEAR, sw, cw, G.dev(bias), N, K)
+    swh, cwh = sw.cpu().numpy(), cw.cpu().numpy()
+    r = workloads.rng(732 + L)
+    table = r.integers(2, 9, (L, 1)).astype(np.uint8)
+    tasq.tasq_set_schedule(ctx.h, table, L, 1)
+    d_layers = G.dev(np.arange(L, dtype=np.int32))
+    x = workloads.normal((M, K), 733 + L)
+    codes, alpha, zc = G.quant_act(ctx, G.dev(x), tasq.TASQ_F32, M, K, 8, tasq.TASQ_SYMRANGE, tasq.TASQ_PER_TOKEN,
+                                   tasq.TASQ_CODES_F16)
+    y = G.empty((M, N), torch.int16)
+    tasq.tasq_masked_gemm_shared_input(ctx.h, d_layers, L, 0, codes, tasq.TASQ_CODES_F16, alpha, zc, M, packed, N, K,
+                                       y, None)
+    rows = np.unique(np.concatenate([[0, M - 1], r.integers(0, M, 6)]))
+    yh = G.bf16_bits_host(y)[rows]
+    s_x, a, z = oracle.quant_act(x)
+    for g in range(L):
+        b = int(table[g, 0])
+        sl = slice(g * Ng, (g + 1) * Ng)
+        ref = oracle.gemm(s_x[rows], swh[sl], b)
+        _, yb = oracle.epilogue_f32(ref, a[rows], z[rows], oracle.row_sums(swh[sl], b), cwh[sl], bias[sl])
+        assert np.array_equal(yh[:, sl], yb), (g, b)
+    assert tasq.tasq_device_status(ctx.h) == tasq.TASQ_OK
+
+
 def test_shared_input_in_a_graph_and_bad_members(ctx, oracle):
     """The member list is read at every replay of a captured call (a later change
     of the list or of the bit table shows in the next replay); a layer index outside
