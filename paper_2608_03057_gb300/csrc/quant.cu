@@ -299,79 +299,79 @@ __global__ void __launch_bounds__(kRegRowWarps * 32) quant_act_rowreg_kernel(con
             reinterpret_cast<uint4*>(out)[c] = pk;
             if constexpr (CODES == TASQ_CODES_F16_E5M2)
                 reinterpret_cast<uint2*>(out8)[c] = make_uint2(ptx::e5m2x4(pk.x, pk.y), ptx::e5m2x4(pk.z, pk.w));
-            continue;
-        }
-        // vb[j]: fp32 bits of Q + 1.5 * 2^23 + 0x6400 with Q = clamp(rint(x / alpha + z),
-        // 0, qmax), so the low 16 bits are 0x6400 + Q (clamping u to the integer bounds
-        // before rounding gives the same Q as rounding first); x / alpha as div_rn_by.  Element pairs: every packed
-        // f32x2 operation rounds each lane exactly as the scalar one (the divide's
-        // remainder fma(-q, a, x) is taken as fma(q, -a, x)).
-        uint32_t vb[EPC];
-#pragma unroll
-        for (int j = 0; j < EPC; j += 2) {
-            const float2 x2 = make_float2(elem(d[k], j), elem(d[k], j + 1));
-            const float2 q2 = ptx::fmul2(x2, ra2);
-            const float2 r2 = ptx::ffma2(q2, na2, x2);
-            const float2 u2 = ptx::fadd2(ptx::ffma2(r2, ra2, q2), z2);
-            // For a finite row whose alpha is a normal float, u stays within (-0.5,
-            // qmax + 0.5) (alpha and z come from the row's own range; the error is a few
-            // ulps of qmax), so the clamp never binds and fp16 codes are clamped once,
-            // packed, after the subtraction below instead (which also keeps codes in
-            // range for inputs outside that class).  Integer codes and code sums take Q
-            // from the bits here, so they clamp u first.
-            float2 c2 = u2;
-            if constexpr (CODES == TASQ_CODES_S8 || SUMS)
-                c2 = make_float2(fminf(fmaxf(u2.x, 0.0f), qmaxf), fminf(fmaxf(u2.y, 0.0f), qmaxf));
-            const float2 v2 = ptx::fadd2(c2, magic2);
-            vb[j] = __float_as_uint(v2.x);
-            vb[j + 1] = __float_as_uint(v2.y);
-        }
-        int q[EPC];
-#pragma unroll
-        for (int j = 0; j < EPC; ++j) q[j] = int(vb[j] & 0xFFFFu) - (0x6400 + half);
-        if constexpr (SUMS) {
-#pragma unroll
-            for (int j = 0; j < EPC; ++j) csum += q[j];
-        }
-        if (CODES == TASQ_CODES_S8) {
-            if (EPC == 8) {
-                uint2 pk;
-                pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((uint32_t)(q[3] & 0xFF) << 24);
-                pk.y = (q[4 % EPC] & 0xFF) | ((q[5 % EPC] & 0xFF) << 8) | ((q[6 % EPC] & 0xFF) << 16) |
-                       ((uint32_t)(q[7 % EPC] & 0xFF) << 24);
-                reinterpret_cast<uint2*>(out)[c] = pk;
-            } else {
-                reinterpret_cast<uint32_t*>(out)[c] =
-                    (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2 % EPC] & 0xFF) << 16) | ((uint32_t)(q[3 % EPC] & 0xFF) << 24);
-            }
         } else {
-            // fp16 of a small integer s: the bits 0x6400 + (s + half) hold 1024 + s + half
-            // exactly; one packed subtraction of 1024 + half leaves s
-            const uint32_t off = 0x6400u + uint32_t(half);
-            const __half2 bias2 = __halves2half2(__ushort_as_half(uint16_t(off)), __ushort_as_half(uint16_t(off)));
-            // the low halves of two vb words, 0x6400 + Q each, are the fp16 values
-            // 1024 + Q; one packed subtraction of 1024 + half leaves the codes s = Q - half
-            const __half2 lo2 = __float2half2_rn(float(-half)), hi2 = __float2half2_rn(float(half - 1));
-            auto sub2 = [&](uint32_t v0, uint32_t v1) -> uint32_t {
-                uint32_t w = __byte_perm(v0, v1, 0x5410);
-                __half2 r = __hsub2(*reinterpret_cast<__half2*>(&w), bias2);
-                if constexpr (!SUMS) r = __hmax2(__hmin2(r, hi2), lo2);
-                return *reinterpret_cast<uint32_t*>(&r);
-            };
-            const uint32_t* h = vb;
-            if (EPC == 8) {
-                uint4 pk;
-                pk.x = sub2(h[0], h[1]);
-                pk.y = sub2(h[2], h[3]);
-                pk.z = sub2(h[4 % EPC], h[5 % EPC]);
-                pk.w = sub2(h[6 % EPC], h[7 % EPC]);
-                reinterpret_cast<uint4*>(out)[c] = pk;
-                if constexpr (CODES == TASQ_CODES_F16_E5M2)
-                    reinterpret_cast<uint2*>(out8)[c] = make_uint2(ptx::e5m2x4(pk.x, pk.y), ptx::e5m2x4(pk.z, pk.w));
+            // vb[j]: fp32 bits of Q + 1.5 * 2^23 + 0x6400 with Q = clamp(rint(x / alpha + z),
+            // 0, qmax), so the low 16 bits are 0x6400 + Q (clamping u to the integer bounds
+            // before rounding gives the same Q as rounding first); x / alpha as div_rn_by.  Element pairs: every packed
+            // f32x2 operation rounds each lane exactly as the scalar one (the divide's
+            // remainder fma(-q, a, x) is taken as fma(q, -a, x)).
+            uint32_t vb[EPC];
+    #pragma unroll
+            for (int j = 0; j < EPC; j += 2) {
+                const float2 x2 = make_float2(elem(d[k], j), elem(d[k], j + 1));
+                const float2 q2 = ptx::fmul2(x2, ra2);
+                const float2 r2 = ptx::ffma2(q2, na2, x2);
+                const float2 u2 = ptx::fadd2(ptx::ffma2(r2, ra2, q2), z2);
+                // For a finite row whose alpha is a normal float, u stays within (-0.5,
+                // qmax + 0.5) (alpha and z come from the row's own range; the error is a few
+                // ulps of qmax), so the clamp never binds and fp16 codes are clamped once,
+                // packed, after the subtraction below instead (which also keeps codes in
+                // range for inputs outside that class).  Integer codes and code sums take Q
+                // from the bits here, so they clamp u first.
+                float2 c2 = u2;
+                if constexpr (CODES == TASQ_CODES_S8 || SUMS)
+                    c2 = make_float2(fminf(fmaxf(u2.x, 0.0f), qmaxf), fminf(fmaxf(u2.y, 0.0f), qmaxf));
+                const float2 v2 = ptx::fadd2(c2, magic2);
+                vb[j] = __float_as_uint(v2.x);
+                vb[j + 1] = __float_as_uint(v2.y);
+            }
+            int q[EPC];
+    #pragma unroll
+            for (int j = 0; j < EPC; ++j) q[j] = int(vb[j] & 0xFFFFu) - (0x6400 + half);
+            if constexpr (SUMS) {
+    #pragma unroll
+                for (int j = 0; j < EPC; ++j) csum += q[j];
+            }
+            if (CODES == TASQ_CODES_S8) {
+                if (EPC == 8) {
+                    uint2 pk;
+                    pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((uint32_t)(q[3] & 0xFF) << 24);
+                    pk.y = (q[4 % EPC] & 0xFF) | ((q[5 % EPC] & 0xFF) << 8) | ((q[6 % EPC] & 0xFF) << 16) |
+                           ((uint32_t)(q[7 % EPC] & 0xFF) << 24);
+                    reinterpret_cast<uint2*>(out)[c] = pk;
+                } else {
+                    reinterpret_cast<uint32_t*>(out)[c] =
+                        (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2 % EPC] & 0xFF) << 16) | ((uint32_t)(q[3 % EPC] & 0xFF) << 24);
+                }
             } else {
-                const uint2 pk = make_uint2(sub2(h[0], h[1]), sub2(h[2 % EPC], h[3 % EPC]));
-                reinterpret_cast<uint2*>(out)[c] = pk;
-                if constexpr (CODES == TASQ_CODES_F16_E5M2) reinterpret_cast<uint32_t*>(out8)[c] = ptx::e5m2x4(pk.x, pk.y);
+                // fp16 of a small integer s: the bits 0x6400 + (s + half) hold 1024 + s + half
+                // exactly; one packed subtraction of 1024 + half leaves s
+                const uint32_t off = 0x6400u + uint32_t(half);
+                const __half2 bias2 = __halves2half2(__ushort_as_half(uint16_t(off)), __ushort_as_half(uint16_t(off)));
+                // the low halves of two vb words, 0x6400 + Q each, are the fp16 values
+                // 1024 + Q; one packed subtraction of 1024 + half leaves the codes s = Q - half
+                const __half2 lo2 = __float2half2_rn(float(-half)), hi2 = __float2half2_rn(float(half - 1));
+                auto sub2 = [&](uint32_t v0, uint32_t v1) -> uint32_t {
+                    uint32_t w = __byte_perm(v0, v1, 0x5410);
+                    __half2 r = __hsub2(*reinterpret_cast<__half2*>(&w), bias2);
+                    if constexpr (!SUMS) r = __hmax2(__hmin2(r, hi2), lo2);
+                    return *reinterpret_cast<uint32_t*>(&r);
+                };
+                const uint32_t* h = vb;
+                if (EPC == 8) {
+                    uint4 pk;
+                    pk.x = sub2(h[0], h[1]);
+                    pk.y = sub2(h[2], h[3]);
+                    pk.z = sub2(h[4 % EPC], h[5 % EPC]);
+                    pk.w = sub2(h[6 % EPC], h[7 % EPC]);
+                    reinterpret_cast<uint4*>(out)[c] = pk;
+                    if constexpr (CODES == TASQ_CODES_F16_E5M2)
+                        reinterpret_cast<uint2*>(out8)[c] = make_uint2(ptx::e5m2x4(pk.x, pk.y), ptx::e5m2x4(pk.z, pk.w));
+                } else {
+                    const uint2 pk = make_uint2(sub2(h[0], h[1]), sub2(h[2 % EPC], h[3 % EPC]));
+                    reinterpret_cast<uint2*>(out)[c] = pk;
+                    if constexpr (CODES == TASQ_CODES_F16_E5M2) reinterpret_cast<uint32_t*>(out8)[c] = ptx::e5m2x4(pk.x, pk.y);
+                }
             }
         }
     }
